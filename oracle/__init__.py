@@ -1,0 +1,195 @@
+"""The oracle: a plain, slow, exact CPU statement of the PEAT error signature.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+``bench.py``'s ``cpu_baseline`` leg may import this package.  It shares no
+code with the CUDA library in ``paper_2609_13544_gb300`` and imports nothing
+from it.
+
+Everything is computed by ``peat_oracle.c`` (see its header comment for the
+definitions, which follow Section IV-B-3 "FI Assessment Scores" and the Err
+step of Alg. 1 / Alg. 2).  This module only marshals numpy arrays.
+"""
+from __future__ import annotations
+
+import ctypes
+from typing import Sequence
+
+import numpy as np
+
+from .build import LIB, build
+
+DTYPES = {"f32": 0, "f16": 1, "bf16": 2}
+ITEMSIZE = {"f32": 4, "f16": 2, "bf16": 2}
+CLASSES = ("exact", "within_tol", "mismatch", "nan_inf_asym", "sign_flip")
+INJECT_KINDS = {
+    "rz": 0, "rv": 1, "bitflip": 2, "nan_inf": 3, "signflip": 4, "rel_gauss": 5,
+    "add_gauss": 6, "bias": 7, "cast_f16_rne": 8, "cast_f16_rtz": 9, "cast_bf16_rne": 10,
+    "cast_bf16_rtz": 11,
+}
+
+
+class Stats(ctypes.Structure):
+    _fields_ = [
+        ("n", ctypes.c_uint64),
+        ("count", ctypes.c_uint64 * 5),
+        ("n_finite", ctypes.c_uint64),
+        ("max_abs", ctypes.c_double),
+        ("argmax_abs", ctypes.c_int64),
+        ("max_rel", ctypes.c_double),
+        ("argmax_rel", ctypes.c_int64),
+        ("max_ulp", ctypes.c_uint64),
+        ("argmax_ulp", ctypes.c_int64),
+        ("sum_abs", ctypes.c_double),
+        ("sum_sq", ctypes.c_double),
+        ("sum_signed", ctypes.c_double),
+        ("rtol_eff", ctypes.c_double),
+        ("atol_eff", ctypes.c_double),
+    ]
+
+
+class InjectModel(ctypes.Structure):
+    _fields_ = [
+        ("kind", ctypes.c_int32),
+        ("k", ctypes.c_int32),
+        ("bit_lo", ctypes.c_int32),
+        ("bit_hi", ctypes.c_int32),
+        ("x", ctypes.c_double),
+    ]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        path = build()
+        L = ctypes.CDLL(str(path))
+        vp, i64, i32, dbl = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_double
+        L.orc_compare.argtypes = [vp, vp, i64, i32, dbl, dbl, ctypes.POINTER(Stats), vp]
+        L.orc_compare.restype = i32
+        L.orc_compare_segmented.argtypes = [vp, vp, vp, i64, i32, dbl, dbl, ctypes.POINTER(Stats), vp]
+        L.orc_compare_segmented.restype = i32
+        L.orc_ulp_key.argtypes = [ctypes.c_uint32, i32]
+        L.orc_ulp_key.restype = i64
+        L.orc_exact_sum.argtypes = [vp, i64]
+        L.orc_exact_sum.restype = dbl
+        L.orc_exact_dot.argtypes = [vp, vp, i64]
+        L.orc_exact_dot.restype = dbl
+        L.orc_inject.argtypes = [vp, vp, i64, i32, ctypes.POINTER(InjectModel), i32, ctypes.c_uint64, vp]
+        L.orc_inject.restype = i32
+        L.orc_philox4x32_10.argtypes = [vp, vp, vp]
+        L.orc_philox4x32_10.restype = None
+        L.orc_normal_from_words.argtypes = [ctypes.c_uint32, ctypes.c_uint32]
+        L.orc_normal_from_words.restype = ctypes.c_float
+        L.orc_logf.argtypes = [ctypes.c_float]
+        L.orc_logf.restype = ctypes.c_float
+        L.orc_cos2pi.argtypes = [ctypes.c_float]
+        L.orc_cos2pi.restype = ctypes.c_float
+        _lib = L
+    return _lib
+
+
+def _bits(x, dtype: str) -> np.ndarray:
+    """Raw bit patterns of x as a contiguous uint16/uint32 array."""
+    if hasattr(x, "detach"):  # a CPU torch tensor (bf16 has no numpy dtype)
+        import torch
+        x = x.detach().cpu().contiguous()
+        x = x.view(torch.int32 if ITEMSIZE[dtype] == 4 else torch.int16).numpy()
+    x = np.ascontiguousarray(x)
+    if x.dtype.itemsize != ITEMSIZE[dtype]:
+        raise ValueError(f"{dtype} needs {ITEMSIZE[dtype]}-byte elements, got {x.dtype}")
+    return x.reshape(-1).view(np.uint32 if ITEMSIZE[dtype] == 4 else np.uint16)
+
+
+def _stats_dict(s: Stats) -> dict:
+    d = {f: getattr(s, f) for f, _ in Stats._fields_ if f != "count"}
+    d["count"] = [int(v) for v in s.count]
+    for name, v in zip(CLASSES, s.count):
+        d[name] = int(v)
+    return d
+
+
+def compare(g, c, dtype: str, rtol: float, atol: float = 0.0):
+    """Signature of one tensor pair: (stats dict, hist uint64[2, 64])."""
+    gb, cb = _bits(g, dtype), _bits(c, dtype)
+    if gb.size != cb.size:
+        raise ValueError("golden and candidate differ in length")
+    st = Stats()
+    hist = np.zeros((2, 64), np.uint64)
+    rc = lib().orc_compare(gb.ctypes.data, cb.ctypes.data, gb.size, DTYPES[dtype], rtol, atol,
+                           ctypes.byref(st), hist.ctypes.data)
+    if rc:
+        raise ValueError(f"oracle rejected the arguments (code {rc})")
+    return _stats_dict(st), hist
+
+
+def compare_segmented(g, c, offsets: Sequence[int], dtype: str, rtol: float, atol: float = 0.0):
+    """Per-segment signatures: (list of stats dicts, hist uint64[nseg, 2, 64])."""
+    gb, cb = _bits(g, dtype), _bits(c, dtype)
+    off = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    nseg = off.size - 1
+    if gb.size != cb.size or nseg < 0 or (nseg >= 0 and off[-1] > gb.size):
+        raise ValueError("bad offsets or lengths")
+    st = (Stats * max(nseg, 1))()
+    hist = np.zeros((max(nseg, 1), 2, 64), np.uint64)
+    rc = lib().orc_compare_segmented(gb.ctypes.data, cb.ctypes.data, off.ctypes.data, nseg,
+                                     DTYPES[dtype], rtol, atol, st, hist.ctypes.data)
+    if rc:
+        raise ValueError(f"oracle rejected the arguments (code {rc})")
+    return [_stats_dict(st[s]) for s in range(nseg)], hist[:nseg]
+
+
+def ulp_key(bits: int, dtype: str) -> int:
+    return int(lib().orc_ulp_key(int(bits), DTYPES[dtype]))
+
+
+def exact_sum(x) -> float:
+    x = np.ascontiguousarray(x, np.float64)
+    return float(lib().orc_exact_sum(x.ctypes.data, x.size))
+
+
+def exact_dot(x, y) -> float:
+    x = np.ascontiguousarray(x, np.float64)
+    y = np.ascontiguousarray(y, np.float64)
+    return float(lib().orc_exact_dot(x.ctypes.data, y.ctypes.data, x.size))
+
+
+def model(kind: str, k: int = 0, bit_lo: int = 0, bit_hi: int = 0, x: float = 0.0) -> dict:
+    return {"kind": kind, "k": k, "bit_lo": bit_lo, "bit_hi": bit_hi, "x": x}
+
+
+def inject(src, dtype: str, models: Sequence[dict], seed: int):
+    """Apply the error models in order; returns (dst bits array, counts uint64[nmodels])."""
+    sb = _bits(src, dtype)
+    dst = np.empty_like(sb)
+    arr = (InjectModel * max(len(models), 1))()
+    for i, m in enumerate(models):
+        arr[i] = InjectModel(INJECT_KINDS[m["kind"]], m.get("k", 0), m.get("bit_lo", 0),
+                             m.get("bit_hi", 0), m.get("x", 0.0))
+    counts = np.zeros(max(len(models), 1), np.uint64)
+    rc = lib().orc_inject(dst.ctypes.data, sb.ctypes.data, sb.size, DTYPES[dtype], arr, len(models),
+                          ctypes.c_uint64(seed), counts.ctypes.data)
+    if rc:
+        raise ValueError(f"oracle rejected the arguments (code {rc})")
+    return dst, counts[: len(models)]
+
+
+def philox(ctr: Sequence[int], key: Sequence[int]) -> list:
+    c = np.array(ctr, np.uint32)
+    k = np.array(key, np.uint32)
+    out = np.zeros(4, np.uint32)
+    lib().orc_philox4x32_10(c.ctypes.data, k.ctypes.data, out.ctypes.data)
+    return [int(v) for v in out]
+
+
+def normal_from_words(w0: int, w1: int) -> float:
+    return float(lib().orc_normal_from_words(w0, w1))
+
+
+def logf(x: float) -> float:
+    return float(lib().orc_logf(x))
+
+
+def cos2pi(u: float) -> float:
+    return float(lib().orc_cos2pi(u))

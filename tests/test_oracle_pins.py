@@ -1,0 +1,474 @@
+"""Pins for the oracle against things other than itself (CPU only).
+
+Each block names what it pins: hand-worked cases (tests/golden), brute force
+over every 16-bit pattern, exact rational arithmetic on random pairs, library
+routines (torch.isclose, torch.argmax, math.fsum, numpy.frexp), invariants
+and closed forms of the synthetic recipes.  The definitions pinned are those
+of Section IV-B-3 (error = |golden - faulty|, scored by max, mean and
+variance) with the readings for the relative error, ULP distance, classes
+and histogram bins recorded in the oracle's header.
+"""
+import json
+import math
+import struct
+from fractions import Fraction
+from pathlib import Path
+
+import numpy as np
+import pytest
+import torch
+
+GOLD = json.loads((Path(__file__).parent / "golden" / "hand_cases.json").read_text())
+CLASS_IDX = {"exact": 0, "within_tol": 1, "mismatch": 2, "nan_inf_asym": 3, "sign_flip": 4}
+NP_BITS = {"f32": np.uint32, "f16": np.uint16, "bf16": np.uint16}
+
+
+# ---------------------------------------------------------------- helpers
+def decode(bits: int, dtype: str) -> float:
+    """Exact value of one bit pattern via the platform's own float formats."""
+    if dtype == "f32":
+        return float(np.array([bits], np.uint32).view(np.float32)[0])
+    if dtype == "f16":
+        return float(np.array([bits], np.uint16).view(np.float16)[0])
+    return float(np.array([bits << 16], np.uint32).view(np.float32)[0])
+
+
+def signbit(bits: int, dtype: str) -> int:
+    return (bits >> (31 if dtype == "f32" else 15)) & 1
+
+
+def rn32(x: float) -> float:
+    return float(np.float32(x))
+
+
+def ref_pair(gb: int, cb: int, dtype: str, rtol: float, atol: float, rank=None):
+    """The definitions evaluated with exact rationals (Python Fractions)."""
+    gv, cv = decode(gb, dtype), decode(cb, dtype)
+    out = {}
+    gfin, cfin = math.isfinite(gv), math.isfinite(cv)
+    if not (gfin and cfin):
+        eq = (math.isnan(gv) and math.isnan(cv)) or (math.isinf(gv) and math.isinf(cv) and gv == cv)
+        out["cls"] = 0 if eq else 3
+        out["relbin"] = 0 if eq else 63
+        out["finite"] = False
+        return out
+    out["finite"] = True
+    d = Fraction(cv) - Fraction(gv)
+    a = abs(d)
+    ag = abs(Fraction(gv))
+    R, A = Fraction(rn32(rtol)), Fraction(rn32(atol))
+    if a == 0:
+        cls = 0
+    elif a <= A + R * ag:
+        cls = 1
+    elif gv != 0 and cv != 0 and signbit(gb, dtype) != signbit(cb, dtype):
+        cls = 4
+    else:
+        cls = 2
+    out["cls"] = cls
+    if a == 0:
+        out["relbin"], out["rel"] = 0, Fraction(0)
+    elif ag == 0:
+        out["relbin"], out["rel"] = 63, None
+    else:
+        rel = a / ag
+        k = 0
+        while Fraction(2) ** k > rel:
+            k -= 1
+        while Fraction(2) ** (k + 1) <= rel:
+            k += 1
+        out["relbin"], out["rel"] = min(max(k + 48, 1), 62), rel
+    out["d"], out["a"] = d, a
+    return out
+
+
+# ---------------------------------------------------------------- hand cases
+@pytest.mark.parametrize("case", GOLD["cases"], ids=lambda c: f"{c['dtype']}:{c['g']}:{c['c']}:{c['why'][:20]}")
+def test_hand_case(oracle, case):
+    dt = case["dtype"]
+    g = np.array([int(case["g"], 16)], NP_BITS[dt])
+    c = np.array([int(case["c"], 16)], NP_BITS[dt])
+    st, h = oracle.compare(g, c, dt, case["rtol"], case["atol"])
+    assert st["count"][CLASS_IDX[case["class"]]] == 1, (case, st["count"])
+    assert h[0][case["relbin"]] == 1 and h[0].sum() == 1, np.nonzero(h[0])
+    assert h[1][case["ulpbin"]] == 1 and h[1].sum() == 1, np.nonzero(h[1])
+    if case["u"] is None and case["class"] != "mismatch":
+        assert st["argmax_ulp"] == -1
+    elif case["u"] is not None:
+        assert st["max_ulp"] == case["u"] and st["argmax_ulp"] == 0
+
+
+@pytest.mark.parametrize("agg", GOLD["aggregates"], ids=lambda a: a["why"][:30])
+def test_hand_aggregate(oracle, agg):
+    npt = {"f32": np.float32, "f16": np.float16}[agg["dtype"]]
+    st, h = oracle.compare(np.array(agg["g"], npt), np.array(agg["c"], npt), agg["dtype"], agg["rtol"], agg["atol"])
+    assert st["count"] == agg["counts"]
+    for k in ("n_finite", "max_abs", "argmax_abs", "max_rel", "argmax_rel", "max_ulp", "argmax_ulp",
+              "sum_signed", "sum_abs", "sum_sq"):
+        assert st[k] == agg[k], k
+    assert {str(i): int(v) for i, v in enumerate(h[0]) if v} == agg["relhist"]
+    assert {str(i): int(v) for i, v in enumerate(h[1]) if v} == agg["ulphist"]
+
+
+# ---------------------------------------------------------------- ULP distance, brute force
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+def test_ulp_key_is_rank_for_every_16bit_pattern(oracle, dtype):
+    """key(x) must equal the signed rank of x among all distinct non-NaN values
+    (both zeros merged).  Since u = |key(c) - key(g)|, this fixes the ULP
+    distance of all 2^32 pairs of the type."""
+    allbits = np.arange(65536, dtype=np.uint32)
+    vals = np.array([decode(int(b), dtype) for b in allbits])
+    ok = ~np.isnan(vals)
+    distinct = np.unique(vals[ok])  # -0.0 == 0.0 merge
+    rank = {v: i for i, v in enumerate(distinct.tolist())}
+    r0 = rank[0.0]
+    keys = np.array([oracle.ulp_key(int(b), dtype) for b in allbits[ok]])
+    ranks = np.array([rank[v] - r0 for v in vals[ok].tolist()])
+    assert np.array_equal(keys, ranks)
+
+
+def test_ulp_key_f32_successor(oracle):
+    rng = np.random.default_rng(1)
+    bits = rng.integers(0, 2 ** 32, 20000, dtype=np.uint64).astype(np.uint32)
+    bits = np.concatenate([bits, np.array([0, 0x80000000, 1, 0x80000001, 0x7f7fffff, 0xff7fffff, 0x00800000], np.uint32)])
+    x = bits.view(np.float32)
+    x = x[np.isfinite(x)]
+    x = x[x < np.float32(3.4028235e38)]
+    up = np.nextafter(x, np.float32(np.inf))
+    for a, b in zip(x.view(np.uint32)[:5000], up.view(np.uint32)[:5000]):
+        assert oracle.ulp_key(int(b), "f32") == oracle.ulp_key(int(a), "f32") + 1
+    assert oracle.ulp_key(0, "f32") == oracle.ulp_key(0x80000000, "f32") == 0
+
+
+# ---------------------------------------------------------------- exact rationals on random pairs
+def _random_pairs(dtype, n, rng):
+    w = 32 if dtype == "f32" else 16
+    top = 2 ** w
+    g = rng.integers(0, top, n, dtype=np.uint64)
+    c = g.copy()
+    kind = rng.integers(0, 6, n)
+    # 0: close in key space, 1: random pattern, 2: sign flipped close, 3: zero candidate,
+    # 4: same value, 5: small values near the subnormal range
+    step = rng.integers(-4, 5, n)
+    c = np.where(kind == 0, (g + step.astype(np.uint64)) % top, c)
+    c = np.where(kind == 1, rng.integers(0, top, n, dtype=np.uint64), c)
+    sign = np.uint64(1 << (w - 1))
+    c = np.where(kind == 2, (g ^ sign) + (step.astype(np.uint64) % np.uint64(3)), c) % top
+    c = np.where(kind == 3, np.uint64(0), c)
+    small = rng.integers(0, 2 ** (w // 2), n, dtype=np.uint64)
+    g = np.where(kind == 5, small, g)
+    c = np.where(kind == 5, small + rng.integers(0, 3, n).astype(np.uint64), c)
+    return g.astype(NP_BITS[dtype]), c.astype(NP_BITS[dtype])
+
+
+_RANKS = {}
+
+
+def rank_table(dtype):
+    """Signed rank of every 16-bit pattern among the distinct non-NaN values."""
+    if dtype not in _RANKS:
+        vals = np.array([decode(b, dtype) for b in range(65536)])
+        distinct = np.unique(vals[~np.isnan(vals)])
+        pos = {v: i for i, v in enumerate(distinct.tolist())}
+        r0 = pos[0.0]
+        _RANKS[dtype] = [None if math.isnan(v) else pos[v] - r0 for v in vals.tolist()]
+    return _RANKS[dtype]
+
+
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+def test_per_pair_ulp_against_rank_distance(oracle, dtype):
+    rng = np.random.default_rng({"f16": 31, "bf16": 32}[dtype])
+    g, c = _random_pairs(dtype, 4000, rng)
+    rank = rank_table(dtype)
+    stats, hist = oracle.compare_segmented(g, c, np.arange(g.size + 1), dtype, 0.0, 0.0)
+    for i in range(g.size):
+        rg, rc = rank[int(g[i])], rank[int(c[i])]
+        if rg is None or rc is None:
+            both = rg is None and rc is None
+            assert stats[i]["argmax_ulp"] == -1 and hist[i][1][0 if both else 63] == 1
+        else:
+            u = abs(rc - rg)
+            assert stats[i]["max_ulp"] == u and stats[i]["argmax_ulp"] == 0
+            assert hist[i][1][min(u, 63)] == 1
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16"])
+def test_per_pair_against_exact_rationals(oracle, dtype):
+    rng = np.random.default_rng({"f32": 11, "f16": 12, "bf16": 13}[dtype])
+    g, c = _random_pairs(dtype, 3000, rng)
+    rtol, atol = 1e-3, 1e-30
+    off = np.arange(g.size + 1)
+    stats, hist = oracle.compare_segmented(g, c, off, dtype, rtol, atol)
+    for i in range(g.size):
+        ref = ref_pair(int(g[i]), int(c[i]), dtype, rtol, atol)
+        st = stats[i]
+        assert st["count"][ref["cls"]] == 1, (i, hex(g[i]), hex(c[i]), ref, st["count"])
+        assert hist[i][0][ref["relbin"]] == 1, (i, ref["relbin"], np.nonzero(hist[i][0]))
+        if ref["finite"]:
+            assert st["n_finite"] == 1
+            assert st["sum_signed"] == float(ref["d"])
+            assert st["sum_abs"] == float(ref["a"])
+            assert st["sum_sq"] == float(ref["d"] ** 2)
+            assert st["max_abs"] == float(ref["a"])
+            exp_rel = math.inf if ref["rel"] is None else float(ref["rel"])
+            assert st["max_rel"] == exp_rel
+        else:
+            assert st["n_finite"] == 0 and st["argmax_abs"] == -1
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16"])
+def test_aggregate_against_exact_rationals(oracle, dtype):
+    rng = np.random.default_rng({"f32": 21, "f16": 22, "bf16": 23}[dtype])
+    g, c = _random_pairs(dtype, 1500, rng)
+    # plant exact ties for the maxima at two indices
+    g[700], c[700] = g[300], c[300]
+    st, hist = oracle.compare(g, c, dtype, 1e-2, 0.0)
+    S0 = S1 = S2 = Fraction(0)
+    best_a = best_r = None
+    ia = ir = -1
+    for i in range(g.size):
+        ref = ref_pair(int(g[i]), int(c[i]), dtype, 1e-2, 0.0)
+        if not ref["finite"]:
+            continue
+        S0 += ref["d"]
+        S1 += ref["a"]
+        S2 += ref["d"] ** 2
+        if best_a is None or ref["a"] > best_a:
+            best_a, ia = ref["a"], i
+        r = ref["rel"] if ref["rel"] is not None else math.inf
+        if best_r is None or r > best_r:
+            best_r, ir = r, i
+    assert st["sum_signed"] == float(S0)
+    assert st["sum_abs"] == float(S1)
+    assert st["sum_sq"] == float(S2)
+    assert st["argmax_abs"] == ia and st["max_abs"] == float(best_a)
+    assert st["argmax_rel"] == ir
+    assert st["max_rel"] == (math.inf if best_r == math.inf else float(best_r))
+
+
+# ---------------------------------------------------------------- library routines
+def _fp16_noise(n, seed, frac_nan=0.0):
+    rng = np.random.default_rng(seed)
+    g = (rng.laplace(0, 0.02, n)).astype(np.float16)
+    c = (g.astype(np.float32) * (1 + 1e-3 * rng.standard_normal(n).astype(np.float32))).astype(np.float16)
+    if frac_nan:
+        idx = rng.choice(n, int(n * frac_nan), replace=False)
+        c[idx] = np.float16(np.nan)
+    return g, c
+
+
+def test_isclose_count_matches_exact_plus_within(oracle):
+    """torch.isclose(c, g, rtol, atol, equal_nan=True) evaluated in float64 is
+    exact for fp16 data with atol = 0, so its count is EXACT + WITHIN_TOL."""
+    g, c = _fp16_noise(50000, 5, frac_nan=0.001)
+    g[:10] = np.float16(np.inf)
+    c[:5] = np.float16(np.inf)
+    st, _ = oracle.compare(g, c, "f16", 1e-3, 0.0)
+    close = torch.isclose(torch.from_numpy(c.astype(np.float64)), torch.from_numpy(g.astype(np.float64)),
+                          rtol=st["rtol_eff"], atol=0.0, equal_nan=True)
+    assert int(close.sum()) == st["exact"] + st["within_tol"]
+
+
+def test_argmax_and_fsum(oracle):
+    g, c = _fp16_noise(40000, 6)
+    c[123] = g[77]  # a large error somewhere
+    st, _ = oracle.compare(g, c, "f16", 1e-3, 0.0)
+    d = c.astype(np.float64) - g.astype(np.float64)  # exact for fp16 operands
+    assert st["argmax_abs"] == int(torch.argmax(torch.from_numpy(np.abs(d))))
+    assert st["max_abs"] == float(np.max(np.abs(d)))
+    assert st["sum_signed"] == math.fsum(d.tolist())
+    assert st["sum_abs"] == math.fsum(np.abs(d).tolist())
+    sq = d * d
+    assert np.all(np.abs(d[d != 0]) < 2.0 ** 12 * np.abs(d[d != 0]).min() * 2 ** 14)  # d*d exact in float64
+    assert st["sum_sq"] == math.fsum(sq.tolist())
+
+
+def test_rel_bin_against_frexp(oracle):
+    g, c = _fp16_noise(30000, 7)
+    _, h = oracle.compare(g, c, "f16", 1e-3, 0.0)
+    gd, cd = g.astype(np.float64), c.astype(np.float64)
+    a, ag = np.abs(cd - gd), np.abs(gd)
+    bins = np.zeros(64, np.int64)
+    ma, ea = np.frexp(a)
+    mg, eg = np.frexp(ag)
+    k = ea - eg - (ma < mg)
+    sel = (a > 0) & (ag > 0)
+    np.add.at(bins, np.clip(k[sel] + 48, 1, 62), 1)
+    bins[0] = int((a == 0).sum())
+    bins[63] = int(((a > 0) & (ag == 0)).sum())
+    assert np.array_equal(h[0].astype(np.int64), bins)
+
+
+def test_exact_accumulator_against_python_integers(oracle):
+    rng = np.random.default_rng(8)
+    for trial in range(40):
+        n = int(rng.integers(1, 60))
+        e = rng.integers(-300, 300, n)
+        x = rng.standard_normal(n) * np.exp2(e)
+        if trial % 4 == 0:  # heavy cancellation
+            x = np.concatenate([x, -x[:-1]])
+        y = rng.standard_normal(x.size) * np.exp2(rng.integers(-200, 200, x.size))
+        assert oracle.exact_sum(x) == float(sum(Fraction(v) for v in x))
+        assert oracle.exact_dot(x, y) == float(sum(Fraction(a) * Fraction(b) for a, b in zip(x, y)))
+    # round-half-even at a tie and just above it
+    assert oracle.exact_sum([1.0, 2.0 ** -53]) == 1.0
+    assert oracle.exact_sum([1.0, 2.0 ** -53, 2.0 ** -300]) == 1.0 + 2.0 ** -52
+    assert oracle.exact_sum([1.0 + 2.0 ** -52, 2.0 ** -53]) == 1.0 + 2.0 ** -51
+
+
+# ---------------------------------------------------------------- invariants
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16"])
+def test_self_compare(oracle, dtype):
+    rng = np.random.default_rng(9)
+    x, _ = _random_pairs(dtype, 4000, rng)
+    st, h = oracle.compare(x, x, dtype, 0.0, 0.0)
+    n = x.size
+    assert st["exact"] == n and sum(st["count"]) == n
+    assert h[0][0] == n and h[1][0] == n
+    assert st["sum_abs"] == st["sum_sq"] == st["sum_signed"] == 0.0
+    vals = np.array([decode(int(b), dtype) for b in x])
+    fin = np.nonzero(np.isfinite(vals))[0]
+    assert st["argmax_abs"] == (fin[0] if fin.size else -1)
+    assert st["argmax_rel"] == st["argmax_abs"]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16"])
+def test_swap_and_concatenation(oracle, dtype):
+    rng = np.random.default_rng(10)
+    g, c = _random_pairs(dtype, 5000, rng)
+    s1, h1 = oracle.compare(g, c, dtype, 0.0, 0.0)
+    s2, h2 = oracle.compare(c, g, dtype, 0.0, 0.0)
+    for k in ("exact", "nan_inf_asym", "sign_flip", "n_finite"):
+        assert s1[k] == s2[k]
+    assert np.array_equal(h1[1], h2[1])
+    assert s1["max_ulp"] == s2["max_ulp"] and s1["argmax_ulp"] == s2["argmax_ulp"]
+    assert s1["sum_abs"] == s2["sum_abs"] and s1["sum_sq"] == s2["sum_sq"]
+    assert s1["sum_signed"] == -s2["sum_signed"]
+    assert s1["max_abs"] == s2["max_abs"] and s1["argmax_abs"] == s2["argmax_abs"]
+    assert sum(s1["count"]) == g.size and h1[0].sum() == g.size and h1[1].sum() == g.size
+    off = np.array([0, 0, 17, 17, 1000, 1001, 4096, 5000])
+    ss, hs = oracle.compare_segmented(g, c, off, dtype, 0.0, 0.0)
+    assert np.array_equal(hs.sum(axis=0), h1)
+    assert [sum(s["count"][j] for s in ss) for j in range(5)] == s1["count"]
+    assert ss[0]["n"] == 0 and ss[0]["argmax_abs"] == -1
+    assert max(s["max_ulp"] for s in ss) == s1["max_ulp"]
+
+
+# ---------------------------------------------------------------- closed forms of the recipes
+def test_closed_form_bf16_rne_vs_rtz(oracle):
+    """RNE and RTZ roundings of the same float32 differ by one bf16 step, so
+    every differing pair has u = 1 and rel in [2^-8, 2^-7) (bin 40), and is
+    within rtol = 2^-7."""
+    from paper_2609_13544_gb300 import workloads as W
+    w = W.c2_bf16_rne_vs_rtz(numel=1 << 18, seed=2)
+    st, h = oracle.compare(w.golden, w.candidate, "bf16", 2.0 ** -7)
+    differ = int((w.golden.view(torch.int16) != w.candidate.view(torch.int16)).sum())
+    assert set(np.nonzero(h[0])[0]) == {0, 40}
+    assert set(np.nonzero(h[1])[0]) == {0, 1}
+    assert h[0][40] == differ == h[1][1]
+    assert st["within_tol"] == differ and st["mismatch"] == st["sign_flip"] == st["nan_inf_asym"] == 0
+    n = w.n
+    assert abs(differ - n / 2) < 5 * math.sqrt(n) / 2
+
+
+def test_closed_form_relative_bias(oracle):
+    """c = g + 1e-4|g| puts every nonzero relative error in [2^-14, 2^-13)."""
+    from paper_2609_13544_gb300 import workloads as W
+    shapes = W.resnet50_param_shapes()[:12]
+    w = W.c3_resnet50(seed=3, shapes=shapes)
+    stats, h = oracle.compare_segmented(w.golden, w.candidate, w.offsets, "f32", 1e-5)
+    for s in range(0, len(shapes), 2):
+        assert set(np.nonzero(h[s][0])[0]) <= {0, 34}
+        assert stats[s]["sum_signed"] > 0
+        gseg = w.golden[w.offsets[s]:w.offsets[s + 1]].double()
+        assert abs(stats[s]["sum_signed"] / (1e-4 * float(gseg.abs().sum())) - 1) < 1e-3
+
+
+def test_closed_form_gaussian_noise_moments(oracle):
+    """c = g(1+e), e ~ N(0, 1e-6): E[sum d^2] = n E[g^2] 1e-12 and
+    E[sum |d|] = n E|g| sqrt(2/pi) 1e-6, up to float32 rounding of c."""
+    from paper_2609_13544_gb300 import workloads as W
+    w = W.c1_single_fp32(n=1 << 16, seed=0, flips=0)
+    st, _ = oracle.compare(w.golden, w.candidate, "f32", 1e-5)
+    g = w.golden.double()
+    n = w.n
+    exp_sq = float((g * g).sum()) * 1e-12
+    exp_abs = float(g.abs().sum()) * math.sqrt(2 / math.pi) * 1e-6
+    assert abs(st["sum_sq"] / exp_sq - 1) < 0.05
+    assert abs(st["sum_abs"] / exp_abs - 1) < 0.05
+    assert st["mismatch"] + st["sign_flip"] + st["nan_inf_asym"] == 0
+
+
+# ---------------------------------------------------------------- injector building blocks
+def test_philox_known_answers(oracle):
+    """Known-answer vectors published with Philox4x32-10 (Random123)."""
+    assert oracle.philox([0, 0, 0, 0], [0, 0]) == [0x6627E8D5, 0xE169C58D, 0xBC57AC4C, 0x9B00DBD8]
+    assert oracle.philox([0xFFFFFFFF] * 4, [0xFFFFFFFF] * 2) == [0x408F276D, 0x41C83B0E, 0xA20BC7C6, 0x6D5451FD]
+    assert oracle.philox([0x243F6A88, 0x85A308D3, 0x13198A2E, 0x03707344], [0xA4093822, 0x299F31D0]) == \
+        [0xD16CFE09, 0x94FDCCEB, 0x5001E420, 0x24126EA1]
+
+
+def test_logf_and_cos2pi_against_libm(oracle):
+    xs = np.concatenate([np.arange(1, 1 << 24, 4099, dtype=np.float64) * 2.0 ** -24, [1.0, 0.5, 2.0 ** -24]])
+    for x in xs:
+        x32 = rn32(x)
+        ref = math.log(x32)
+        assert abs(oracle.logf(x32) - ref) <= 3e-7 * max(1.0, abs(ref)), x32
+    for u in np.arange(0, 1 << 24, 3001) * 2.0 ** -24:
+        assert abs(oracle.cos2pi(float(u)) - math.cos(2 * math.pi * u)) < 4e-7, u
+
+
+def test_box_muller_moments(oracle):
+    n = 100000
+    w = [oracle.philox([i, 0, 7, 1], [5, 0]) for i in range(n)]
+    z = np.array([oracle.normal_from_words(a[0], a[1]) for a in w])
+    assert abs(z.mean()) < 5 / math.sqrt(n)
+    assert abs(z.var() - 1) < 5 * math.sqrt(2 / n)
+    kurt = ((z - z.mean()) ** 4).mean() / z.var() ** 2
+    assert abs(kurt - 3) < 5 * math.sqrt(24 / n)
+    assert abs((np.abs(z) < 1).mean() - 0.6826894921) < 5 * math.sqrt(0.22 / n)
+
+
+def test_inject_fixed_count_models(oracle):
+    rng = np.random.default_rng(12)
+    src = rng.standard_normal(5000).astype(np.float32)
+    models = [oracle.model("rz", k=3), oracle.model("rv", k=5), oracle.model("bitflip", k=16, bit_lo=0, bit_hi=31)]
+    for m in models:
+        dst, cnt = oracle.inject(src, "f32", [m], seed=42)
+        diff = np.nonzero(dst != src.view(np.uint32))[0]
+        assert cnt[0] == m["k"] and diff.size <= m["k"]
+        if m["kind"] == "rz":
+            assert diff.size == 3 and np.all(dst[diff] == 0)
+        if m["kind"] == "rv":
+            assert all(dst[i] in set(src.view(np.uint32).tolist()) for i in diff)
+        if m["kind"] == "bitflip":
+            assert diff.size == 16
+            x = dst[diff] ^ src.view(np.uint32)[diff]
+            assert all(bin(int(v)).count("1") == 1 for v in x)
+    dst2, _ = oracle.inject(src, "f32", models, seed=42)
+    dst3, _ = oracle.inject(src, "f32", models, seed=42)
+    assert np.array_equal(dst2, dst3)
+
+
+def test_inject_rate_and_noise_models(oracle):
+    rng = np.random.default_rng(13)
+    n = 200000
+    src = rng.standard_normal(n).astype(np.float32)
+    dst, cnt = oracle.inject(src, "f32", [oracle.model("nan_inf", x=1e-3)], seed=1)
+    v = dst.view(np.float32)
+    assert abs(int(cnt[0]) - n * 1e-3) < 5 * math.sqrt(n * 1e-3)
+    assert int(np.isnan(v).sum() + np.isinf(v).sum()) == cnt[0]
+    dst, cnt = oracle.inject(src, "f32", [oracle.model("rel_gauss", x=1e-3)], seed=2)
+    e = (dst.view(np.float32).astype(np.float64) / src - 1) / 1e-3
+    assert cnt[0] == n and abs(e.mean()) < 5 / math.sqrt(n) and abs(e.std() - 1) < 0.01
+    dst, _ = oracle.inject(src, "f32", [oracle.model("cast_f16_rne")], seed=0)
+    assert np.array_equal(dst.view(np.float32), src.astype(np.float16).astype(np.float32))
+    dst, _ = oracle.inject(src, "f32", [oracle.model("cast_bf16_rne")], seed=0)
+    ref = torch.from_numpy(src).to(torch.bfloat16).to(torch.float32).numpy()
+    assert np.array_equal(dst.view(np.float32), ref)
+    dst, _ = oracle.inject(src, "f32", [oracle.model("cast_bf16_rtz")], seed=0)
+    assert np.array_equal(dst, src.view(np.uint32) & np.uint32(0xFFFF0000))
+    dst, _ = oracle.inject(src, "f32", [oracle.model("cast_f16_rtz")], seed=0)
+    y = dst.view(np.float32).astype(np.float16)
+    up = np.nextafter(y, np.where(src >= 0, np.float16(np.inf), np.float16(-np.inf)))
+    assert np.all(np.abs(y.astype(np.float64)) <= np.abs(src)) and np.all(np.abs(up.astype(np.float64)) > np.abs(src))

@@ -1,0 +1,384 @@
+"""Throughput of the golden-vs-candidate error signature (peat_compare) on GB300.
+
+One step = one full pass of the compare (stage 1 stream over both tensors +
+stage 2 per-segment merge) over one synthetic workload resident in HBM.
+Default workload: the [8,2048,4096] bf16 activation (67,108,864 pairs,
+RNE vs RTZ candidate).  Prints ONE JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c1..c5] [--impl reference]
+
+For N > 1 it runs under torch.distributed.run, one rank per GPU; every rank
+compares its own copy of the workload (weak scaling: the compare of one
+tensor is independent per rank, no data-path collective); time = max over
+ranks between barriers.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+METRIC = "element-pairs/s and achieved HBM GB/s (fraction of ~8 TB/s) for peat_compare"
+WORKLOAD_NAMES = {
+    "c1": "single fp32 tensor n=1,048,576, N(0,1) golden, rel noise 1e-6 + 16 bit flips, rtol 1e-5",
+    "c2": "bf16 activation [8,2048,4096] (67,108,864 pairs): RNE vs RTZ rounding of N(0,2^2) fp32, rtol 2^-7",
+    "c3": "ResNet-50 parameter list, 161 fp32 segments (25,557,032 pairs), Kaiming-normal, bias/noise candidate",
+    "c4": "GPT-2-medium parameter list, 292 fp16 segments (354,823,168 pairs), Laplace(0,0.02), noise+NaN/Inf+sign flips",
+    "c5": "playback sweep step 63 of a 268,435,456-element bf16 tensor, rel noise 1e-4*sqrt(s)",
+}
+NOMINAL_HBM_GBS = 8000.0
+
+
+def measured_peaks() -> dict:
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        return json.loads(p.read_text())
+    return {"hbm_gbs": 6800.0, "fallback": True}
+
+
+def kernel_source_sha() -> str:
+    h = hashlib.sha256()
+    for f in ("compare.cu", "peat_internal.h"):
+        h.update((ROOT / "paper_2609_13544_gb300" / "csrc" / f).read_bytes())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per stage-1 launch from the committed ncu summary, if it was
+    taken on the current kernel source."""
+    p = ROOT / "profiles" / "traffic.json"
+    if not p.exists():
+        return None
+    d = json.loads(p.read_text()).get(workload)
+    if not d or d.get("source_sha") != kernel_source_sha():
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 200 ms."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = Path(os.environ.get("TMPDIR", "/tmp")) / f"peat_clocks_{os.getpid()}.csv"
+
+    def __enter__(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self) -> dict:
+        if self.proc is None or not self.path.exists():
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        for line in self.path.read_text().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append(parts)
+            except ValueError:
+                pass
+        self.path.unlink(missing_ok=True)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i, v in enumerate(r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def make_workload(name: str, device: str):
+    from paper_2609_13544_gb300 import workloads as W
+    if name == "c1":
+        return W.c1_single_fp32(device=device)
+    if name == "c2":
+        return W.c2_bf16_rne_vs_rtz(device=device)
+    if name == "c3":
+        return W.c3_resnet50(device=device)
+    if name == "c4":
+        return W.c4_gpt2_medium(device=device)
+    if name == "c5":
+        return W.PlaybackSweep(device=device).workload(63)
+    raise ValueError(name)
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+# --------------------------------------------------------------------------- oracle timing
+def _oracle_slice(args):
+    import numpy as np
+    import oracle
+    g, c, dtype, rtol, atol, segs = args
+    t0 = time.perf_counter()
+    if segs is None:
+        oracle.compare(g, c, dtype, rtol, atol)
+    else:
+        oracle.compare_segmented(g, c, segs, dtype, rtol, atol)
+    return time.perf_counter() - t0
+
+
+def host_bits(t, dtype):
+    import numpy as np
+    import torch
+    it = torch.int32 if dtype == "f32" else torch.int16
+    return t.contiguous().view(it).cpu().numpy().view(np.uint32 if dtype == "f32" else np.uint16)
+
+
+def oracle_rate(w, pool, cores: int, pairs: int) -> tuple:
+    """Oracle pairs/s on the first `pairs` pairs, split across `cores` processes."""
+    import numpy as np
+    pairs = min(pairs, w.n)
+    gb, cb = host_bits(w.golden[:pairs], w.dtype), host_bits(w.candidate[:pairs], w.dtype)
+    bounds = np.linspace(0, pairs, cores + 1).astype(np.int64)
+    jobs = [(gb[a:b], cb[a:b], w.dtype, w.rtol, w.atol, None) for a, b in zip(bounds[:-1], bounds[1:]) if b > a]
+    t0 = time.perf_counter()
+    list(pool.map(_oracle_slice, jobs))
+    dt = time.perf_counter() - t0
+    return pairs / dt, dt, pairs
+
+
+def make_pool(cores):
+    import multiprocessing as mp
+    from concurrent.futures import ProcessPoolExecutor
+    return ProcessPoolExecutor(max_workers=cores, mp_context=mp.get_context("spawn"))
+
+
+def run_reference(args) -> None:
+    """Reference arm: the oracle, as it stands, on the host cores."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    w = make_workload(args.workload, "cpu")
+    cores = os.cpu_count() or 1
+    with make_pool(cores) as pool:
+        # size each step's sample so the whole run stays within about a minute of wall time
+        rate, _, _ = oracle_rate(w, pool, cores, min(w.n, 200_000 * cores))
+        per_step = int(max(4096 * cores, min(w.n, rate * 60.0 / max(1, args.steps + args.warmup))))
+        for _ in range(args.warmup):
+            oracle_rate(w, pool, cores, per_step)
+        t0 = time.perf_counter()
+        done = 0
+        for _ in range(args.steps):
+            _, _, p = oracle_rate(w, pool, cores, per_step)
+            done += p
+        dt = time.perf_counter() - t0
+    value = done / dt
+    sample = f"first {per_step} pairs of {args.workload} per step, split over {cores} processes"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "pairs/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / max(1, args.steps),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64+exact int",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD_NAMES[args.workload], "element": w.dtype, "pairs_per_step": per_step},
+        "cpu_baseline": {"value": value, "unit": "pairs/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "pairs/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- the CUDA path
+def run_gpu(args) -> None:
+    import numpy as np
+    import torch
+
+    import paper_2609_13544_gb300 as peat
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    peat.load()
+    w = make_workload(args.workload, "cuda")
+    g, c = w.golden.to(dev), w.candidate.to(dev)
+    nseg = 1 if w.offsets is None else len(w.offsets) - 1
+    h = peat.Handle(local, max_segments=max(4096, nseg))
+    stats = torch.empty(nseg * peat.STATS_BYTES, dtype=torch.uint8, device=dev)
+    hist = torch.empty(nseg * peat.HIST_BINS, dtype=torch.int64, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        if w.offsets is None:
+            peat.peat_compare_raw(h, g, c, w.rtol, w.atol, stats, hist, stream)
+        else:
+            peat.peat_compare_segmented_raw(h, g, c, w.offsets, w.rtol, w.atol, stats, hist, stream)
+
+    # sanity before timing: counts add up
+    step()
+    torch.cuda.synchronize()
+    st = peat.stats_to_dicts(stats.cpu().numpy())
+    assert sum(sum(s["count"]) for s in st) == w.n, "counts do not add up to n"
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        time.sleep(0.25)
+        barrier()
+        wall0 = time.perf_counter()
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        barrier()
+        wall = time.perf_counter() - wall0
+        time.sleep(0.25)
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    clocks = clk.summary()
+    ms_per_step = ms / args.steps
+    pairs = w.n * world
+    value = pairs * args.steps / (ms * 1e-3)
+    bytes_per_step = 2 * w.n * (4 if w.dtype == "f32" else 2)
+    gbs = bytes_per_step / (ms_per_step * 1e-3) / 1e9
+    peaks = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", 6800.0))
+
+    # end to end through the C ABI with host buffers: H2D of both tensors from
+    # pinned memory, the compare, D2H of the stats and histograms, every step
+    e2e = None
+    if rank == 0 or world > 1:
+        gh = torch.empty_like(g, device="cpu").pin_memory()
+        ch = torch.empty_like(c, device="cpu").pin_memory()
+        gh.copy_(g)
+        ch.copy_(c)
+        sh = torch.empty_like(stats, device="cpu").pin_memory()
+        hh = torch.empty_like(hist, device="cpu").pin_memory()
+        e2e_steps = max(3, min(args.steps, 50))
+
+        def e2e_step():
+            g.copy_(gh, non_blocking=True)
+            c.copy_(ch, non_blocking=True)
+            step()
+            sh.copy_(stats, non_blocking=True)
+            hh.copy_(hist, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        barrier()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(e2e_steps):
+            e2e_step()
+        f1.record(stream)
+        barrier()
+        ems = f0.elapsed_time(f1)
+        if world > 1:
+            import torch.distributed as dist
+            t = torch.tensor([ems], device=dev, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        e2e = {"value": w.n * world * e2e_steps / (ems * 1e-3), "unit": "pairs/s",
+               "h2d_bytes_per_step": bytes_per_step, "d2h_bytes_per_step": int(stats.numel() + hist.numel() * 8),
+               "ms_per_step": ems / e2e_steps}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        cores = os.cpu_count() or 1
+        wc = w
+        with make_pool(cores) as pool:
+            r0, _, _ = oracle_rate(wc, pool, cores, min(wc.n, 100_000 * cores))
+            target = int(min(wc.n, max(1_000_000, r0 * 20.0)))  # about 20 s of CPU work in total
+            rate, dt, done = oracle_rate(wc, pool, cores, target)
+        cpu = {"value": rate, "unit": "pairs/s", "cores": cores, "kind": "oracle",
+               "sample": f"first {done} pairs of the same workload, {cores} processes, {dt:.1f} s wall"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "pairs/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32+int (exact)", "data": "synthetic",
+            "config": {"workload": WORKLOAD_NAMES[args.workload], "element": w.dtype, "pairs": w.n,
+                       "segments": nseg, "l2": "inputs larger than L2 (no flush)" if bytes_per_step > 135e6
+                       else "inputs smaller than L2: steps re-read from L2", "parallelism": f"replicas x{world}"},
+            "hbm_gbs": gbs, "frac_of_8tbs": gbs / NOMINAL_HBM_GBS,
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
+                         "traffic": recorded_traffic(args.workload),
+                         "kernel": "compare_stage1 + compare_stage2 per call (event-timed on the launch stream)",
+                         "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy)" if not peaks.get("fallback")
+                         else "fallback 6.8 TB/s"},
+            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": 2 * args.steps, "clocks": clocks,
+            "wall_s_timed": wall,
+        }
+        print(json.dumps(line), flush=True)
+    h.close()
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default="c2", choices=sorted(WORKLOAD_NAMES))
+    ap.add_argument("--impl", default="peat", choices=["peat", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.steps is None:
+        args.steps = {"c1": 20000, "c2": 20000, "c3": 20000, "c4": 3000, "c5": 4000}[args.workload]
+        if args.impl == "reference":
+            args.steps = 10
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,218 @@
+/*
+ * peat.h -- C ABI of libpeat, the GB300 (sm_103a) golden-vs-candidate error
+ * signature library.
+ *
+ * PEAT's Analyzer scores the error between a golden tensor and a
+ * fault-injected (candidate) tensor recorded during training: the error is
+ * their absolute difference, scored per recorded tensor by its maximum, its
+ * mean and its variance (Section IV-B-3, "FI Assessment Scores"; the Err(...)
+ * step that ends Alg. 1 and Alg. 2).  This library computes that signature,
+ * extended per element with the relative error, the ordered-integer ULP
+ * distance and a five-way classification, in one pass over both tensors.
+ *
+ * Definitions (exact over the reals, then rounded once to nearest-even):
+ *   non-finite pairs  EXACT if both NaN or both infinite with equal sign,
+ *                     NAN_INF_ASYM otherwise; excluded from sums and from
+ *                     the abs/rel maxima.
+ *   finite pairs      d = c - g, a = |d|.  EXACT iff a = 0.  WITHIN_TOL iff
+ *                     0 < a <= atol + rtol*|g| (torch.isclose form, golden as
+ *                     reference, Section III-A; rtol/atol rounded to float32).
+ *                     SIGN_FLIP iff not yet classified, g != 0, c != 0 and
+ *                     the sign bits differ.  MISMATCH otherwise.
+ *   relative error    a/|g|; 0 when a = 0; +inf when g = 0 < a.
+ *   rel histogram     bin 0: a = 0 (and equal non-finite pairs); bins 1..62:
+ *                     k = floor(log2(a/|g|)) at clamp(k+48, 1, 62); bin 63:
+ *                     g = 0 < a, and every NAN_INF_ASYM pair.
+ *   ULP distance      u = |key(c) - key(g)|, key(x) = +/-(bits without sign)
+ *                     by the sign bit (both zeros -> 0).  Bin min(u, 63).  A
+ *                     pair with a NaN has no u: bin 63 (bin 0 if both NaN),
+ *                     and it is left out of max_ulp.
+ *   maxima            lowest index wins ties (exact comparison).
+ *   sums              over finite pairs: sum |d|, sum d^2, sum d, exact, then
+ *                     rounded to nearest-even binary64.
+ * Derived scores (host side): mean = sum_abs/n_finite, bias =
+ * sum_signed/n_finite, L2 = sqrt(sum_sq), variance of |e| =
+ * sum_sq/n_finite - mean^2.
+ *
+ * Conventions for every entry point
+ *  - Pointers named golden/candidate/src/dst/stats_out/hist_out/counts_out
+ *    are DEVICE pointers (cudaMalloc or managed memory) owned by the caller;
+ *    `offsets` and `models` are HOST arrays the call copies before returning.
+ *  - Every call is asynchronous on `stream` (NULL = legacy default stream);
+ *    outputs are valid once the stream has been synchronised.
+ *  - A handle is not thread-safe: use one handle per host thread.  Calls on
+ *    one handle must not overlap on the GPU (the handle's workspace is reused
+ *    call after call; issue them on one stream, or order the streams).
+ *  - Errors are returned as peat_status_t; nothing is thrown across the ABI.
+ *    peat_last_error(h) gives the text of the last error on that handle.
+ *    CUDA errors map to PEAT_ERR_CUDA.
+ */
+#ifndef PEAT_H
+#define PEAT_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA stream (layout-compatible with cudaStream_t / CUstream). */
+typedef struct CUstream_st* peat_stream_t;
+
+typedef enum { PEAT_F32 = 0, PEAT_F16 = 1, PEAT_BF16 = 2 } peat_dtype_t;
+
+typedef enum {
+  PEAT_OK = 0,
+  PEAT_ERR_INVALID_ARG = 1, /* null pointer, negative size, bad dtype, bad offsets, ... */
+  PEAT_ERR_UNSUPPORTED = 2, /* a valid request this build does not serve */
+  PEAT_ERR_ALLOC = 3,       /* device or pinned allocation failed */
+  PEAT_ERR_CUDA = 4,        /* a CUDA runtime call failed (text in peat_last_error) */
+  PEAT_ERR_TIMEOUT = 5,     /* a bounded device-side wait expired */
+  PEAT_ERR_INTERNAL = 6     /* an internal consistency check failed */
+} peat_status_t;
+
+/* Classes, in the order of peat_stats_t.count. */
+enum {
+  PEAT_EXACT = 0,
+  PEAT_WITHIN_TOL = 1,
+  PEAT_MISMATCH = 2,
+  PEAT_NAN_INF_ASYM = 3,
+  PEAT_SIGN_FLIP = 4,
+  PEAT_NCLASS = 5
+};
+
+/* Tolerances of the WITHIN_TOL test; both are rounded to float32 (round to
+ * nearest even) and must then be finite and >= 0. */
+typedef struct {
+  double rtol;
+  double atol;
+} peat_tol_t;
+
+/* Handle configuration.  device: CUDA ordinal the handle's calls run on.
+ * max_segments: the largest nseg a segmented call may pass (0 = 4096).
+ * flags: reserved, must be 0. */
+typedef struct {
+  int32_t device;
+  int32_t reserved0;
+  int64_t max_segments;
+  uint32_t flags;
+  uint32_t reserved1;
+} peat_config_t;
+
+/* Signature of one tensor (or one segment).  144 bytes, no padding holes. */
+typedef struct {
+  uint64_t n;                   /* pairs compared */
+  uint64_t count[PEAT_NCLASS];  /* class counts; they sum to n */
+  uint64_t n_finite;            /* pairs with both operands finite */
+  double max_abs;               /* RN64(max |d|) over finite pairs, 0 if none */
+  int64_t argmax_abs;           /* lowest index attaining it, -1 if no finite pair */
+  double max_rel;               /* RN64(max a/|g|) over finite pairs; may be +inf */
+  int64_t argmax_rel;           /* -1 if no finite pair */
+  uint64_t max_ulp;             /* max u over pairs without a NaN */
+  int64_t argmax_ulp;           /* -1 if every pair has a NaN */
+  double sum_abs;               /* RN64(sum |d|) over finite pairs */
+  double sum_sq;                /* RN64(sum d^2) */
+  double sum_signed;            /* RN64(sum d) */
+  double rtol_eff;              /* the float32 tolerances actually used */
+  double atol_eff;
+} peat_stats_t;
+
+/* Histograms of one tensor: 128 uint64 counters, [0..63] log2-relative-error
+ * bins then [64..127] ULP bins.  Each half sums to n. */
+#define PEAT_HIST_BINS 128
+
+typedef struct peat_handle_s* peat_handle_t;
+
+/* Create a handle bound to cfg->device (cfg may be NULL: device 0, defaults).
+ * Allocates the handle's device workspace.  Errors: INVALID_ARG, CUDA, ALLOC. */
+peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg);
+
+/* Release the handle and its workspace; waits for the handle's work to finish.
+ * NULL is accepted and ignored. */
+peat_status_t peat_signature_destroy(peat_handle_t h);
+
+/* Signature of one tensor pair (the Err step of Alg. 1 / Alg. 2 over one
+ * recorded tensor; scores of Section IV-B-3).
+ *   golden, candidate  device arrays of n elements of `dtype`, any alignment
+ *                      (16-byte aligned arrays with equal alignment run the
+ *                      vectorised path); contiguous, element i at byte
+ *                      i*sizeof(dtype).
+ *   n                  >= 0; n = 0 yields zero counts and argmax -1.
+ *   tol                see peat_tol_t.
+ *   stats_out          device pointer to one peat_stats_t.
+ *   hist_out           device pointer to PEAT_HIST_BINS uint64 (or NULL).
+ * Errors: INVALID_ARG (null pointer with n > 0, n < 0, bad dtype, bad tol),
+ * CUDA. */
+peat_status_t peat_compare(peat_handle_t h, const void* golden, const void* candidate, int64_t n,
+                           peat_dtype_t dtype, peat_tol_t tol, peat_stats_t* stats_out,
+                           uint64_t* hist_out, peat_stream_t stream);
+
+/* Per-segment signatures of a packed list of tensors (e.g. every parameter
+ * of a model, recorded per epoch as in Alg. 1).  Segment s is elements
+ * [offsets[s], offsets[s+1]) of golden/candidate; argmax indices are local
+ * to the segment.
+ *   offsets    HOST array of nseg+1 int64, offsets[0] = 0, non-decreasing;
+ *              copied during the call.  Empty segments are allowed.
+ *   nseg       0 <= nseg <= the handle's max_segments.
+ *   stats_out  device array of nseg peat_stats_t.
+ *   hist_out   device array of nseg*PEAT_HIST_BINS uint64 (or NULL).
+ * Errors: INVALID_ARG (as above, or offsets not non-decreasing from 0),
+ * UNSUPPORTED (nseg above max_segments), CUDA. */
+peat_status_t peat_compare_segmented(peat_handle_t h, const void* golden, const void* candidate,
+                                     const int64_t* offsets, int64_t nseg, peat_dtype_t dtype,
+                                     peat_tol_t tol, peat_stats_t* stats_out, uint64_t* hist_out,
+                                     peat_stream_t stream);
+
+/* Pseudo-error models (Section IV-A: FP16 cast, random value RV, random zero
+ * RZ with num_pos positions; Section II-B: random bit flip, random NaN; plus
+ * multiplicative and additive Gaussian noise, a relative bias and sign flips). */
+typedef enum {
+  PEAT_INJ_RZ = 0,        /* k distinct positions set to +0 */
+  PEAT_INJ_RV = 1,        /* k distinct positions take the value of a uniformly drawn element of src */
+  PEAT_INJ_BITFLIP = 2,   /* k distinct positions, one bit in [bit_lo, bit_hi] flipped */
+  PEAT_INJ_NAN_INF = 3,   /* each element with probability x: NaN (1/2), +Inf (1/4), -Inf (1/4) */
+  PEAT_INJ_SIGNFLIP = 4,  /* each element with probability x: sign bit flipped */
+  PEAT_INJ_REL_GAUSS = 5, /* v <- RN(v * RN32(1 + x*z)), z ~ N(0,1) */
+  PEAT_INJ_ADD_GAUSS = 6, /* v <- RN(RN32(v + x*z)) */
+  PEAT_INJ_BIAS = 7,      /* v <- RN(RN32(v + x*|v|)) */
+  PEAT_INJ_CAST_F16_RNE = 8, /* float32 tensors only: round to binary16 (nearest even) and back */
+  PEAT_INJ_CAST_F16_RTZ = 9, /* ... toward zero */
+  PEAT_INJ_CAST_BF16_RNE = 10,
+  PEAT_INJ_CAST_BF16_RTZ = 11
+} peat_inject_kind_t;
+
+typedef struct {
+  int32_t kind;   /* peat_inject_kind_t */
+  int32_t k;      /* RZ/RV/BITFLIP: number of distinct positions, 0 <= k <= min(n, 2^20) */
+  int32_t bit_lo; /* BITFLIP: inclusive bit range within the element */
+  int32_t bit_hi;
+  double x;       /* NAN_INF/SIGNFLIP: probability in [0,1]; GAUSS: sigma; BIAS: alpha (rounded to float32) */
+} peat_inject_t;
+
+/* Seeded pseudo-error generator (the Inject step of Alg. 1 / Alg. 2).
+ * dst = src with models[0..nmodels) applied in array order; each model sees
+ * the previous model's output, except that RV copies from src.  Noise,
+ * bias and cast models leave NaN/Inf elements unchanged.  Randomness is
+ * Philox4x32-10 keyed by `seed`: element i of model m uses counter
+ * (i lo, i hi, m, 0x454C454D); the j-th position draw of a fixed-count model
+ * uses (j lo, j hi, m, 0x504F5331).  Results are bit-identical run to run.
+ *   dst, src     device arrays of n elements (dst == src allowed; partial
+ *                overlap is not).
+ *   models       HOST array of nmodels (0 <= nmodels <= 64).
+ *   counts_out   device array of nmodels uint64: how many elements each
+ *                model fired on (k for the fixed-count models; the number
+ *                of finite elements for noise/bias/cast).
+ * Errors: INVALID_ARG (bad model parameters, cast on a non-float32 tensor,
+ * k > n), CUDA, ALLOC. */
+peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* src, int64_t n,
+                                       peat_dtype_t dtype, const peat_inject_t* models, int nmodels,
+                                       uint64_t seed, uint64_t* counts_out, peat_stream_t stream);
+
+/* Text of the last error reported on h (never NULL; "" if none).  With
+ * h == NULL, the last error of a failed peat_signature_create on this thread. */
+const char* peat_last_error(peat_handle_t h);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PEAT_H */

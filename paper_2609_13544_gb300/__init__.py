@@ -1,0 +1,259 @@
+"""Python binding of libpeat (include/peat.h): argument marshalling only.
+
+Every step of the compare and of the injector runs in the CUDA library;
+this module turns torch tensors into device pointers and sizes, calls the C
+ABI through ctypes, and unpacks the result records.  It raises if the
+library has not been built (there is no CPU fallback).
+
+Names follow the C ABI: ``peat_signature_create``, ``peat_compare``,
+``peat_compare_segmented``, ``peat_pseudo_error_inject``, ``peat_last_error``.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+from typing import Optional, Sequence
+
+import numpy as np
+
+from .buildlib import LIB, build  # noqa: F401
+
+DTYPE_CODES = {"f32": 0, "f16": 1, "bf16": 2}
+CLASSES = ("exact", "within_tol", "mismatch", "nan_inf_asym", "sign_flip")
+HIST_BINS = 128
+STATS_BYTES = 144
+INJECT_KINDS = {
+    "rz": 0, "rv": 1, "bitflip": 2, "nan_inf": 3, "signflip": 4, "rel_gauss": 5,
+    "add_gauss": 6, "bias": 7, "cast_f16_rne": 8, "cast_f16_rtz": 9, "cast_bf16_rne": 10,
+    "cast_bf16_rtz": 11,
+}
+STATUS = {0: "PEAT_OK", 1: "PEAT_ERR_INVALID_ARG", 2: "PEAT_ERR_UNSUPPORTED", 3: "PEAT_ERR_ALLOC",
+          4: "PEAT_ERR_CUDA", 5: "PEAT_ERR_TIMEOUT", 6: "PEAT_ERR_INTERNAL"}
+
+# numpy view of peat_stats_t
+STATS_DTYPE = np.dtype([
+    ("n", "<u8"), ("count", "<u8", (5,)), ("n_finite", "<u8"),
+    ("max_abs", "<f8"), ("argmax_abs", "<i8"), ("max_rel", "<f8"), ("argmax_rel", "<i8"),
+    ("max_ulp", "<u8"), ("argmax_ulp", "<i8"), ("sum_abs", "<f8"), ("sum_sq", "<f8"),
+    ("sum_signed", "<f8"), ("rtol_eff", "<f8"), ("atol_eff", "<f8"),
+])
+assert STATS_DTYPE.itemsize == STATS_BYTES
+
+
+class PeatError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("device", ctypes.c_int32), ("reserved0", ctypes.c_int32), ("max_segments", ctypes.c_int64),
+                ("flags", ctypes.c_uint32), ("reserved1", ctypes.c_uint32)]
+
+
+class Tol(ctypes.Structure):
+    _fields_ = [("rtol", ctypes.c_double), ("atol", ctypes.c_double)]
+
+
+class InjectModel(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("k", ctypes.c_int32), ("bit_lo", ctypes.c_int32),
+                ("bit_hi", ctypes.c_int32), ("x", ctypes.c_double)]
+
+
+EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
+           "peat_pseudo_error_inject", "peat_last_error")
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def load(path: Optional[Path] = None) -> ctypes.CDLL:
+    """Load libpeat.so; raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    p = Path(path) if path else LIB
+    if not p.exists():
+        raise RuntimeError(f"{p} is missing: build it with paper_2609_13544_gb300.buildlib.build() "
+                           "(or __graft_entry__.build()); there is no fallback")
+    L = ctypes.CDLL(str(p))
+    vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+    L.peat_signature_create.argtypes = [ctypes.POINTER(vp), ctypes.POINTER(Config)]
+    L.peat_signature_create.restype = i32
+    L.peat_signature_destroy.argtypes = [vp]
+    L.peat_signature_destroy.restype = i32
+    L.peat_compare.argtypes = [vp, vp, vp, i64, i32, Tol, vp, vp, vp]
+    L.peat_compare.restype = i32
+    L.peat_compare_segmented.argtypes = [vp, vp, vp, vp, i64, i32, Tol, vp, vp, vp]
+    L.peat_compare_segmented.restype = i32
+    L.peat_pseudo_error_inject.argtypes = [vp, vp, vp, i64, i32, ctypes.POINTER(InjectModel), i32,
+                                           ctypes.c_uint64, vp, vp]
+    L.peat_pseudo_error_inject.restype = i32
+    L.peat_last_error.argtypes = [vp]
+    L.peat_last_error.restype = ctypes.c_char_p
+    _lib = L
+    return L
+
+
+def peat_last_error(h=None) -> str:
+    return load().peat_last_error(h.ptr if isinstance(h, Handle) else h).decode()
+
+
+def _check(rc: int, h) -> None:
+    if rc != 0:
+        raise PeatError(rc, peat_last_error(h))
+
+
+class Handle:
+    """Owns one peat_handle_t (peat_signature_create / peat_signature_destroy)."""
+
+    def __init__(self, device: int = 0, max_segments: int = 0):
+        self.ptr = ctypes.c_void_p()
+        cfg = Config(device, 0, max_segments, 0, 0)
+        _check(load().peat_signature_create(ctypes.byref(self.ptr), ctypes.byref(cfg)), None)
+        self.device = device
+
+    def close(self) -> None:
+        if self.ptr:
+            load().peat_signature_destroy(self.ptr)
+            self.ptr = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *a):
+        self.close()
+
+
+def peat_signature_create(device: int = 0, max_segments: int = 0) -> Handle:
+    return Handle(device, max_segments)
+
+
+def peat_signature_destroy(h: Handle) -> None:
+    h.close()
+
+
+def dtype_code(t) -> int:
+    import torch
+    m = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2}
+    if t.dtype not in m:
+        raise TypeError(f"unsupported dtype {t.dtype}")
+    return m[t.dtype]
+
+
+def _stream_ptr(stream) -> Optional[int]:
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def _dev_tensor_check(*ts):
+    for t in ts:
+        if not t.is_cuda:
+            raise ValueError("golden/candidate must be CUDA tensors")
+        if not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+
+
+def peat_compare_raw(h: Handle, golden, candidate, rtol: float, atol: float, stats_out, hist_out=None,
+                     stream=None) -> None:
+    """peat_compare on preallocated device outputs (stats_out: uint8[144], hist_out: int64[128])."""
+    _dev_tensor_check(golden, candidate)
+    if golden.numel() != candidate.numel() or golden.dtype != candidate.dtype:
+        raise ValueError("golden and candidate differ in size or dtype")
+    rc = load().peat_compare(h.ptr, golden.data_ptr(), candidate.data_ptr(), golden.numel(), dtype_code(golden),
+                             Tol(rtol, atol), stats_out.data_ptr(),
+                             hist_out.data_ptr() if hist_out is not None else None, _stream_ptr(stream))
+    _check(rc, h)
+
+
+def peat_compare_segmented_raw(h: Handle, golden, candidate, offsets, rtol: float, atol: float, stats_out,
+                               hist_out=None, stream=None) -> None:
+    _dev_tensor_check(golden, candidate)
+    off = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    if golden.numel() != candidate.numel() or golden.dtype != candidate.dtype:
+        raise ValueError("golden and candidate differ in size or dtype")
+    if off.size < 1 or off[-1] > golden.numel():
+        raise ValueError("offsets exceed the tensors")
+    rc = load().peat_compare_segmented(h.ptr, golden.data_ptr(), candidate.data_ptr(), off.ctypes.data,
+                                       off.size - 1, dtype_code(golden), Tol(rtol, atol), stats_out.data_ptr(),
+                                       hist_out.data_ptr() if hist_out is not None else None,
+                                       _stream_ptr(stream))
+    _check(rc, h)
+
+
+def stats_to_dicts(raw: np.ndarray) -> list:
+    """Unpack host bytes (k*144) into dicts (same keys as the oracle's)."""
+    arr = np.frombuffer(np.ascontiguousarray(raw).tobytes(), dtype=STATS_DTYPE)
+    out = []
+    for r in arr:
+        d = {k: (r[k].item() if k != "count" else [int(v) for v in r[k]]) for k in STATS_DTYPE.names}
+        for name, v in zip(CLASSES, d["count"]):
+            d[name] = v
+        out.append(d)
+    return out
+
+
+def peat_compare(h: Handle, golden, candidate, rtol: float, atol: float = 0.0, stream=None):
+    """Signature of one tensor pair: (stats dict, hist numpy uint64[2, 64]); synchronises."""
+    import torch
+    dev = golden.device
+    stats = torch.empty(STATS_BYTES, dtype=torch.uint8, device=dev)
+    hist = torch.empty(HIST_BINS, dtype=torch.int64, device=dev)
+    peat_compare_raw(h, golden, candidate, rtol, atol, stats, hist, stream)
+    s = stats_to_dicts(stats.cpu().numpy())[0]
+    return s, hist.cpu().numpy().view(np.uint64).reshape(2, 64)
+
+
+def peat_compare_segmented(h: Handle, golden, candidate, offsets: Sequence[int], rtol: float, atol: float = 0.0,
+                           stream=None):
+    """Per-segment signatures: (list of dicts, hist numpy uint64[nseg, 2, 64]); synchronises."""
+    import torch
+    dev = golden.device
+    nseg = len(offsets) - 1
+    stats = torch.empty(max(nseg, 1) * STATS_BYTES, dtype=torch.uint8, device=dev)
+    hist = torch.empty(max(nseg, 1) * HIST_BINS, dtype=torch.int64, device=dev)
+    peat_compare_segmented_raw(h, golden, candidate, offsets, rtol, atol, stats, hist, stream)
+    if nseg == 0:
+        return [], np.zeros((0, 2, 64), np.uint64)
+    s = stats_to_dicts(stats.cpu().numpy()[: nseg * STATS_BYTES])
+    return s, hist.cpu().numpy()[: nseg * HIST_BINS].view(np.uint64).reshape(nseg, 2, 64)
+
+
+def inject_model(kind: str, k: int = 0, bit_lo: int = 0, bit_hi: int = 0, x: float = 0.0) -> dict:
+    return {"kind": kind, "k": k, "bit_lo": bit_lo, "bit_hi": bit_hi, "x": x}
+
+
+def peat_pseudo_error_inject(h: Handle, src, models: Sequence[dict], seed: int, dst=None, stream=None):
+    """Apply error models to src on the GPU; returns (dst tensor, counts numpy uint64)."""
+    import torch
+    _dev_tensor_check(src)
+    if dst is None:
+        dst = torch.empty_like(src)
+    arr = (InjectModel * max(len(models), 1))()
+    for i, m in enumerate(models):
+        arr[i] = InjectModel(INJECT_KINDS[m["kind"]], m.get("k", 0), m.get("bit_lo", 0), m.get("bit_hi", 0),
+                             float(m.get("x", 0.0)))
+    counts = torch.zeros(max(len(models), 1), dtype=torch.int64, device=src.device)
+    rc = load().peat_pseudo_error_inject(h.ptr, dst.data_ptr(), src.data_ptr(), src.numel(), dtype_code(src), arr,
+                                         len(models), ctypes.c_uint64(seed), counts.data_ptr(),
+                                         _stream_ptr(stream))
+    _check(rc, h)
+    return dst, counts[: len(models)].cpu().numpy().view(np.uint64)
+
+
+def derived_scores(st: dict) -> dict:
+    """Host-side scores of Section IV-B-3 from one signature: mean, variance of |e|, bias, L2, RMS."""
+    import math
+    nf = st["n_finite"]
+    mean = st["sum_abs"] / nf if nf else 0.0
+    out = {"max": st["max_abs"], "mean": mean, "bias": st["sum_signed"] / nf if nf else 0.0,
+           "l2": math.sqrt(st["sum_sq"]), "rms": math.sqrt(st["sum_sq"] / nf) if nf else 0.0,
+           "var": (st["sum_sq"] / nf - mean * mean) if nf else 0.0}
+    return out

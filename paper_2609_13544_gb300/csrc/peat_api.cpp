@@ -1,0 +1,405 @@
+// Host runtime behind the C ABI declared in include/peat.h: handles,
+// workspace, argument checks, launch planning and error reporting.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <string>
+#include <unordered_set>
+#include <vector>
+
+#include "peat.h"
+#include "peat_internal.h"
+
+struct peat_handle_s {
+  int device = 0;
+  int nsm = 0;
+  int64_t max_segments = 4096;
+  int max_ctas = 0;
+  // compare workspace
+  peat::Partial* partials = nullptr;
+  int64_t* d_offsets = nullptr;
+  int64_t* h_offsets = nullptr;  // pinned staging
+  cudaEvent_t staged = nullptr;  // the last staging copy has been consumed
+  bool staged_pending = false;
+  // injector staging (grown on demand)
+  int64_t* d_inj = nullptr;
+  int64_t* h_inj = nullptr;
+  size_t inj_cap = 0;  // in int64 elements
+  std::string err;
+};
+
+namespace {
+
+thread_local std::string g_create_error;
+
+struct DeviceGuard {
+  int prev = -1;
+  bool ok = true;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+peat_status_t fail(peat_handle_t h, peat_status_t st, const std::string& msg) {
+  if (h) h->err = msg;
+  return st;
+}
+
+peat_status_t cuda_fail(peat_handle_t h, cudaError_t e, const char* what) {
+  cudaGetLastError();  // clear a sticky non-fatal error state
+  return fail(h, PEAT_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+int dtype_bytes(int dt) { return dt == PEAT_F32 ? 4 : (dt == PEAT_F16 || dt == PEAT_BF16 ? 2 : 0); }
+
+bool round_tol(peat_tol_t tol, float* r, float* a) {
+  if (!(tol.rtol >= 0.0) || !(tol.atol >= 0.0)) return false;  // rejects NaN too
+  *r = (float)tol.rtol;
+  *a = (float)tol.atol;
+  return std::isfinite(*r) && std::isfinite(*a);
+}
+
+// wait until the pinned staging buffers may be rewritten
+peat_status_t wait_staging(peat_handle_t h) {
+  if (h->staged_pending) {
+    cudaError_t e = cudaEventSynchronize(h->staged);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventSynchronize");
+    h->staged_pending = false;
+  }
+  return PEAT_OK;
+}
+
+peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const int64_t* offsets,
+                           int64_t nseg, peat_dtype_t dtype, peat_tol_t tol, peat_stats_t* stats,
+                           uint64_t* hist, peat_stream_t stream) {
+  if (!h) return PEAT_ERR_INVALID_ARG;
+  int B = dtype_bytes(dtype);
+  if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
+  float rtol, atol;
+  if (!round_tol(tol, &rtol, &atol))
+    return fail(h, PEAT_ERR_INVALID_ARG, "rtol and atol must be finite and >= 0 after rounding to float32");
+  if (nseg < 0) return fail(h, PEAT_ERR_INVALID_ARG, "nseg < 0");
+  if (nseg > h->max_segments)
+    return fail(h, PEAT_ERR_UNSUPPORTED, "nseg exceeds the handle's max_segments");
+  if (!offsets) return fail(h, PEAT_ERR_INVALID_ARG, "offsets is NULL");
+  if (offsets[0] != 0) return fail(h, PEAT_ERR_INVALID_ARG, "offsets[0] must be 0");
+  for (int64_t s = 0; s < nseg; s++)
+    if (offsets[s + 1] < offsets[s]) return fail(h, PEAT_ERR_INVALID_ARG, "offsets must be non-decreasing");
+  const int64_t n = offsets[nseg];
+  if (n > 0 && (!g || !c)) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
+  if (nseg > 0 && !stats) return fail(h, PEAT_ERR_INVALID_ARG, "stats_out is NULL");
+  if (nseg == 0) return PEAT_OK;
+  DeviceGuard dg(h->device);
+  if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+
+  peat_status_t ps = wait_staging(h);
+  if (ps != PEAT_OK) return ps;
+  std::memcpy(h->h_offsets, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
+  cudaError_t e = cudaMemcpyAsync(h->d_offsets, h->h_offsets, sizeof(int64_t) * (size_t)(nseg + 1),
+                                  cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(offsets)");
+  e = cudaEventRecord(h->staged, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
+  h->staged_pending = true;
+
+  peat::CompareParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.g = g;
+  p.c = c;
+  p.n_total = n;
+  p.offsets = h->d_offsets;
+  p.nseg = nseg;
+  uintptr_t ag = reinterpret_cast<uintptr_t>(g), ac = reinterpret_cast<uintptr_t>(c);
+  if (n > 0 && ag % B == 0 && ac % B == 0 && ag % 16 == ac % 16)
+    p.p0 = (int64_t)(((16 - ag % 16) % 16) / B);
+  else
+    p.p0 = -1;
+  // persistent grid, at most one CTA per ~4K elements for small inputs
+  int64_t want = (n + 4095) / 4096;
+  p.nctas = (int)std::max<int64_t>(1, std::min<int64_t>(h->max_ctas, want));
+  p.partials = h->partials;
+  p.rtol = rtol;
+  p.atol = atol;
+  p.stats = stats;
+  p.hist = hist;
+  e = peat::launch_compare(dtype, p, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "compare launch");
+  return PEAT_OK;
+}
+
+// ---- host Philox4x32-10 for the fixed-count position draws ----
+void philox_host(const uint32_t ctr[4], uint64_t seed, uint32_t out[4]) {
+  uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
+  uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+  for (int r = 0; r < 10; r++) {
+    if (r) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    uint64_t p0 = (uint64_t)0xD2511F53u * c0, p1 = (uint64_t)0xCD9E8D57u * c2;
+    uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ k0, n2 = (uint32_t)(p0 >> 32) ^ c3 ^ k1;
+    c1 = (uint32_t)p1;
+    c3 = (uint32_t)p0;
+    c0 = n0;
+    c2 = n2;
+  }
+  out[0] = c0;
+  out[1] = c1;
+  out[2] = c2;
+  out[3] = c3;
+}
+
+uint64_t mulhi64(uint64_t w, uint64_t n) { return (uint64_t)(((unsigned __int128)w * n) >> 64); }
+
+peat_status_t grow_inject(peat_handle_t h, size_t need) {
+  if (need <= h->inj_cap) return PEAT_OK;
+  peat_status_t ps = wait_staging(h);
+  if (ps != PEAT_OK) return ps;
+  size_t cap = std::max(need, (size_t)4096);
+  if (h->d_inj) cudaFree(h->d_inj);
+  if (h->h_inj) cudaFreeHost(h->h_inj);
+  h->d_inj = nullptr;
+  h->h_inj = nullptr;
+  h->inj_cap = 0;
+  if (cudaMalloc(&h->d_inj, cap * sizeof(int64_t)) != cudaSuccess ||
+      cudaMallocHost(&h->h_inj, cap * sizeof(int64_t)) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(h, PEAT_ERR_ALLOC, "injector staging allocation failed");
+  }
+  h->inj_cap = cap;
+  return PEAT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg) {
+  g_create_error.clear();
+  if (!out) {
+    g_create_error = "out is NULL";
+    return PEAT_ERR_INVALID_ARG;
+  }
+  *out = nullptr;
+  peat_config_t c;
+  std::memset(&c, 0, sizeof(c));
+  if (cfg) c = *cfg;
+  if (c.flags != 0 || c.max_segments < 0) {
+    g_create_error = "bad config (flags must be 0, max_segments >= 0)";
+    return PEAT_ERR_INVALID_ARG;
+  }
+  int ndev = 0;
+  cudaError_t e = cudaGetDeviceCount(&ndev);
+  if (e != cudaSuccess || c.device < 0 || c.device >= ndev) {
+    cudaGetLastError();
+    g_create_error = std::string("no such CUDA device: ") + (e != cudaSuccess ? cudaGetErrorString(e) : "");
+    return e != cudaSuccess ? PEAT_ERR_CUDA : PEAT_ERR_INVALID_ARG;
+  }
+  peat_handle_t h = new peat_handle_s();
+  h->device = c.device;
+  h->max_segments = c.max_segments > 0 ? c.max_segments : 4096;
+  DeviceGuard dg(h->device);
+  if (!dg.ok) {
+    g_create_error = "cudaSetDevice failed";
+    delete h;
+    return PEAT_ERR_CUDA;
+  }
+  cudaDeviceGetAttribute(&h->nsm, cudaDevAttrMultiProcessorCount, h->device);
+  h->max_ctas = std::max(1, h->nsm * peat::compare_ctas_per_sm());
+  size_t slots = (size_t)h->max_segments + (size_t)h->max_ctas;
+  bool ok = cudaMalloc(&h->partials, slots * peat::compare_partial_bytes()) == cudaSuccess &&
+            cudaMalloc(&h->d_offsets, sizeof(int64_t) * (size_t)(h->max_segments + 1)) == cudaSuccess &&
+            cudaMallocHost(&h->h_offsets, sizeof(int64_t) * (size_t)(h->max_segments + 1)) == cudaSuccess &&
+            cudaEventCreateWithFlags(&h->staged, cudaEventDisableTiming) == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    g_create_error = "workspace allocation failed";
+    peat_signature_destroy(h);
+    return PEAT_ERR_ALLOC;
+  }
+  *out = h;
+  return PEAT_OK;
+}
+
+peat_status_t peat_signature_destroy(peat_handle_t h) {
+  if (!h) return PEAT_OK;
+  {
+    DeviceGuard dg(h->device);
+    if (h->staged) cudaEventSynchronize(h->staged);
+    cudaDeviceSynchronize();
+    if (h->partials) cudaFree(h->partials);
+    if (h->d_offsets) cudaFree(h->d_offsets);
+    if (h->h_offsets) cudaFreeHost(h->h_offsets);
+    if (h->d_inj) cudaFree(h->d_inj);
+    if (h->h_inj) cudaFreeHost(h->h_inj);
+    if (h->staged) cudaEventDestroy(h->staged);
+    cudaGetLastError();
+  }
+  delete h;
+  return PEAT_OK;
+}
+
+peat_status_t peat_compare(peat_handle_t h, const void* golden, const void* candidate, int64_t n,
+                           peat_dtype_t dtype, peat_tol_t tol, peat_stats_t* stats_out, uint64_t* hist_out,
+                           peat_stream_t stream) {
+  if (!h) return PEAT_ERR_INVALID_ARG;
+  if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
+  int64_t off[2] = {0, n};
+  return compare_impl(h, golden, candidate, off, 1, dtype, tol, stats_out, hist_out, stream);
+}
+
+peat_status_t peat_compare_segmented(peat_handle_t h, const void* golden, const void* candidate,
+                                     const int64_t* offsets, int64_t nseg, peat_dtype_t dtype,
+                                     peat_tol_t tol, peat_stats_t* stats_out, uint64_t* hist_out,
+                                     peat_stream_t stream) {
+  return compare_impl(h, golden, candidate, offsets, nseg, dtype, tol, stats_out, hist_out, stream);
+}
+
+peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* src, int64_t n,
+                                       peat_dtype_t dtype, const peat_inject_t* models, int nmodels,
+                                       uint64_t seed, uint64_t* counts_out, peat_stream_t stream) {
+  if (!h) return PEAT_ERR_INVALID_ARG;
+  int B = dtype_bytes(dtype);
+  if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "bad dtype");
+  if (n < 0 || nmodels < 0 || nmodels > 64) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0 or nmodels outside [0, 64]");
+  if (nmodels > 0 && (!models || !counts_out)) return fail(h, PEAT_ERR_INVALID_ARG, "models/counts_out is NULL");
+  if (n > 0 && (!dst || !src)) return fail(h, PEAT_ERR_INVALID_ARG, "dst/src is NULL");
+  if (dst != src && n > 0) {
+    uintptr_t a = (uintptr_t)dst, b = (uintptr_t)src, len = (uintptr_t)n * B;
+    if (a < b + len && b < a + len) return fail(h, PEAT_ERR_INVALID_ARG, "dst and src overlap partially");
+  }
+  const int width = B * 8;
+  size_t need = 0;
+  for (int m = 0; m < nmodels; m++) {
+    const peat_inject_t& md = models[m];
+    if (md.kind < PEAT_INJ_RZ || md.kind > PEAT_INJ_CAST_BF16_RTZ) return fail(h, PEAT_ERR_INVALID_ARG, "bad model kind");
+    if (md.kind <= PEAT_INJ_BITFLIP) {
+      if (md.k < 0 || md.k > n || md.k > (1 << 20)) return fail(h, PEAT_ERR_INVALID_ARG, "k outside [0, min(n, 2^20)]");
+      if (md.kind == PEAT_INJ_BITFLIP && (md.bit_lo < 0 || md.bit_hi < md.bit_lo || md.bit_hi >= width))
+        return fail(h, PEAT_ERR_INVALID_ARG, "bit range outside the element");
+      need += 3 * (size_t)md.k;
+    } else if (md.kind <= PEAT_INJ_SIGNFLIP) {
+      if (!(md.x >= 0.0 && md.x <= 1.0)) return fail(h, PEAT_ERR_INVALID_ARG, "rate outside [0, 1]");
+    } else if (md.kind <= PEAT_INJ_BIAS) {
+      if (!std::isfinite(md.x) || !std::isfinite((float)md.x)) return fail(h, PEAT_ERR_INVALID_ARG, "parameter not finite");
+    } else if (dtype != PEAT_F32) {
+      return fail(h, PEAT_ERR_INVALID_ARG, "cast models apply to float32 tensors only");
+    }
+  }
+  DeviceGuard dg(h->device);
+  if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (nmodels > 0) {
+    e = cudaMemsetAsync(counts_out, 0, sizeof(uint64_t) * (size_t)nmodels, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemsetAsync(counts)");
+  }
+  // Draw every fixed-count model's positions up front.  Staging layout per
+  // model m: [positions k | aux k | values k] int64, then nmodels counts.
+  // aux = RV source index; values = RV source values (filled on the device)
+  // or, for BITFLIP, the bit indices as uint32.
+  peat_status_t ps = grow_inject(h, need + (size_t)nmodels);
+  if (ps != PEAT_OK) return ps;
+  ps = wait_staging(h);
+  if (ps != PEAT_OK) return ps;
+  std::vector<size_t> base(nmodels, 0);
+  size_t used = 0;
+  for (int m = 0; m < nmodels; m++) {
+    const peat_inject_t& md = models[m];
+    h->h_inj[need + (size_t)m] = 0;
+    if (md.kind > PEAT_INJ_BITFLIP) continue;
+    int64_t k = md.k;
+    base[m] = used;
+    int64_t* pos = h->h_inj + used;
+    int64_t* aux = pos + k;
+    uint32_t* bits = reinterpret_cast<uint32_t*>(pos + 2 * k);
+    std::unordered_set<int64_t> taken;
+    taken.reserve((size_t)k * 2 + 1);
+    int64_t got = 0;
+    for (uint64_t j = 0; got < k; j++) {
+      uint32_t ctr[4] = {(uint32_t)j, (uint32_t)(j >> 32), (uint32_t)m, 0x504F5331u}, w[4];
+      philox_host(ctr, seed, w);
+      int64_t p = (int64_t)mulhi64(((uint64_t)w[1] << 32) | w[0], (uint64_t)n);
+      if (!taken.insert(p).second) continue;
+      pos[got] = p;
+      aux[got] = 0;
+      if (md.kind == PEAT_INJ_RV)
+        aux[got] = (int64_t)mulhi64(((uint64_t)w[3] << 32) | w[2], (uint64_t)n);
+      else if (md.kind == PEAT_INJ_BITFLIP)
+        bits[got] = (uint32_t)md.bit_lo + (uint32_t)(((uint64_t)w[2] * (uint64_t)(md.bit_hi - md.bit_lo + 1)) >> 32);
+      got++;
+    }
+    h->h_inj[need + (size_t)m] = k;
+    used += 3 * (size_t)k;
+  }
+  if (nmodels > 0) {
+    e = cudaMemcpyAsync(h->d_inj, h->h_inj, (need + (size_t)nmodels) * sizeof(int64_t), cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(positions)");
+  }
+  // RV source values come from src before any model runs (src may be dst)
+  for (int m = 0; m < nmodels; m++)
+    if (models[m].kind == PEAT_INJ_RV && models[m].k > 0) {
+      int64_t k = models[m].k;
+      e = peat::launch_gather(dtype, src, h->d_inj + base[m] + k, h->d_inj + base[m] + 2 * k, k, st);
+      if (e != cudaSuccess) return cuda_fail(h, e, "gather launch");
+    }
+  if (dst != src && n > 0) {
+    e = cudaMemcpyAsync(dst, src, (size_t)n * B, cudaMemcpyDeviceToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(dst <- src)");
+  }
+  for (int m = 0; m < nmodels; m++) {
+    const peat_inject_t& md = models[m];
+    if (md.kind <= PEAT_INJ_BITFLIP) {
+      int64_t k = md.k;
+      if (k > 0) {
+        peat::InjectScatterParams sp;
+        sp.dst = dst;
+        sp.src = src;
+        sp.n = n;
+        sp.kind = md.kind;
+        sp.pos = h->d_inj + base[m];
+        sp.from = h->d_inj + base[m] + 2 * k;
+        sp.bit = reinterpret_cast<const uint32_t*>(h->d_inj + base[m] + 2 * k);
+        sp.k = k;
+        e = peat::launch_inject_scatter(dtype, sp, st);
+        if (e != cudaSuccess) return cuda_fail(h, e, "inject scatter launch");
+      }
+      e = cudaMemcpyAsync(counts_out + m, h->d_inj + need + m, sizeof(uint64_t), cudaMemcpyDeviceToDevice, st);
+      if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(count)");
+    } else {
+      peat::InjectElemParams ep;
+      ep.dst = dst;
+      ep.src = src;
+      ep.n = n;
+      ep.kind = md.kind;
+      ep.model = (uint32_t)m;
+      ep.seed = seed;
+      double t = std::floor(md.x * 4294967296.0);
+      ep.threshold = (uint64_t)std::min(std::max(t, 0.0), 4294967296.0);
+      ep.x = (float)md.x;
+      ep.count = reinterpret_cast<unsigned long long*>(counts_out + m);
+      e = peat::launch_inject_elem(dtype, ep, st);
+      if (e != cudaSuccess) return cuda_fail(h, e, "inject launch");
+    }
+  }
+  e = cudaEventRecord(h->staged, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
+  h->staged_pending = true;
+  return PEAT_OK;
+}
+
+const char* peat_last_error(peat_handle_t h) {
+  if (!h) return g_create_error.c_str();
+  return h->err.c_str();
+}
+
+}  // extern "C"

@@ -90,7 +90,7 @@ typedef struct {
 
 /* Handle configuration.  device: CUDA ordinal the handle's calls run on.
  * max_segments: the largest nseg a segmented call may pass (0 = 4096).
- * flags: reserved, must be 0. */
+ * flags: 0, or PEAT_FLAG_TEST_EXPIRE_WAITS. */
 typedef struct {
   int32_t device;
   int32_t reserved0;
@@ -98,6 +98,12 @@ typedef struct {
   uint32_t flags;
   uint32_t reserved1;
 } peat_config_t;
+
+/* Testing aid: every bounded device-side wait of the compare pipeline gives
+ * up at its first poll, so the timeout path (error flag, drained copies,
+ * PEAT_ERR_TIMEOUT on the next call) can be exercised without a real stall.
+ * Outputs of calls on such a handle are not valid. */
+#define PEAT_FLAG_TEST_EXPIRE_WAITS 0x80000000u
 
 /* Signature of one tensor (or one segment).  144 bytes, no padding holes. */
 typedef struct {
@@ -142,7 +148,8 @@ peat_status_t peat_signature_destroy(peat_handle_t h);
  *   stats_out          device pointer to one peat_stats_t.
  *   hist_out           device pointer to PEAT_HIST_BINS uint64 (or NULL).
  * Errors: INVALID_ARG (null pointer with n > 0, n < 0, bad dtype, bad tol),
- * CUDA. */
+ * CUDA, TIMEOUT (a bounded device wait of an EARLIER call on this handle
+ * expired; that call's outputs are invalid; the flag is cleared). */
 peat_status_t peat_compare(peat_handle_t h, const void* golden, const void* candidate, int64_t n,
                            peat_dtype_t dtype, peat_tol_t tol, peat_stats_t* stats_out,
                            uint64_t* hist_out, peat_stream_t stream);

@@ -27,6 +27,7 @@ INJECT_KINDS = {
     "add_gauss": 6, "bias": 7, "cast_f16_rne": 8, "cast_f16_rtz": 9, "cast_bf16_rne": 10,
     "cast_bf16_rtz": 11,
 }
+PEAT_FLAG_TEST_EXPIRE_WAITS = 0x80000000
 STATUS = {0: "PEAT_OK", 1: "PEAT_ERR_INVALID_ARG", 2: "PEAT_ERR_UNSUPPORTED", 3: "PEAT_ERR_ALLOC",
           4: "PEAT_ERR_CUDA", 5: "PEAT_ERR_TIMEOUT", 6: "PEAT_ERR_INTERNAL"}
 
@@ -106,9 +107,9 @@ def _check(rc: int, h) -> None:
 class Handle:
     """Owns one peat_handle_t (peat_signature_create / peat_signature_destroy)."""
 
-    def __init__(self, device: int = 0, max_segments: int = 0):
+    def __init__(self, device: int = 0, max_segments: int = 0, flags: int = 0):
         self.ptr = ctypes.c_void_p()
-        cfg = Config(device, 0, max_segments, 0, 0)
+        cfg = Config(device, 0, max_segments, flags, 0)
         _check(load().peat_signature_create(ctypes.byref(self.ptr), ctypes.byref(cfg)), None)
         self.device = device
 
@@ -130,8 +131,8 @@ class Handle:
         self.close()
 
 
-def peat_signature_create(device: int = 0, max_segments: int = 0) -> Handle:
-    return Handle(device, max_segments)
+def peat_signature_create(device: int = 0, max_segments: int = 0, flags: int = 0) -> Handle:
+    return Handle(device, max_segments, flags)
 
 
 def peat_signature_destroy(h: Handle) -> None:

@@ -8,23 +8,29 @@
 // sums as the exact real sum rounded once to nearest-even binary64.
 //
 // Stage 1 (compare_stage1): a persistent grid streams both tensors once.
-// CTA b owns the contiguous element range [lo_b, lo_{b+1}) and writes one
-// Partial per segment piece it touches (slot s + b).  Per element pair:
+// CTA b owns the contiguous element range [lo_b, lo_{b+1}); per segment piece
+// it touches it adds its integer totals (counts, histograms, sum digits) to
+// the segment's accumulator with atomics and writes its maxima to slot s + b.
+// Per element pair:
 //   - bitwise-equal vectors are counted and skipped;
-//   - a "window" lane (same sign and binade, golden exponent inside the CTA's
-//     window of binades) is exact in float32 arithmetic and integer ops:
-//     d = +-u * 2^E with u = |bits(c) - bits(g)| the ULP distance, so
-//     sum |d|, sum d, sum d^2 accumulate as integers u << (e - Lb) and
-//     (u << (e - Lb))^2; the log2-relative bin is the exponent difference
-//     of |d| and |g|; the tolerance test is one float32 fma (exact except
-//     at equality, which goes to the general path);
-//   - every other lane (non-finite, sign change, other binades, outside the
-//     window, tolerance ties) takes the general path, which evaluates the
-//     definitions exactly in binary64 (TwoSum) and adds its sum terms to a
-//     CTA-wide carry-save fixed-point accumulator in shared memory.
-// Stage 2 (compare_stage2): one CTA per segment merges that segment's
-// partials in a fixed order; all merged quantities are integers or exact
-// values, so the result does not depend on the grid.
+//   - a "window" lane -- same sign, at most one binade apart (ULP distance
+//     u < 2^UB), both operands' steps at least 2^Lexp, |d| < 2^(24+Lexp) --
+//     is exact in float32 and integer arithmetic: d = c - g is exact in
+//     float32, V = |d| / 2^Lexp is an integer below 2^24, so sum |d|, sum d
+//     and sum d^2 accumulate as integers; the log2-relative bin is the
+//     exponent difference of |d| and |g| read from their bit patterns; the
+//     tolerance test is one float32 fma, exact except at equality;
+//   - every other lane (non-finite, sign change, zeros, wide gaps, outside
+//     the window, tolerance ties) takes the general path, which evaluates the
+//     definitions exactly with float32 error-free transforms and integer
+//     digits, adding its sum terms to a CTA-wide carry-save fixed-point
+//     accumulator in shared memory.
+// Binary64 arithmetic is avoided in stage 1 (GB300 runs it at a small
+// fraction of float32 rate); binary64 values appear only as containers.
+// Stage 2 (compare_stage2): one CTA per segment merges the maxima of that
+// segment's pieces, rounds the exact sums once and clears the accumulator;
+// all merged quantities are integers or exact values, so the result does not
+// depend on the grid or on the order of the atomics.
 #include <cuda_fp16.h>
 
 #include <cstdint>
@@ -42,34 +48,36 @@ struct Tr;
 template <>
 struct Tr<PEAT_F32> {
   static constexpr int BYTES = 4, VEC = 4, MB = 23, BIAS = 127, EMAX = 255;
-  static constexpr int UB = 12;      // window lanes need u < 2^UB
-  static constexpr int LBMIN = 24;   // |d| >= 2^(e-150) stays a normal float32
-  static constexpr uint32_t SIGN = 0x80000000u, MAG = 0x7FFFFFFFu, SE = 0xFF800000u, INF = 0x7F800000u;
+  static constexpr int UB = 12;       // window lanes need u < 2^UB
+  static constexpr int LBMIN = 24;    // keeps 2^Lexp >= 2^-126 (normal float32)
+  static constexpr int LBMAX = 221;   // keeps |g| < 2^126 (normal reciprocal)
+  static constexpr uint32_t SIGN = 0x80000000u, MAG = 0x7FFFFFFFu, INF = 0x7F800000u;
 };
 template <>
 struct Tr<PEAT_F16> {
   static constexpr int BYTES = 2, VEC = 8, MB = 10, BIAS = 15, EMAX = 31;
-  static constexpr int UB = 10, LBMIN = 1;
-  static constexpr uint32_t SIGN = 0x8000u, MAG = 0x7FFFu, SE = 0xFC00u, INF = 0x7C00u;
+  static constexpr int UB = 10, LBMIN = 1, LBMAX = 30;
+  static constexpr uint32_t SIGN = 0x8000u, MAG = 0x7FFFu, INF = 0x7C00u;
 };
 template <>
 struct Tr<PEAT_BF16> {
   static constexpr int BYTES = 2, VEC = 8, MB = 7, BIAS = 127, EMAX = 255;
-  static constexpr int UB = 7, LBMIN = 8;
-  static constexpr uint32_t SIGN = 0x8000u, MAG = 0x7FFFu, SE = 0xFF80u, INF = 0x7F80u;
+  static constexpr int UB = 7, LBMIN = 8, LBMAX = 221;
+  static constexpr uint32_t SIGN = 0x8000u, MAG = 0x7FFFu, INF = 0x7F80u;
 };
 
-// Window of binades [Lb, Lb + SHMAX]: u << (e - Lb) stays below 2^32.
+// Private per-thread histogram rows: ULP bins 1..NU, then the log2-relative
+// bins window lanes reach, k in [KLO, KHI] (fp16 goldens may be subnormal,
+// whose ratios reach 2^MB).  ULP bins above NU use shared counters.
+constexpr int NU = 15;
 template <int DT>
-struct Win {
-  static constexpr int SHMAX = 32 - Tr<DT>::UB;
-  // keep |g| < 2^126 inside the window so the reciprocal in the rel filter stays normal
-  static constexpr int LBMAX = (Tr<DT>::EMAX == 255 ? 252 : Tr<DT>::EMAX - 1) - SHMAX;
-  static constexpr int NPB = 63 + Tr<DT>::UB + 1;  // private rows: ULP 1..63, rel k in [-(MB+1), UB-MB-1]
+struct Rows {
+  static constexpr int KLO = -(Tr<DT>::MB + 1);
+  static constexpr int KHI = DT == PEAT_F16 ? Tr<DT>::MB - 1 : Tr<DT>::UB - Tr<DT>::MB;
+  static constexpr int NPB = NU + KHI - KLO + 1;
 };
-
 constexpr int HALF = BLOCK / 2;
-constexpr int NPB_MAX = 63 + 12 + 1;
+constexpr int NPB_MAX = NU + 9 + 11 + 1;
 
 template <int DT>
 __device__ __forceinline__ float to_f32(uint32_t b) {
@@ -106,17 +114,57 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return r;
 }
 
-// ---------------------------------------------------------------------------
-// exact arithmetic helpers (binary64; used off the hot path)
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ void two_sum(double x, double y, double& s, double& t) {
-  s = __dadd_rn(x, y);
-  double yv = __dsub_rn(s, x);
-  double xv = __dsub_rn(s, yv);
-  t = __dadd_rn(__dsub_rn(x, xv), __dsub_rn(y, yv));
+// ---- bulk-copy (TMA) staging: mbarrier + cp.async.bulk, waits bounded -----
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void mbar_init(unsigned long long* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
 }
+__device__ __forceinline__ void mbar_init_fence() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+__device__ __forceinline__ void mbar_expect_tx(unsigned long long* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+// global -> shared bulk copy of `bytes` (16-byte aligned, multiple of 16), completing on bar
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, unsigned long long* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_addr(dst)),
+               "l"(src), "r"(bytes), "r"(smem_addr(bar))
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_test(unsigned long long* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// wait for phase `parity` of bar to complete, giving up after `limit` polls
+// (limit 0: give up without polling)
+__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, uint32_t parity, uint32_t limit) {
+  for (uint32_t it = 0; it < limit; it++)
+    if (mbar_test(bar, parity)) return true;
+  return false;
+}
+// order earlier generic-proxy accesses of the stage before the next bulk write into it
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+constexpr uint32_t DRAIN_LIMIT = 1u << 26;  // polls before a drain wait gives up (far beyond any copy)
 
-// x = m * 2^e, m a 53-bit integer (x finite, nonzero)
+// ---------------------------------------------------------------------------
+// exact integer digits
+// ---------------------------------------------------------------------------
+// x = m * 2^e with m an integer (x finite, nonzero); float32 and binary64
+__device__ __forceinline__ uint32_t split_float(float x, int& e) {
+  uint32_t b = __float_as_uint(x) & 0x7FFFFFFFu;
+  uint32_t be = b >> 23, m = b & 0x7FFFFFu;
+  if (be == 0) {
+    e = -149;
+    return m;
+  }
+  e = (int)be - 150;
+  return m | 0x800000u;
+}
 __device__ __forceinline__ uint64_t split_double(double x, int& e) {
   uint64_t b = (uint64_t)__double_as_longlong(x) & 0x7FFFFFFFFFFFFFFFull;
   int be = (int)(b >> 52);
@@ -129,9 +177,8 @@ __device__ __forceinline__ uint64_t split_double(double x, int& e) {
   return m | (1ull << 52);
 }
 
-// Signed 32-bit digits of +-m * 2^e, m < 2^106, delivered to a callback
-// (digit index, signed value).  LIMB_LSB <= e and the top digit stays in range
-// for every value that occurs (checked by construction of the callers).
+// Signed 32-bit digits of +-m * 2^e (m < 2^128), delivered to f(digit, value).
+// Every value that occurs is a multiple of 2^LIMB_LSB and below 2^352.
 template <class F>
 __device__ __forceinline__ void for_digits(unsigned __int128 m, int e, bool neg, F&& f) {
   if (m == 0) return;
@@ -148,7 +195,7 @@ __device__ __forceinline__ void for_digits(unsigned __int128 m, int e, bool neg,
     if (out[k] && j + k < NLIMB) f(j + k, neg ? -(int64_t)out[k] : (int64_t)out[k]);
 }
 
-// A local exact accumulator (off the hot path: rare comparisons, stage 2).
+// A local exact accumulator: integer digits only (off the hot path).
 struct XAcc {
   int64_t d[NLIMB];
   __device__ void zero() {
@@ -157,6 +204,19 @@ struct XAcc {
   }
   __device__ void add_m(unsigned __int128 m, int e, bool neg) {
     for_digits(m, e, neg, [&](int j, int64_t v) { d[j] += v; });
+  }
+  // +-x * 2^sc
+  __device__ void add_f(float x, bool neg = false, int sc = 0) {
+    if (x == 0.0f) return;
+    int e;
+    uint32_t m = split_float(x, e);
+    add_m(m, e + sc, neg ^ (x < 0));
+  }
+  __device__ void add_prod_f(float x, float y, bool neg = false, int sc = 0) {
+    if (x == 0.0f || y == 0.0f) return;
+    int ex, ey;
+    uint32_t mx = split_float(x, ex), my = split_float(y, ey);
+    add_m((unsigned __int128)((uint64_t)mx * my), ex + ey + sc, neg ^ (x < 0) ^ (y < 0));
   }
   __device__ void add_double(double x, bool neg = false) {
     if (x == 0.0) return;
@@ -202,17 +262,15 @@ struct XAcc {
         break;
       }
     if (top < 0) return 0.0;
-    // gather the value's leading 96 bits into hi:mid:lo digits
     uint64_t dtop = (uint64_t)d[top];
-    int lz = __clzll(dtop);  // >= 0; dtop < 2^63
-    int msb = top * 32 + 63 - lz;  // bit index of the leading one
-    // take bits [msb-63, msb] as a 64-bit window, plus a sticky flag below
+    int msb = top * 32 + 63 - __clzll(dtop);  // bit index of the leading one
+    // the 64 bits [msb-63, msb], plus a sticky flag for everything below
     uint64_t win = 0;
-    bool sticky = false;
     for (int bit = msb; bit > msb - 64; bit--) {
       win <<= 1;
       if (bit >= 0) win |= ((uint64_t)d[bit >> 5] >> (bit & 31)) & 1ull;
     }
+    bool sticky = false;
     for (int j = 0; j < NLIMB && !sticky; j++) {
       int lo_bit = j * 32, hi_bit = j * 32 + 31;
       if (hi_bit <= msb - 64) sticky = d[j] != 0;
@@ -222,8 +280,8 @@ struct XAcc {
         sticky = ((uint64_t)d[j] & mask) != 0;
       }
     }
-    uint64_t mant = win >> 11;              // 53 bits
-    uint64_t rest = win & 0x7FFull;         // 11 bits below
+    uint64_t mant = win >> 11;
+    uint64_t rest = win & 0x7FFull;
     bool round = (rest >> 10) & 1;
     bool st = sticky || (rest & 0x3FF);
     if (round && (st || (mant & 1))) mant++;
@@ -232,373 +290,543 @@ struct XAcc {
   }
 };
 
-// sign(a1/g1 - a2/g2) for exact pairs a = hi + lo >= 0 and g >= 0, where
-// g = 0 with a > 0 means +inf and a = 0 means 0.
-__device__ int cmp_rel(double h1, double l1, double g1, double h2, double l2, double g2) {
-  int k1 = h1 == 0.0 ? 0 : (g1 == 0.0 ? 2 : 1);
-  int k2 = h2 == 0.0 ? 0 : (g2 == 0.0 ? 2 : 1);
-  if (k1 != k2) return k1 > k2 ? 1 : -1;
-  if (k1 != 1) return 0;
-  XAcc x;
-  x.zero();
-  x.add_prod(h1, g2);
-  x.add_prod(l1, g2);
-  x.add_prod(h2, g1, true);
-  x.add_prod(l2, g1, true);
-  x.normalize();
-  return x.sign();
+// ---------------------------------------------------------------------------
+// exact magnitudes as float32 pairs
+// ---------------------------------------------------------------------------
+// |d| is carried as (hi + lo) * 2^sc with hi = RN32(|d| 2^-sc), |lo| <= half a
+// step of hi, sc in {0, 1} (sc = 1 only when |d| exceeds the float32 range).
+
+__device__ __forceinline__ void two_sum_f(float x, float y, float& s, float& t) {
+  s = __fadd_rn(x, y);
+  float yv = __fsub_rn(s, x);
+  float xv = __fsub_rn(s, yv);
+  t = __fadd_rn(__fsub_rn(x, xv), __fsub_rn(y, yv));
 }
 
-// sign(pair - y) for a normalised binary64 pair and a double
-__device__ __forceinline__ int cmp_pair_dbl(double hi, double lo, double y) {
-  if (hi != y) return hi > y ? 1 : -1;
-  return lo > 0 ? 1 : (lo < 0 ? -1 : 0);
-}
-__device__ __forceinline__ int cmp_pair(double h1, double l1, double h2, double l2) {
+// sign(x - y) for two exact pair magnitudes
+__device__ __forceinline__ int cmp_mag(float h1, float l1, int s1, float h2, float l2, int s2) {
+  if (s1 != s2) return s1 > s2 ? 1 : -1;  // scaled values exceed every unscaled float32
   if (h1 != h2) return h1 > h2 ? 1 : -1;
   return l1 > l2 ? 1 : (l1 < l2 ? -1 : 0);
 }
 
-// float32 lower bound of a nonnegative pair value
-__device__ __forceinline__ float pair_to_f32_rd(double hi, double lo) {
-  float f = __double2float_rd(hi);
-  if ((double)f == hi && lo < 0) f = nextafterf(f, 0.0f);
-  return f;
+// sign(a1/g1 - a2/g2), a = (hi + lo) 2^sc >= 0, g >= 0; g = 0 < a means +inf
+__device__ int cmp_rel_exact(float h1, float l1, int s1, float g1, float h2, float l2, int s2, float g2) {
+  int k1 = h1 == 0.0f ? 0 : (g1 == 0.0f ? 2 : 1);
+  int k2 = h2 == 0.0f ? 0 : (g2 == 0.0f ? 2 : 1);
+  if (k1 != k2) return k1 > k2 ? 1 : -1;
+  if (k1 != 1) return 0;
+  XAcc x;
+  x.zero();
+  x.add_prod_f(h1, g2, false, s1);
+  x.add_prod_f(l1, g2, false, s1);
+  x.add_prod_f(h2, g1, true, s2);
+  x.add_prod_f(l2, g1, true, s2);
+  x.normalize();
+  return x.sign();
+}
+
+// sign(a1/g1 - a2/g2) for positive normal float32 values (a2 may be 0):
+// compares the 48-bit products of the significands.
+__device__ __forceinline__ int cmp_ratio_f(float a1, float g1, float a2, float g2) {
+  if (a2 == 0.0f) return 1;
+  uint32_t b1 = __float_as_uint(a1), c1 = __float_as_uint(g1), b2 = __float_as_uint(a2), c2 = __float_as_uint(g2);
+  uint64_t P1 = (uint64_t)((b1 & 0x7FFFFFu) | 0x800000u) * ((c2 & 0x7FFFFFu) | 0x800000u);
+  uint64_t P2 = (uint64_t)((b2 & 0x7FFFFFu) | 0x800000u) * ((c1 & 0x7FFFFFu) | 0x800000u);
+  int x1 = (int)(b1 >> 23) + (int)(c2 >> 23), x2 = (int)(b2 >> 23) + (int)(c1 >> 23);
+  if (x1 > x2 + 1) return 1;
+  if (x2 > x1 + 1) return -1;
+  if (x1 > x2) P1 <<= 1;
+  else if (x2 > x1) P2 <<= 1;
+  return P1 > P2 ? 1 : (P1 < P2 ? -1 : 0);
+}
+
+// float32 filter for a rel best: a value <= rel with a margin for the
+// approximate per-lane ratio a * rcp(|g|)
+__device__ __forceinline__ float rel_filter(float hi, int sc, float g) {
+  if (g == 0.0f) return __int_as_float(0x7F800000);
+  float q = __fdiv_rd(hi, g);
+  if (sc) q = __fmul_rd(q, 2.0f);
+  return __fmul_rd(q, 0.99999809265136719f);  // 1 - 2^-19
 }
 
 // ---------------------------------------------------------------------------
 // shared memory
 // ---------------------------------------------------------------------------
-struct Smem {
+// Per-thread state touched only on the rare paths: the general-path counters
+// and the exact maxima records.
+struct Cold {
+  float abs_hi, abs_lo;
+  float rel_hi, rel_lo, rel_g;
+  float rel_f;  // filter of the rel best
+  uint32_t ulp;
+  uint32_t n_gw, n_gm, n_ga, n_gf, n_nf, n_geq;
+  int abs_sc, rel_sc;
+  uint32_t pad;
+  long long abs_idx, rel_idx, ulp_idx;
+};
+
+// Per-warp staging ring for the bulk copies: NSTAGE stages, each one warp
+// tile of CHV 16-byte vectors of each tensor (two vectors per lane).
+constexpr int NW = BLOCK / 32;
+constexpr int NSTAGE = 3;
+constexpr int CHV = 64;
+
+struct __align__(128) Smem {
+  uint4 ring_g[NW][NSTAGE][CHV];
+  uint4 ring_c[NW][NSTAGE][CHV];
+  unsigned long long bar[NW][NSTAGE];
   unsigned long long hist[HBINS];
   unsigned long long sacc[NSUM][NLIMB];
   unsigned long long cnt[8];
-  MaxAbs wabs[BLOCK / 32];
-  MaxRel wrel[BLOCK / 32];
-  MaxUlp wulp[BLOCK / 32];
-  long long wff[BLOCK / 32], wfu[BLOCK / 32];
+  Partial wbest[NW];
   int lb;
+  uint32_t ovf[64];               // ULP bins NU+1..63 of window lanes (CTA-wide)
+  Cold cold[BLOCK];
   uint32_t priv[NPB_MAX * HALF];  // per-thread 16-bit counters, two threads per word
+  unsigned short qp[NW][CHV * 8]; // per-warp queue: tile positions of the unequal lanes
 };
 
 __device__ __forceinline__ void sacc_add(Smem& sm, int which, unsigned __int128 m, int e, bool neg) {
-  for_digits(m, e, neg, [&](int j, int64_t v) {
-    atomicAdd(&sm.sacc[which][j], (unsigned long long)v);
-  });
+  for_digits(m, e, neg, [&](int j, int64_t v) { atomicAdd(&sm.sacc[which][j], (unsigned long long)v); });
 }
-__device__ __forceinline__ void sacc_add_double(Smem& sm, int which, double x) {
-  if (x == 0.0) return;
+__device__ __forceinline__ void sacc_add_f(Smem& sm, int which, float x, bool neg, int sc) {
+  if (x == 0.0f) return;
   int e;
-  uint64_t m = split_double(x, e);
-  sacc_add(sm, which, m, e, x < 0);
+  uint32_t m = split_float(x, e);
+  sacc_add(sm, which, m, e + sc, neg ^ (x < 0));
 }
-__device__ __forceinline__ void sacc_add_prod(Smem& sm, int which, double x, double y) {
-  if (x == 0.0 || y == 0.0) return;
+__device__ __forceinline__ void sacc_add_prod_f(Smem& sm, int which, float x, float y, int sc) {
+  if (x == 0.0f || y == 0.0f) return;
   int ex, ey;
-  uint64_t mx = split_double(x, ex), my = split_double(y, ey);
-  sacc_add(sm, which, (unsigned __int128)mx * my, ex + ey, (x < 0) ^ (y < 0));
+  uint32_t mx = split_float(x, ex), my = split_float(y, ey);
+  sacc_add(sm, which, (unsigned __int128)((uint64_t)mx * my), ex + ey + sc, (x < 0) ^ (y < 0));
 }
 
 // ---------------------------------------------------------------------------
-// per-thread state
+// per-thread hot state (registers)
 // ---------------------------------------------------------------------------
 struct Ctx {
+  Cold* cold;         // this thread's rare-path record
   float rtol, atol;
   uint32_t lb_shift;  // Lb << MB
-  uint32_t win_span;  // (SHMAX + 1) << MB
+  uint32_t c0;        // 158 + Lexp: V = ((bits(|d|) << 8) | 2^31) >> (c0 - exponent(|d|))
   uint32_t col, inc;  // private histogram column and increment
 };
 
-struct LaneState {
-  uint32_t n_eq, n_simple, n_within, n_nonfinite;
-  uint32_t n_gw, n_gm, n_ga, n_gf;  // general path: within, mismatch, asym, flip
+struct Hot {
+  uint32_t n_eq, n_win, n_within;
   uint64_t P, N, Q;
-  uint32_t Qh;
-  float abs_f, rel_f;
+  float abs_f;         // best |d|: exact when abs_x, else a lower bound
+  float rel_f;         // filter: <= best rel
+  float rel_a, rel_g;  // best rel = rel_a / rel_g exactly when rel_x
   uint32_t ulp_f;
-  MaxAbs mabs;
-  MaxRel mrel;
-  int64_t ulp_idx;
+  bool abs_x, rel_x;
   int64_t first_fin, first_ulp;
 };
 
-__device__ __forceinline__ void state_init(LaneState& st) {
-  st.n_eq = st.n_simple = st.n_within = st.n_nonfinite = 0;
-  st.n_gw = st.n_gm = st.n_ga = st.n_gf = 0;
-  st.P = st.N = st.Q = 0;
-  st.Qh = 0;
-  st.abs_f = 0.0f;
-  st.rel_f = 0.0f;
-  st.ulp_f = 0;
-  st.mabs = MaxAbs{0.0, 0.0, -1};
-  st.mrel = MaxRel{0.0, 0.0, 1.0, -1};
-  st.ulp_idx = -1;
-  st.first_fin = st.first_ulp = -1;
+__device__ __forceinline__ void hot_init(Hot& h) {
+  h.n_eq = h.n_win = h.n_within = 0;
+  h.P = h.N = h.Q = 0;
+  h.abs_f = 0.0f;
+  h.rel_f = 0.0f;
+  h.rel_a = 0.0f;
+  h.rel_g = 1.0f;
+  h.ulp_f = 0;
+  h.abs_x = h.rel_x = true;
+  h.first_fin = h.first_ulp = -1;
+}
+
+__device__ __forceinline__ void cold_init(Cold& c) {
+  c.abs_hi = c.abs_lo = 0.0f;
+  c.rel_hi = c.rel_lo = 0.0f;
+  c.rel_g = 1.0f;
+  c.rel_f = 0.0f;
+  c.ulp = 0;
+  c.n_gw = c.n_gm = c.n_ga = c.n_gf = c.n_nf = c.n_geq = 0;
+  c.abs_sc = c.rel_sc = 0;
+  c.abs_idx = c.rel_idx = c.ulp_idx = -1;
+}
+
+// after the general path ran, refresh the hot copies from the cold records
+__device__ __forceinline__ void hot_reload(Hot& h, const Cold& c) {
+  h.abs_x = c.abs_lo == 0.0f && c.abs_sc == 0;
+  h.abs_f = (c.abs_lo < 0.0f && c.abs_sc == 0) ? nextafterf(c.abs_hi, 0.0f) : c.abs_hi;
+  // the integer ratio compare needs normal float32 operands
+  h.rel_x = c.rel_lo == 0.0f && c.rel_sc == 0 &&
+            (c.rel_idx < 0 || (c.rel_g >= 1.17549435e-38f && c.rel_hi >= 1.17549435e-38f));
+  h.rel_a = c.rel_hi;
+  h.rel_g = c.rel_g;
+  h.rel_f = c.rel_f;
+  h.ulp_f = c.ulp;
 }
 
 template <int DT>
-__device__ __forceinline__ void note_first(LaneState& st, uint32_t G, uint32_t C, int64_t idx) {
+__device__ __forceinline__ void note_first(Hot& h, uint32_t G, uint32_t C, int64_t idx) {
   using T = Tr<DT>;
   uint32_t ag = G & T::MAG, ac = C & T::MAG;
-  if (st.first_fin < 0 && ag < T::INF && ac < T::INF) st.first_fin = idx;
-  if (st.first_ulp < 0 && ag <= T::INF && ac <= T::INF) st.first_ulp = idx;
+  if (h.first_fin < 0 && ag < T::INF && ac < T::INF) h.first_fin = idx;
+  if (h.first_ulp < 0 && ag <= T::INF && ac <= T::INF) h.first_ulp = idx;
 }
 
-// rel filter value for a new best: RD(rel) * (1 - 2^-20)
-__device__ __forceinline__ float rel_filter(double hi, double lo, double g) {
-  if (g == 0.0) return __int_as_float(0x7F800000);
-  double q = __ddiv_rd(hi, g);
-  (void)lo;
-  return __fmul_rd(__double2float_rd(q), 0.99999904632568359375f);
-}
-
-// Exact update of the maxima for a window lane (index order: idx is larger
-// than every index seen so far by this thread).
-template <int DT>
-__device__ __noinline__ LaneState window_candidate(LaneState st, uint32_t G, uint32_t C, int64_t idx) {
-  using T = Tr<DT>;
-  float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
-  float a = fabsf(__fsub_rn(cf, gf)), ag = fabsf(gf);
-  uint32_t u = (uint32_t)abs((int32_t)C - (int32_t)G);
-  if (a > st.abs_f) {
-    double ad = (double)a;
-    bool gt = st.mabs.idx < 0 || cmp_pair_dbl(st.mabs.hi, st.mabs.lo, ad) < 0;
+// Exact maxima update for a window lane; idx exceeds every index this thread
+// has seen, so ties keep the current best.
+__device__ __forceinline__ void window_update(Hot& h, Cold& cd, float a, float ag, uint32_t u, int64_t idx) {
+  if (a > h.abs_f) {
+    bool gt = h.abs_x || cmp_mag(a, 0.0f, 0, cd.abs_hi, cd.abs_lo, cd.abs_sc) > 0;
     if (gt) {
-      st.mabs = MaxAbs{ad, 0.0, idx};
-      st.abs_f = a;
+      cd.abs_hi = a;
+      cd.abs_lo = 0.0f;
+      cd.abs_sc = 0;
+      cd.abs_idx = idx;
+      h.abs_f = a;
+      h.abs_x = true;
     }
   }
-  if (u > st.ulp_f) {
-    st.ulp_f = u;
-    st.ulp_idx = idx;
+  if (u > h.ulp_f) {
+    h.ulp_f = u;
+    cd.ulp = u;
+    cd.ulp_idx = idx;
   }
   float r = __fmul_rn(a, rcp_approx(ag));
-  if (r > st.rel_f) {
-    bool gt = st.mrel.idx < 0 || cmp_rel((double)a, 0.0, (double)ag, st.mrel.hi, st.mrel.lo, st.mrel.g) > 0;
-    if (gt) {
-      st.mrel = MaxRel{(double)a, 0.0, (double)ag, idx};
-      st.rel_f = rel_filter((double)a, 0.0, (double)ag);
+  if (r > h.rel_f) {
+    int c = h.rel_x ? cmp_ratio_f(a, ag, h.rel_a, h.rel_g)
+                    : cmp_rel_exact(a, 0.0f, 0, ag, cd.rel_hi, cd.rel_lo, cd.rel_sc, cd.rel_g);
+    if (c > 0) {
+      cd.rel_hi = a;
+      cd.rel_lo = 0.0f;
+      cd.rel_sc = 0;
+      cd.rel_g = ag;
+      cd.rel_idx = idx;
+      h.rel_a = a;
+      h.rel_g = ag;
+      h.rel_x = true;
+      h.rel_f = rel_filter(a, 0, ag);
+      cd.rel_f = h.rel_f;
     }
   }
-  (void)T::MB;
-  return st;
 }
 
-// The general path: the definitions evaluated exactly, any pair.
+// floor(log2(a / g)) for a = (hi + lo) 2^sc > 0 and g > 0 (float32 pair, any range)
+__device__ int log2_ratio(float hi, float lo, int sc, float g) {
+  float hs = hi, gs = g;
+  if (hs < 1.17549435e-38f || gs < 1.17549435e-38f) {  // scale subnormals by 2^64
+    if (hs >= 1.8446744e19f) return 200;              // ratio far above the clamp
+    if (gs >= 1.8446744e19f) return -200;
+    hs = __fmul_rn(hs, 1.8446744e19f);
+    gs = __fmul_rn(gs, 1.8446744e19f);
+  }
+  uint32_t bh = __float_as_uint(hs), bg = __float_as_uint(gs);
+  int k = ((int)(bh - bg)) >> 23;
+  if (lo < 0.0f && (bh & 0x7FFFFFu) == (bg & 0x7FFFFFu)) k--;  // a just below 2^k g
+  return k + sc;
+}
+
+// The general path: the definitions evaluated exactly, for any pair.
 template <int DT>
-__device__ __noinline__ LaneState general_lane(LaneState st, uint32_t G, uint32_t C, int64_t idx, float rtol,
-                                               float atol, Smem& sm) {
+__device__ __noinline__ void general_lane(Smem& sm, Cold& cd, uint32_t G, uint32_t C, int64_t idx, float rtol,
+                                          float atol) {
   using T = Tr<DT>;
-  uint32_t ag = G & T::MAG, ac = C & T::MAG;
-  bool gnan = ag > T::INF, cnan = ac > T::INF, ginf = ag == T::INF, cinf = ac == T::INF;
+  uint32_t ag_m = G & T::MAG, ac_m = C & T::MAG;
+  bool gnan = ag_m > T::INF, cnan = ac_m > T::INF, ginf = ag_m == T::INF, cinf = ac_m == T::INF;
   bool gs = (G & T::SIGN) != 0, cs = (C & T::SIGN) != 0;
-  int64_t kg = gs ? -(int64_t)ag : (int64_t)ag, kc = cs ? -(int64_t)ac : (int64_t)ac;
+  int64_t kg = gs ? -(int64_t)ag_m : (int64_t)ag_m, kc = cs ? -(int64_t)ac_m : (int64_t)ac_m;
   uint64_t u = (uint64_t)(kc > kg ? kc - kg : kg - kc);
   bool ulpdef = !gnan && !cnan;
+  if (ulpdef && u > 0 && (u > cd.ulp || (u == cd.ulp && idx < cd.ulp_idx))) {
+    cd.ulp = (uint32_t)u;
+    cd.ulp_idx = idx;
+  }
   if (gnan || cnan || ginf || cinf) {
-    st.n_nonfinite++;
+    cd.n_nf++;
     bool equal = (gnan && cnan) || (ginf && cinf && gs == cs);
     if (equal) {
-      st.n_eq++;
-      return st;
+      cd.n_geq++;
+      return;
     }
-    st.n_ga++;
+    cd.n_ga++;
     atomicAdd(&sm.hist[63], 1ull);
     atomicAdd(&sm.hist[64 + (ulpdef ? (u < 63 ? (int)u : 63) : 63)], 1ull);
-    if (ulpdef && u > 0) {
-      if (u > st.ulp_f || (u == st.ulp_f && idx < st.ulp_idx)) {
-        st.ulp_f = (uint32_t)u;
-        st.ulp_idx = idx;
-      }
-    }
-    return st;
+    return;
   }
-  double gv = (double)to_f32<DT>(G), cv = (double)to_f32<DT>(C);
-  double s, t;
-  two_sum(cv, -gv, s, t);
-  double ahi = fabs(s), alo = s < 0 ? -t : t;
-  double absg = fabs(gv);
-  if (ahi == 0.0) {  // numerically equal (e.g. +0 and -0)
-    st.n_eq++;
-    return st;
+  float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
+  if (gf == cf) {  // +0 and -0
+    cd.n_geq++;
+    return;
   }
-  // tolerance: a <= atol + rtol*|g|, exactly (rtol*|g| is exact in binary64)
-  double P = (double)rtol * absg, Tt, tt;
-  two_sum((double)atol, P, Tt, tt);
-  int cls;
-  if (cmp_pair(ahi, alo, Tt, tt) <= 0) cls = PEAT_WITHIN_TOL;
-  else if (gv != 0.0 && cv != 0.0 && gs != cs) cls = PEAT_SIGN_FLIP;
-  else cls = PEAT_MISMATCH;
-  if (cls == PEAT_WITHIN_TOL) st.n_gw++;
-  else if (cls == PEAT_SIGN_FLIP) st.n_gf++;
-  else st.n_gm++;
-  // log2-relative bin
+  float s, t;
+  int sc = 0;
+  two_sum_f(cf, -gf, s, t);
+  if (!(fabsf(s) < __int_as_float(0x7F800000))) {  // |d| above the float32 range: halve exactly
+    two_sum_f(__fmul_rn(cf, 0.5f), __fmul_rn(-gf, 0.5f), s, t);
+    sc = 1;
+  }
+  float hi = fabsf(s), lo = s < 0.0f ? -t : t;
+  float ag = fabsf(gf);
+  // WITHIN_TOL: a <= atol + rtol |g|, decided in float32 when clear, exactly otherwise
+  bool within;
+  float thr = __fmaf_rn(rtol, ag, atol);
+  if (sc == 0 && hi >= 1e-30f && thr >= 1e-30f && __fmul_rn(hi, 1.0000005f) < __fmul_rn(thr, 0.9999995f)) {
+    within = true;
+  } else if (sc == 0 && hi >= 1e-30f && __fmul_rn(hi, 0.9999995f) > __fmul_rn(thr, 1.0000005f)) {
+    within = false;
+  } else {
+    XAcc x;
+    x.zero();
+    x.add_f(hi, false, sc);
+    x.add_f(lo, false, sc);
+    x.add_f(atol, true);
+    x.add_prod_f(rtol, ag, true);
+    x.normalize();
+    within = x.sign() <= 0;
+  }
+  if (within) cd.n_gw++;
+  else if (gf != 0.0f && cf != 0.0f && gs != cs) cd.n_gf++;
+  else cd.n_gm++;
+  // log2-relative bin and ULP bin
   int rb;
-  if (absg == 0.0) {
+  if (ag == 0.0f) {
     rb = 63;
   } else {
-    int k = ilogb(ahi) - ilogb(absg);
-    while (cmp_pair_dbl(ahi, alo, ldexp(absg, k)) < 0) k--;
-    while (cmp_pair_dbl(ahi, alo, ldexp(absg, k + 1)) >= 0) k++;
-    k += 48;
+    int k = log2_ratio(hi, lo, sc, ag) + 48;
     rb = k < 1 ? 1 : (k > 62 ? 62 : k);
   }
   atomicAdd(&sm.hist[rb], 1ull);
   atomicAdd(&sm.hist[64 + (u < 63 ? (int)u : 63)], 1ull);
   // maxima, full (value, index) order
   {
-    int c = st.mabs.idx < 0 ? 1 : cmp_pair(ahi, alo, st.mabs.hi, st.mabs.lo);
-    if (c > 0 || (c == 0 && idx < st.mabs.idx)) {
-      st.mabs = MaxAbs{ahi, alo, idx};
-      st.abs_f = pair_to_f32_rd(ahi, alo);
+    int c = cd.abs_idx < 0 ? 1 : cmp_mag(hi, lo, sc, cd.abs_hi, cd.abs_lo, cd.abs_sc);
+    if (c > 0 || (c == 0 && idx < cd.abs_idx)) {
+      cd.abs_hi = hi;
+      cd.abs_lo = lo;
+      cd.abs_sc = sc;
+      cd.abs_idx = idx;
     }
   }
   {
-    int c = st.mrel.idx < 0 ? 1 : cmp_rel(ahi, alo, absg, st.mrel.hi, st.mrel.lo, st.mrel.g);
-    if (c > 0 || (c == 0 && idx < st.mrel.idx)) {
-      st.mrel = MaxRel{ahi, alo, absg, idx};
-      st.rel_f = rel_filter(ahi, alo, absg);
-    }
-  }
-  if (u > 0 && (u > st.ulp_f || (u == st.ulp_f && idx < st.ulp_idx))) {
-    st.ulp_f = (uint32_t)u;
-    st.ulp_idx = idx;
-  }
-  // exact sums: d = s + t, |d| = ahi + alo, d^2 = s^2 + 2st + t^2
-  sacc_add_double(sm, 0, s);
-  sacc_add_double(sm, 0, t);
-  sacc_add_double(sm, 1, ahi);
-  sacc_add_double(sm, 1, alo);
-  sacc_add_prod(sm, 2, s, s);
-  sacc_add_prod(sm, 2, s, t);
-  sacc_add_prod(sm, 2, s, t);
-  sacc_add_prod(sm, 2, t, t);
-  return st;
-}
-
-// One lane of the fast path.  Returns via bit masks which lanes need the
-// general path (gen) or an exact maxima check (cand).
-template <int DT>
-__device__ __forceinline__ void window_lane(LaneState& st, uint32_t G, uint32_t C, int j, const Ctx& cx,
-                                            Smem& sm, uint32_t& gen, uint32_t& cand) {
-  using T = Tr<DT>;
-  uint32_t ag = G & T::MAG;
-  bool eq = G == C;
-  bool eqf = eq && ag < T::INF;
-  uint32_t rel_e = ag - cx.lb_shift;
-  bool inwin = rel_e < cx.win_span;
-  bool sse = ((G ^ C) & T::SE) == 0;
-  int32_t delta = (int32_t)C - (int32_t)G;
-  uint32_t u = (uint32_t)abs(delta);
-  bool simple = !eq && sse && inwin;
-  if constexpr (T::UB < T::MB) simple = simple && u < (1u << T::UB);
-  float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
-  float s = __fsub_rn(cf, gf);
-  float a = fabsf(s), agf = fabsf(gf);
-  float thr = __fmaf_rn(cx.rtol, agf, cx.atol);
-  bool within = a < thr;
-  bool tie = a == thr;
-  st.n_eq += eqf ? 1u : 0u;
-  bool go = simple && !tie;
-  if (!go && !eqf) gen |= 1u << j;
-  if (go) {
-    st.n_simple++;
-    st.n_within += within ? 1u : 0u;
-    int k = (int)(__float_as_uint(a) - __float_as_uint(agf)) >> 23;  // floor(log2(a/|g|))
-    uint32_t ub = u < 63u ? u : 63u;
-    atomicAdd(&sm.priv[(ub - 1) * HALF + cx.col], cx.inc);
-    atomicAdd(&sm.priv[(63 + k + T::MB + 1) * HALF + cx.col], cx.inc);
-    uint32_t sh = rel_e >> T::MB;
-    uint32_t V = u << sh;
-    if (s > 0.0f) st.P += V;
-    else st.N += V;
-    uint64_t v2 = (uint64_t)V * V;
-    uint64_t q = st.Q + v2;
-    st.Qh += q < st.Q ? 1u : 0u;
-    st.Q = q;
-    float r = __fmul_rn(a, rcp_approx(agf));
-    if ((a > st.abs_f) | (u > st.ulp_f) | (r > st.rel_f)) cand |= 1u << j;
-  }
-}
-
-template <int DT>
-__device__ __forceinline__ uint32_t nonfinite_count(const uint4& v) {
-  using T = Tr<DT>;
-  uint32_t n = 0;
-#pragma unroll
-  for (int j = 0; j < T::VEC; j++) n += (lane_bits<DT>(v, j) & T::MAG) >= T::INF ? 1u : 0u;
-  return n;
-}
-
-template <int DT>
-__device__ __forceinline__ void do_vector(LaneState& st, const uint4& gv, const uint4& cv, int64_t base,
-                                          const Ctx& cx, Smem& sm) {
-  using T = Tr<DT>;
-  bool alleq = (gv.x == cv.x) & (gv.y == cv.y) & (gv.z == cv.z) & (gv.w == cv.w);
-  if ((st.first_fin | st.first_ulp) < 0) {
-#pragma unroll
-    for (int j = 0; j < T::VEC; j++) note_first<DT>(st, lane_bits<DT>(gv, j), lane_bits<DT>(cv, j), base + j);
-  }
-  if (alleq) {
-    st.n_eq += T::VEC;
-    uint32_t nf = nonfinite_count<DT>(gv);
-    st.n_eq -= nf;              // non-finite equal lanes are counted by the general path
-    if (nf) {
-#pragma unroll
-      for (int j = 0; j < T::VEC; j++) {
-        uint32_t G = lane_bits<DT>(gv, j);
-        if ((G & T::MAG) >= T::INF) st = general_lane<DT>(st, G, G, base + j, cx.rtol, cx.atol, sm);
+    bool maybe = cd.rel_idx < 0 || ag == 0.0f || sc ||
+                 __fmul_rn(__fmul_rn(hi, rcp_approx(ag)), 1.00001f) >= cd.rel_f;
+    if (maybe) {
+      int c = cd.rel_idx < 0 ? 1 : cmp_rel_exact(hi, lo, sc, ag, cd.rel_hi, cd.rel_lo, cd.rel_sc, cd.rel_g);
+      if (c > 0 || (c == 0 && idx < cd.rel_idx)) {
+        cd.rel_hi = hi;
+        cd.rel_lo = lo;
+        cd.rel_sc = sc;
+        cd.rel_g = ag;
+        cd.rel_idx = idx;
+        cd.rel_f = rel_filter(hi, sc, ag);
       }
     }
+  }
+  // exact sums: d = (s + t) 2^sc, |d| = (hi + lo) 2^sc, d^2 = (s^2 + 2st + t^2) 4^sc
+  sacc_add_f(sm, 0, s, false, sc);
+  sacc_add_f(sm, 0, t, false, sc);
+  sacc_add_f(sm, 1, hi, false, sc);
+  sacc_add_f(sm, 1, lo, false, sc);
+  sacc_add_prod_f(sm, 2, s, s, 2 * sc);
+  sacc_add_prod_f(sm, 2, s, t, 2 * sc + 1);
+  sacc_add_prod_f(sm, 2, t, t, 2 * sc);
+}
+
+template <int DT>
+__device__ __forceinline__ void window_cand(Hot& h, Cold& cd, uint32_t G, uint32_t C, int64_t idx) {
+  float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
+  float a = fabsf(__fsub_rn(cf, gf)), ag = fabsf(gf);
+  uint32_t u = (uint32_t)abs((int32_t)C - (int32_t)G);
+  window_update(h, cd, a, ag, u, idx);
+}
+
+// bitmask of the lanes of a vector whose value is NaN or Inf
+template <int DT>
+__device__ __forceinline__ uint32_t nonfinite_mask(const uint4& v) {
+  using T = Tr<DT>;
+  if constexpr (T::BYTES == 2) {
+    constexpr uint32_t ADD = (0x8000u - T::INF) * 0x10001u;  // sets bit 15 of a half iff mag >= INF
+    uint32_t any = (((v.x & 0x7FFF7FFFu) + ADD) | ((v.y & 0x7FFF7FFFu) + ADD) | ((v.z & 0x7FFF7FFFu) + ADD) |
+                    ((v.w & 0x7FFF7FFFu) + ADD)) & 0x80008000u;
+    if (!any) return 0;
+  }
+  uint32_t m = 0;
+#pragma unroll
+  for (int j = 0; j < T::VEC; j++) m |= ((lane_bits<DT>(v, j) & T::MAG) >= T::INF ? 1u : 0u) << j;
+  return m;
+}
+
+// One unequal lane: the window fast path, or the general path.
+template <int DT>
+__device__ __forceinline__ void lane_proc(Hot& h, uint32_t G, uint32_t C, int64_t idx, const Ctx& cx, Smem& sm) {
+  using T = Tr<DT>;
+  const uint32_t ag = G & T::MAG, ac = C & T::MAG;
+  const uint32_t u = (uint32_t)abs((int32_t)C - (int32_t)G);  // ULP distance for same-sign pairs
+  uint32_t mg = ag, mc = ac;
+  if constexpr (DT == PEAT_F16) {  // subnormal steps equal binade 1's
+    mg = max(mg, 1u << T::MB);
+    mc = max(mc, 1u << T::MB);
+  }
+  bool ok = ((G ^ C) & T::SIGN) == 0 && u < (1u << T::UB) && ag != 0u && mg >= cx.lb_shift && mc >= cx.lb_shift;
+  const float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
+  const float s = __fsub_rn(cf, gf);
+  const float a = fabsf(s), agf = fabsf(gf);
+  const uint32_t ab = __float_as_uint(a);
+  const uint32_t sh = cx.c0 - (ab >> 23);
+  const float thr = __fmaf_rn(cx.rtol, agf, cx.atol);
+  ok = ok && (sh - 8u) <= 23u && a != thr;  // 1 <= V < 2^24; tolerance ties go to the general path
+  if (ok) {
+    h.n_win++;
+    h.n_within += a < thr ? 1u : 0u;
+    const int k = (int)(ab - __float_as_uint(agf)) >> 23;  // floor(log2(|d| / |g|))
+    uint32_t* uctr = u <= (uint32_t)NU ? &sm.priv[(u - 1) * HALF + cx.col] : &sm.ovf[u < 63u ? u : 63u];
+    atomicAdd(uctr, u <= (uint32_t)NU ? cx.inc : 1u);
+    atomicAdd(&sm.priv[(NU + k - Rows<DT>::KLO) * HALF + cx.col], cx.inc);
+    const uint32_t V = ((ab << 8) | 0x80000000u) >> sh;  // |d| / 2^Lexp, exact
+    if (s > 0.0f) h.P += V;
+    else h.N += V;
+    h.Q += (uint64_t)V * V;
+    if ((a > h.abs_f) | (u > h.ulp_f) | (__fmul_rn(a, rcp_approx(agf)) > h.rel_f))
+      window_update(h, *cx.cold, a, agf, u, idx);
+  } else {
+    Cold& cd = *cx.cold;
+    general_lane<DT>(sm, cd, G, C, idx, cx.rtol, cx.atol);
+    hot_reload(h, cd);
+  }
+}
+
+// lanes of one vector whose golden value is NaN or Inf, as a bitmask
+template <int DT>
+__device__ __forceinline__ uint32_t nonfinite_lanes(const uint4& v) {
+  using T = Tr<DT>;
+  uint32_t m = 0;
+#pragma unroll
+  for (int j = 0; j < T::VEC; j++) m |= ((lane_bits<DT>(v, j) & T::MAG) >= T::INF ? 1u : 0u) << j;
+  return m;
+}
+// any NaN/Inf among the lanes of one vector (cheap test)
+template <int DT>
+__device__ __forceinline__ bool any_nonfinite(const uint4& v) {
+  using T = Tr<DT>;
+  if constexpr (T::BYTES == 2) {
+    constexpr uint32_t ADD = (0x8000u - T::INF) * 0x10001u;  // sets bit 15 of a half iff its magnitude >= INF
+    return ((((v.x & 0x7FFF7FFFu) + ADD) | ((v.y & 0x7FFF7FFFu) + ADD) | ((v.z & 0x7FFF7FFFu) + ADD) |
+             ((v.w & 0x7FFF7FFFu) + ADD)) & 0x80008000u) != 0u;
+  } else {
+    uint32_t m = max(max(v.x & T::MAG, v.y & T::MAG), max(v.z & T::MAG, v.w & T::MAG));
+    return m >= T::INF;
+  }
+}
+// bitmask of the lanes whose bit patterns differ
+template <int DT>
+__device__ __forceinline__ uint32_t unequal_mask(const uint4& g, const uint4& c) {
+  const uint32_t x[4] = {g.x ^ c.x, g.y ^ c.y, g.z ^ c.z, g.w ^ c.w};
+  uint32_t m = 0;
+  if constexpr (Tr<DT>::BYTES == 4) {
+#pragma unroll
+    for (int j = 0; j < 4; j++) m |= (x[j] != 0u ? 1u : 0u) << j;
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; j++) m |= ((x[j] & 0xFFFFu) != 0u ? 1u : 0u) << (2 * j) | (x[j] > 0xFFFFu ? 2u : 0u) << (2 * j);
+  }
+  return m;
+}
+
+// Equal lanes of one vector: every bitwise-equal pair is EXACT; the ones
+// holding NaN/Inf also count as non-finite pairs.
+template <int DT>
+__device__ __forceinline__ void count_equal(Hot& h, const uint4& g, uint32_t eqm, int64_t base, Cold& cd) {
+  h.n_eq += __popc(eqm);
+  if (eqm && any_nonfinite<DT>(g)) {
+    const uint32_t nf = nonfinite_lanes<DT>(g) & eqm;
+    cd.n_nf += __popc(nf);
+  }
+  (void)base;
+}
+
+// One warp tile of CHV vectors staged in shared memory: lane L owns vectors L
+// and L + 32.  Equal lanes are counted in place; unequal lanes are queued (in
+// element order) and processed 32 at a time, so every thread does useful work.
+template <int DT>
+__device__ __forceinline__ void do_tile(Hot& h, const uint4* gt, const uint4* ct, int nvalid, int64_t tile_base,
+                                        const Ctx& cx, Smem& sm) {
+  using T = Tr<DT>;
+  constexpr int VEC = T::VEC;
+  constexpr uint32_t FULL = (1u << VEC) - 1u;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const bool okA = lane < nvalid, okB = lane + 32 < nvalid;
+  const uint4 z = make_uint4(0, 0, 0, 0);
+  const uint4 gA = okA ? gt[lane] : z, cA = okA ? ct[lane] : z;
+  const uint4 gB = okB ? gt[lane + 32] : z, cB = okB ? ct[lane + 32] : z;
+  const int64_t baseA = tile_base + (int64_t)lane * VEC, baseB = baseA + 32 * VEC;
+  if ((h.first_fin | h.first_ulp) < 0) {
+    if (okA)
+      for (int j = 0; j < VEC; j++) note_first<DT>(h, lane_bits<DT>(gA, j), lane_bits<DT>(cA, j), baseA + j);
+    if (okB)
+      for (int j = 0; j < VEC; j++) note_first<DT>(h, lane_bits<DT>(gB, j), lane_bits<DT>(cB, j), baseB + j);
+  }
+  const bool diff = ((gA.x ^ cA.x) | (gA.y ^ cA.y) | (gA.z ^ cA.z) | (gA.w ^ cA.w) | (gB.x ^ cB.x) | (gB.y ^ cB.y) |
+                     (gB.z ^ cB.z) | (gB.w ^ cB.w)) != 0u;
+  Cold& cd = *cx.cold;
+  if (!__any_sync(0xFFFFFFFFu, diff)) {  // the whole warp tile is bitwise equal
+    if (okA) count_equal<DT>(h, gA, FULL, baseA, cd);
+    if (okB) count_equal<DT>(h, gB, FULL, baseB, cd);
     return;
   }
-  uint32_t gen = 0, cand = 0;
+  const uint32_t nA = okA ? unequal_mask<DT>(gA, cA) : 0u, nB = okB ? unequal_mask<DT>(gB, cB) : 0u;
+  if (okA) count_equal<DT>(h, gA, FULL & ~nA, baseA, cd);
+  if (okB) count_equal<DT>(h, gB, FULL & ~nB, baseB, cd);
+  // one scan of the packed counts gives the A-queue and B-queue offsets
+  const uint32_t packed = __popc(nA) | (__popc(nB) << 16);
+  uint32_t incl = packed;
 #pragma unroll
-  for (int j = 0; j < T::VEC; j++)
-    window_lane<DT>(st, lane_bits<DT>(gv, j), lane_bits<DT>(cv, j), j, cx, sm, gen, cand);
-  while (cand) {
-    int j = __ffs(cand) - 1;
-    cand &= cand - 1;
-    st = window_candidate<DT>(st, lane_bits<DT>(gv, j), lane_bits<DT>(cv, j), base + j);
+  for (int o = 1; o < 32; o <<= 1) {
+    uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane >= o) incl += t;
   }
-  while (gen) {
-    int j = __ffs(gen) - 1;
-    gen &= gen - 1;
-    st = general_lane<DT>(st, lane_bits<DT>(gv, j), lane_bits<DT>(cv, j), base + j, cx.rtol, cx.atol, sm);
+  const uint32_t tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
+  const uint32_t totA = tot & 0xFFFFu, total = totA + (tot >> 16);
+  uint32_t posA = (incl & 0xFFFFu) - (packed & 0xFFFFu);
+  uint32_t posB = totA + (incl >> 16) - (packed >> 16);
+  unsigned short* q = sm.qp[warp];
+#pragma unroll
+  for (int j = 0; j < VEC; j++) {
+    if ((nA >> j) & 1u) q[posA++] = (unsigned short)(lane * VEC + j);
+    if ((nB >> j) & 1u) q[posB++] = (unsigned short)((lane + 32) * VEC + j);
   }
+  __syncwarp();
+  for (uint32_t e = lane; e < total; e += 32) {
+    const uint32_t pos = q[e];
+    uint32_t G, C;
+    if constexpr (T::BYTES == 2) {
+      G = reinterpret_cast<const unsigned short*>(gt)[pos];
+      C = reinterpret_cast<const unsigned short*>(ct)[pos];
+    } else {
+      G = reinterpret_cast<const uint32_t*>(gt)[pos];
+      C = reinterpret_cast<const uint32_t*>(ct)[pos];
+    }
+    lane_proc<DT>(h, G, C, tile_base + pos, cx, sm);
+  }
+  __syncwarp();
 }
 
+// one element outside the vector grid
 template <int DT>
-__device__ __forceinline__ void do_scalar(LaneState& st, uint32_t G, uint32_t C, int64_t idx, const Ctx& cx,
-                                          Smem& sm) {
-  if ((st.first_fin | st.first_ulp) < 0) note_first<DT>(st, G, C, idx);
-  uint32_t gen = 0, cand = 0;
-  window_lane<DT>(st, G, C, 0, cx, sm, gen, cand);
-  if (cand) st = window_candidate<DT>(st, G, C, idx);
-  if (gen) st = general_lane<DT>(st, G, C, idx, cx.rtol, cx.atol, sm);
+__device__ __forceinline__ void do_scalar(Hot& h, uint32_t G, uint32_t C, int64_t idx, const Ctx& cx, Smem& sm) {
+  using T = Tr<DT>;
+  if ((h.first_fin | h.first_ulp) < 0) note_first<DT>(h, G, C, idx);
+  if (G == C) {
+    h.n_eq++;
+    if ((G & T::MAG) >= T::INF) cx.cold->n_nf++;
+    return;
+  }
+  lane_proc<DT>(h, G, C, idx, cx, sm);
 }
 
 // ---------------------------------------------------------------------------
-// CTA ranges
+// CTA ranges: boundaries precomputed on the host
 // ---------------------------------------------------------------------------
-template <int DT>
-__host__ __device__ __forceinline__ int64_t cta_lo(int64_t b, const CompareParams& p) {
-  if (b <= 0) return 0;
-  if (b >= p.nctas) return p.n_total;
-  constexpr int VEC = Tr<DT>::VEC;
-  if (p.p0 < 0 || p.p0 >= p.n_total) return (p.n_total / p.nctas) * b + (p.n_total % p.nctas) * b / p.nctas;
-  int64_t nv = (p.n_total - p.p0) / VEC;
-  int64_t lo = p.p0 + ((nv / p.nctas) * b + (nv % p.nctas) * b / p.nctas) * VEC;
-  return lo < p.n_total ? lo : p.n_total;
-}
-
-// the CTA whose range holds element i (0 <= i < n_total)
-template <int DT>
-__device__ int cta_of(int64_t i, const CompareParams& p) {
+__device__ __forceinline__ int cta_of(int64_t i, const CompareParams& p) {
   int lo = 0, hi = p.nctas - 1;
   while (lo < hi) {
     int mid = (lo + hi + 1) >> 1;
-    if (cta_lo<DT>(mid, p) <= i) lo = mid;
+    if (p.bounds[mid] <= i) lo = mid;
     else hi = mid - 1;
   }
   return lo;
@@ -616,74 +844,113 @@ __device__ int64_t seg_of(int64_t i, const int64_t* off, int64_t nseg) {
 }
 
 // ---------------------------------------------------------------------------
-// reductions
+// merging maxima records
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ uint64_t shfl64(uint64_t v, int src) {
-  uint32_t lo = __shfl_sync(0xFFFFFFFFu, (uint32_t)v, src);
-  uint32_t hi = __shfl_sync(0xFFFFFFFFu, (uint32_t)(v >> 32), src);
-  return ((uint64_t)hi << 32) | lo;
-}
-__device__ __forceinline__ uint64_t warp_sum64(uint64_t v) {
-  for (int o = 16; o > 0; o >>= 1) {
-    uint32_t lo = __shfl_down_sync(0xFFFFFFFFu, (uint32_t)v, o);
-    uint32_t hi = __shfl_down_sync(0xFFFFFFFFu, (uint32_t)(v >> 32), o);
-    v += ((uint64_t)hi << 32) | lo;
-  }
-  return v;
-}
-__device__ __forceinline__ double shfl_d(double v, int o) {
-  return __longlong_as_double((long long)
-      ((uint64_t)__shfl_down_sync(0xFFFFFFFFu, (uint32_t)__double_as_longlong(v), o) |
-       ((uint64_t)__shfl_down_sync(0xFFFFFFFFu, (uint32_t)((uint64_t)__double_as_longlong(v) >> 32), o) << 32)));
-}
-__device__ __forceinline__ int64_t shfl_i64(int64_t v, int o) {
-  return (int64_t)((uint64_t)__shfl_down_sync(0xFFFFFFFFu, (uint32_t)v, o) |
-                   ((uint64_t)__shfl_down_sync(0xFFFFFFFFu, (uint32_t)((uint64_t)v >> 32), o) << 32));
+__device__ __forceinline__ void part_none(Partial& r) {
+  r.abs_hi = r.abs_lo = 0.0f;
+  r.abs_sc = r.pad0 = 0;
+  r.abs_idx = -1;
+  r.rel_hi = r.rel_lo = 0.0f;
+  r.rel_g = 1.0f;
+  r.rel_sc = 0;
+  r.rel_idx = -1;
+  r.ulp = 0;
+  r.ulp_idx = -1;
+  r.first_fin = r.first_ulp = -1;
 }
 
-__device__ __forceinline__ bool abs_better(const MaxAbs& x, const MaxAbs& y) {  // x beats y
-  if (x.idx < 0) return false;
-  if (y.idx < 0) return true;
-  int c = cmp_pair(x.hi, x.lo, y.hi, y.lo);
-  return c > 0 || (c == 0 && x.idx < y.idx);
-}
-__device__ __forceinline__ bool rel_better(const MaxRel& x, const MaxRel& y) {
-  if (x.idx < 0) return false;
-  if (y.idx < 0) return true;
-  int c = cmp_rel(x.hi, x.lo, x.g, y.hi, y.lo, y.g);
-  return c > 0 || (c == 0 && x.idx < y.idx);
-}
-__device__ __forceinline__ bool ulp_better(const MaxUlp& x, const MaxUlp& y) {
-  if (x.idx < 0) return false;
-  if (y.idx < 0) return true;
-  return x.u > y.u || (x.u == y.u && x.idx < y.idx);
-}
 __device__ __forceinline__ int64_t min_idx(int64_t a, int64_t b) {
   if (a < 0) return b;
   if (b < 0) return a;
   return a < b ? a : b;
 }
 
+__device__ int cmp_rel_rec(float h1, float l1, int s1, float g1, float h2, float l2, int s2, float g2) {
+  const float tiny = 1.17549435e-38f;
+  if (l1 == 0.0f && l2 == 0.0f && s1 == 0 && s2 == 0 && h1 >= tiny && h2 >= tiny && g1 >= tiny && g2 >= tiny)
+    return cmp_ratio_f(h1, g1, h2, g2);
+  return cmp_rel_exact(h1, l1, s1, g1, h2, l2, s2, g2);
+}
+
+// x <- the better of x and y, field by field; ties to the lower index
+__device__ void part_merge(Partial& x, const Partial& y) {
+  if (y.abs_idx >= 0) {
+    int c = x.abs_idx < 0 ? 1 : cmp_mag(y.abs_hi, y.abs_lo, y.abs_sc, x.abs_hi, x.abs_lo, x.abs_sc);
+    if (c > 0 || (c == 0 && y.abs_idx < x.abs_idx)) {
+      x.abs_hi = y.abs_hi;
+      x.abs_lo = y.abs_lo;
+      x.abs_sc = y.abs_sc;
+      x.abs_idx = y.abs_idx;
+    }
+  }
+  if (y.rel_idx >= 0) {
+    int c = x.rel_idx < 0 ? 1 : cmp_rel_rec(y.rel_hi, y.rel_lo, y.rel_sc, y.rel_g, x.rel_hi, x.rel_lo, x.rel_sc, x.rel_g);
+    if (c > 0 || (c == 0 && y.rel_idx < x.rel_idx)) {
+      x.rel_hi = y.rel_hi;
+      x.rel_lo = y.rel_lo;
+      x.rel_sc = y.rel_sc;
+      x.rel_g = y.rel_g;
+      x.rel_idx = y.rel_idx;
+    }
+  }
+  if (y.ulp_idx >= 0 && (x.ulp_idx < 0 || y.ulp > x.ulp || (y.ulp == x.ulp && y.ulp_idx < x.ulp_idx))) {
+    x.ulp = y.ulp;
+    x.ulp_idx = y.ulp_idx;
+  }
+  x.first_fin = min_idx(x.first_fin, y.first_fin);
+  x.first_ulp = min_idx(x.first_ulp, y.first_ulp);
+}
+
+__device__ __forceinline__ int64_t shfl_i64(int64_t v, int o) {
+  return (int64_t)((uint64_t)__shfl_down_sync(0xFFFFFFFFu, (uint32_t)v, o) |
+                   ((uint64_t)__shfl_down_sync(0xFFFFFFFFu, (uint32_t)((uint64_t)v >> 32), o) << 32));
+}
+__device__ __forceinline__ float shfl_f(float v, int o) { return __shfl_down_sync(0xFFFFFFFFu, v, o); }
+__device__ __forceinline__ int shfl_int(int v, int o) { return __shfl_down_sync(0xFFFFFFFFu, v, o); }
+
+// warp tournament; lane 0 ends with the warp's best
+__device__ void part_warp_reduce(Partial& x) {
+  const int lane = threadIdx.x & 31;
+  for (int o = 16; o > 0; o >>= 1) {
+    Partial y;
+    y.abs_hi = shfl_f(x.abs_hi, o);
+    y.abs_lo = shfl_f(x.abs_lo, o);
+    y.abs_sc = shfl_int(x.abs_sc, o);
+    y.abs_idx = shfl_i64(x.abs_idx, o);
+    y.rel_hi = shfl_f(x.rel_hi, o);
+    y.rel_lo = shfl_f(x.rel_lo, o);
+    y.rel_g = shfl_f(x.rel_g, o);
+    y.rel_sc = shfl_int(x.rel_sc, o);
+    y.rel_idx = shfl_i64(x.rel_idx, o);
+    y.ulp = (uint64_t)shfl_i64((int64_t)x.ulp, o);
+    y.ulp_idx = shfl_i64(x.ulp_idx, o);
+    y.first_fin = shfl_i64(x.first_fin, o);
+    y.first_ulp = shfl_i64(x.first_ulp, o);
+    if (lane + o < 32) part_merge(x, y);
+  }
+}
+
+__device__ __forceinline__ uint64_t warp_sum64(uint64_t v) {
+  for (int o = 16; o > 0; o >>= 1) v += (uint64_t)shfl_i64((int64_t)v, o);
+  return v;
+}
+
 // Fold the per-thread 16-bit histograms and the window sums into the CTA
-// totals.  All threads call it; ends with the private counters zeroed.
+// totals.  All threads call it; it ends with the private counters zeroed.
 template <int DT>
-__device__ void fold_round(LaneState& st, Smem& sm, int lb) {
-  using T = Tr<DT>;
-  constexpr int NPB = Win<DT>::NPB;
+__device__ void fold_round(Hot& h, Smem& sm, int lexp) {
+  constexpr int NPB = Rows<DT>::NPB;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  // window sums: P, N (< 2^48 per round), Q as 96 bits
-  uint64_t P = warp_sum64(st.P), N = warp_sum64(st.N);
-  uint64_t q0 = warp_sum64(st.Q & 0xFFFFFFFFull), q1 = warp_sum64(st.Q >> 32), q2 = warp_sum64(st.Qh);
+  // window sums: P, N < 2^40 and Q < 2^64 per thread per round; warp sums in 128 bits
+  uint64_t P = warp_sum64(h.P), N = warp_sum64(h.N);
+  uint64_t qlo = warp_sum64(h.Q & 0xFFFFFFFFull), qhi = warp_sum64(h.Q >> 32);
   if (lane == 0) {
-    const int lexp = lb - T::BIAS - T::MB;  // weight of V's bit 0
     if (P >= N) sacc_add(sm, 0, (unsigned __int128)(P - N), lexp, false);
     else sacc_add(sm, 0, (unsigned __int128)(N - P), lexp, true);
     sacc_add(sm, 1, (unsigned __int128)P + N, lexp, false);
-    unsigned __int128 Q = (unsigned __int128)q0 + ((unsigned __int128)q1 << 32) + ((unsigned __int128)q2 << 64);
-    sacc_add(sm, 2, Q, 2 * lexp, false);
+    sacc_add(sm, 2, (unsigned __int128)qlo + ((unsigned __int128)qhi << 32), 2 * lexp, false);
   }
-  st.P = st.N = st.Q = 0;
-  st.Qh = 0;
+  h.P = h.N = h.Q = 0;
   __syncthreads();
   // private histograms: one warp per row
   for (int r = warp; r < NPB; r += BLOCK / 32) {
@@ -695,91 +962,65 @@ __device__ void fold_round(LaneState& st, Smem& sm, int lb) {
     }
     sum = __reduce_add_sync(0xFFFFFFFFu, sum);
     if (lane == 0 && sum) {
-      int bin = r < 63 ? 64 + r + 1 : (r - 63) - T::MB - 1 + 48;
+      int bin = r < NU ? 64 + r + 1 : 48 + (r - NU) + Rows<DT>::KLO;
       sm.hist[bin] += sum;
     }
+  }
+  for (int b = threadIdx.x; b < 64; b += BLOCK) {  // ULP bins above NU
+    if (b > NU && sm.ovf[b]) sm.hist[64 + b] += sm.ovf[b];
+    sm.ovf[b] = 0;
   }
   __syncthreads();
 }
 
+// End of one segment piece: the integer totals go to the segment's
+// accumulator (global atomics), the maxima to the CTA's partial slot.
 template <int DT>
-__device__ void finish_piece(LaneState& st, Smem& sm, int lb, Partial* out, int64_t n_piece) {
-  fold_round<DT>(st, sm, lb);
+__device__ void finish_piece(Hot& h, Cold& cd, Smem& sm, int lexp, Partial* out, SegAcc* acc) {
+  fold_round<DT>(h, sm, lexp);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  // counts
-  uint32_t c[8] = {st.n_eq, st.n_simple, st.n_within, st.n_nonfinite, st.n_gw, st.n_gm, st.n_ga, st.n_gf};
+  uint32_t c[8] = {h.n_eq + cd.n_geq, h.n_win, h.n_within, cd.n_nf, cd.n_gw, cd.n_gm, cd.n_ga, cd.n_gf};
 #pragma unroll
   for (int k = 0; k < 8; k++) {
     uint32_t v = __reduce_add_sync(0xFFFFFFFFu, c[k]);
     if (lane == 0 && v) atomicAdd(&sm.cnt[k], (unsigned long long)v);
   }
-  // maxima: warp tournament, then across warps
-  MaxAbs ma = st.mabs;
-  MaxRel mr = st.mrel;
-  MaxUlp mu = MaxUlp{st.ulp_f, st.ulp_idx};
-  int64_t ff = st.first_fin, fu = st.first_ulp;
-  for (int o = 16; o > 0; o >>= 1) {
-    MaxAbs oa{shfl_d(ma.hi, o), shfl_d(ma.lo, o), shfl_i64(ma.idx, o)};
-    MaxRel orl{shfl_d(mr.hi, o), shfl_d(mr.lo, o), shfl_d(mr.g, o), shfl_i64(mr.idx, o)};
-    MaxUlp ou{(uint64_t)shfl_i64((int64_t)mu.u, o), shfl_i64(mu.idx, o)};
-    int64_t off = shfl_i64(ff, o), ofu = shfl_i64(fu, o);
-    if (lane + o < 32) {
-      if (abs_better(oa, ma)) ma = oa;
-      if (rel_better(orl, mr)) mr = orl;
-      if (ulp_better(ou, mu)) mu = ou;
-      ff = min_idx(ff, off);
-      fu = min_idx(fu, ofu);
-    }
-  }
-  if (lane == 0) {
-    sm.wabs[warp] = ma;
-    sm.wrel[warp] = mr;
-    sm.wulp[warp] = mu;
-    sm.wff[warp] = ff;
-    sm.wfu[warp] = fu;
-  }
+  Partial x;
+  x.abs_hi = cd.abs_hi;
+  x.abs_lo = cd.abs_lo;
+  x.abs_sc = cd.abs_sc;
+  x.pad0 = 0;
+  x.abs_idx = cd.abs_idx;
+  x.rel_hi = cd.rel_hi;
+  x.rel_lo = cd.rel_lo;
+  x.rel_g = cd.rel_g;
+  x.rel_sc = cd.rel_sc;
+  x.rel_idx = cd.rel_idx;
+  x.ulp = cd.ulp;
+  x.ulp_idx = cd.ulp_idx;
+  x.first_fin = h.first_fin;
+  x.first_ulp = h.first_ulp;
+  part_warp_reduce(x);
+  if (lane == 0) sm.wbest[warp] = x;
   __syncthreads();
   if (threadIdx.x == 0) {
-    for (int w = 1; w < BLOCK / 32; w++) {
-      if (abs_better(sm.wabs[w], ma)) ma = sm.wabs[w];
-      if (rel_better(sm.wrel[w], mr)) mr = sm.wrel[w];
-      if (ulp_better(sm.wulp[w], mu)) mu = sm.wulp[w];
-      ff = min_idx(ff, sm.wff[w]);
-      fu = min_idx(fu, sm.wfu[w]);
-    }
-    out->mabs = ma;
-    out->mrel = mr;
-    out->mulp = mu;
-    out->first_fin = ff;
-    out->first_ulp = fu;
-    unsigned long long* cn = sm.cnt;
-    out->cnt[PEAT_EXACT] = cn[0];
-    out->cnt[PEAT_WITHIN_TOL] = cn[2] + cn[4];
-    out->cnt[PEAT_MISMATCH] = (cn[1] - cn[2]) + cn[5];
-    out->cnt[PEAT_NAN_INF_ASYM] = cn[6];
-    out->cnt[PEAT_SIGN_FLIP] = cn[7];
-    out->nonfinite = cn[3];
-    out->n = (uint64_t)n_piece;
+    for (int w = 1; w < BLOCK / 32; w++) part_merge(x, sm.wbest[w]);
+    *out = x;
   }
-  if (threadIdx.x < NSUM) {  // normalise the carry-save digits of one sum
-    int k = threadIdx.x;
-    long long carry = 0;
-    for (int j = 0; j < NLIMB; j++) {
-      long long v = (long long)sm.sacc[k][j] + carry;
-      if (j < NLIMB - 1) {
-        carry = v >> 32;
-        v &= 0xFFFFFFFFll;
-      }
-      out->limbs[k][j] = v;
-    }
+  for (int b = threadIdx.x; b < HBINS; b += BLOCK)
+    if (sm.hist[b]) atomicAdd(&acc->hist[b], sm.hist[b]);
+  if (threadIdx.x < 8 && sm.cnt[threadIdx.x]) atomicAdd(&acc->cnt[threadIdx.x], sm.cnt[threadIdx.x]);
+  for (int j = threadIdx.x; j < NSUM * NLIMB; j += BLOCK) {
+    unsigned long long v = (&sm.sacc[0][0])[j];
+    if (v) atomicAdd(reinterpret_cast<unsigned long long*>(&acc->limbs[0][0]) + j, v);
   }
-  for (int b = threadIdx.x; b < HBINS; b += BLOCK) out->hist[b] = sm.hist[b];
   __syncthreads();
   // reset the CTA totals for the next piece
   for (int b = threadIdx.x; b < HBINS; b += BLOCK) sm.hist[b] = 0;
   for (int j = threadIdx.x; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
   if (threadIdx.x < 8) sm.cnt[threadIdx.x] = 0;
-  state_init(st);
+  hot_init(h);
+  cold_init(cd);
   __syncthreads();
 }
 
@@ -790,28 +1031,39 @@ template <int DT>
 __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
   using T = Tr<DT>;
   constexpr int VEC = T::VEC;
-  constexpr int SHMAX = Win<DT>::SHMAX;
-  // lanes per thread per round stay below 2^16 (16-bit private counters)
-  constexpr int64_t ROUND_VECS = (int64_t)BLOCK * (65535 / VEC);
-  __shared__ Smem sm;
-  const int tid = threadIdx.x;
+  // lanes per thread per round stay below 2^16 (16-bit private counters): each
+  // warp tile gives a thread at most 2 VEC lanes
+  constexpr int64_t ROUND_CHUNKS = (int64_t)NW * (65535 / (2 * VEC));
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int b = tid; b < HBINS; b += BLOCK) sm.hist[b] = 0;
   for (int j = tid; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
-  for (int j = tid; j < Win<DT>::NPB * HALF; j += BLOCK) sm.priv[j] = 0;
+  for (int j = tid; j < Rows<DT>::NPB * HALF; j += BLOCK) sm.priv[j] = 0;
   if (tid < 8) sm.cnt[tid] = 0;
-  const int64_t lo = cta_lo<DT>(blockIdx.x, p), hi = cta_lo<DT>((int64_t)blockIdx.x + 1, p);
-  LaneState st;
-  state_init(st);
+  if (tid < 64) sm.ovf[tid] = 0;
+  if (lane == 0) {
+    for (int st = 0; st < NSTAGE; st++) mbar_init(&sm.bar[warp][st], 1);
+    mbar_init_fence();
+  }
   Ctx cx;
+  cx.cold = &sm.cold[tid];
+  cold_init(*cx.cold);
+  const int64_t lo = p.bounds[blockIdx.x], hi = p.bounds[blockIdx.x + 1];
+  Hot h;
+  hot_init(h);
   cx.rtol = p.rtol;
   cx.atol = p.atol;
-  cx.win_span = (uint32_t)(SHMAX + 1) << T::MB;
   cx.col = tid & (HALF - 1);
   cx.inc = tid < HALF ? 1u : 65536u;
   __syncthreads();
   if (lo >= hi) return;
+  uint32_t seq = 0;      // this warp's bulk-copy stage uses so far (stage = seq % NSTAGE)
+  bool failed = false;   // a pipeline wait expired: skip the data, keep the barriers
   int64_t s = seg_of(lo, p.offsets, p.nseg);
   int64_t pb = lo;
+  const char* gbase = reinterpret_cast<const char*>(p.g);
+  const char* cbase = reinterpret_cast<const char*>(p.c);
   while (pb < hi) {
     while (p.offsets[s + 1] <= pb) s++;  // skip empty segments
     const int64_t pe = min(hi, p.offsets[s + 1]);
@@ -823,6 +1075,21 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
       if (a0 < a1) vb = a0, ve = a1;
     }
     const int64_t nvec = (ve - vb) / VEC;
+    const int64_t nchunk = (nvec + CHV - 1) / CHV;
+    // start this warp's copies (chunk k = warp + NW * i) before anything else
+    auto issue = [&](uint32_t sq, int64_t k) {
+      const int st = (int)(sq % NSTAGE);
+      const int64_t v0 = k * CHV;
+      const uint32_t bytes = (uint32_t)(min((int64_t)CHV, nvec - v0) * 16);
+      const int64_t off = (vb + v0 * VEC) * T::BYTES;
+      fence_proxy_async();
+      mbar_expect_tx(&sm.bar[warp][st], 2 * bytes);
+      bulk_load(&sm.ring_g[warp][st][0], gbase + off, bytes, &sm.bar[warp][st]);
+      bulk_load(&sm.ring_c[warp][st][0], cbase + off, bytes, &sm.bar[warp][st]);
+    };
+    const int64_t my_chunks = nchunk > warp ? (nchunk - warp + NW - 1) / NW : 0;
+    if (lane == 0 && !failed)
+      for (int64_t i = 0; i < NSTAGE && i < my_chunks; i++) issue(seq + (uint32_t)i, warp + NW * i);
     // window of binades from the largest golden exponent in the first vectors
     if (tid == 0) sm.lb = 0;
     __syncthreads();
@@ -837,9 +1104,12 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
       atomicMax(&sm.lb, (int)emax);
     }
     __syncthreads();
-    int lb = sm.lb + 2 - SHMAX;
-    lb = lb < T::LBMIN ? T::LBMIN : (lb > Win<DT>::LBMAX ? Win<DT>::LBMAX : lb);
+    // V = |d| / 2^Lexp < 2^24 for u < 2^UB and golden binades up to 2 above the largest seen
+    int lb = sm.lb + T::UB - 22;
+    lb = lb < T::LBMIN ? T::LBMIN : (lb > T::LBMAX ? T::LBMAX : lb);
+    const int lexp = lb - T::BIAS - T::MB;  // weight of V's unit
     cx.lb_shift = (uint32_t)lb << T::MB;
+    cx.c0 = (uint32_t)(158 + lexp);
     // scalar head: fewer than VEC elements, or the whole piece in scalar mode
     // (then in rounds of at most 65535 elements per thread)
     {
@@ -848,46 +1118,64 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
       for (int64_t r0 = pb; r0 < h_end; r0 += ROUND_ELEMS) {
         const int64_t r1 = min(h_end, r0 + ROUND_ELEMS);
         for (int64_t i = r0 + tid; i < r1; i += BLOCK)
-          do_scalar<DT>(st, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), i, cx, sm);
-        if (r1 < h_end) fold_round<DT>(st, sm, lb);
+          do_scalar<DT>(h, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), i, cx, sm);
+        if (r1 < h_end) fold_round<DT>(h, sm, lexp);
       }
     }
-    // vector body in rounds
-    for (int64_t r0 = 0; r0 < nvec; r0 += ROUND_VECS) {
-      const int64_t r1 = min(nvec, r0 + ROUND_VECS);
-      int64_t v = r0 + tid;
-      // two vectors in flight per thread
-      for (; v + BLOCK < r1; v += 2 * BLOCK) {
-        const int64_t e0 = vb + v * VEC, e1 = vb + (v + BLOCK) * VEC;
-        uint4 g0 = load_vec(p.g, e0 * T::BYTES), c0 = load_vec(p.c, e0 * T::BYTES);
-        uint4 g1 = load_vec(p.g, e1 * T::BYTES), c1 = load_vec(p.c, e1 * T::BYTES);
-        do_vector<DT>(st, g0, c0, e0, cx, sm);
-        do_vector<DT>(st, g1, c1, e1, cx, sm);
+    // vector body: warp w takes chunks w, w + NW, ... of CHV vectors from its
+    // staging ring; NSTAGE chunks are in flight ahead of the one processed
+    int64_t i = 0;  // this warp's chunk counter within the piece
+    int64_t fail_i = -1;
+    uint32_t fail_seq = 0;
+    for (int64_t r0 = 0; r0 < nchunk; r0 += ROUND_CHUNKS) {
+      const int64_t r1 = min(nchunk, r0 + ROUND_CHUNKS);
+      for (int64_t k = warp + NW * i; k < r1; k = warp + NW * (++i)) {
+        const int st = (int)(seq % NSTAGE);
+        const uint32_t parity = (seq / NSTAGE) & 1u;
+        if (!failed && !mbar_wait(&sm.bar[warp][st], parity, p.wait_limit)) {
+          failed = true;  // chunks fail_i .. fail_i + NSTAGE - 1 may still be in flight
+          fail_i = i;
+          fail_seq = seq;
+          if (lane == 0) atomicOr(p.status, 1u);
+        }
+        if (!failed) {
+          const int64_t v0 = k * CHV;
+          const int nvalid = (int)min((int64_t)CHV, nvec - v0);
+          do_tile<DT>(h, sm.ring_g[warp][st], sm.ring_c[warp][st], nvalid, vb + v0 * VEC, cx, sm);
+          if (lane == 0 && i + NSTAGE < my_chunks) issue(seq + NSTAGE, warp + NW * (i + NSTAGE));
+        }
+        seq++;
       }
-      if (v < r1) {
-        const int64_t e0 = vb + v * VEC;
-        uint4 g0 = load_vec(p.g, e0 * T::BYTES), c0 = load_vec(p.c, e0 * T::BYTES);
-        do_vector<DT>(st, g0, c0, e0, cx, sm);
+      if (r1 < nchunk) fold_round<DT>(h, sm, lexp);
+    }
+    if (fail_i >= 0) {
+      // copies this warp issued but never consumed: wait for them before the
+      // staging memory is reused or the CTA exits
+      for (int64_t j = fail_i; j < my_chunks && j < fail_i + NSTAGE; j++) {
+        const uint32_t sq = fail_seq + (uint32_t)(j - fail_i);
+        mbar_wait(&sm.bar[warp][sq % NSTAGE], (sq / NSTAGE) & 1u, DRAIN_LIMIT);
       }
-      if (r1 < nvec) fold_round<DT>(st, sm, lb);
     }
     // scalar tail (fewer than VEC elements), after the body: lanes stay in index order
     if (vb < ve && ve < pe)
-      for (int64_t i = ve + tid; i < pe; i += BLOCK)
-        do_scalar<DT>(st, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), i, cx, sm);
-    finish_piece<DT>(st, sm, lb, p.partials + s + blockIdx.x, pe - pb);
+      for (int64_t e = ve + tid; e < pe; e += BLOCK)
+        do_scalar<DT>(h, load_scalar<DT>(p.g, e), load_scalar<DT>(p.c, e), e, cx, sm);
+    finish_piece<DT>(h, *cx.cold, sm, lexp, p.partials + s + blockIdx.x, p.acc + s);
     pb = pe;
   }
 }
 
 // ---------------------------------------------------------------------------
-// stage 2: one CTA per segment, fixed-order merge, exact finalisation
+// stage 2: one CTA per segment: merge the maxima of the segment's pieces,
+// round the exact sums once, write the outputs, clear the accumulator
 // ---------------------------------------------------------------------------
-__device__ double rel_value(const MaxRel& m) {
-  if (m.hi == 0.0) return 0.0;
-  if (m.g == 0.0) return __longlong_as_double(0x7FF0000000000000ll);
-  // RN64((hi+lo)/g): the candidate with the smallest exact residual, ties to even
-  double q0 = __ddiv_rn(m.hi, m.g);
+// RN64 of the quotient (hi + lo) 2^sc / g > 0: the candidate with the smallest
+// exact residual, ties to the even significand
+__device__ double rel_value(float hi, float lo, int sc, float g) {
+  if (hi == 0.0f) return 0.0;
+  if (g == 0.0f) return __longlong_as_double(0x7FF0000000000000ll);
+  double num = __dadd_rn((double)hi, (double)lo) * (sc ? 2.0 : 1.0);
+  double q0 = __ddiv_rn(num, (double)g);  // within a few units of the exact quotient
   double q = q0;
   for (int i = 0; i < 3; i++) q = nextafter(q, 0.0);
   double best = q;
@@ -896,9 +1184,9 @@ __device__ double rel_value(const MaxRel& m) {
   for (int step = 0; step < 7; step++, q = nextafter(q, __longlong_as_double(0x7FF0000000000000ll))) {
     XAcc r;
     r.zero();
-    r.add_double(m.hi);
-    r.add_double(m.lo);
-    r.add_prod(q, m.g, true);
+    r.add_f(hi, false, sc);
+    r.add_f(lo, false, sc);
+    r.add_prod(q, (double)g, true);
     r.normalize();
     if (r.sign() < 0) r.negate();
     if (!have) {
@@ -914,157 +1202,107 @@ __device__ double rel_value(const MaxRel& m) {
   return best;
 }
 
-template <int DT>
 __global__ void __launch_bounds__(BLOCK) compare_stage2(CompareParams p) {
   const int64_t s = blockIdx.x;
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t s0 = p.offsets[s], s1 = p.offsets[s + 1];
-  __shared__ MaxAbs wabs[BLOCK / 32];
-  __shared__ MaxRel wrel[BLOCK / 32];
-  __shared__ MaxUlp wulp[BLOCK / 32];
-  __shared__ long long wff[BLOCK / 32], wfu[BLOCK / 32];
-  __shared__ unsigned long long hist[HBINS];
+  SegAcc* acc = p.acc + s;
   __shared__ unsigned long long cnt[8];
   __shared__ long long limbs[NSUM][NLIMB];
-  peat_stats_t* out = p.stats + s;
-  if (s1 <= s0) {  // empty segment
-    if (tid == 0) {
-      peat_stats_t z;
-      memset(&z, 0, sizeof(z));
-      z.argmax_abs = z.argmax_rel = z.argmax_ulp = -1;
-      z.rtol_eff = p.rtol;
-      z.atol_eff = p.atol;
-      *out = z;
-    }
-    if (p.hist)
-      for (int b = tid; b < HBINS; b += BLOCK) p.hist[s * HBINS + b] = 0;
-    return;
-  }
-  const int b0 = cta_of<DT>(s0, p), b1 = cta_of<DT>(s1 - 1, p);
-  auto slot = [&](int b) -> const Partial* { return p.partials + s + b; };
-  auto nonempty = [&](int b) { return cta_lo<DT>(b, p) < cta_lo<DT>((int64_t)b + 1, p); };
-  // integer parts: one thread per counter / bin / digit, partials in order
+  __shared__ double sums[NSUM];
+  __shared__ Partial wbest[BLOCK / 32];
+  // integer totals, then clear them for the next call
+  unsigned long long hv = 0;
   if (tid < HBINS) {
-    unsigned long long h = 0;
-    for (int b = b0; b <= b1; b++)
-      if (nonempty(b)) h += slot(b)->hist[tid];
-    hist[tid] = h;
+    hv = acc->hist[tid];
+    acc->hist[tid] = 0;
   }
-  if (tid >= HBINS && tid < HBINS + 7) {
-    int k = tid - HBINS;
-    unsigned long long v = 0;
-    for (int b = b0; b <= b1; b++)
-      if (nonempty(b)) v += k < 5 ? slot(b)->cnt[k] : (k == 5 ? slot(b)->nonfinite : slot(b)->n);
-    cnt[k] = v;
+  if (tid >= HBINS && tid < HBINS + 8) {
+    cnt[tid - HBINS] = acc->cnt[tid - HBINS];
+    acc->cnt[tid - HBINS] = 0;
   }
   if (tid >= 160 && tid < 160 + NSUM * NLIMB) {
-    int k = (tid - 160) / NLIMB, j = (tid - 160) % NLIMB;
-    long long v = 0;
-    for (int b = b0; b <= b1; b++)
-      if (nonempty(b)) v += slot(b)->limbs[k][j];
-    limbs[k][j] = v;
+    int j = tid - 160;
+    (&limbs[0][0])[j] = (&acc->limbs[0][0])[j];
+    (&acc->limbs[0][0])[j] = 0;
   }
-  // maxima
-  MaxAbs ma{0.0, 0.0, -1};
-  MaxRel mr{0.0, 0.0, 1.0, -1};
-  MaxUlp mu{0, -1};
-  int64_t ff = -1, fu = -1;
-  for (int b = b0 + tid; b <= b1; b += BLOCK) {
-    if (!nonempty(b)) continue;
-    const Partial* q = slot(b);
-    if (abs_better(q->mabs, ma)) ma = q->mabs;
-    if (rel_better(q->mrel, mr)) mr = q->mrel;
-    if (ulp_better(q->mulp, mu)) mu = q->mulp;
-    ff = min_idx(ff, q->first_fin);
-    fu = min_idx(fu, q->first_ulp);
+  // maxima over the segment's pieces, in CTA order
+  Partial x;
+  part_none(x);
+  if (s1 > s0) {
+    const int b0 = cta_of(s0, p), b1 = cta_of(s1 - 1, p);
+    for (int b = b0 + tid; b <= b1; b += BLOCK)
+      if (p.bounds[b] < p.bounds[b + 1]) part_merge(x, p.partials[s + b]);
   }
-  const int lane = tid & 31, warp = tid >> 5;
-  for (int o = 16; o > 0; o >>= 1) {
-    MaxAbs oa{shfl_d(ma.hi, o), shfl_d(ma.lo, o), shfl_i64(ma.idx, o)};
-    MaxRel orl{shfl_d(mr.hi, o), shfl_d(mr.lo, o), shfl_d(mr.g, o), shfl_i64(mr.idx, o)};
-    MaxUlp ou{(uint64_t)shfl_i64((int64_t)mu.u, o), shfl_i64(mu.idx, o)};
-    int64_t off = shfl_i64(ff, o), ofu = shfl_i64(fu, o);
-    if (lane + o < 32) {
-      if (abs_better(oa, ma)) ma = oa;
-      if (rel_better(orl, mr)) mr = orl;
-      if (ulp_better(ou, mu)) mu = ou;
-      ff = min_idx(ff, off);
-      fu = min_idx(fu, ofu);
-    }
-  }
-  if (lane == 0) {
-    wabs[warp] = ma;
-    wrel[warp] = mr;
-    wulp[warp] = mu;
-    wff[warp] = ff;
-    wfu[warp] = fu;
+  part_warp_reduce(x);
+  if (lane == 0) wbest[warp] = x;
+  __syncthreads();
+  if (tid < NSUM) {
+    XAcc a;
+    for (int j = 0; j < NLIMB; j++) a.d[j] = limbs[tid][j];
+    sums[tid] = a.to_double();
   }
   __syncthreads();
   if (tid == 0) {
-    for (int w = 1; w < BLOCK / 32; w++) {
-      if (abs_better(wabs[w], ma)) ma = wabs[w];
-      if (rel_better(wrel[w], mr)) mr = wrel[w];
-      if (ulp_better(wulp[w], mu)) mu = wulp[w];
-      ff = min_idx(ff, wff[w]);
-      fu = min_idx(fu, wfu[w]);
-    }
+    for (int w = 1; w < BLOCK / 32; w++) part_merge(x, wbest[w]);
     peat_stats_t r;
-    r.n = cnt[6];
+    const uint64_t n = (uint64_t)(s1 - s0);
+    r.n = n;
     r.count[PEAT_EXACT] = cnt[0];
-    for (int k = 1; k < PEAT_NCLASS; k++) r.count[k] = cnt[k];
-    r.n_finite = cnt[6] - cnt[5];
-    // maxima: only strictly positive errors are recorded; a zero maximum is
-    // attained first at the first finite (or ULP-defined) pair
-    if (ma.idx >= 0) {
-      r.max_abs = ma.hi;  // hi = RN64(|d|)
-      r.argmax_abs = ma.idx - s0;
+    r.count[PEAT_WITHIN_TOL] = cnt[2] + cnt[4];
+    r.count[PEAT_MISMATCH] = (cnt[1] - cnt[2]) + cnt[5];
+    r.count[PEAT_NAN_INF_ASYM] = cnt[6];
+    r.count[PEAT_SIGN_FLIP] = cnt[7];
+    r.n_finite = n - cnt[3];
+    if (x.abs_idx >= 0) {
+      r.max_abs = __dadd_rn((double)x.abs_hi, (double)x.abs_lo) * (x.abs_sc ? 2.0 : 1.0);
+      r.argmax_abs = x.abs_idx - s0;
     } else {
       r.max_abs = 0.0;
-      r.argmax_abs = ff >= 0 ? ff - s0 : -1;
+      r.argmax_abs = x.first_fin >= 0 ? x.first_fin - s0 : -1;
     }
-    if (mr.idx >= 0) {
-      r.max_rel = rel_value(mr);
-      r.argmax_rel = mr.idx - s0;
+    if (x.rel_idx >= 0) {
+      r.max_rel = rel_value(x.rel_hi, x.rel_lo, x.rel_sc, x.rel_g);
+      r.argmax_rel = x.rel_idx - s0;
     } else {
       r.max_rel = 0.0;
-      r.argmax_rel = ff >= 0 ? ff - s0 : -1;
+      r.argmax_rel = x.first_fin >= 0 ? x.first_fin - s0 : -1;
     }
-    if (mu.idx >= 0) {
-      r.max_ulp = mu.u;
-      r.argmax_ulp = mu.idx - s0;
+    if (x.ulp_idx >= 0) {
+      r.max_ulp = x.ulp;
+      r.argmax_ulp = x.ulp_idx - s0;
     } else {
       r.max_ulp = 0;
-      r.argmax_ulp = fu >= 0 ? fu - s0 : -1;
-    }
-    double sums[NSUM];
-    for (int k = 0; k < NSUM; k++) {
-      XAcc x;
-      for (int j = 0; j < NLIMB; j++) x.d[j] = limbs[k][j];
-      sums[k] = x.to_double();
+      r.argmax_ulp = x.first_ulp >= 0 ? x.first_ulp - s0 : -1;
     }
     r.sum_signed = sums[0];
     r.sum_abs = sums[1];
     r.sum_sq = sums[2];
     r.rtol_eff = p.rtol;
     r.atol_eff = p.atol;
-    *out = r;
+    p.stats[s] = r;
   }
-  if (p.hist) {
-    for (int b = tid; b < HBINS; b += BLOCK) {
-      unsigned long long h = hist[b];
-      if (b == 0 || b == 64) h += cnt[0];  // EXACT pairs: rel bin 0 and ULP bin 0
-      p.hist[s * HBINS + b] = h;
-    }
-  }
+  if (p.hist && tid < HBINS) p.hist[s * HBINS + tid] = hv + ((tid == 0 || tid == 64) ? cnt[0] : 0ull);
 }
 
 template <int DT>
 cudaError_t launch_t(const CompareParams& p, cudaStream_t st) {
-  compare_stage1<DT><<<p.nctas, BLOCK, 0, st>>>(p);
+  compare_stage1<DT><<<p.nctas, BLOCK, sizeof(Smem), st>>>(p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if (p.nseg > 0) compare_stage2<DT><<<(unsigned)p.nseg, BLOCK, 0, st>>>(p);
+  if (p.nseg > 0) compare_stage2<<<(unsigned)p.nseg, BLOCK, 0, st>>>(p);
   return cudaGetLastError();
+}
+
+template <int DT>
+int64_t bound_t(int64_t b, int nctas, int64_t n, int64_t p0) {
+  if (b <= 0) return 0;
+  if (b >= nctas) return n;
+  constexpr int VEC = Tr<DT>::VEC;
+  if (p0 < 0 || p0 >= n) return (n / nctas) * b + (n % nctas) * b / nctas;
+  int64_t nv = (n - p0) / VEC;
+  int64_t lo = p0 + ((nv / nctas) * b + (nv % nctas) * b / nctas) * VEC;
+  return lo < n ? lo : n;
 }
 
 }  // namespace
@@ -1078,7 +1316,29 @@ cudaError_t launch_compare(int dtype, const CompareParams& p, cudaStream_t s) {
   return cudaErrorInvalidValue;
 }
 
+int64_t compare_cta_bound(int dtype, int64_t b, int nctas, int64_t n, int64_t p0) {
+  switch (dtype) {
+    case PEAT_F32: return bound_t<PEAT_F32>(b, nctas, n, p0);
+    case PEAT_F16: return bound_t<PEAT_F16>(b, nctas, n, p0);
+    default: return bound_t<PEAT_BF16>(b, nctas, n, p0);
+  }
+}
+
+// once per device, before the first launch
+cudaError_t compare_prepare() {
+  cudaError_t e = cudaFuncSetAttribute(compare_stage1<PEAT_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)sizeof(Smem));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(compare_stage1<PEAT_F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(Smem));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(compare_stage1<PEAT_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)sizeof(Smem));
+  return e;
+}
+
 int compare_ctas_per_sm() { return 2; }
 size_t compare_partial_bytes() { return sizeof(Partial); }
+size_t compare_segacc_bytes() { return sizeof(SegAcc); }
+size_t compare_cold_bytes() { return sizeof(Cold) * BLOCK; }
 
 }  // namespace peat

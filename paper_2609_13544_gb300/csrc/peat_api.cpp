@@ -20,8 +20,13 @@ struct peat_handle_s {
   int max_ctas = 0;
   // compare workspace
   peat::Partial* partials = nullptr;
-  int64_t* d_offsets = nullptr;
-  int64_t* h_offsets = nullptr;  // pinned staging
+  peat::SegAcc* acc = nullptr;   // per-segment integer totals, zero between calls
+  void* cold = nullptr;          // per-thread rare-path records of stage 1
+  unsigned int* status_host = nullptr;  // mapped pinned error word written by the kernels
+  unsigned int* status_dev = nullptr;
+  unsigned int wait_limit = 1u << 24;   // polls before a pipeline wait gives up
+  int64_t* d_offsets = nullptr;  // offsets (nseg + 1) then CTA bounds (nctas + 1)
+  int64_t* h_offsets = nullptr;  // pinned staging of the same
   cudaEvent_t staged = nullptr;  // the last staging copy has been consumed
   bool staged_pending = false;
   // injector staging (grown on demand)
@@ -96,43 +101,59 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   const int64_t n = offsets[nseg];
   if (n > 0 && (!g || !c)) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
   if (nseg > 0 && !stats) return fail(h, PEAT_ERR_INVALID_ARG, "stats_out is NULL");
+  if (h->status_host && *(volatile unsigned int*)h->status_host) {
+    *(volatile unsigned int*)h->status_host = 0;
+    return fail(h, PEAT_ERR_TIMEOUT,
+                "a bounded device-side wait expired in an earlier call on this handle; its outputs are invalid");
+  }
   if (nseg == 0) return PEAT_OK;
   DeviceGuard dg(h->device);
   if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-
-  peat_status_t ps = wait_staging(h);
-  if (ps != PEAT_OK) return ps;
-  std::memcpy(h->h_offsets, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
-  cudaError_t e = cudaMemcpyAsync(h->d_offsets, h->h_offsets, sizeof(int64_t) * (size_t)(nseg + 1),
-                                  cudaMemcpyHostToDevice, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(offsets)");
-  e = cudaEventRecord(h->staged, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
-  h->staged_pending = true;
 
   peat::CompareParams p;
   std::memset(&p, 0, sizeof(p));
   p.g = g;
   p.c = c;
   p.n_total = n;
-  p.offsets = h->d_offsets;
   p.nseg = nseg;
   uintptr_t ag = reinterpret_cast<uintptr_t>(g), ac = reinterpret_cast<uintptr_t>(c);
   if (n > 0 && ag % B == 0 && ac % B == 0 && ag % 16 == ac % 16)
     p.p0 = (int64_t)(((16 - ag % 16) % 16) / B);
   else
     p.p0 = -1;
-  // persistent grid, at most one CTA per ~4K elements for small inputs
-  int64_t want = (n + 4095) / 4096;
+  // persistent grid; small inputs get about one CTA per 32K elements
+  int64_t want = (n + 32767) / 32768;
   p.nctas = (int)std::max<int64_t>(1, std::min<int64_t>(h->max_ctas, want));
+
+  peat_status_t ps = wait_staging(h);
+  if (ps != PEAT_OK) return ps;
+  std::memcpy(h->h_offsets, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
+  int64_t* hb = h->h_offsets + nseg + 1;
+  for (int b = 0; b <= p.nctas; b++) hb[b] = peat::compare_cta_bound(dtype, b, p.nctas, n, p.p0);
+  cudaError_t e = cudaMemcpyAsync(h->d_offsets, h->h_offsets, sizeof(int64_t) * (size_t)(nseg + 2 + p.nctas),
+                                  cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(offsets)");
+  e = cudaEventRecord(h->staged, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
+  h->staged_pending = true;
+  p.offsets = h->d_offsets;
+  p.bounds = h->d_offsets + nseg + 1;
+  p.acc = h->acc;
   p.partials = h->partials;
+  p.cold = h->cold;
+  p.status = h->status_dev;
+  p.wait_limit = h->wait_limit;
   p.rtol = rtol;
   p.atol = atol;
   p.stats = stats;
   p.hist = hist;
   e = peat::launch_compare(dtype, p, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "compare launch");
+  if (e != cudaSuccess) {
+    // the accumulators may hold a partial stage 1: clear them for the next call
+    cudaMemsetAsync(h->acc, 0, peat::compare_segacc_bytes() * (size_t)nseg, st);
+    return cuda_fail(h, e, "compare launch");
+  }
   return PEAT_OK;
 }
 
@@ -193,8 +214,8 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
   peat_config_t c;
   std::memset(&c, 0, sizeof(c));
   if (cfg) c = *cfg;
-  if (c.flags != 0 || c.max_segments < 0) {
-    g_create_error = "bad config (flags must be 0, max_segments >= 0)";
+  if ((c.flags & ~PEAT_FLAG_TEST_EXPIRE_WAITS) != 0 || c.max_segments < 0) {
+    g_create_error = "bad config (unknown flags, or max_segments < 0)";
     return PEAT_ERR_INVALID_ARG;
   }
   int ndev = 0;
@@ -207,6 +228,7 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
   peat_handle_t h = new peat_handle_s();
   h->device = c.device;
   h->max_segments = c.max_segments > 0 ? c.max_segments : 4096;
+  if (c.flags & PEAT_FLAG_TEST_EXPIRE_WAITS) h->wait_limit = 0;
   DeviceGuard dg(h->device);
   if (!dg.ok) {
     g_create_error = "cudaSetDevice failed";
@@ -214,12 +236,26 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
     return PEAT_ERR_CUDA;
   }
   cudaDeviceGetAttribute(&h->nsm, cudaDevAttrMultiProcessorCount, h->device);
+  if (peat::compare_prepare() != cudaSuccess) {
+    cudaGetLastError();
+    g_create_error = "could not configure the compare kernels";
+    delete h;
+    return PEAT_ERR_CUDA;
+  }
   h->max_ctas = std::max(1, h->nsm * peat::compare_ctas_per_sm());
   size_t slots = (size_t)h->max_segments + (size_t)h->max_ctas;
+  size_t staging = (size_t)h->max_segments + 2 + (size_t)h->max_ctas;
+  size_t acc_bytes = (size_t)h->max_segments * peat::compare_segacc_bytes();
   bool ok = cudaMalloc(&h->partials, slots * peat::compare_partial_bytes()) == cudaSuccess &&
-            cudaMalloc(&h->d_offsets, sizeof(int64_t) * (size_t)(h->max_segments + 1)) == cudaSuccess &&
-            cudaMallocHost(&h->h_offsets, sizeof(int64_t) * (size_t)(h->max_segments + 1)) == cudaSuccess &&
-            cudaEventCreateWithFlags(&h->staged, cudaEventDisableTiming) == cudaSuccess;
+            cudaMalloc(&h->acc, acc_bytes) == cudaSuccess &&
+            cudaMalloc(&h->cold, (size_t)h->max_ctas * peat::compare_cold_bytes()) == cudaSuccess &&
+            cudaHostAlloc((void**)&h->status_host, sizeof(unsigned int), cudaHostAllocMapped) == cudaSuccess &&
+            cudaHostGetDevicePointer((void**)&h->status_dev, h->status_host, 0) == cudaSuccess &&
+            cudaMemset(h->acc, 0, acc_bytes) == cudaSuccess &&
+            cudaMalloc(&h->d_offsets, sizeof(int64_t) * staging) == cudaSuccess &&
+            cudaMallocHost(&h->h_offsets, sizeof(int64_t) * staging) == cudaSuccess &&
+            cudaEventCreateWithFlags(&h->staged, cudaEventDisableTiming) == cudaSuccess &&
+            cudaDeviceSynchronize() == cudaSuccess;
   if (!ok) {
     cudaGetLastError();
     g_create_error = "workspace allocation failed";
@@ -237,6 +273,9 @@ peat_status_t peat_signature_destroy(peat_handle_t h) {
     if (h->staged) cudaEventSynchronize(h->staged);
     cudaDeviceSynchronize();
     if (h->partials) cudaFree(h->partials);
+    if (h->acc) cudaFree(h->acc);
+    if (h->cold) cudaFree(h->cold);
+    if (h->status_host) cudaFreeHost(h->status_host);
     if (h->d_offsets) cudaFree(h->d_offsets);
     if (h->h_offsets) cudaFreeHost(h->h_offsets);
     if (h->d_inj) cudaFree(h->d_inj);

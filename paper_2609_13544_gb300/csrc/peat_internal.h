@@ -19,33 +19,34 @@ constexpr int NSUM = 3;  // 0: sum d, 1: sum |d|, 2: sum d^2
 constexpr int BLOCK = 256;    // threads per compare CTA
 constexpr int HBINS = 128;    // 64 rel bins + 64 ULP bins
 
-// Exact maxima records.  abs: |d| = hi + lo (binary64 pair, hi = RN(|d|)).
-// rel: (hi + lo) / g with g = |golden| (g = 0 means +inf).  idx = -1: none.
-struct MaxAbs {
-  double hi, lo;
-  int64_t idx;
-};
-struct MaxRel {
-  double hi, lo, g;
-  int64_t idx;
-};
-struct MaxUlp {
-  uint64_t u;
-  int64_t idx;
+// Exact maxima of one CTA piece (element indices are global).  |d| is kept
+// as (hi + lo) * 2^sc with hi = RN32(|d| 2^-sc), |lo| at most half a float32
+// step of hi, and sc = 1 only when |d| exceeds the float32 range.  The rel
+// record is (hi + lo) 2^sc / g with g = |golden| (g = 0: +inf).  idx = -1:
+// no record.  Only strictly positive errors and ULP distances are recorded;
+// first_fin / first_ulp give the argmax when every error is zero.
+struct Partial {
+  float abs_hi, abs_lo;
+  int32_t abs_sc, pad0;
+  int64_t abs_idx;
+  float rel_hi, rel_lo, rel_g;
+  int32_t rel_sc;
+  int64_t rel_idx;
+  uint64_t ulp;
+  int64_t ulp_idx;
+  int64_t first_fin;  // lowest index of a finite pair (-1 none)
+  int64_t first_ulp;  // lowest index of a pair without NaN (-1 none)
 };
 
-// One CTA's contribution to one segment.  Element indices are global.
-struct Partial {
-  uint64_t cnt[PEAT_NCLASS];
-  uint64_t nonfinite;  // pairs with a NaN or Inf operand
-  uint64_t n;
-  uint64_t hist[HBINS];
-  MaxAbs mabs;
-  MaxRel mrel;
-  MaxUlp mulp;         // only u > 0 is recorded
-  int64_t first_fin;   // lowest index of a finite pair (-1 none)
-  int64_t first_ulp;   // lowest index of a pair without NaN (-1 none)
-  int64_t limbs[NSUM][NLIMB];  // normalised: digits 0..NLIMB-2 in [0, 2^32), top signed
+// Integer totals of one segment: stage 1 adds into them with atomics (all
+// integers, so the order does not matter), stage 2 reads and clears them.
+// cnt: 0 EXACT, 1 window lanes, 2 window lanes within tol, 3 non-finite
+// pairs, 4 general within, 5 general mismatch, 6 NaN/Inf asymmetric,
+// 7 sign flip.  limbs: carry-save digits of the three exact sums.
+struct SegAcc {
+  unsigned long long hist[HBINS];
+  unsigned long long cnt[8];
+  long long limbs[NSUM][NLIMB];
 };
 
 struct CompareParams {
@@ -53,10 +54,15 @@ struct CompareParams {
   const void* c;
   int64_t n_total;
   const int64_t* offsets;  // device copy, nseg + 1 entries
+  const int64_t* bounds;   // device copy, nctas + 1 CTA range boundaries
   int64_t nseg;
   int64_t p0;              // first element index of the aligned vector grid; -1: scalar only
   int nctas;
   Partial* partials;       // nseg + nctas slots; slot s + b holds CTA b's part of segment s
+  SegAcc* acc;             // nseg accumulators, all zero between calls
+  void* cold;              // per-thread rare-path state, nctas * BLOCK records
+  unsigned int* status;    // device-visible error word (bit 0: a bounded wait expired)
+  unsigned int wait_limit; // iteration bound of a pipeline wait (0: give up at once, for tests)
   float rtol, atol;        // float32 tolerances
   peat_stats_t* stats;
   uint64_t* hist;          // may be null
@@ -65,7 +71,13 @@ struct CompareParams {
 // Host-side launchers (compare.cu / inject.cu).
 cudaError_t launch_compare(int dtype, const CompareParams& p, cudaStream_t s);
 int compare_ctas_per_sm();
+cudaError_t compare_prepare();
+// CTA b of a grid of nctas owns elements [bound(b), bound(b+1)); boundaries
+// lie on the 16-byte vector grid that starts at element p0 (p0 < 0: none)
+int64_t compare_cta_bound(int dtype, int64_t b, int nctas, int64_t n, int64_t p0);
 size_t compare_partial_bytes();
+size_t compare_segacc_bytes();
+size_t compare_cold_bytes();  // per CTA
 
 struct InjectElemParams {
   void* dst;

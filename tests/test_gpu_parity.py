@@ -153,3 +153,22 @@ def test_invalid_arguments(peat_gpu, h):
         peat_gpu.peat_compare_segmented_raw(small, g, g, [0, 1, 2, 10], 0.0, 0.0, s)
     assert e.value.status == 2
     small.close()
+
+
+def test_forced_wait_expiry_reports_timeout_and_context_survives(peat_gpu, oracle, h):
+    """The pipeline's bounded waits: with the test flag every wait gives up at
+    once; the kernel drains its copies, returns, and the next call on that
+    handle reports PEAT_ERR_TIMEOUT.  The GPU context stays usable."""
+    import torch
+    gb, cb = noise_pairs("bf16", 1_000_003, seed=17)
+    g, c = to_device(gb, "bf16"), to_device(cb, "bf16")
+    s = torch.empty(144, dtype=torch.uint8, device="cuda")
+    bad = peat_gpu.Handle(0, flags=peat_gpu.PEAT_FLAG_TEST_EXPIRE_WAITS)
+    peat_gpu.peat_compare_raw(bad, g, c, 1e-3, 0.0, s)
+    torch.cuda.synchronize()
+    with pytest.raises(peat_gpu.PeatError) as e:
+        peat_gpu.peat_compare_raw(bad, g, c, 1e-3, 0.0, s)
+    assert e.value.status == 5
+    torch.cuda.synchronize()
+    bad.close()
+    check_pair(peat_gpu, oracle, h, gb, cb, "bf16", 1e-3, 0.0, ctx="after forced expiry")

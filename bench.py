@@ -140,6 +140,22 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The slowest replica sets the step time: MAX over ranks (identity at N = 1)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: int, world: int, steps: int, ms: float) -> float:
+    """Units all ranks processed in `steps` steps, per second of the max-over-ranks time."""
+    return units_per_rank * world * steps / (ms * 1e-3)
+
+
 # --------------------------------------------------------------------------- oracle timing
 def _oracle_slice(args):
     import numpy as np
@@ -269,16 +285,10 @@ def run_gpu(args) -> None:
         barrier()
         wall = time.perf_counter() - wall0
         time.sleep(0.25)
-    ms = e0.elapsed_time(e1)
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
     clocks = clk.summary()
     ms_per_step = ms / args.steps
-    pairs = w.n * world
-    value = pairs * args.steps / (ms * 1e-3)
+    value = whole_job_rate(w.n, world, args.steps, ms)
     bytes_per_step = 2 * w.n * (4 if w.dtype == "f32" else 2)
     gbs = bytes_per_step / (ms_per_step * 1e-3) / 1e9
     peaks = measured_peaks()
@@ -312,13 +322,8 @@ def run_gpu(args) -> None:
             e2e_step()
         f1.record(stream)
         barrier()
-        ems = f0.elapsed_time(f1)
-        if world > 1:
-            import torch.distributed as dist
-            t = torch.tensor([ems], device=dev, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
-        e2e = {"value": w.n * world * e2e_steps / (ems * 1e-3), "unit": "pairs/s",
+        ems = max_over_ranks(f0.elapsed_time(f1), dev)
+        e2e = {"value": whole_job_rate(w.n, world, e2e_steps, ems), "unit": "pairs/s",
                "h2d_bytes_per_step": bytes_per_step, "d2h_bytes_per_step": int(stats.numel() + hist.numel() * 8),
                "ms_per_step": ems / e2e_steps}
 

@@ -7,30 +7,35 @@
 // 64-bin histograms.  Every output is exact: integer outputs bit for bit,
 // sums as the exact real sum rounded once to nearest-even binary64.
 //
-// Stage 1 (compare_stage1): a persistent grid streams both tensors once.
-// CTA b owns the contiguous element range [lo_b, lo_{b+1}); per segment piece
-// it touches it adds its integer totals (counts, histograms, sum digits) to
-// the segment's accumulator with atomics and writes its maxima to slot s + b.
+// Stage 1 (compare_stage1): a persistent grid streams both tensors once
+// through per-warp rings of bulk copies (cp.async.bulk + mbarrier).  CTA b
+// owns the contiguous element range [lo_b, lo_{b+1}); per segment piece it
+// touches it adds its integer totals (counts, histograms, sum digits) to the
+// segment's accumulator with atomics and writes its maxima to slot s + b.
 // Per element pair:
-//   - bitwise-equal vectors are counted and skipped;
-//   - a "window" lane -- same sign, at most one binade apart (ULP distance
-//     u < 2^UB), both operands' steps at least 2^Lexp, |d| < 2^(24+Lexp) --
-//     is exact in float32 and integer arithmetic: d = c - g is exact in
-//     float32, V = |d| / 2^Lexp is an integer below 2^24, so sum |d|, sum d
-//     and sum d^2 accumulate as integers; the log2-relative bin is the
-//     exponent difference of |d| and |g| read from their bit patterns; the
-//     tolerance test is one float32 fma, exact except at equality;
-//   - every other lane (non-finite, sign change, zeros, wide gaps, outside
-//     the window, tolerance ties) takes the general path, which evaluates the
-//     definitions exactly with float32 error-free transforms and integer
-//     digits, adding its sum terms to a CTA-wide carry-save fixed-point
-//     accumulator in shared memory.
+//   - bitwise-equal pairs are counted (whole warp tiles at once when equal);
+//   - unequal pairs of a tile are processed in place when most of the tile
+//     differs, else compacted into a per-warp queue first;
+//   - a "window" pair -- same sign, ULP distance u < 2^UB (so c is within a
+//     factor 2 of g and c - g is exact in float32, Sterbenz), |g| at least
+//     2^(Lb+1-bias), |d| < 2^(Lexp+22) -- is finished in float32 and
+//     integer arithmetic: V = |d| / 2^Lexp is an integer below 2^22, read
+//     from the bits of |d| + 1.5 * 2^(Lexp+23), so sum |d|, sum d and sum d^2
+//     accumulate as integers; the log2-relative bin is the exponent
+//     difference of |d| and |g|; the tolerance test is one float32 fma, exact
+//     except at equality; the maxima are exact float32 comparisons (the
+//     significands are short enough for exact products, or error-free
+//     products for float32 input);
+//   - every other pair (non-finite, sign change, zeros, wide gaps, outside
+//     the window, tolerance ties) is deferred to a per-warp buffer and
+//     evaluated exactly, 32 at a time, with float32 error-free transforms and
+//     integer digits added to a CTA-wide carry-save fixed-point accumulator.
 // Binary64 arithmetic is avoided in stage 1 (GB300 runs it at a small
 // fraction of float32 rate); binary64 values appear only as containers.
 // Stage 2 (compare_stage2): one CTA per segment merges the maxima of that
-// segment's pieces, rounds the exact sums once and clears the accumulator;
-// all merged quantities are integers or exact values, so the result does not
-// depend on the grid or on the order of the atomics.
+// segment's pieces in CTA order, rounds the exact sums once and clears the
+// accumulator; all merged quantities are integers or exact values, so the
+// result does not depend on the grid or on the order of the atomics.
 #include <cuda_fp16.h>
 
 #include <cstdint>
@@ -43,41 +48,45 @@ namespace {
 // ---------------------------------------------------------------------------
 // element types
 // ---------------------------------------------------------------------------
+// UBMAX: the largest window ULP bound (u < 2^UB keeps c within a factor 2 of
+// g; the per-piece UB is sampled from the data and capped here).  LBMIN and
+// LBMAX bound the window's floor binade Lb so that 2^Lexp is a normal float32
+// (Lexp = Lb - BIAS - MB) and 1.5 * 2^(Lexp+23) is finite.
 template <int DT>
 struct Tr;
 template <>
 struct Tr<PEAT_F32> {
   static constexpr int BYTES = 4, VEC = 4, MB = 23, BIAS = 127, EMAX = 255;
-  static constexpr int UB = 12;       // window lanes need u < 2^UB
-  static constexpr int LBMIN = 24;    // keeps 2^Lexp >= 2^-126 (normal float32)
-  static constexpr int LBMAX = 221;   // keeps |g| < 2^126 (normal reciprocal)
+  static constexpr int UBMAX = 12, LBMIN = 24, LBMAX = 221;
   static constexpr uint32_t SIGN = 0x80000000u, MAG = 0x7FFFFFFFu, INF = 0x7F800000u;
 };
 template <>
 struct Tr<PEAT_F16> {
   static constexpr int BYTES = 2, VEC = 8, MB = 10, BIAS = 15, EMAX = 31;
-  static constexpr int UB = 10, LBMIN = 1, LBMAX = 30;
+  static constexpr int UBMAX = 10, LBMIN = 1, LBMAX = 30;
   static constexpr uint32_t SIGN = 0x8000u, MAG = 0x7FFFu, INF = 0x7C00u;
 };
 template <>
 struct Tr<PEAT_BF16> {
   static constexpr int BYTES = 2, VEC = 8, MB = 7, BIAS = 127, EMAX = 255;
-  static constexpr int UB = 7, LBMIN = 8, LBMAX = 221;
+  static constexpr int UBMAX = 7, LBMIN = 8, LBMAX = 221;
   static constexpr uint32_t SIGN = 0x8000u, MAG = 0x7FFFu, INF = 0x7F80u;
 };
 
-// Private per-thread histogram rows: ULP bins 1..NU, then the log2-relative
-// bins window lanes reach, k in [KLO, KHI] (fp16 goldens may be subnormal,
-// whose ratios reach 2^MB).  ULP bins above NU use shared counters.
+// Private per-thread histogram rows (16-bit counters, two threads per word):
+// ULP bins 1..NU, then ULP bin 63, then the log2-relative bins window pairs
+// reach, k in [KLO, KHI] (fp16 goldens may be subnormal, whose ratios reach
+// 2^(MB-1)).  ULP bins NU+1..62 use CTA-wide shared counters.
 constexpr int NU = 15;
 template <int DT>
 struct Rows {
   static constexpr int KLO = -(Tr<DT>::MB + 1);
-  static constexpr int KHI = DT == PEAT_F16 ? Tr<DT>::MB - 1 : Tr<DT>::UB - Tr<DT>::MB;
-  static constexpr int NPB = NU + KHI - KLO + 1;
+  static constexpr int KHI = DT == PEAT_F16 ? Tr<DT>::MB - 1 : Tr<DT>::UBMAX - Tr<DT>::MB;
+  static constexpr int NPB = NU + 1 + KHI - KLO + 1;
 };
 constexpr int HALF = BLOCK / 2;
-constexpr int NPB_MAX = NU + 9 + 11 + 1;
+constexpr int ROWB = HALF * 4;  // bytes per private row
+constexpr int NPB_MAX = NU + 1 + 9 + 11 + 1;
 
 template <int DT>
 __device__ __forceinline__ float to_f32(uint32_t b) {
@@ -250,44 +259,6 @@ struct XAcc {
     for (int j = 0; j < NLIMB; j++) d[j] = -d[j];
     normalize();
   }
-  // round-to-nearest-even binary64 of the exact value
-  __device__ double to_double() {
-    normalize();
-    bool neg = sign() < 0;
-    if (neg) negate();
-    int top = -1;
-    for (int j = NLIMB - 1; j >= 0; j--)
-      if (d[j]) {
-        top = j;
-        break;
-      }
-    if (top < 0) return 0.0;
-    uint64_t dtop = (uint64_t)d[top];
-    int msb = top * 32 + 63 - __clzll(dtop);  // bit index of the leading one
-    // the 64 bits [msb-63, msb], plus a sticky flag for everything below
-    uint64_t win = 0;
-    for (int bit = msb; bit > msb - 64; bit--) {
-      win <<= 1;
-      if (bit >= 0) win |= ((uint64_t)d[bit >> 5] >> (bit & 31)) & 1ull;
-    }
-    bool sticky = false;
-    for (int j = 0; j < NLIMB && !sticky; j++) {
-      int lo_bit = j * 32, hi_bit = j * 32 + 31;
-      if (hi_bit <= msb - 64) sticky = d[j] != 0;
-      else if (lo_bit <= msb - 64) {
-        int nb = msb - 64 - lo_bit + 1;
-        uint64_t mask = nb >= 32 ? 0xFFFFFFFFull : ((1ull << nb) - 1);
-        sticky = ((uint64_t)d[j] & mask) != 0;
-      }
-    }
-    uint64_t mant = win >> 11;
-    uint64_t rest = win & 0x7FFull;
-    bool round = (rest >> 10) & 1;
-    bool st = sticky || (rest & 0x3FF);
-    if (round && (st || (mant & 1))) mant++;
-    double r = ldexp((double)mant, msb - 52 + LIMB_LSB);
-    return neg ? -r : r;
-  }
 };
 
 // ---------------------------------------------------------------------------
@@ -353,8 +324,8 @@ __device__ __forceinline__ float rel_filter(float hi, int sc, float g) {
 // ---------------------------------------------------------------------------
 // shared memory
 // ---------------------------------------------------------------------------
-// Per-thread state touched only on the rare paths: the general-path counters
-// and the exact maxima records.
+// Per-thread state of the general path: its class counters and its exact
+// maxima records (|d| as (hi + lo) 2^sc, see Partial).
 struct Cold {
   float abs_hi, abs_lo;
   float rel_hi, rel_lo, rel_g;
@@ -364,6 +335,7 @@ struct Cold {
   int abs_sc, rel_sc;
   uint32_t pad;
   long long abs_idx, rel_idx, ulp_idx;
+  long long first_fin, first_ulp;  // lowest index of a finite pair / of a pair without NaN
 };
 
 // Per-warp staging ring for the bulk copies: NSTAGE stages, each one warp
@@ -380,11 +352,14 @@ struct __align__(128) Smem {
   unsigned long long sacc[NSUM][NLIMB];
   unsigned long long cnt[8];
   Partial wbest[NW];
-  int lb;
-  uint32_t ovf[64];               // ULP bins NU+1..63 of window lanes (CTA-wide)
+  int lb, ub;
+  long long lo;                    // the CTA's first element
+  uint32_t* glist;                 // this CTA's list of general pairs (offsets), GCAP entries
+  uint32_t gn;                     // entries appended in this piece (may exceed GCAP)
+  uint32_t ovf[64];                // ULP bins NU+1..62 of window pairs (CTA-wide)
   Cold cold[BLOCK];
-  uint32_t priv[NPB_MAX * HALF];  // per-thread 16-bit counters, two threads per word
-  unsigned short qp[NW][CHV * 8]; // per-warp queue: tile positions of the unequal lanes
+  uint32_t priv[NPB_MAX * HALF];   // per-thread 16-bit counters, two threads per word
+  unsigned short qp[NW][CHV * 8];  // per-warp queue: tile positions of the unequal pairs
 };
 
 __device__ __forceinline__ void sacc_add(Smem& sm, int which, unsigned __int128 m, int e, bool neg) {
@@ -401,110 +376,6 @@ __device__ __forceinline__ void sacc_add_prod_f(Smem& sm, int which, float x, fl
   int ex, ey;
   uint32_t mx = split_float(x, ex), my = split_float(y, ey);
   sacc_add(sm, which, (unsigned __int128)((uint64_t)mx * my), ex + ey + sc, (x < 0) ^ (y < 0));
-}
-
-// ---------------------------------------------------------------------------
-// per-thread hot state (registers)
-// ---------------------------------------------------------------------------
-struct Ctx {
-  Cold* cold;         // this thread's rare-path record
-  float rtol, atol;
-  uint32_t lb_shift;  // Lb << MB
-  uint32_t c0;        // 158 + Lexp: V = ((bits(|d|) << 8) | 2^31) >> (c0 - exponent(|d|))
-  uint32_t col, inc;  // private histogram column and increment
-};
-
-struct Hot {
-  uint32_t n_eq, n_win, n_within;
-  uint64_t P, N, Q;
-  float abs_f;         // best |d|: exact when abs_x, else a lower bound
-  float rel_f;         // filter: <= best rel
-  float rel_a, rel_g;  // best rel = rel_a / rel_g exactly when rel_x
-  uint32_t ulp_f;
-  bool abs_x, rel_x;
-  int64_t first_fin, first_ulp;
-};
-
-__device__ __forceinline__ void hot_init(Hot& h) {
-  h.n_eq = h.n_win = h.n_within = 0;
-  h.P = h.N = h.Q = 0;
-  h.abs_f = 0.0f;
-  h.rel_f = 0.0f;
-  h.rel_a = 0.0f;
-  h.rel_g = 1.0f;
-  h.ulp_f = 0;
-  h.abs_x = h.rel_x = true;
-  h.first_fin = h.first_ulp = -1;
-}
-
-__device__ __forceinline__ void cold_init(Cold& c) {
-  c.abs_hi = c.abs_lo = 0.0f;
-  c.rel_hi = c.rel_lo = 0.0f;
-  c.rel_g = 1.0f;
-  c.rel_f = 0.0f;
-  c.ulp = 0;
-  c.n_gw = c.n_gm = c.n_ga = c.n_gf = c.n_nf = c.n_geq = 0;
-  c.abs_sc = c.rel_sc = 0;
-  c.abs_idx = c.rel_idx = c.ulp_idx = -1;
-}
-
-// after the general path ran, refresh the hot copies from the cold records
-__device__ __forceinline__ void hot_reload(Hot& h, const Cold& c) {
-  h.abs_x = c.abs_lo == 0.0f && c.abs_sc == 0;
-  h.abs_f = (c.abs_lo < 0.0f && c.abs_sc == 0) ? nextafterf(c.abs_hi, 0.0f) : c.abs_hi;
-  // the integer ratio compare needs normal float32 operands
-  h.rel_x = c.rel_lo == 0.0f && c.rel_sc == 0 &&
-            (c.rel_idx < 0 || (c.rel_g >= 1.17549435e-38f && c.rel_hi >= 1.17549435e-38f));
-  h.rel_a = c.rel_hi;
-  h.rel_g = c.rel_g;
-  h.rel_f = c.rel_f;
-  h.ulp_f = c.ulp;
-}
-
-template <int DT>
-__device__ __forceinline__ void note_first(Hot& h, uint32_t G, uint32_t C, int64_t idx) {
-  using T = Tr<DT>;
-  uint32_t ag = G & T::MAG, ac = C & T::MAG;
-  if (h.first_fin < 0 && ag < T::INF && ac < T::INF) h.first_fin = idx;
-  if (h.first_ulp < 0 && ag <= T::INF && ac <= T::INF) h.first_ulp = idx;
-}
-
-// Exact maxima update for a window lane; idx exceeds every index this thread
-// has seen, so ties keep the current best.
-__device__ __forceinline__ void window_update(Hot& h, Cold& cd, float a, float ag, uint32_t u, int64_t idx) {
-  if (a > h.abs_f) {
-    bool gt = h.abs_x || cmp_mag(a, 0.0f, 0, cd.abs_hi, cd.abs_lo, cd.abs_sc) > 0;
-    if (gt) {
-      cd.abs_hi = a;
-      cd.abs_lo = 0.0f;
-      cd.abs_sc = 0;
-      cd.abs_idx = idx;
-      h.abs_f = a;
-      h.abs_x = true;
-    }
-  }
-  if (u > h.ulp_f) {
-    h.ulp_f = u;
-    cd.ulp = u;
-    cd.ulp_idx = idx;
-  }
-  float r = __fmul_rn(a, rcp_approx(ag));
-  if (r > h.rel_f) {
-    int c = h.rel_x ? cmp_ratio_f(a, ag, h.rel_a, h.rel_g)
-                    : cmp_rel_exact(a, 0.0f, 0, ag, cd.rel_hi, cd.rel_lo, cd.rel_sc, cd.rel_g);
-    if (c > 0) {
-      cd.rel_hi = a;
-      cd.rel_lo = 0.0f;
-      cd.rel_sc = 0;
-      cd.rel_g = ag;
-      cd.rel_idx = idx;
-      h.rel_a = a;
-      h.rel_g = ag;
-      h.rel_x = true;
-      h.rel_f = rel_filter(a, 0, ag);
-      cd.rel_f = h.rel_f;
-    }
-  }
 }
 
 // floor(log2(a / g)) for a = (hi + lo) 2^sc > 0 and g > 0 (float32 pair, any range)
@@ -628,66 +499,201 @@ __device__ __noinline__ void general_lane(Smem& sm, Cold& cd, uint32_t G, uint32
   sacc_add_prod_f(sm, 2, t, t, 2 * sc);
 }
 
-template <int DT>
-__device__ __forceinline__ void window_cand(Hot& h, Cold& cd, uint32_t G, uint32_t C, int64_t idx) {
-  float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
-  float a = fabsf(__fsub_rn(cf, gf)), ag = fabsf(gf);
-  uint32_t u = (uint32_t)abs((int32_t)C - (int32_t)G);
-  window_update(h, cd, a, ag, u, idx);
+// ---------------------------------------------------------------------------
+// per-thread window state (registers) and per-piece window constants
+// ---------------------------------------------------------------------------
+// Maxima of the window pairs this thread saw, in increasing index order (so a
+// tie keeps the earlier index).  Indices are offsets from the CTA's first
+// element.  The rel record keeps the ratio in normalised form, an / mg with
+// mg = |g| / 2^e(g) in [1, 2) and an = |d| / 2^e(g); it is turned back into
+// (|d|, |g|) from the element itself at the end of the piece.
+struct Lane {
+  float amax;
+  uint32_t aidx;
+  uint32_t umax, uidx;  // umax in the unit of ud (bf16: u * 2^16)
+  float ra, rm;
+  uint32_t ridx;
+  uint32_t sa, sn;      // this tile's sum of V, and of V over negative d
+  uint32_t within;      // window pairs within tolerance
+  uint32_t uneq;        // unequal pairs seen (the piece length minus them are bitwise equal)
+  uint64_t A, N, Q;     // this round's sums of V, V over negative d, V^2
+};
+
+struct Win {
+  float rtol, atol;
+  float gmin;       // smallest |g| of a window pair: 2^(Lb + 1 - BIAS)
+  float lim;        // |d| < 2^(Lexp + 22)
+  float M;          // 1.5 * 2^(Lexp + 23): bits(|d| + M) - bits(M) = |d| / 2^Lexp
+  uint32_t udmax;   // window bound on ud (u < 2^UB)
+  uint32_t base;    // shared address of this thread's counter in private row 0
+  uint32_t inc;     // 1 (low half of the word) or 65536 (high half)
+};
+
+__device__ __forceinline__ void lane_init(Lane& L) {
+  L.amax = 0.0f;
+  L.aidx = 0;
+  L.umax = L.uidx = 0;
+  L.ra = 0.0f;
+  L.rm = 1.0f;
+  L.ridx = 0;
+  L.sa = L.sn = 0;
+  L.within = L.uneq = 0;
+  L.A = L.N = L.Q = 0;
 }
 
-// bitmask of the lanes of a vector whose value is NaN or Inf
-template <int DT>
-__device__ __forceinline__ uint32_t nonfinite_mask(const uint4& v) {
-  using T = Tr<DT>;
-  if constexpr (T::BYTES == 2) {
-    constexpr uint32_t ADD = (0x8000u - T::INF) * 0x10001u;  // sets bit 15 of a half iff mag >= INF
-    uint32_t any = (((v.x & 0x7FFF7FFFu) + ADD) | ((v.y & 0x7FFF7FFFu) + ADD) | ((v.z & 0x7FFF7FFFu) + ADD) |
-                    ((v.w & 0x7FFF7FFFu) + ADD)) & 0x80008000u;
-    if (!any) return 0;
-  }
-  uint32_t m = 0;
-#pragma unroll
-  for (int j = 0; j < T::VEC; j++) m |= ((lane_bits<DT>(v, j) & T::MAG) >= T::INF ? 1u : 0u) << j;
-  return m;
+__device__ __forceinline__ void cold_init(Cold& c) {
+  c.abs_hi = c.abs_lo = 0.0f;
+  c.rel_hi = c.rel_lo = 0.0f;
+  c.rel_g = 1.0f;
+  c.rel_f = 0.0f;
+  c.ulp = 0;
+  c.n_gw = c.n_gm = c.n_ga = c.n_gf = c.n_nf = c.n_geq = 0;
+  c.abs_sc = c.rel_sc = 0;
+  c.abs_idx = c.rel_idx = c.ulp_idx = -1;
+  c.first_fin = c.first_ulp = -1;
 }
 
-// One unequal lane: the window fast path, or the general path.
+__device__ __forceinline__ void red_shared(uint32_t addr, uint32_t v) {
+  asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
 template <int DT>
-__device__ __forceinline__ void lane_proc(Hot& h, uint32_t G, uint32_t C, int64_t idx, const Ctx& cx, Smem& sm) {
+__device__ __forceinline__ void note_first(Cold& cd, uint32_t G, uint32_t C, int64_t idx) {
   using T = Tr<DT>;
-  const uint32_t ag = G & T::MAG, ac = C & T::MAG;
-  const uint32_t u = (uint32_t)abs((int32_t)C - (int32_t)G);  // ULP distance for same-sign pairs
-  uint32_t mg = ag, mc = ac;
-  if constexpr (DT == PEAT_F16) {  // subnormal steps equal binade 1's
-    mg = max(mg, 1u << T::MB);
-    mc = max(mc, 1u << T::MB);
-  }
-  bool ok = ((G ^ C) & T::SIGN) == 0 && u < (1u << T::UB) && ag != 0u && mg >= cx.lb_shift && mc >= cx.lb_shift;
-  const float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
-  const float s = __fsub_rn(cf, gf);
-  const float a = fabsf(s), agf = fabsf(gf);
-  const uint32_t ab = __float_as_uint(a);
-  const uint32_t sh = cx.c0 - (ab >> 23);
-  const float thr = __fmaf_rn(cx.rtol, agf, cx.atol);
-  ok = ok && (sh - 8u) <= 23u && a != thr;  // 1 <= V < 2^24; tolerance ties go to the general path
-  if (ok) {
-    h.n_win++;
-    h.n_within += a < thr ? 1u : 0u;
-    const int k = (int)(ab - __float_as_uint(agf)) >> 23;  // floor(log2(|d| / |g|))
-    uint32_t* uctr = u <= (uint32_t)NU ? &sm.priv[(u - 1) * HALF + cx.col] : &sm.ovf[u < 63u ? u : 63u];
-    atomicAdd(uctr, u <= (uint32_t)NU ? cx.inc : 1u);
-    atomicAdd(&sm.priv[(NU + k - Rows<DT>::KLO) * HALF + cx.col], cx.inc);
-    const uint32_t V = ((ab << 8) | 0x80000000u) >> sh;  // |d| / 2^Lexp, exact
-    if (s > 0.0f) h.P += V;
-    else h.N += V;
-    h.Q += (uint64_t)V * V;
-    if ((a > h.abs_f) | (u > h.ulp_f) | (__fmul_rn(a, rcp_approx(agf)) > h.rel_f))
-      window_update(h, *cx.cold, a, agf, u, idx);
+  uint32_t ag = G & T::MAG, ac = C & T::MAG;
+  if (cd.first_fin < 0 && ag < T::INF && ac < T::INF) cd.first_fin = idx;
+  if (cd.first_ulp < 0 && ag <= T::INF && ac <= T::INF) cd.first_ulp = idx;
+}
+
+// raw element bits from the form pair_proc receives (bf16: float32 bits)
+template <int DT>
+__device__ __forceinline__ uint32_t raw_of(uint32_t x) {
+  if constexpr (DT == PEAT_BF16) return x >> 16;
+  else return x;
+}
+
+// sign(an1 / m1 - an2 / m2) > 0 for the normalised ratios of window pairs
+template <int DT>
+__device__ __forceinline__ bool rel_greater(float an1, float m1, float an2, float m2) {
+  const float p = __fmul_rn(an1, m2), q = __fmul_rn(an2, m1);
+  if constexpr (DT == PEAT_F32) {
+    // an has at most UB + 2 significant bits, m 24: the products need an
+    // error term, which is exact (no underflow: both products exceed 2^-26)
+    const float ep = __fmaf_rn(an1, m2, -p), eq = __fmaf_rn(an2, m1, -q);
+    return p > q || (p == q && ep > eq);
   } else {
-    Cold& cd = *cx.cold;
-    general_lane<DT>(sm, cd, G, C, idx, cx.rtol, cx.atol);
-    hot_reload(h, cd);
+    // at most (UB + 2) + (MB + 1) <= 24 significant bits: both products exact
+    return p > q;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// one unequal pair
+// ---------------------------------------------------------------------------
+// private row layout: ULP bins 1..NU in rows 0..NU-1, ULP bin 63 in row NU,
+// log2-relative bin k in row NU + 1 + k - KLO
+constexpr uint32_t ROW_U63 = NU * ROWB;
+
+__device__ __forceinline__ void ulp_overflow_bin(uint32_t u, const Win& W, Smem& sm) {
+  if (u >= 63u) red_shared(W.base + ROW_U63, W.inc);
+  else atomicAdd(&sm.ovf[u], 1u);
+}
+
+// The window test.  gr, cr: raw bits (bf16: the float32 bits, i.e. raw << 16);
+// gf, cf: the values.  Also returns ud, s = c - g, a = |s| and thr.
+template <int DT>
+__device__ __forceinline__ bool in_window(uint32_t gr, uint32_t cr, float gf, float cf, const Win& W, uint32_t& ud,
+                                          float& s, float& a, float& thr) {
+  const uint32_t gb = __float_as_uint(gf), cb = __float_as_uint(cf);
+  {
+    const uint32_t dd = DT == PEAT_F16 ? cr - gr : cb - gb;
+    ud = (int32_t)dd < 0 ? 0u - dd : dd;  // ULP distance of a same-sign pair (bf16: scaled by 2^16)
+  }
+  s = __fsub_rn(cf, gf);
+  a = fabsf(s);
+  const float ag = fabsf(gf);
+  thr = __fmaf_rn(W.rtol, ag, W.atol);
+  return (int32_t)(gb ^ cb) >= 0 && ud < W.udmax && ag >= W.gmin && a < W.lim && a != thr;
+}
+
+// a pair outside the window: append its offset to the CTA's general list
+// (evaluated at the end of the piece; past GCAP entries the piece is rescanned)
+__device__ __forceinline__ void defer_pair(uint32_t li, Smem& sm) {
+  const uint32_t slot = atomicAdd(&sm.gn, 1u);
+  if (slot < (uint32_t)GCAP) sm.glist[slot] = li;
+}
+
+template <int DT>
+__device__ __forceinline__ void pair_proc(Lane& L, uint32_t gr, uint32_t cr, float gf, float cf, uint32_t li,
+                                          const Win& W, Smem& sm) {
+  uint32_t ud;
+  float s, a, thr;
+  if (in_window<DT>(gr, cr, gf, cf, W, ud, s, a, thr)) {
+    const uint32_t gb = __float_as_uint(gf);
+    L.within += a < thr ? 1u : 0u;
+    // |d| / |g| = an / mg with mg in [1, 2); floor(log2) from the bit patterns
+    const uint32_t ef = gb & 0x7F800000u;
+    const float an = __uint_as_float(__float_as_uint(a) - ef + 0x3F800000u);
+    const float mg = __uint_as_float((gb & 0x007FFFFFu) | 0x3F800000u);
+    const int k = (int)(__float_as_uint(an) - __float_as_uint(mg)) >> 23;
+    red_shared(W.base + (uint32_t)((NU + 1 - Rows<DT>::KLO + k) * ROWB), W.inc);
+    const uint32_t u = DT == PEAT_BF16 ? ud >> 16 : ud;
+    if (u <= (uint32_t)NU) red_shared(W.base + (u - 1) * ROWB, W.inc);
+    else ulp_overflow_bin(u, W, sm);
+    // exact sums in units of 2^Lexp
+    const uint32_t V = __float_as_uint(__fadd_rn(a, W.M)) - __float_as_uint(W.M);
+    L.sa += V;
+    L.sn += s < 0.0f ? V : 0u;
+    L.Q += (uint64_t)V * V;
+    // maxima (selects, no branches)
+    const bool pa = a > L.amax, pu = ud > L.umax, pr = rel_greater<DT>(an, mg, L.ra, L.rm);
+    L.amax = pa ? a : L.amax;
+    L.aidx = pa ? li : L.aidx;
+    L.umax = pu ? ud : L.umax;
+    L.uidx = pu ? li : L.uidx;
+    L.ra = pr ? an : L.ra;
+    L.rm = pr ? mg : L.rm;
+    L.ridx = pr ? li : L.ridx;
+  } else {
+    defer_pair(li, sm);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// tiles
+// ---------------------------------------------------------------------------
+// element j of a 16-byte vector: raw bits in the form pair_proc takes, and value
+template <int DT>
+__device__ __forceinline__ void elem(const uint4& v, int j, uint32_t& r, float& f) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  if constexpr (DT == PEAT_F32) {
+    r = w[j];
+    f = __uint_as_float(r);
+  } else if constexpr (DT == PEAT_BF16) {
+    const uint32_t x = w[j >> 1];
+    r = (j & 1) ? (x & 0xFFFF0000u) : (x << 16);
+    f = __uint_as_float(r);
+  } else {
+    const uint32_t x = w[j >> 1];
+    const __half2 h = *reinterpret_cast<const __half2*>(&x);
+    r = (j & 1) ? (x >> 16) : (x & 0xFFFFu);
+    f = (j & 1) ? __high2float(h) : __low2float(h);
+  }
+}
+
+// element at position pos of a staged tile
+template <int DT>
+__device__ __forceinline__ void elem_at(const uint4* t, uint32_t pos, uint32_t& r, float& f) {
+  if constexpr (DT == PEAT_F32) {
+    r = reinterpret_cast<const uint32_t*>(t)[pos];
+    f = __uint_as_float(r);
+  } else if constexpr (DT == PEAT_BF16) {
+    r = (uint32_t)reinterpret_cast<const unsigned short*>(t)[pos] << 16;
+    f = __uint_as_float(r);
+  } else {
+    const unsigned short x = reinterpret_cast<const unsigned short*>(t)[pos];
+    r = x;
+    f = __half2float(__ushort_as_half(x));
   }
 }
 
@@ -731,21 +737,18 @@ __device__ __forceinline__ uint32_t unequal_mask(const uint4& g, const uint4& c)
 // Equal lanes of one vector: every bitwise-equal pair is EXACT; the ones
 // holding NaN/Inf also count as non-finite pairs.
 template <int DT>
-__device__ __forceinline__ void count_equal(Hot& h, const uint4& g, uint32_t eqm, int64_t base, Cold& cd) {
-  h.n_eq += __popc(eqm);
-  if (eqm && any_nonfinite<DT>(g)) {
-    const uint32_t nf = nonfinite_lanes<DT>(g) & eqm;
-    cd.n_nf += __popc(nf);
-  }
-  (void)base;
+__device__ __forceinline__ void count_equal(const uint4& g, uint32_t eqm, Cold& cd) {
+  if (eqm && any_nonfinite<DT>(g)) cd.n_nf += __popc(nonfinite_lanes<DT>(g) & eqm);
 }
 
 // One warp tile of CHV vectors staged in shared memory: lane L owns vectors L
-// and L + 32.  Equal lanes are counted in place; unequal lanes are queued (in
-// element order) and processed 32 at a time, so every thread does useful work.
+// and L + 32; tile element e sits at offset tli + e from the CTA's first
+// element.  Equal pairs are counted in place.  When most pairs differ, each
+// lane processes its own unequal pairs; otherwise they are queued (in element
+// order) and processed 32 at a time, so every thread does useful work.
 template <int DT>
-__device__ __forceinline__ void do_tile(Hot& h, const uint4* gt, const uint4* ct, int nvalid, int64_t tile_base,
-                                        const Ctx& cx, Smem& sm) {
+__device__ __forceinline__ void do_tile(Lane& L, const uint4* gt, const uint4* ct, int nvalid, uint32_t tli,
+                                        const Win& W, Smem& sm) {
   using T = Tr<DT>;
   constexpr int VEC = T::VEC;
   constexpr uint32_t FULL = (1u << VEC) - 1u;
@@ -754,69 +757,119 @@ __device__ __forceinline__ void do_tile(Hot& h, const uint4* gt, const uint4* ct
   const uint4 z = make_uint4(0, 0, 0, 0);
   const uint4 gA = okA ? gt[lane] : z, cA = okA ? ct[lane] : z;
   const uint4 gB = okB ? gt[lane + 32] : z, cB = okB ? ct[lane + 32] : z;
-  const int64_t baseA = tile_base + (int64_t)lane * VEC, baseB = baseA + 32 * VEC;
-  if ((h.first_fin | h.first_ulp) < 0) {
+  const uint32_t liA = tli + (uint32_t)(lane * VEC), liB = liA + 32 * VEC;
+  Cold& cd = sm.cold[threadIdx.x];
+  if ((cd.first_fin | cd.first_ulp) < 0) {
+    const int64_t lo = sm.lo;
     if (okA)
-      for (int j = 0; j < VEC; j++) note_first<DT>(h, lane_bits<DT>(gA, j), lane_bits<DT>(cA, j), baseA + j);
+      for (int j = 0; j < VEC; j++) note_first<DT>(cd, lane_bits<DT>(gA, j), lane_bits<DT>(cA, j), lo + liA + j);
     if (okB)
-      for (int j = 0; j < VEC; j++) note_first<DT>(h, lane_bits<DT>(gB, j), lane_bits<DT>(cB, j), baseB + j);
+      for (int j = 0; j < VEC; j++) note_first<DT>(cd, lane_bits<DT>(gB, j), lane_bits<DT>(cB, j), lo + liB + j);
   }
   const bool diff = ((gA.x ^ cA.x) | (gA.y ^ cA.y) | (gA.z ^ cA.z) | (gA.w ^ cA.w) | (gB.x ^ cB.x) | (gB.y ^ cB.y) |
                      (gB.z ^ cB.z) | (gB.w ^ cB.w)) != 0u;
-  Cold& cd = *cx.cold;
   if (!__any_sync(0xFFFFFFFFu, diff)) {  // the whole warp tile is bitwise equal
-    if (okA) count_equal<DT>(h, gA, FULL, baseA, cd);
-    if (okB) count_equal<DT>(h, gB, FULL, baseB, cd);
+    if (okA) count_equal<DT>(gA, FULL, cd);
+    if (okB) count_equal<DT>(gB, FULL, cd);
     return;
   }
   const uint32_t nA = okA ? unequal_mask<DT>(gA, cA) : 0u, nB = okB ? unequal_mask<DT>(gB, cB) : 0u;
-  if (okA) count_equal<DT>(h, gA, FULL & ~nA, baseA, cd);
-  if (okB) count_equal<DT>(h, gB, FULL & ~nB, baseB, cd);
-  // one scan of the packed counts gives the A-queue and B-queue offsets
-  const uint32_t packed = __popc(nA) | (__popc(nB) << 16);
-  uint32_t incl = packed;
+  if (okA) count_equal<DT>(gA, FULL & ~nA, cd);
+  if (okB) count_equal<DT>(gB, FULL & ~nB, cd);
+  const uint32_t mine = __popc(nA) + __popc(nB);
+  L.uneq += mine;
+  const uint32_t total = __reduce_add_sync(0xFFFFFFFFu, mine);
+  if (total * 16u >= 11u * (64u * VEC)) {
+    // dense: every lane works through its own unequal pairs
 #pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-    if (lane >= o) incl += t;
-  }
-  const uint32_t tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
-  const uint32_t totA = tot & 0xFFFFu, total = totA + (tot >> 16);
-  uint32_t posA = (incl & 0xFFFFu) - (packed & 0xFFFFu);
-  uint32_t posB = totA + (incl >> 16) - (packed >> 16);
-  unsigned short* q = sm.qp[warp];
+    for (int j = 0; j < VEC; j++)
+      if ((nA >> j) & 1u) {
+        uint32_t gr, cr;
+        float gf, cf;
+        elem<DT>(gA, j, gr, gf);
+        elem<DT>(cA, j, cr, cf);
+        pair_proc<DT>(L, gr, cr, gf, cf, liA + j, W, sm);
+      }
 #pragma unroll
-  for (int j = 0; j < VEC; j++) {
-    if ((nA >> j) & 1u) q[posA++] = (unsigned short)(lane * VEC + j);
-    if ((nB >> j) & 1u) q[posB++] = (unsigned short)((lane + 32) * VEC + j);
-  }
-  __syncwarp();
-  for (uint32_t e = lane; e < total; e += 32) {
-    const uint32_t pos = q[e];
-    uint32_t G, C;
-    if constexpr (T::BYTES == 2) {
-      G = reinterpret_cast<const unsigned short*>(gt)[pos];
-      C = reinterpret_cast<const unsigned short*>(ct)[pos];
-    } else {
-      G = reinterpret_cast<const uint32_t*>(gt)[pos];
-      C = reinterpret_cast<const uint32_t*>(ct)[pos];
+    for (int j = 0; j < VEC; j++)
+      if ((nB >> j) & 1u) {
+        uint32_t gr, cr;
+        float gf, cf;
+        elem<DT>(gB, j, gr, gf);
+        elem<DT>(cB, j, cr, cf);
+        pair_proc<DT>(L, gr, cr, gf, cf, liB + j, W, sm);
+      }
+  } else {
+    // sparse: queue the unequal positions; one scan of the packed counts
+    // gives the A-queue and B-queue offsets
+    const uint32_t packed = __popc(nA) | (__popc(nB) << 16);
+    uint32_t incl = packed;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane >= o) incl += t;
     }
-    lane_proc<DT>(h, G, C, tile_base + pos, cx, sm);
+    const uint32_t tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
+    const uint32_t totA = tot & 0xFFFFu;
+    uint32_t posA = (incl & 0xFFFFu) - (packed & 0xFFFFu);
+    uint32_t posB = totA + (incl >> 16) - (packed >> 16);
+    unsigned short* q = sm.qp[warp];
+#pragma unroll
+    for (int j = 0; j < VEC; j++) {
+      if ((nA >> j) & 1u) q[posA++] = (unsigned short)(lane * VEC + j);
+      if ((nB >> j) & 1u) q[posB++] = (unsigned short)((lane + 32) * VEC + j);
+    }
+    __syncwarp();
+    // two queue entries per iteration (e, e + 32: still in index order per lane)
+    for (uint32_t e = lane; e < total; e += 64) {
+      const uint32_t pos0 = q[e];
+      const bool two = e + 32 < total;
+      const uint32_t pos1 = two ? q[e + 32] : pos0;
+      uint32_t gr0, cr0, gr1, cr1;
+      float gf0, cf0, gf1, cf1;
+      elem_at<DT>(gt, pos0, gr0, gf0);
+      elem_at<DT>(ct, pos0, cr0, cf0);
+      elem_at<DT>(gt, pos1, gr1, gf1);
+      elem_at<DT>(ct, pos1, cr1, cf1);
+      pair_proc<DT>(L, gr0, cr0, gf0, cf0, tli + pos0, W, sm);
+      if (two) pair_proc<DT>(L, gr1, cr1, gf1, cf1, tli + pos1, W, sm);
+    }
+    __syncwarp();
   }
-  __syncwarp();
+  L.A += L.sa;
+  L.N += L.sn;
+  L.sa = L.sn = 0;
 }
 
-// one element outside the vector grid
+// one element outside the vector grid (li: offset from the CTA's first element)
 template <int DT>
-__device__ __forceinline__ void do_scalar(Hot& h, uint32_t G, uint32_t C, int64_t idx, const Ctx& cx, Smem& sm) {
+__device__ __forceinline__ void do_scalar(Lane& L, uint32_t G, uint32_t C, uint32_t li, const Win& W, Smem& sm) {
   using T = Tr<DT>;
-  if ((h.first_fin | h.first_ulp) < 0) note_first<DT>(h, G, C, idx);
+  Cold& cd = sm.cold[threadIdx.x];
+  if ((cd.first_fin | cd.first_ulp) < 0) note_first<DT>(cd, G, C, sm.lo + li);
   if (G == C) {
-    h.n_eq++;
-    if ((G & T::MAG) >= T::INF) cx.cold->n_nf++;
+    if ((G & T::MAG) >= T::INF) cd.n_nf++;
     return;
   }
-  lane_proc<DT>(h, G, C, idx, cx, sm);
+  L.uneq++;
+  uint32_t gr = G, cr = C;
+  float gf, cf;
+  if constexpr (DT == PEAT_F32) {
+    gf = __uint_as_float(G);
+    cf = __uint_as_float(C);
+  } else if constexpr (DT == PEAT_BF16) {
+    gr = G << 16;
+    cr = C << 16;
+    gf = __uint_as_float(gr);
+    cf = __uint_as_float(cr);
+  } else {
+    gf = __half2float(__ushort_as_half((unsigned short)G));
+    cf = __half2float(__ushort_as_half((unsigned short)C));
+  }
+  pair_proc<DT>(L, gr, cr, gf, cf, li, W, sm);
+  L.A += L.sa;
+  L.N += L.sn;
+  L.sa = L.sn = 0;
 }
 
 // ---------------------------------------------------------------------------
@@ -935,38 +988,73 @@ __device__ __forceinline__ uint64_t warp_sum64(uint64_t v) {
   return v;
 }
 
+// The general pairs of a piece [pb, pe), evaluated exactly by every thread of
+// the CTA: from the list when it held them all, else found again by a rescan
+// of the piece with the same window test.  Kept out of line so that the hot
+// loop carries no call.
+template <int DT>
+__device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p, int64_t pb, int64_t pe) {
+  __syncthreads();
+  const uint32_t n = sm.gn;
+  const int64_t lo = sm.lo;
+  Cold& cd = sm.cold[threadIdx.x];
+  if (n <= (uint32_t)GCAP) {
+    for (uint32_t e = threadIdx.x; e < n; e += BLOCK) {
+      const int64_t i = lo + sm.glist[e];
+      general_lane<DT>(sm, cd, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), i, W.rtol, W.atol);
+    }
+  } else {
+    for (int64_t i = pb + threadIdx.x; i < pe; i += BLOCK) {
+      const uint32_t G = load_scalar<DT>(p.g, i), C = load_scalar<DT>(p.c, i);
+      if (G == C) continue;
+      uint32_t gr = G, cr = C;
+      if constexpr (DT == PEAT_BF16) {
+        gr = G << 16;
+        cr = C << 16;
+      }
+      uint32_t ud;
+      float s, a, thr;
+      if (!in_window<DT>(gr, cr, to_f32<DT>(G), to_f32<DT>(C), W, ud, s, a, thr))
+        general_lane<DT>(sm, cd, G, C, i, W.rtol, W.atol);
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) sm.gn = 0;
+}
+
 // Fold the per-thread 16-bit histograms and the window sums into the CTA
 // totals.  All threads call it; it ends with the private counters zeroed.
 template <int DT>
-__device__ void fold_round(Hot& h, Smem& sm, int lexp) {
+__device__ void fold_round(Lane& L, Smem& sm, int lexp) {
   constexpr int NPB = Rows<DT>::NPB;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  // window sums: P, N < 2^40 and Q < 2^64 per thread per round; warp sums in 128 bits
-  uint64_t P = warp_sum64(h.P), N = warp_sum64(h.N);
-  uint64_t qlo = warp_sum64(h.Q & 0xFFFFFFFFull), qhi = warp_sum64(h.Q >> 32);
+  // window sums: A, N < 2^38 and Q < 2^60 per thread per round; warp sums in 128 bits
+  const uint64_t A = warp_sum64(L.A), N = warp_sum64(L.N);
+  const uint64_t qlo = warp_sum64(L.Q & 0xFFFFFFFFull), qhi = warp_sum64(L.Q >> 32);
   if (lane == 0) {
+    const uint64_t P = A - N;  // sum of V over positive d
     if (P >= N) sacc_add(sm, 0, (unsigned __int128)(P - N), lexp, false);
     else sacc_add(sm, 0, (unsigned __int128)(N - P), lexp, true);
-    sacc_add(sm, 1, (unsigned __int128)P + N, lexp, false);
+    sacc_add(sm, 1, (unsigned __int128)A, lexp, false);
     sacc_add(sm, 2, (unsigned __int128)qlo + ((unsigned __int128)qhi << 32), 2 * lexp, false);
   }
-  h.P = h.N = h.Q = 0;
+  L.A = L.N = L.Q = 0;
   __syncthreads();
-  // private histograms: one warp per row
-  for (int r = warp; r < NPB; r += BLOCK / 32) {
+  // private rows: one warp per row
+  for (int r = warp; r < NPB; r += NW) {
     uint32_t sum = 0;
     for (int w = lane; w < HALF; w += 32) {
-      uint32_t v = sm.priv[r * HALF + w];
+      const uint32_t v = sm.priv[r * HALF + w];
       sum += (v & 0xFFFFu) + (v >> 16);
       sm.priv[r * HALF + w] = 0;
     }
     sum = __reduce_add_sync(0xFFFFFFFFu, sum);
     if (lane == 0 && sum) {
-      int bin = r < NU ? 64 + r + 1 : 48 + (r - NU) + Rows<DT>::KLO;
+      const int bin = r < NU ? 64 + r + 1 : (r == NU ? 127 : 48 + Rows<DT>::KLO + (r - NU - 1));
       sm.hist[bin] += sum;
     }
   }
-  for (int b = threadIdx.x; b < 64; b += BLOCK) {  // ULP bins above NU
+  for (int b = threadIdx.x; b < 64; b += BLOCK) {  // ULP bins NU+1..62
     if (b > NU && sm.ovf[b]) sm.hist[64 + b] += sm.ovf[b];
     sm.ovf[b] = 0;
   }
@@ -976,15 +1064,31 @@ __device__ void fold_round(Hot& h, Smem& sm, int lexp) {
 // End of one segment piece: the integer totals go to the segment's
 // accumulator (global atomics), the maxima to the CTA's partial slot.
 template <int DT>
-__device__ void finish_piece(Hot& h, Cold& cd, Smem& sm, int lexp, Partial* out, SegAcc* acc) {
-  fold_round<DT>(h, sm, lexp);
+__device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, int lexp, const CompareParams& p,
+                                             int64_t pb, int64_t pe, Partial* out, SegAcc* acc) {
+  const int64_t plen = pe - pb;
+  run_general<DT>(W, sm, p, pb, pe);
+  fold_round<DT>(L, sm, lexp);
+  Cold& cd = sm.cold[threadIdx.x];
+  const int64_t lo = sm.lo;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t c[8] = {h.n_eq + cd.n_geq, h.n_win, h.n_within, cd.n_nf, cd.n_gw, cd.n_gm, cd.n_ga, cd.n_gf};
+  // window pairs = unequal pairs - general pairs (per warp: a warp runs the
+  // general pairs it deferred, so its difference is never negative); EXACT =
+  // the piece length - unequal pairs + general pairs found equal.  Per-thread
+  // terms wrap modulo 2^32; the CTA totals lie in [0, 2^31).
+  const uint32_t gen = cd.n_gw + cd.n_gm + cd.n_ga + cd.n_gf + cd.n_geq;
+  const uint32_t c[8] = {cd.n_geq - L.uneq + (threadIdx.x == 0 ? (uint32_t)plen : 0u), L.uneq - gen, L.within,
+                         cd.n_nf, cd.n_gw, cd.n_gm, cd.n_ga, cd.n_gf};
+  __shared__ uint32_t cnt32[8];
+  if (threadIdx.x < 8) cnt32[threadIdx.x] = 0;
+  __syncthreads();
 #pragma unroll
   for (int k = 0; k < 8; k++) {
-    uint32_t v = __reduce_add_sync(0xFFFFFFFFu, c[k]);
-    if (lane == 0 && v) atomicAdd(&sm.cnt[k], (unsigned long long)v);
+    const uint32_t v = __reduce_add_sync(0xFFFFFFFFu, c[k]);
+    if (lane == 0 && v) atomicAdd(&cnt32[k], v);
   }
+  __syncthreads();
+  if (threadIdx.x < 8) sm.cnt[threadIdx.x] += cnt32[threadIdx.x];
   Partial x;
   x.abs_hi = cd.abs_hi;
   x.abs_lo = cd.abs_lo;
@@ -998,20 +1102,41 @@ __device__ void finish_piece(Hot& h, Cold& cd, Smem& sm, int lexp, Partial* out,
   x.rel_idx = cd.rel_idx;
   x.ulp = cd.ulp;
   x.ulp_idx = cd.ulp_idx;
-  x.first_fin = h.first_fin;
-  x.first_ulp = h.first_ulp;
+  x.first_fin = cd.first_fin;
+  x.first_ulp = cd.first_ulp;
+  {
+    // the window records of this thread, as exact values
+    Partial w;
+    part_none(w);
+    if (L.amax > 0.0f) {
+      w.abs_hi = L.amax;
+      w.abs_idx = lo + L.aidx;
+    }
+    if (L.ra > 0.0f) {
+      const int64_t i = lo + L.ridx;
+      const float gf = to_f32<DT>(load_scalar<DT>(p.g, i)), cf = to_f32<DT>(load_scalar<DT>(p.c, i));
+      w.rel_hi = fabsf(__fsub_rn(cf, gf));
+      w.rel_g = fabsf(gf);
+      w.rel_idx = i;
+    }
+    if (L.umax > 0u) {
+      w.ulp = DT == PEAT_BF16 ? L.umax >> 16 : L.umax;
+      w.ulp_idx = lo + L.uidx;
+    }
+    part_merge(x, w);
+  }
   part_warp_reduce(x);
   if (lane == 0) sm.wbest[warp] = x;
   __syncthreads();
   if (threadIdx.x == 0) {
-    for (int w = 1; w < BLOCK / 32; w++) part_merge(x, sm.wbest[w]);
+    for (int w = 1; w < NW; w++) part_merge(x, sm.wbest[w]);
     *out = x;
   }
   for (int b = threadIdx.x; b < HBINS; b += BLOCK)
     if (sm.hist[b]) atomicAdd(&acc->hist[b], sm.hist[b]);
   if (threadIdx.x < 8 && sm.cnt[threadIdx.x]) atomicAdd(&acc->cnt[threadIdx.x], sm.cnt[threadIdx.x]);
   for (int j = threadIdx.x; j < NSUM * NLIMB; j += BLOCK) {
-    unsigned long long v = (&sm.sacc[0][0])[j];
+    const unsigned long long v = (&sm.sacc[0][0])[j];
     if (v) atomicAdd(reinterpret_cast<unsigned long long*>(&acc->limbs[0][0]) + j, v);
   }
   __syncthreads();
@@ -1019,7 +1144,7 @@ __device__ void finish_piece(Hot& h, Cold& cd, Smem& sm, int lexp, Partial* out,
   for (int b = threadIdx.x; b < HBINS; b += BLOCK) sm.hist[b] = 0;
   for (int j = threadIdx.x; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
   if (threadIdx.x < 8) sm.cnt[threadIdx.x] = 0;
-  hot_init(h);
+  lane_init(L);
   cold_init(cd);
   __syncthreads();
 }
@@ -1030,32 +1155,37 @@ __device__ void finish_piece(Hot& h, Cold& cd, Smem& sm, int lexp, Partial* out,
 template <int DT>
 __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
   using T = Tr<DT>;
+  using R = Rows<DT>;
   constexpr int VEC = T::VEC;
-  // lanes per thread per round stay below 2^16 (16-bit private counters): each
-  // warp tile gives a thread at most 2 VEC lanes
+  // pairs per thread per round stay below 2^16 (16-bit private counters): each
+  // warp tile gives a thread at most 2 VEC pairs
   constexpr int64_t ROUND_CHUNKS = (int64_t)NW * (65535 / (2 * VEC));
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int b = tid; b < HBINS; b += BLOCK) sm.hist[b] = 0;
   for (int j = tid; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
-  for (int j = tid; j < Rows<DT>::NPB * HALF; j += BLOCK) sm.priv[j] = 0;
+  for (int j = tid; j < R::NPB * HALF; j += BLOCK) sm.priv[j] = 0;
   if (tid < 8) sm.cnt[tid] = 0;
   if (tid < 64) sm.ovf[tid] = 0;
+  if (tid == 0) {
+    sm.gn = 0;
+    sm.glist = p.glist + (size_t)blockIdx.x * GCAP;
+  }
   if (lane == 0) {
     for (int st = 0; st < NSTAGE; st++) mbar_init(&sm.bar[warp][st], 1);
     mbar_init_fence();
   }
-  Ctx cx;
-  cx.cold = &sm.cold[tid];
-  cold_init(*cx.cold);
   const int64_t lo = p.bounds[blockIdx.x], hi = p.bounds[blockIdx.x + 1];
-  Hot h;
-  hot_init(h);
-  cx.rtol = p.rtol;
-  cx.atol = p.atol;
-  cx.col = tid & (HALF - 1);
-  cx.inc = tid < HALF ? 1u : 65536u;
+  if (tid == 0) sm.lo = lo;
+  Win W;
+  W.rtol = p.rtol;
+  W.atol = p.atol;
+  W.base = smem_addr(&sm.priv[tid & (HALF - 1)]);
+  W.inc = tid < HALF ? 1u : 65536u;
+  cold_init(sm.cold[tid]);
+  Lane L;
+  lane_init(L);
   __syncthreads();
   if (lo >= hi) return;
   uint32_t seq = 0;      // this warp's bulk-copy stage uses so far (stage = seq % NSTAGE)
@@ -1090,26 +1220,44 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
     const int64_t my_chunks = nchunk > warp ? (nchunk - warp + NW - 1) / NW : 0;
     if (lane == 0 && !failed)
       for (int64_t i = 0; i < NSTAGE && i < my_chunks; i++) issue(seq + (uint32_t)i, warp + NW * i);
-    // window of binades from the largest golden exponent in the first vectors
-    if (tid == 0) sm.lb = 0;
+    // the window from a sample of the piece: the largest finite golden
+    // exponent and the largest same-sign ULP distance of the first vectors
+    if (tid == 0) sm.lb = sm.ub = 0;
     __syncthreads();
     if (tid < nvec) {
-      uint4 gv = load_vec(p.g, (vb + (int64_t)tid * VEC) * T::BYTES);
-      uint32_t emax = 0;
+      const uint4 gv = load_vec(p.g, (vb + (int64_t)tid * VEC) * T::BYTES);
+      const uint4 cv = load_vec(p.c, (vb + (int64_t)tid * VEC) * T::BYTES);
+      uint32_t emax = 0, umax = 0;
 #pragma unroll
       for (int j = 0; j < VEC; j++) {
-        uint32_t e = (lane_bits<DT>(gv, j) & T::MAG) >> T::MB;
+        const uint32_t G = lane_bits<DT>(gv, j), C = lane_bits<DT>(cv, j);
+        const uint32_t e = (G & T::MAG) >> T::MB;
         if (e < (uint32_t)T::EMAX && e > emax) emax = e;
+        if (((G ^ C) & T::SIGN) == 0u && (G & T::MAG) < T::INF && (C & T::MAG) < T::INF) {
+          const uint32_t u = G > C ? G - C : C - G;
+          umax = u > umax ? u : umax;
+        }
       }
       atomicMax(&sm.lb, (int)emax);
+      atomicMax(&sm.ub, (int)(32 - __clz(umax)));
     }
     __syncthreads();
-    // V = |d| / 2^Lexp < 2^24 for u < 2^UB and golden binades up to 2 above the largest seen
-    int lb = sm.lb + T::UB - 22;
+    // u < 2^UB with one bit to spare over the sample; V = |d| / 2^Lexp < 2^22
+    // for such pairs with goldens up to 2 binades above the largest seen
+    int UB = sm.ub + 1;
+    UB = UB > T::UBMAX ? T::UBMAX : UB;
+    int lb = sm.lb + UB - 20;
     lb = lb < T::LBMIN ? T::LBMIN : (lb > T::LBMAX ? T::LBMAX : lb);
     const int lexp = lb - T::BIAS - T::MB;  // weight of V's unit
-    cx.lb_shift = (uint32_t)lb << T::MB;
-    cx.c0 = (uint32_t)(158 + lexp);
+    W.gmin = (DT == PEAT_F16 && lb == T::LBMIN) ? __uint_as_float((uint32_t)(127 - 24) << 23)
+                                                  : __uint_as_float((uint32_t)(lb + 1 - T::BIAS + 127) << 23);
+    W.lim = __uint_as_float((uint32_t)(lexp + 22 + 127) << 23);
+    W.M = __uint_as_float(((uint32_t)(lexp + 23 + 127) << 23) | 0x400000u);
+    W.udmax = (1u << UB) << (DT == PEAT_BF16 ? 16 : 0);
+    auto scalar_range = [&](int64_t b0, int64_t b1) {
+      for (int64_t i = b0 + tid; i < b1; i += BLOCK)
+        do_scalar<DT>(L, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), (uint32_t)(i - lo), W, sm);
+    };
     // scalar head: fewer than VEC elements, or the whole piece in scalar mode
     // (then in rounds of at most 65535 elements per thread)
     {
@@ -1117,9 +1265,8 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
       constexpr int64_t ROUND_ELEMS = (int64_t)BLOCK * 65535;
       for (int64_t r0 = pb; r0 < h_end; r0 += ROUND_ELEMS) {
         const int64_t r1 = min(h_end, r0 + ROUND_ELEMS);
-        for (int64_t i = r0 + tid; i < r1; i += BLOCK)
-          do_scalar<DT>(h, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), i, cx, sm);
-        if (r1 < h_end) fold_round<DT>(h, sm, lexp);
+        scalar_range(r0, r1);
+        if (r1 < h_end) fold_round<DT>(L, sm, lexp);
       }
     }
     // vector body: warp w takes chunks w, w + NW, ... of CHV vectors from its
@@ -1141,12 +1288,12 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
         if (!failed) {
           const int64_t v0 = k * CHV;
           const int nvalid = (int)min((int64_t)CHV, nvec - v0);
-          do_tile<DT>(h, sm.ring_g[warp][st], sm.ring_c[warp][st], nvalid, vb + v0 * VEC, cx, sm);
+          do_tile<DT>(L, sm.ring_g[warp][st], sm.ring_c[warp][st], nvalid, (uint32_t)(vb + v0 * VEC - lo), W, sm);
           if (lane == 0 && i + NSTAGE < my_chunks) issue(seq + NSTAGE, warp + NW * (i + NSTAGE));
         }
         seq++;
       }
-      if (r1 < nchunk) fold_round<DT>(h, sm, lexp);
+      if (r1 < nchunk) fold_round<DT>(L, sm, lexp);
     }
     if (fail_i >= 0) {
       // copies this warp issued but never consumed: wait for them before the
@@ -1156,11 +1303,9 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
         mbar_wait(&sm.bar[warp][sq % NSTAGE], (sq / NSTAGE) & 1u, DRAIN_LIMIT);
       }
     }
-    // scalar tail (fewer than VEC elements), after the body: lanes stay in index order
-    if (vb < ve && ve < pe)
-      for (int64_t e = ve + tid; e < pe; e += BLOCK)
-        do_scalar<DT>(h, load_scalar<DT>(p.g, e), load_scalar<DT>(p.c, e), e, cx, sm);
-    finish_piece<DT>(h, *cx.cold, sm, lexp, p.partials + s + blockIdx.x, p.acc + s);
+    // scalar tail (fewer than VEC elements), after the body: pairs stay in index order
+    if (vb < ve && ve < pe) scalar_range(ve, pe);
+    finish_piece<DT>(L, W, sm, lexp, p, pb, pe, p.partials + s + blockIdx.x, p.acc + s);
     pb = pe;
   }
 }
@@ -1169,14 +1314,17 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
 // stage 2: one CTA per segment: merge the maxima of the segment's pieces,
 // round the exact sums once, write the outputs, clear the accumulator
 // ---------------------------------------------------------------------------
-// RN64 of the quotient (hi + lo) 2^sc / g > 0: the candidate with the smallest
-// exact residual, ties to the even significand
+// RN64 of the quotient (hi + lo) 2^sc / g > 0.  When hi + lo is a binary64
+// number (always, unless lo is more than 29 binades below hi) the numerator
+// is exact and one correctly rounded division gives the answer; otherwise the
+// candidate with the smallest exact residual wins, ties to the even significand.
 __device__ double rel_value(float hi, float lo, int sc, float g) {
   if (hi == 0.0f) return 0.0;
   if (g == 0.0f) return __longlong_as_double(0x7FF0000000000000ll);
-  double num = __dadd_rn((double)hi, (double)lo) * (sc ? 2.0 : 1.0);
-  double q0 = __ddiv_rn(num, (double)g);  // within a few units of the exact quotient
-  double q = q0;
+  const double dh = hi, dl = lo;
+  const double num = __dadd_rn(dh, dl);
+  if (__dsub_rn(num, dh) == dl) return __ddiv_rn(sc ? num * 2.0 : num, (double)g);
+  double q = __ddiv_rn(sc ? num * 2.0 : num, (double)g);  // within a few units of the exact quotient
   for (int i = 0; i < 3; i++) q = nextafter(q, 0.0);
   double best = q;
   XAcc bres;
@@ -1196,10 +1344,67 @@ __device__ double rel_value(float hi, float lo, int sc, float g) {
     int c = 0;
     for (int j = NLIMB - 1; j >= 0 && c == 0; j--)
       if (r.d[j] != bres.d[j]) c = r.d[j] > bres.d[j] ? 1 : -1;
-    bool qeven = (__double_as_longlong(q) & 1) == 0, beven = (__double_as_longlong(best) & 1) == 0;
+    const bool qeven = (__double_as_longlong(q) & 1) == 0, beven = (__double_as_longlong(best) & 1) == 0;
     if (c < 0 || (c == 0 && qeven && !beven)) best = q, bres = r;
   }
   return best;
+}
+
+// RN-even binary64 of the exact value of NLIMB carry-save digits (digit j
+// weighs 2^(32 j + LIMB_LSB)).  Loops are unrolled with constant indices so
+// the digits stay in registers.
+__device__ double limbs_to_double(const long long* src) {
+  int64_t d[NLIMB];
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++) d[j] = src[j];
+  // carry-propagate: digits 0..NLIMB-2 into [0, 2^32), the top digit signed
+  int64_t carry = 0;
+#pragma unroll
+  for (int j = 0; j < NLIMB - 1; j++) {
+    const int64_t v = d[j] + carry;
+    carry = v >> 32;
+    d[j] = v & 0xFFFFFFFFll;
+  }
+  d[NLIMB - 1] += carry;
+  const bool neg = d[NLIMB - 1] < 0;
+  if (neg) {
+    carry = 0;
+#pragma unroll
+    for (int j = 0; j < NLIMB - 1; j++) {
+      const int64_t v = -d[j] + carry;
+      carry = v >> 32;
+      d[j] = v & 0xFFFFFFFFll;
+    }
+    d[NLIMB - 1] = -d[NLIMB - 1] + carry;
+  }
+  // the top nonzero digit, the two below it, and a sticky bit for the rest
+  int top = -1;
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++)
+    if (d[j] != 0) top = j;
+  if (top < 0) return 0.0;
+  uint64_t w2 = 0, w1 = 0, w0 = 0;
+  bool sticky = false;
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++) {
+    if (j == top) w2 = (uint64_t)d[j];
+    if (j == top - 1) w1 = (uint64_t)d[j];
+    if (j == top - 2) w0 = (uint64_t)d[j];
+    if (j < top - 2 && d[j] != 0) sticky = true;
+  }
+  // after normalisation every digit is below 2^32 (the sums stay below 2^352):
+  // W = w2 2^64 + w1 2^32 + w0 < 2^96, value = W 2^(32 (top - 2) + LIMB_LSB)
+  const int b = 31 - __clz((uint32_t)w2);  // leading one of w2
+  const unsigned __int128 W = ((unsigned __int128)w2 << 64) | ((unsigned __int128)w1 << 32) | w0;
+  const int shift = b + 1;                 // W >> shift has its leading one at bit 63
+  const uint64_t m = (uint64_t)(W >> shift);
+  if ((W & (((unsigned __int128)1 << shift) - 1)) != 0) sticky = true;
+  uint64_t mant = m >> 11;
+  const uint64_t rbits = m & 0x7FFull;
+  if (rbits > 0x400ull || (rbits == 0x400ull && (sticky || (mant & 1ull)))) mant++;
+  const int e = 11 + shift + 32 * (top - 2) + LIMB_LSB;
+  const double r = ldexp((double)mant, e);
+  return neg ? -r : r;
 }
 
 __global__ void __launch_bounds__(BLOCK) compare_stage2(CompareParams p) {
@@ -1222,11 +1427,11 @@ __global__ void __launch_bounds__(BLOCK) compare_stage2(CompareParams p) {
     acc->cnt[tid - HBINS] = 0;
   }
   if (tid >= 160 && tid < 160 + NSUM * NLIMB) {
-    int j = tid - 160;
+    const int j = tid - 160;
     (&limbs[0][0])[j] = (&acc->limbs[0][0])[j];
     (&acc->limbs[0][0])[j] = 0;
   }
-  // maxima over the segment's pieces, in CTA order
+  // maxima over the segment's pieces
   Partial x;
   part_none(x);
   if (s1 > s0) {
@@ -1237,11 +1442,7 @@ __global__ void __launch_bounds__(BLOCK) compare_stage2(CompareParams p) {
   part_warp_reduce(x);
   if (lane == 0) wbest[warp] = x;
   __syncthreads();
-  if (tid < NSUM) {
-    XAcc a;
-    for (int j = 0; j < NLIMB; j++) a.d[j] = limbs[tid][j];
-    sums[tid] = a.to_double();
-  }
+  if (tid < NSUM) sums[tid] = limbs_to_double(limbs[tid]);
   __syncthreads();
   if (tid == 0) {
     for (int w = 1; w < BLOCK / 32; w++) part_merge(x, wbest[w]);
@@ -1339,6 +1540,5 @@ cudaError_t compare_prepare() {
 int compare_ctas_per_sm() { return 2; }
 size_t compare_partial_bytes() { return sizeof(Partial); }
 size_t compare_segacc_bytes() { return sizeof(SegAcc); }
-size_t compare_cold_bytes() { return sizeof(Cold) * BLOCK; }
 
 }  // namespace peat

@@ -21,7 +21,7 @@ struct peat_handle_s {
   // compare workspace
   peat::Partial* partials = nullptr;
   peat::SegAcc* acc = nullptr;   // per-segment integer totals, zero between calls
-  void* cold = nullptr;          // per-thread rare-path records of stage 1
+  uint32_t* glist = nullptr;      // per-CTA lists of general-path pairs (stage 1 scratch)
   unsigned int* status_host = nullptr;  // mapped pinned error word written by the kernels
   unsigned int* status_dev = nullptr;
   unsigned int wait_limit = 1u << 24;   // polls before a pipeline wait gives up
@@ -122,9 +122,12 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
     p.p0 = (int64_t)(((16 - ag % 16) % 16) / B);
   else
     p.p0 = -1;
-  // persistent grid; small inputs get about one CTA per 32K elements
-  int64_t want = (n + 32767) / 32768;
+  // persistent grid; small inputs get about one CTA per 4K elements
+  int64_t want = (n + 4095) / 4096;
   p.nctas = (int)std::max<int64_t>(1, std::min<int64_t>(h->max_ctas, want));
+  // stage 1 keeps element offsets within a CTA's range in 32 bits
+  if (n / p.nctas >= ((int64_t)1 << 31) - 64)
+    return fail(h, PEAT_ERR_UNSUPPORTED, "n is too large for one call (more than 2^31 elements per CTA)");
 
   peat_status_t ps = wait_staging(h);
   if (ps != PEAT_OK) return ps;
@@ -141,7 +144,7 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   p.bounds = h->d_offsets + nseg + 1;
   p.acc = h->acc;
   p.partials = h->partials;
-  p.cold = h->cold;
+  p.glist = h->glist;
   p.status = h->status_dev;
   p.wait_limit = h->wait_limit;
   p.rtol = rtol;
@@ -248,7 +251,7 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
   size_t acc_bytes = (size_t)h->max_segments * peat::compare_segacc_bytes();
   bool ok = cudaMalloc(&h->partials, slots * peat::compare_partial_bytes()) == cudaSuccess &&
             cudaMalloc(&h->acc, acc_bytes) == cudaSuccess &&
-            cudaMalloc(&h->cold, (size_t)h->max_ctas * peat::compare_cold_bytes()) == cudaSuccess &&
+            cudaMalloc(&h->glist, sizeof(uint32_t) * (size_t)peat::GCAP * (size_t)h->max_ctas) == cudaSuccess &&
             cudaHostAlloc((void**)&h->status_host, sizeof(unsigned int), cudaHostAllocMapped) == cudaSuccess &&
             cudaHostGetDevicePointer((void**)&h->status_dev, h->status_host, 0) == cudaSuccess &&
             cudaMemset(h->acc, 0, acc_bytes) == cudaSuccess &&
@@ -274,7 +277,7 @@ peat_status_t peat_signature_destroy(peat_handle_t h) {
     cudaDeviceSynchronize();
     if (h->partials) cudaFree(h->partials);
     if (h->acc) cudaFree(h->acc);
-    if (h->cold) cudaFree(h->cold);
+    if (h->glist) cudaFree(h->glist);
     if (h->status_host) cudaFreeHost(h->status_host);
     if (h->d_offsets) cudaFree(h->d_offsets);
     if (h->h_offsets) cudaFreeHost(h->h_offsets);

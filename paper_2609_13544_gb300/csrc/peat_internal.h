@@ -17,6 +17,7 @@ constexpr int LIMB_LSB = -416;
 constexpr int NSUM = 3;  // 0: sum d, 1: sum |d|, 2: sum d^2
 
 constexpr int BLOCK = 256;    // threads per compare CTA
+constexpr int GCAP = 16384;   // general-path pairs a CTA lists per segment piece (more: the piece is rescanned)
 constexpr int HBINS = 128;    // 64 rel bins + 64 ULP bins
 
 // Exact maxima of one CTA piece (element indices are global).  |d| is kept
@@ -60,7 +61,7 @@ struct CompareParams {
   int nctas;
   Partial* partials;       // nseg + nctas slots; slot s + b holds CTA b's part of segment s
   SegAcc* acc;             // nseg accumulators, all zero between calls
-  void* cold;              // per-thread rare-path state, nctas * BLOCK records
+  uint32_t* glist;         // nctas * GCAP offsets: each CTA's general pairs of the current piece
   unsigned int* status;    // device-visible error word (bit 0: a bounded wait expired)
   unsigned int wait_limit; // iteration bound of a pipeline wait (0: give up at once, for tests)
   float rtol, atol;        // float32 tolerances
@@ -77,7 +78,6 @@ cudaError_t compare_prepare();
 int64_t compare_cta_bound(int dtype, int64_t b, int nctas, int64_t n, int64_t p0);
 size_t compare_partial_bytes();
 size_t compare_segacc_bytes();
-size_t compare_cold_bytes();  // per CTA
 
 struct InjectElemParams {
   void* dst;

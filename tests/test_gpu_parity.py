@@ -55,6 +55,15 @@ def test_noise_ragged_large(peat_gpu, oracle, h, dtype):
 
 
 @pytest.mark.parametrize("dtype", DTYPES)
+def test_general_pairs_beyond_the_list(peat_gpu, oracle, h, dtype):
+    """Random bit patterns: most pairs leave the window, so every CTA piece
+    holds more general pairs than its list (16384) and is rescanned."""
+    n = 12_000_017
+    gb, cb = random_pairs(dtype, n, seed=4242)
+    check_pair(peat_gpu, oracle, h, gb, cb, dtype, 1e-3, 0.0, ctx=f"{dtype} rescan")
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
 @pytest.mark.parametrize("offs", [(1, 1), (3, 3), (1, 2), (0, 5)])
 def test_misaligned_bases(peat_gpu, oracle, h, dtype, offs):
     gb, cb = noise_pairs(dtype, 50021, seed=11, rel=1e-2)

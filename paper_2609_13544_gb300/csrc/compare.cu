@@ -74,19 +74,19 @@ struct Tr<PEAT_BF16> {
 };
 
 // Private per-thread histogram rows (16-bit counters, two threads per word):
-// ULP bins 1..NU, then ULP bin 63, then the log2-relative bins window pairs
-// reach, k in [KLO, KHI] (fp16 goldens may be subnormal, whose ratios reach
-// 2^(MB-1)).  ULP bins NU+1..62 use CTA-wide shared counters.
-constexpr int NU = 15;
+// ULP bins 1..63 in rows 0..62, then the log2-relative bins window pairs
+// reach, k in [KLO, KHI] in rows 63 + k - KLO (fp16 goldens may be subnormal,
+// whose ratios reach 2^(MB-1)).
+constexpr int NUR = 63;  // ULP rows
 template <int DT>
 struct Rows {
   static constexpr int KLO = -(Tr<DT>::MB + 1);
   static constexpr int KHI = DT == PEAT_F16 ? Tr<DT>::MB - 1 : Tr<DT>::UBMAX - Tr<DT>::MB;
-  static constexpr int NPB = NU + 1 + KHI - KLO + 1;
+  static constexpr int NPB = NUR + KHI - KLO + 1;
 };
 constexpr int HALF = BLOCK / 2;
 constexpr int ROWB = HALF * 4;  // bytes per private row
-constexpr int NPB_MAX = NU + 1 + 9 + 11 + 1;
+constexpr int NPB_MAX = NUR + 9 + 11 + 1;
 
 template <int DT>
 __device__ __forceinline__ float to_f32(uint32_t b) {
@@ -282,7 +282,7 @@ __device__ __forceinline__ int cmp_mag(float h1, float l1, int s1, float h2, flo
 }
 
 // sign(a1/g1 - a2/g2), a = (hi + lo) 2^sc >= 0, g >= 0; g = 0 < a means +inf
-__device__ int cmp_rel_exact(float h1, float l1, int s1, float g1, float h2, float l2, int s2, float g2) {
+__device__ __noinline__ int cmp_rel_exact(float h1, float l1, int s1, float g1, float h2, float l2, int s2, float g2) {
   int k1 = h1 == 0.0f ? 0 : (g1 == 0.0f ? 2 : 1);
   int k2 = h2 == 0.0f ? 0 : (g2 == 0.0f ? 2 : 1);
   if (k1 != k2) return k1 > k2 ? 1 : -1;
@@ -324,18 +324,25 @@ __device__ __forceinline__ float rel_filter(float hi, int sc, float g) {
 // ---------------------------------------------------------------------------
 // shared memory
 // ---------------------------------------------------------------------------
-// Per-thread state of the general path: its class counters and its exact
-// maxima records (|d| as (hi + lo) 2^sc, see Partial).
-struct Cold {
+// Exact maxima records and class counters of the general path (|d| as
+// (hi + lo) 2^sc, see Partial); registers of run_general.
+struct GenRec {
   float abs_hi, abs_lo;
   float rel_hi, rel_lo, rel_g;
   float rel_f;  // filter of the rel best
   uint32_t ulp;
   uint32_t n_gw, n_gm, n_ga, n_gf, n_nf, n_geq;
   int abs_sc, rel_sc;
-  uint32_t pad;
   long long abs_idx, rel_idx, ulp_idx;
-  long long first_fin, first_ulp;  // lowest index of a finite pair / of a pair without NaN
+};
+
+// Maxima of the window pairs one thread evaluated exactly (offsets from the
+// CTA's first element; ties to the lower offset).  The rel record keeps the
+// ratio in normalised form an / mg with mg = |g| / 2^e(g) in [1, 2) and
+// an = |d| / 2^e(g).
+struct WinRec {
+  float amax, ra, rm;
+  uint32_t aidx, umax, uidx, ridx, pad;
 };
 
 // Per-warp staging ring for the bulk copies: NSTAGE stages, each one warp
@@ -352,12 +359,13 @@ struct __align__(128) Smem {
   unsigned long long sacc[NSUM][NLIMB];
   unsigned long long cnt[8];
   Partial wbest[NW];
-  int lb, ub;
   long long lo;                    // the CTA's first element
+  long long ff, fu;                // first finite pair, first pair without NaN (search result)
   uint32_t* glist;                 // this CTA's list of general pairs (offsets), GCAP entries
   uint32_t gn;                     // entries appended in this piece (may exceed GCAP)
-  uint32_t ovf[64];                // ULP bins NU+1..62 of window pairs (CTA-wide)
-  Cold cold[BLOCK];
+  uint32_t nfe;                    // bitwise-equal pairs holding NaN or Inf
+  int lb, ub;
+  WinRec rec[BLOCK];
   uint32_t priv[NPB_MAX * HALF];   // per-thread 16-bit counters, two threads per word
   unsigned short qp[NW][CHV * 8];  // per-warp queue: tile positions of the unequal pairs
 };
@@ -395,7 +403,7 @@ __device__ int log2_ratio(float hi, float lo, int sc, float g) {
 
 // The general path: the definitions evaluated exactly, for any pair.
 template <int DT>
-__device__ __noinline__ void general_lane(Smem& sm, Cold& cd, uint32_t G, uint32_t C, int64_t idx, float rtol,
+__device__ __forceinline__ void general_lane(Smem& sm, GenRec& cd, uint32_t G, uint32_t C, int64_t idx, float rtol,
                                           float atol) {
   using T = Tr<DT>;
   uint32_t ag_m = G & T::MAG, ac_m = C & T::MAG;
@@ -500,23 +508,22 @@ __device__ __noinline__ void general_lane(Smem& sm, Cold& cd, uint32_t G, uint32
 }
 
 // ---------------------------------------------------------------------------
-// per-thread window state (registers) and per-piece window constants
+// per-thread window state and per-piece window constants (registers)
 // ---------------------------------------------------------------------------
-// Maxima of the window pairs this thread saw, in increasing index order (so a
-// tie keeps the earlier index).  Indices are offsets from the CTA's first
-// element.  The rel record keeps the ratio in normalised form, an / mg with
-// mg = |g| / 2^e(g) in [1, 2) and an = |d| / 2^e(g); it is turned back into
-// (|d|, |g|) from the element itself at the end of the piece.
 struct Lane {
-  float amax;
-  uint32_t aidx;
-  uint32_t umax, uidx;  // umax in the unit of ud (bf16: u * 2^16)
-  float ra, rm;
-  uint32_t ridx;
-  uint32_t sa, sn;      // this tile's sum of V, and of V over negative d
-  uint32_t within;      // window pairs within tolerance
-  uint32_t uneq;        // unequal pairs seen (the piece length minus them are bitwise equal)
-  uint64_t A, N, Q;     // this round's sums of V, V over negative d, V^2
+  uint32_t sa, sn;   // this tile's sum of V, and of V over negative d
+  uint32_t within;   // window pairs within tolerance
+  uint32_t uneq;     // unequal pairs seen (the rest of the piece is bitwise equal)
+  uint64_t A, N, Q;  // this round's sums of V, of V over negative d, of V^2
+};
+
+// This thread's window maxima so far (its pairs come in increasing index
+// order): a later pair at or below them cannot be a maximum of the piece, so
+// only pairs strictly above one of them are evaluated exactly.
+struct Thr {
+  float ta;       // |d|
+  uint32_t tu;    // ud
+  float tra, trm; // ratio tra / trm
 };
 
 struct Win {
@@ -530,18 +537,24 @@ struct Win {
 };
 
 __device__ __forceinline__ void lane_init(Lane& L) {
-  L.amax = 0.0f;
-  L.aidx = 0;
-  L.umax = L.uidx = 0;
-  L.ra = 0.0f;
-  L.rm = 1.0f;
-  L.ridx = 0;
   L.sa = L.sn = 0;
   L.within = L.uneq = 0;
   L.A = L.N = L.Q = 0;
 }
-
-__device__ __forceinline__ void cold_init(Cold& c) {
+__device__ __forceinline__ void thr_init(Thr& T) {
+  T.ta = 0.0f;
+  T.tu = 0;
+  T.tra = 0.0f;
+  T.trm = 1.0f;
+}
+__device__ __forceinline__ void rec_init(WinRec& r) {
+  r.amax = r.ra = 0.0f;
+  r.rm = 1.0f;
+  r.aidx = r.uidx = r.ridx = 0xFFFFFFFFu;
+  r.umax = 0;
+  r.pad = 0;
+}
+__device__ __forceinline__ void gen_init(GenRec& c) {
   c.abs_hi = c.abs_lo = 0.0f;
   c.rel_hi = c.rel_lo = 0.0f;
   c.rel_g = 1.0f;
@@ -550,26 +563,10 @@ __device__ __forceinline__ void cold_init(Cold& c) {
   c.n_gw = c.n_gm = c.n_ga = c.n_gf = c.n_nf = c.n_geq = 0;
   c.abs_sc = c.rel_sc = 0;
   c.abs_idx = c.rel_idx = c.ulp_idx = -1;
-  c.first_fin = c.first_ulp = -1;
 }
 
 __device__ __forceinline__ void red_shared(uint32_t addr, uint32_t v) {
   asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-
-template <int DT>
-__device__ __forceinline__ void note_first(Cold& cd, uint32_t G, uint32_t C, int64_t idx) {
-  using T = Tr<DT>;
-  uint32_t ag = G & T::MAG, ac = C & T::MAG;
-  if (cd.first_fin < 0 && ag < T::INF && ac < T::INF) cd.first_fin = idx;
-  if (cd.first_ulp < 0 && ag <= T::INF && ac <= T::INF) cd.first_ulp = idx;
-}
-
-// raw element bits from the form pair_proc receives (bf16: float32 bits)
-template <int DT>
-__device__ __forceinline__ uint32_t raw_of(uint32_t x) {
-  if constexpr (DT == PEAT_BF16) return x >> 16;
-  else return x;
 }
 
 // sign(an1 / m1 - an2 / m2) > 0 for the normalised ratios of window pairs
@@ -590,30 +587,31 @@ __device__ __forceinline__ bool rel_greater(float an1, float m1, float an2, floa
 // ---------------------------------------------------------------------------
 // one unequal pair
 // ---------------------------------------------------------------------------
-// private row layout: ULP bins 1..NU in rows 0..NU-1, ULP bin 63 in row NU,
-// log2-relative bin k in row NU + 1 + k - KLO
-constexpr uint32_t ROW_U63 = NU * ROWB;
-
-__device__ __forceinline__ void ulp_overflow_bin(uint32_t u, const Win& W, Smem& sm) {
-  if (u >= 63u) red_shared(W.base + ROW_U63, W.inc);
-  else atomicAdd(&sm.ovf[u], 1u);
-}
 
 // The window test.  gr, cr: raw bits (bf16: the float32 bits, i.e. raw << 16);
-// gf, cf: the values.  Also returns ud, s = c - g, a = |s| and thr.
+// gf, cf: the values.  Also returns ud (the ULP distance, bf16: scaled by
+// 2^16), s = c - g, a = |s| and thr.  No sign test is needed: a pair of
+// opposite signs has ud >= 2^23 (bf16 scaled, float32) or >= 2^10 (fp16),
+// beyond every window bound.
 template <int DT>
 __device__ __forceinline__ bool in_window(uint32_t gr, uint32_t cr, float gf, float cf, const Win& W, uint32_t& ud,
                                           float& s, float& a, float& thr) {
-  const uint32_t gb = __float_as_uint(gf), cb = __float_as_uint(cf);
   {
-    const uint32_t dd = DT == PEAT_F16 ? cr - gr : cb - gb;
-    ud = (int32_t)dd < 0 ? 0u - dd : dd;  // ULP distance of a same-sign pair (bf16: scaled by 2^16)
+    const uint32_t dd = DT == PEAT_F16 ? cr - gr : __float_as_uint(cf) - __float_as_uint(gf);
+    ud = (int32_t)dd < 0 ? 0u - dd : dd;
   }
   s = __fsub_rn(cf, gf);
   a = fabsf(s);
   const float ag = fabsf(gf);
   thr = __fmaf_rn(W.rtol, ag, W.atol);
-  return (int32_t)(gb ^ cb) >= 0 && ud < W.udmax && ag >= W.gmin && a < W.lim && a != thr;
+  return ud < W.udmax && ag >= W.gmin && a < W.lim && a != thr;
+}
+
+// normalised ratio |d| / |g| = an / mg, mg in [1, 2)
+__device__ __forceinline__ void norm_ratio(float a, float gf, float& an, float& mg) {
+  const uint32_t gb = __float_as_uint(gf);
+  an = __uint_as_float(__float_as_uint(a) - (gb & 0x7F800000u) + 0x3F800000u);
+  mg = __uint_as_float((gb & 0x007FFFFFu) | 0x3F800000u);
 }
 
 // a pair outside the window: append its offset to the CTA's general list
@@ -623,45 +621,63 @@ __device__ __forceinline__ void defer_pair(uint32_t li, Smem& sm) {
   if (slot < (uint32_t)GCAP) sm.glist[slot] = li;
 }
 
+
+// Everything of one unequal pair except its maxima; returns whether the pair
+// lies strictly above one of the warp's maxima (it is then evaluated exactly
+// by rescan_pair).
 template <int DT>
-__device__ __forceinline__ void pair_proc(Lane& L, uint32_t gr, uint32_t cr, float gf, float cf, uint32_t li,
-                                          const Win& W, Smem& sm) {
+__device__ __forceinline__ bool pair_proc(Lane& L, const Thr& T, uint32_t gr, uint32_t cr, float gf, float cf,
+                                          uint32_t li, const Win& W, Smem& sm) {
   uint32_t ud;
   float s, a, thr;
-  if (in_window<DT>(gr, cr, gf, cf, W, ud, s, a, thr)) {
-    const uint32_t gb = __float_as_uint(gf);
-    L.within += a < thr ? 1u : 0u;
-    // |d| / |g| = an / mg with mg in [1, 2); floor(log2) from the bit patterns
-    const uint32_t ef = gb & 0x7F800000u;
-    const float an = __uint_as_float(__float_as_uint(a) - ef + 0x3F800000u);
-    const float mg = __uint_as_float((gb & 0x007FFFFFu) | 0x3F800000u);
-    const int k = (int)(__float_as_uint(an) - __float_as_uint(mg)) >> 23;
-    red_shared(W.base + (uint32_t)((NU + 1 - Rows<DT>::KLO + k) * ROWB), W.inc);
-    const uint32_t u = DT == PEAT_BF16 ? ud >> 16 : ud;
-    if (u <= (uint32_t)NU) red_shared(W.base + (u - 1) * ROWB, W.inc);
-    else ulp_overflow_bin(u, W, sm);
-    // exact sums in units of 2^Lexp
-    const uint32_t V = __float_as_uint(__fadd_rn(a, W.M)) - __float_as_uint(W.M);
-    L.sa += V;
-    L.sn += s < 0.0f ? V : 0u;
-    L.Q += (uint64_t)V * V;
-    // maxima (selects, no branches)
-    const bool pa = a > L.amax, pu = ud > L.umax, pr = rel_greater<DT>(an, mg, L.ra, L.rm);
-    L.amax = pa ? a : L.amax;
-    L.aidx = pa ? li : L.aidx;
-    L.umax = pu ? ud : L.umax;
-    L.uidx = pu ? li : L.uidx;
-    L.ra = pr ? an : L.ra;
-    L.rm = pr ? mg : L.rm;
-    L.ridx = pr ? li : L.ridx;
-  } else {
+  if (!in_window<DT>(gr, cr, gf, cf, W, ud, s, a, thr)) {
     defer_pair(li, sm);
+    return false;
+  }
+  L.within += a < thr ? 1u : 0u;
+  float an, mg;
+  norm_ratio(a, gf, an, mg);
+  const int k = (int)(__float_as_uint(an) - __float_as_uint(mg)) >> 23;  // floor(log2(|d| / |g|))
+  red_shared(W.base + (uint32_t)((NUR - Rows<DT>::KLO + k) * ROWB), W.inc);
+  const uint32_t u = min(DT == PEAT_BF16 ? ud >> 16 : ud, (uint32_t)NUR);  // ULP bin, 63 = 63 or more
+  red_shared(W.base + (u - 1) * ROWB, W.inc);
+  // exact sums in units of 2^Lexp
+  const uint32_t V = __float_as_uint(__fadd_rn(a, W.M)) - __float_as_uint(W.M);
+  L.sa += V;
+  L.sn += s < 0.0f ? V : 0u;
+  L.Q += (uint64_t)V * V;
+  return (a > T.ta) | (ud > T.tu) | rel_greater<DT>(an, mg, T.tra, T.trm);
+}
+
+// a candidate pair (a window pair strictly above one of this thread's maxima,
+// later in index than all of them): update the exact records and thresholds
+template <int DT>
+__device__ __forceinline__ void rescan_pair(uint32_t gr, uint32_t cr, float gf, float cf, uint32_t li, const Win& W,
+                                            WinRec& r, Thr& T) {
+  uint32_t ud;
+  float s, a, thr;
+  in_window<DT>(gr, cr, gf, cf, W, ud, s, a, thr);
+  float an, mg;
+  norm_ratio(a, gf, an, mg);
+  if (a > T.ta) {
+    T.ta = a;
+    r.amax = a;
+    r.aidx = li;
+  }
+  if (ud > T.tu) {
+    T.tu = ud;
+    r.umax = ud;
+    r.uidx = li;
+  }
+  if (rel_greater<DT>(an, mg, T.tra, T.trm)) {
+    T.tra = an;
+    T.trm = mg;
+    r.ra = an;
+    r.rm = mg;
+    r.ridx = li;
   }
 }
 
-// ---------------------------------------------------------------------------
-// tiles
-// ---------------------------------------------------------------------------
 // element j of a 16-byte vector: raw bits in the form pair_proc takes, and value
 template <int DT>
 __device__ __forceinline__ void elem(const uint4& v, int j, uint32_t& r, float& f) {
@@ -737,118 +753,109 @@ __device__ __forceinline__ uint32_t unequal_mask(const uint4& g, const uint4& c)
 // Equal lanes of one vector: every bitwise-equal pair is EXACT; the ones
 // holding NaN/Inf also count as non-finite pairs.
 template <int DT>
-__device__ __forceinline__ void count_equal(const uint4& g, uint32_t eqm, Cold& cd) {
-  if (eqm && any_nonfinite<DT>(g)) cd.n_nf += __popc(nonfinite_lanes<DT>(g) & eqm);
+__device__ __forceinline__ void count_equal(const uint4& g, uint32_t eqm, Smem& sm) {
+  if (eqm && any_nonfinite<DT>(g)) atomicAdd(&sm.nfe, (uint32_t)__popc(nonfinite_lanes<DT>(g) & eqm));
 }
 
 // One warp tile of CHV vectors staged in shared memory: lane L owns vectors L
 // and L + 32; tile element e sits at offset tli + e from the CTA's first
-// element.  Equal pairs are counted in place.  When most pairs differ, each
-// lane processes its own unequal pairs; otherwise they are queued (in element
-// order) and processed 32 at a time, so every thread does useful work.
+// element.  Equal pairs are counted in place; unequal pairs are queued (in
+// element order) and processed 32 at a time, so every thread does useful
+// work.  Pairs above the warp's maxima are then evaluated exactly.
 template <int DT>
-__device__ __forceinline__ void do_tile(Lane& L, const uint4* gt, const uint4* ct, int nvalid, uint32_t tli,
-                                        const Win& W, Smem& sm) {
-  using T = Tr<DT>;
-  constexpr int VEC = T::VEC;
+__device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nvalid, uint32_t tli, const Win& W,
+                                        Smem& sm) {
+  // the candidate ring sits a fixed distance after the golden ring
+  const uint4* ct = gt + (offsetof(Smem, ring_c) - offsetof(Smem, ring_g)) / sizeof(uint4);
+  using Ty = Tr<DT>;
+  constexpr int VEC = Ty::VEC;
   constexpr uint32_t FULL = (1u << VEC) - 1u;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const bool okA = lane < nvalid, okB = lane + 32 < nvalid;
   const uint4 z = make_uint4(0, 0, 0, 0);
   const uint4 gA = okA ? gt[lane] : z, cA = okA ? ct[lane] : z;
   const uint4 gB = okB ? gt[lane + 32] : z, cB = okB ? ct[lane + 32] : z;
-  const uint32_t liA = tli + (uint32_t)(lane * VEC), liB = liA + 32 * VEC;
-  Cold& cd = sm.cold[threadIdx.x];
-  if ((cd.first_fin | cd.first_ulp) < 0) {
-    const int64_t lo = sm.lo;
-    if (okA)
-      for (int j = 0; j < VEC; j++) note_first<DT>(cd, lane_bits<DT>(gA, j), lane_bits<DT>(cA, j), lo + liA + j);
-    if (okB)
-      for (int j = 0; j < VEC; j++) note_first<DT>(cd, lane_bits<DT>(gB, j), lane_bits<DT>(cB, j), lo + liB + j);
-  }
   const bool diff = ((gA.x ^ cA.x) | (gA.y ^ cA.y) | (gA.z ^ cA.z) | (gA.w ^ cA.w) | (gB.x ^ cB.x) | (gB.y ^ cB.y) |
                      (gB.z ^ cB.z) | (gB.w ^ cB.w)) != 0u;
   if (!__any_sync(0xFFFFFFFFu, diff)) {  // the whole warp tile is bitwise equal
-    if (okA) count_equal<DT>(gA, FULL, cd);
-    if (okB) count_equal<DT>(gB, FULL, cd);
+    if (okA) count_equal<DT>(gA, FULL, sm);
+    if (okB) count_equal<DT>(gB, FULL, sm);
     return;
   }
   const uint32_t nA = okA ? unequal_mask<DT>(gA, cA) : 0u, nB = okB ? unequal_mask<DT>(gB, cB) : 0u;
-  if (okA) count_equal<DT>(gA, FULL & ~nA, cd);
-  if (okB) count_equal<DT>(gB, FULL & ~nB, cd);
-  const uint32_t mine = __popc(nA) + __popc(nB);
-  L.uneq += mine;
-  const uint32_t total = __reduce_add_sync(0xFFFFFFFFu, mine);
-  if (total * 16u >= 11u * (64u * VEC)) {
-    // dense: every lane works through its own unequal pairs
+  if (okA) count_equal<DT>(gA, FULL & ~nA, sm);
+  if (okB) count_equal<DT>(gB, FULL & ~nB, sm);
+  // queue the unequal positions; one scan of the packed counts gives the
+  // A-queue and B-queue offsets
+  const uint32_t packed = __popc(nA) | (__popc(nB) << 16);
+  uint32_t incl = packed;
 #pragma unroll
-    for (int j = 0; j < VEC; j++)
-      if ((nA >> j) & 1u) {
-        uint32_t gr, cr;
-        float gf, cf;
-        elem<DT>(gA, j, gr, gf);
-        elem<DT>(cA, j, cr, cf);
-        pair_proc<DT>(L, gr, cr, gf, cf, liA + j, W, sm);
-      }
-#pragma unroll
-    for (int j = 0; j < VEC; j++)
-      if ((nB >> j) & 1u) {
-        uint32_t gr, cr;
-        float gf, cf;
-        elem<DT>(gB, j, gr, gf);
-        elem<DT>(cB, j, cr, cf);
-        pair_proc<DT>(L, gr, cr, gf, cf, liB + j, W, sm);
-      }
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  const uint32_t tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
+  const uint32_t totA = tot & 0xFFFFu, total = totA + (tot >> 16);
+  L.uneq += __popc(nA) + __popc(nB);
+  uint32_t posA = (incl & 0xFFFFu) - (packed & 0xFFFFu);
+  uint32_t posB = totA + (incl >> 16) - (packed >> 16);
+  unsigned short* q = sm.qp[warp];
+  if (total * 4u <= 64u * VEC) {
+    // sparse tile: visit only the set bits
+    for (uint32_t m = nA; m; m &= m - 1u) q[posA++] = (unsigned short)(lane * VEC + __ffs(m) - 1);
+    for (uint32_t m = nB; m; m &= m - 1u) q[posB++] = (unsigned short)((lane + 32) * VEC + __ffs(m) - 1);
   } else {
-    // sparse: queue the unequal positions; one scan of the packed counts
-    // gives the A-queue and B-queue offsets
-    const uint32_t packed = __popc(nA) | (__popc(nB) << 16);
-    uint32_t incl = packed;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-      if (lane >= o) incl += t;
-    }
-    const uint32_t tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
-    const uint32_t totA = tot & 0xFFFFu;
-    uint32_t posA = (incl & 0xFFFFu) - (packed & 0xFFFFu);
-    uint32_t posB = totA + (incl >> 16) - (packed >> 16);
-    unsigned short* q = sm.qp[warp];
 #pragma unroll
     for (int j = 0; j < VEC; j++) {
       if ((nA >> j) & 1u) q[posA++] = (unsigned short)(lane * VEC + j);
       if ((nB >> j) & 1u) q[posB++] = (unsigned short)((lane + 32) * VEC + j);
     }
-    __syncwarp();
-    // two queue entries per iteration (e, e + 32: still in index order per lane)
-    for (uint32_t e = lane; e < total; e += 64) {
-      const uint32_t pos0 = q[e];
-      const bool two = e + 32 < total;
-      const uint32_t pos1 = two ? q[e + 32] : pos0;
-      uint32_t gr0, cr0, gr1, cr1;
-      float gf0, cf0, gf1, cf1;
-      elem_at<DT>(gt, pos0, gr0, gf0);
-      elem_at<DT>(ct, pos0, cr0, cf0);
-      elem_at<DT>(gt, pos1, gr1, gf1);
-      elem_at<DT>(ct, pos1, cr1, cf1);
-      pair_proc<DT>(L, gr0, cr0, gf0, cf0, tli + pos0, W, sm);
-      if (two) pair_proc<DT>(L, gr1, cr1, gf1, cf1, tli + pos1, W, sm);
-    }
-    __syncwarp();
+  }
+  __syncwarp();
+  // two queue entries per iteration (e, e + 32: in index order per lane);
+  // bit o of cm marks this lane's o-th entry as a maxima candidate
+  uint32_t cm = 0;
+  uint32_t ob = 1;
+  for (uint32_t e = lane; e < total; e += 64, ob <<= 2) {
+    const uint32_t pos0 = q[e];
+    const bool two = e + 32 < total;
+    const uint32_t pos1 = two ? q[e + 32] : pos0;
+    uint32_t gr0, cr0, gr1, cr1;
+    float gf0, cf0, gf1, cf1;
+    elem_at<DT>(gt, pos0, gr0, gf0);
+    elem_at<DT>(ct, pos0, cr0, cf0);
+    elem_at<DT>(gt, pos1, gr1, gf1);
+    elem_at<DT>(ct, pos1, cr1, cf1);
+    if (pair_proc<DT>(L, T, gr0, cr0, gf0, cf0, tli + pos0, W, sm)) cm |= ob;
+    if (two && pair_proc<DT>(L, T, gr1, cr1, gf1, cf1, tli + pos1, W, sm)) cm |= ob << 1;
   }
   L.A += L.sa;
   L.N += L.sn;
   L.sa = L.sn = 0;
+  if (cm) {
+    WinRec& r = sm.rec[threadIdx.x];
+    do {
+      const uint32_t o = __ffs(cm) - 1;
+      cm &= cm - 1u;
+      const uint32_t pos = q[lane + 32 * o];
+      uint32_t gr, cr;
+      float gf, cf;
+      elem_at<DT>(gt, pos, gr, gf);
+      elem_at<DT>(ct, pos, cr, cf);
+      rescan_pair<DT>(gr, cr, gf, cf, tli + pos, W, r, T);
+    } while (cm);
+  }
+  __syncwarp();
 }
 
-// one element outside the vector grid (li: offset from the CTA's first element)
+// one element outside the vector grid (li: offset from the CTA's first
+// element), with its maxima evaluated exactly
 template <int DT>
-__device__ __forceinline__ void do_scalar(Lane& L, uint32_t G, uint32_t C, uint32_t li, const Win& W, Smem& sm) {
-  using T = Tr<DT>;
-  Cold& cd = sm.cold[threadIdx.x];
-  if ((cd.first_fin | cd.first_ulp) < 0) note_first<DT>(cd, G, C, sm.lo + li);
+__device__ __forceinline__ void do_scalar(Lane& L, Thr& T, uint32_t G, uint32_t C, uint32_t li, const Win& W,
+                                          Smem& sm) {
+  using Ty = Tr<DT>;
   if (G == C) {
-    if ((G & T::MAG) >= T::INF) cd.n_nf++;
+    if ((G & Ty::MAG) >= Ty::INF) atomicAdd(&sm.nfe, 1u);
     return;
   }
   L.uneq++;
@@ -866,7 +873,7 @@ __device__ __forceinline__ void do_scalar(Lane& L, uint32_t G, uint32_t C, uint3
     gf = __half2float(__ushort_as_half((unsigned short)G));
     cf = __half2float(__ushort_as_half((unsigned short)C));
   }
-  pair_proc<DT>(L, gr, cr, gf, cf, li, W, sm);
+  if (pair_proc<DT>(L, T, gr, cr, gf, cf, li, W, sm)) rescan_pair<DT>(gr, cr, gf, cf, li, W, sm.rec[threadIdx.x], T);
   L.A += L.sa;
   L.N += L.sn;
   L.sa = L.sn = 0;
@@ -918,7 +925,7 @@ __device__ __forceinline__ int64_t min_idx(int64_t a, int64_t b) {
   return a < b ? a : b;
 }
 
-__device__ int cmp_rel_rec(float h1, float l1, int s1, float g1, float h2, float l2, int s2, float g2) {
+__device__ __forceinline__ int cmp_rel_rec(float h1, float l1, int s1, float g1, float h2, float l2, int s2, float g2) {
   const float tiny = 1.17549435e-38f;
   if (l1 == 0.0f && l2 == 0.0f && s1 == 0 && s2 == 0 && h1 >= tiny && h2 >= tiny && g1 >= tiny && g2 >= tiny)
     return cmp_ratio_f(h1, g1, h2, g2);
@@ -926,7 +933,7 @@ __device__ int cmp_rel_rec(float h1, float l1, int s1, float g1, float h2, float
 }
 
 // x <- the better of x and y, field by field; ties to the lower index
-__device__ void part_merge(Partial& x, const Partial& y) {
+__device__ __forceinline__ void part_merge(Partial& x, const Partial& y) {
   if (y.abs_idx >= 0) {
     int c = x.abs_idx < 0 ? 1 : cmp_mag(y.abs_hi, y.abs_lo, y.abs_sc, x.abs_hi, x.abs_lo, x.abs_sc);
     if (c > 0 || (c == 0 && y.abs_idx < x.abs_idx)) {
@@ -962,7 +969,7 @@ __device__ __forceinline__ float shfl_f(float v, int o) { return __shfl_down_syn
 __device__ __forceinline__ int shfl_int(int v, int o) { return __shfl_down_sync(0xFFFFFFFFu, v, o); }
 
 // warp tournament; lane 0 ends with the warp's best
-__device__ void part_warp_reduce(Partial& x) {
+__device__ __forceinline__ void part_warp_reduce(Partial& x) {
   const int lane = threadIdx.x & 31;
   for (int o = 16; o > 0; o >>= 1) {
     Partial y;
@@ -988,16 +995,36 @@ __device__ __forceinline__ uint64_t warp_sum64(uint64_t v) {
   return v;
 }
 
+// warp sums of the general path's class counters into the CTA counters
+__device__ __forceinline__ void gen_counts(const GenRec& g, Smem& sm) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t gen = g.n_gw + g.n_gm + g.n_ga + g.n_gf + g.n_geq;
+  const uint32_t c[7] = {g.n_geq, gen, g.n_nf, g.n_gw, g.n_gm, g.n_ga, g.n_gf};
+  uint32_t v[7];
+#pragma unroll
+  for (int k = 0; k < 7; k++) v[k] = __reduce_add_sync(0xFFFFFFFFu, c[k]);
+  if (lane == 0) {
+    if (v[0]) atomicAdd(&sm.cnt[0], (unsigned long long)v[0]);
+    if (v[1]) atomicAdd(&sm.cnt[1], 0ull - (unsigned long long)v[1]);  // general pairs are not window pairs
+    if (v[2]) atomicAdd(&sm.cnt[3], (unsigned long long)v[2]);
+    if (v[3]) atomicAdd(&sm.cnt[4], (unsigned long long)v[3]);
+    if (v[4]) atomicAdd(&sm.cnt[5], (unsigned long long)v[4]);
+    if (v[5]) atomicAdd(&sm.cnt[6], (unsigned long long)v[5]);
+    if (v[6]) atomicAdd(&sm.cnt[7], (unsigned long long)v[6]);
+  }
+}
+
 // The general pairs of a piece [pb, pe), evaluated exactly by every thread of
 // the CTA: from the list when it held them all, else found again by a rescan
-// of the piece with the same window test.  Kept out of line so that the hot
-// loop carries no call.
+// of the piece with the same window test.  Out of line, so that the hot loop
+// carries no call.  Leaves each warp's general maxima in sm.wbest[warp].
 template <int DT>
 __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p, int64_t pb, int64_t pe) {
   __syncthreads();
   const uint32_t n = sm.gn;
   const int64_t lo = sm.lo;
-  Cold& cd = sm.cold[threadIdx.x];
+  GenRec cd;
+  gen_init(cd);
   if (n <= (uint32_t)GCAP) {
     for (uint32_t e = threadIdx.x; e < n; e += BLOCK) {
       const int64_t i = lo + sm.glist[e];
@@ -1018,8 +1045,44 @@ __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p
         general_lane<DT>(sm, cd, G, C, i, W.rtol, W.atol);
     }
   }
+  gen_counts(cd, sm);
+  Partial x;
+  part_none(x);
+  x.abs_hi = cd.abs_hi;
+  x.abs_lo = cd.abs_lo;
+  x.abs_sc = cd.abs_sc;
+  x.abs_idx = cd.abs_idx;
+  x.rel_hi = cd.rel_hi;
+  x.rel_lo = cd.rel_lo;
+  x.rel_g = cd.rel_g;
+  x.rel_sc = cd.rel_sc;
+  x.rel_idx = cd.rel_idx;
+  x.ulp = cd.ulp;
+  x.ulp_idx = cd.ulp_idx;
+  part_warp_reduce(x);
+  if ((threadIdx.x & 31) == 0) sm.wbest[threadIdx.x >> 5] = x;
   __syncthreads();
   if (threadIdx.x == 0) sm.gn = 0;
+}
+
+// [pb, pe): the lowest index of a finite pair and of a pair without NaN
+// (the argmax when every error is zero), searched BLOCK elements at a time
+template <int DT>
+__device__ __noinline__ void first_pairs(Smem& sm, const CompareParams& p, int64_t pb, int64_t pe) {
+  using Ty = Tr<DT>;
+  constexpr long long NONE = 0x7FFFFFFFFFFFFFFFll;
+  if (threadIdx.x == 0) sm.ff = sm.fu = NONE;
+  for (int64_t base = pb;; base += BLOCK) {
+    __syncthreads();
+    if (base >= pe || (sm.ff != NONE && sm.fu != NONE)) break;
+    const int64_t i = base + threadIdx.x;
+    if (i < pe) {
+      const uint32_t ag = load_scalar<DT>(p.g, i) & Ty::MAG, ac = load_scalar<DT>(p.c, i) & Ty::MAG;
+      if (ag < Ty::INF && ac < Ty::INF) atomicMin(&sm.ff, (long long)i);
+      if (ag <= Ty::INF && ac <= Ty::INF) atomicMin(&sm.fu, (long long)i);
+    }
+  }
+  __syncthreads();
 }
 
 // Fold the per-thread 16-bit histograms and the window sums into the CTA
@@ -1050,87 +1113,80 @@ __device__ void fold_round(Lane& L, Smem& sm, int lexp) {
     }
     sum = __reduce_add_sync(0xFFFFFFFFu, sum);
     if (lane == 0 && sum) {
-      const int bin = r < NU ? 64 + r + 1 : (r == NU ? 127 : 48 + Rows<DT>::KLO + (r - NU - 1));
+      const int bin = r < NUR ? 64 + r + 1 : 48 + Rows<DT>::KLO + (r - NUR);
       sm.hist[bin] += sum;
     }
-  }
-  for (int b = threadIdx.x; b < 64; b += BLOCK) {  // ULP bins NU+1..62
-    if (b > NU && sm.ovf[b]) sm.hist[64 + b] += sm.ovf[b];
-    sm.ovf[b] = 0;
   }
   __syncthreads();
 }
 
-// End of one segment piece: the integer totals go to the segment's
+// End of one segment piece [pb, pe): the integer totals go to the segment's
 // accumulator (global atomics), the maxima to the CTA's partial slot.
 template <int DT>
 __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, int lexp, const CompareParams& p,
                                              int64_t pb, int64_t pe, Partial* out, SegAcc* acc) {
-  const int64_t plen = pe - pb;
   run_general<DT>(W, sm, p, pb, pe);
   fold_round<DT>(L, sm, lexp);
-  Cold& cd = sm.cold[threadIdx.x];
-  const int64_t lo = sm.lo;
+  first_pairs<DT>(sm, p, pb, pe);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  // window pairs = unequal pairs - general pairs (per warp: a warp runs the
-  // general pairs it deferred, so its difference is never negative); EXACT =
-  // the piece length - unequal pairs + general pairs found equal.  Per-thread
-  // terms wrap modulo 2^32; the CTA totals lie in [0, 2^31).
-  const uint32_t gen = cd.n_gw + cd.n_gm + cd.n_ga + cd.n_gf + cd.n_geq;
-  const uint32_t c[8] = {cd.n_geq - L.uneq + (threadIdx.x == 0 ? (uint32_t)plen : 0u), L.uneq - gen, L.within,
-                         cd.n_nf, cd.n_gw, cd.n_gm, cd.n_ga, cd.n_gf};
-  __shared__ uint32_t cnt32[8];
-  if (threadIdx.x < 8) cnt32[threadIdx.x] = 0;
-  __syncthreads();
-#pragma unroll
-  for (int k = 0; k < 8; k++) {
-    const uint32_t v = __reduce_add_sync(0xFFFFFFFFu, c[k]);
-    if (lane == 0 && v) atomicAdd(&cnt32[k], v);
-  }
-  __syncthreads();
-  if (threadIdx.x < 8) sm.cnt[threadIdx.x] += cnt32[threadIdx.x];
-  Partial x;
-  x.abs_hi = cd.abs_hi;
-  x.abs_lo = cd.abs_lo;
-  x.abs_sc = cd.abs_sc;
-  x.pad0 = 0;
-  x.abs_idx = cd.abs_idx;
-  x.rel_hi = cd.rel_hi;
-  x.rel_lo = cd.rel_lo;
-  x.rel_g = cd.rel_g;
-  x.rel_sc = cd.rel_sc;
-  x.rel_idx = cd.rel_idx;
-  x.ulp = cd.ulp;
-  x.ulp_idx = cd.ulp_idx;
-  x.first_fin = cd.first_fin;
-  x.first_ulp = cd.first_ulp;
+  const int64_t lo = sm.lo;
+  // window pairs = unequal pairs - general pairs; EXACT = the piece length -
+  // unequal pairs + general pairs found equal (64-bit wrapping adds; the
+  // totals are non-negative)
   {
-    // the window records of this thread, as exact values
+    const uint32_t vu = __reduce_add_sync(0xFFFFFFFFu, L.uneq), vw = __reduce_add_sync(0xFFFFFFFFu, L.within);
+    if (lane == 0) {
+      if (vu) {
+        atomicAdd(&sm.cnt[1], (unsigned long long)vu);
+        atomicAdd(&sm.cnt[0], 0ull - (unsigned long long)vu);
+      }
+      if (vw) atomicAdd(&sm.cnt[2], (unsigned long long)vw);
+    }
+    if (threadIdx.x == 0) {
+      atomicAdd(&sm.cnt[0], (unsigned long long)(pe - pb));
+      atomicAdd(&sm.cnt[3], (unsigned long long)sm.nfe);
+    }
+  }
+  // maxima: this thread's window record, then the warp's, merged with the
+  // warp's general best
+  {
+    const WinRec r = sm.rec[threadIdx.x];
     Partial w;
     part_none(w);
-    if (L.amax > 0.0f) {
-      w.abs_hi = L.amax;
-      w.abs_idx = lo + L.aidx;
+    if (r.amax > 0.0f) {
+      w.abs_hi = r.amax;
+      w.abs_idx = lo + r.aidx;
     }
-    if (L.ra > 0.0f) {
-      const int64_t i = lo + L.ridx;
+    if (r.ra > 0.0f) {
+      const int64_t i = lo + r.ridx;
       const float gf = to_f32<DT>(load_scalar<DT>(p.g, i)), cf = to_f32<DT>(load_scalar<DT>(p.c, i));
       w.rel_hi = fabsf(__fsub_rn(cf, gf));
       w.rel_g = fabsf(gf);
       w.rel_idx = i;
     }
-    if (L.umax > 0u) {
-      w.ulp = DT == PEAT_BF16 ? L.umax >> 16 : L.umax;
-      w.ulp_idx = lo + L.uidx;
+    if (r.umax > 0u) {
+      w.ulp = DT == PEAT_BF16 ? r.umax >> 16 : r.umax;
+      w.ulp_idx = lo + r.uidx;
     }
-    part_merge(x, w);
+    part_warp_reduce(w);
+    if (lane == 0) {
+      Partial x = sm.wbest[warp];
+      part_merge(x, w);
+      sm.wbest[warp] = x;
+    }
   }
-  part_warp_reduce(x);
-  if (lane == 0) sm.wbest[warp] = x;
   __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int w = 1; w < NW; w++) part_merge(x, sm.wbest[w]);
-    *out = x;
+  if (warp == 0) {
+    Partial x;
+    if (lane < NW) x = sm.wbest[lane];
+    else part_none(x);
+    part_warp_reduce(x);
+    if (lane == 0) {
+      constexpr long long NONE = 0x7FFFFFFFFFFFFFFFll;
+      x.first_fin = sm.ff == NONE ? -1 : sm.ff;
+      x.first_ulp = sm.fu == NONE ? -1 : sm.fu;
+      *out = x;
+    }
   }
   for (int b = threadIdx.x; b < HBINS; b += BLOCK)
     if (sm.hist[b]) atomicAdd(&acc->hist[b], sm.hist[b]);
@@ -1144,19 +1200,22 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, in
   for (int b = threadIdx.x; b < HBINS; b += BLOCK) sm.hist[b] = 0;
   for (int j = threadIdx.x; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
   if (threadIdx.x < 8) sm.cnt[threadIdx.x] = 0;
+  if (threadIdx.x == 0) sm.nfe = 0;
+  rec_init(sm.rec[threadIdx.x]);
   lane_init(L);
-  cold_init(cd);
   __syncthreads();
 }
 
 // ---------------------------------------------------------------------------
 // stage 1
 // ---------------------------------------------------------------------------
+constexpr int CTAS_PER_SM = 2;
+
 template <int DT>
-__global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
-  using T = Tr<DT>;
+__global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(CompareParams p) {
+  using Ty = Tr<DT>;
   using R = Rows<DT>;
-  constexpr int VEC = T::VEC;
+  constexpr int VEC = Ty::VEC;
   // pairs per thread per round stay below 2^16 (16-bit private counters): each
   // warp tile gives a thread at most 2 VEC pairs
   constexpr int64_t ROUND_CHUNKS = (int64_t)NW * (65535 / (2 * VEC));
@@ -1167,23 +1226,23 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
   for (int j = tid; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
   for (int j = tid; j < R::NPB * HALF; j += BLOCK) sm.priv[j] = 0;
   if (tid < 8) sm.cnt[tid] = 0;
-  if (tid < 64) sm.ovf[tid] = 0;
+  rec_init(sm.rec[tid]);
+  const int64_t lo = p.bounds[blockIdx.x], hi = p.bounds[blockIdx.x + 1];
   if (tid == 0) {
+    sm.lo = lo;
     sm.gn = 0;
+    sm.nfe = 0;
     sm.glist = p.glist + (size_t)blockIdx.x * GCAP;
   }
   if (lane == 0) {
     for (int st = 0; st < NSTAGE; st++) mbar_init(&sm.bar[warp][st], 1);
     mbar_init_fence();
   }
-  const int64_t lo = p.bounds[blockIdx.x], hi = p.bounds[blockIdx.x + 1];
-  if (tid == 0) sm.lo = lo;
   Win W;
   W.rtol = p.rtol;
   W.atol = p.atol;
   W.base = smem_addr(&sm.priv[tid & (HALF - 1)]);
   W.inc = tid < HALF ? 1u : 65536u;
-  cold_init(sm.cold[tid]);
   Lane L;
   lane_init(L);
   __syncthreads();
@@ -1211,7 +1270,7 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
       const int st = (int)(sq % NSTAGE);
       const int64_t v0 = k * CHV;
       const uint32_t bytes = (uint32_t)(min((int64_t)CHV, nvec - v0) * 16);
-      const int64_t off = (vb + v0 * VEC) * T::BYTES;
+      const int64_t off = (vb + v0 * VEC) * Ty::BYTES;
       fence_proxy_async();
       mbar_expect_tx(&sm.bar[warp][st], 2 * bytes);
       bulk_load(&sm.ring_g[warp][st][0], gbase + off, bytes, &sm.bar[warp][st]);
@@ -1225,15 +1284,15 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
     if (tid == 0) sm.lb = sm.ub = 0;
     __syncthreads();
     if (tid < nvec) {
-      const uint4 gv = load_vec(p.g, (vb + (int64_t)tid * VEC) * T::BYTES);
-      const uint4 cv = load_vec(p.c, (vb + (int64_t)tid * VEC) * T::BYTES);
+      const uint4 gv = load_vec(p.g, (vb + (int64_t)tid * VEC) * Ty::BYTES);
+      const uint4 cv = load_vec(p.c, (vb + (int64_t)tid * VEC) * Ty::BYTES);
       uint32_t emax = 0, umax = 0;
 #pragma unroll
       for (int j = 0; j < VEC; j++) {
         const uint32_t G = lane_bits<DT>(gv, j), C = lane_bits<DT>(cv, j);
-        const uint32_t e = (G & T::MAG) >> T::MB;
-        if (e < (uint32_t)T::EMAX && e > emax) emax = e;
-        if (((G ^ C) & T::SIGN) == 0u && (G & T::MAG) < T::INF && (C & T::MAG) < T::INF) {
+        const uint32_t e = (G & Ty::MAG) >> Ty::MB;
+        if (e < (uint32_t)Ty::EMAX && e > emax) emax = e;
+        if (((G ^ C) & Ty::SIGN) == 0u && (G & Ty::MAG) < Ty::INF && (C & Ty::MAG) < Ty::INF) {
           const uint32_t u = G > C ? G - C : C - G;
           umax = u > umax ? u : umax;
         }
@@ -1245,18 +1304,20 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
     // u < 2^UB with one bit to spare over the sample; V = |d| / 2^Lexp < 2^22
     // for such pairs with goldens up to 2 binades above the largest seen
     int UB = sm.ub + 1;
-    UB = UB > T::UBMAX ? T::UBMAX : UB;
+    UB = UB > Ty::UBMAX ? Ty::UBMAX : UB;
     int lb = sm.lb + UB - 20;
-    lb = lb < T::LBMIN ? T::LBMIN : (lb > T::LBMAX ? T::LBMAX : lb);
-    const int lexp = lb - T::BIAS - T::MB;  // weight of V's unit
-    W.gmin = (DT == PEAT_F16 && lb == T::LBMIN) ? __uint_as_float((uint32_t)(127 - 24) << 23)
-                                                  : __uint_as_float((uint32_t)(lb + 1 - T::BIAS + 127) << 23);
+    lb = lb < Ty::LBMIN ? Ty::LBMIN : (lb > Ty::LBMAX ? Ty::LBMAX : lb);
+    const int lexp = lb - Ty::BIAS - Ty::MB;  // weight of V's unit
+    W.gmin = (DT == PEAT_F16 && lb == Ty::LBMIN) ? __uint_as_float((uint32_t)(127 - 24) << 23)
+                                                   : __uint_as_float((uint32_t)(lb + 1 - Ty::BIAS + 127) << 23);
     W.lim = __uint_as_float((uint32_t)(lexp + 22 + 127) << 23);
     W.M = __uint_as_float(((uint32_t)(lexp + 23 + 127) << 23) | 0x400000u);
     W.udmax = (1u << UB) << (DT == PEAT_BF16 ? 16 : 0);
+    Thr T;
+    thr_init(T);
     auto scalar_range = [&](int64_t b0, int64_t b1) {
       for (int64_t i = b0 + tid; i < b1; i += BLOCK)
-        do_scalar<DT>(L, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), (uint32_t)(i - lo), W, sm);
+        do_scalar<DT>(L, T, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), (uint32_t)(i - lo), W, sm);
     };
     // scalar head: fewer than VEC elements, or the whole piece in scalar mode
     // (then in rounds of at most 65535 elements per thread)
@@ -1288,7 +1349,7 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
         if (!failed) {
           const int64_t v0 = k * CHV;
           const int nvalid = (int)min((int64_t)CHV, nvec - v0);
-          do_tile<DT>(L, sm.ring_g[warp][st], sm.ring_c[warp][st], nvalid, (uint32_t)(vb + v0 * VEC - lo), W, sm);
+          do_tile<DT>(L, T, sm.ring_g[warp][st], nvalid, (uint32_t)(vb + v0 * VEC - lo), W, sm);
           if (lane == 0 && i + NSTAGE < my_chunks) issue(seq + NSTAGE, warp + NW * (i + NSTAGE));
         }
         seq++;
@@ -1303,7 +1364,7 @@ __global__ void __launch_bounds__(BLOCK, 2) compare_stage1(CompareParams p) {
         mbar_wait(&sm.bar[warp][sq % NSTAGE], (sq / NSTAGE) & 1u, DRAIN_LIMIT);
       }
     }
-    // scalar tail (fewer than VEC elements), after the body: pairs stay in index order
+    // scalar tail (fewer than VEC elements), after the body
     if (vb < ve && ve < pe) scalar_range(ve, pe);
     finish_piece<DT>(L, W, sm, lexp, p, pb, pe, p.partials + s + blockIdx.x, p.acc + s);
     pb = pe;
@@ -1442,10 +1503,14 @@ __global__ void __launch_bounds__(BLOCK) compare_stage2(CompareParams p) {
   part_warp_reduce(x);
   if (lane == 0) wbest[warp] = x;
   __syncthreads();
-  if (tid < NSUM) sums[tid] = limbs_to_double(limbs[tid]);
+  if (warp == 1 && lane < NSUM) sums[lane] = limbs_to_double(limbs[lane]);
+  if (warp == 0) {
+    if (lane < BLOCK / 32) x = wbest[lane];
+    else part_none(x);
+    part_warp_reduce(x);
+  }
   __syncthreads();
   if (tid == 0) {
-    for (int w = 1; w < BLOCK / 32; w++) part_merge(x, wbest[w]);
     peat_stats_t r;
     const uint64_t n = (uint64_t)(s1 - s0);
     r.n = n;
@@ -1526,18 +1591,23 @@ int64_t compare_cta_bound(int dtype, int64_t b, int nctas, int64_t n, int64_t p0
 }
 
 // once per device, before the first launch
-cudaError_t compare_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(compare_stage1<PEAT_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)sizeof(Smem));
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(compare_stage1<PEAT_F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(Smem));
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(compare_stage1<PEAT_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)sizeof(Smem));
+template <int DT>
+cudaError_t prepare_t() {
+  cudaError_t e =
+      cudaFuncSetAttribute(compare_stage1<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(Smem));
+  if (e == cudaSuccess)  // as much shared memory as the SM offers: CTAS_PER_SM CTAs of sizeof(Smem) each
+    e = cudaFuncSetAttribute(compare_stage1<DT>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
   return e;
 }
 
-int compare_ctas_per_sm() { return 2; }
+cudaError_t compare_prepare() {
+  cudaError_t e = prepare_t<PEAT_F32>();
+  if (e == cudaSuccess) e = prepare_t<PEAT_F16>();
+  if (e == cudaSuccess) e = prepare_t<PEAT_BF16>();
+  return e;
+}
+
+int compare_ctas_per_sm() { return CTAS_PER_SM; }
 size_t compare_partial_bytes() { return sizeof(Partial); }
 size_t compare_segacc_bytes() { return sizeof(SegAcc); }
 

@@ -7,35 +7,36 @@
 // 64-bin histograms.  Every output is exact: integer outputs bit for bit,
 // sums as the exact real sum rounded once to nearest-even binary64.
 //
-// Stage 1 (compare_stage1): a persistent grid streams both tensors once
-// through per-warp rings of bulk copies (cp.async.bulk + mbarrier).  CTA b
-// owns the contiguous element range [lo_b, lo_{b+1}); per segment piece it
-// touches it adds its integer totals (counts, histograms, sum digits) to the
-// segment's accumulator with atomics and writes its maxima to slot s + b.
-// Per element pair:
+// One kernel (compare_stage1) per call: a persistent grid streams both
+// tensors once through per-warp rings of bulk copies (cp.async.bulk +
+// mbarrier).  CTA b owns the contiguous element range [lo_b, lo_{b+1}); per
+// segment piece it touches it adds its integer totals (counts, histograms,
+// sum digits) to the segment's accumulator with atomics and writes its maxima
+// to slot s + b; the CTA that finishes a segment's last piece merges the
+// slots in CTA order, rounds the exact sums once, writes the outputs and
+// clears the accumulator.  All merged quantities are integers or exact
+// values, so the result depends neither on the grid nor on the order of the
+// atomics.  Per element pair:
 //   - bitwise-equal pairs are counted (whole warp tiles at once when equal);
-//   - unequal pairs of a tile are processed in place when most of the tile
-//     differs, else compacted into a per-warp queue first;
-//   - a "window" pair -- same sign, ULP distance u < 2^UB (so c is within a
-//     factor 2 of g and c - g is exact in float32, Sterbenz), |g| at least
-//     2^(Lb+1-bias), |d| < 2^(Lexp+22) -- is finished in float32 and
+//   - unequal pairs of a tile are compacted into a per-warp queue (element
+//     order) and processed 32 at a time;
+//   - a "window" pair -- ULP distance u < 2^UB (so the signs agree and c is
+//     within a factor 2 of g: c - g is exact in float32, Sterbenz), |g| at
+//     least 2^(Lb+1-bias), |d| < 2^(Lexp+22) -- is finished in float32 and
 //     integer arithmetic: V = |d| / 2^Lexp is an integer below 2^22, read
 //     from the bits of |d| + 1.5 * 2^(Lexp+23), so sum |d|, sum d and sum d^2
 //     accumulate as integers; the log2-relative bin is the exponent
 //     difference of |d| and |g|; the tolerance test is one float32 fma, exact
-//     except at equality; the maxima are exact float32 comparisons (the
-//     significands are short enough for exact products, or error-free
-//     products for float32 input);
+//     except at equality; a pair updates the exact maxima only when it lies
+//     strictly above the thread's current ones (its pairs arrive in index
+//     order, so ties keep the earlier index);
 //   - every other pair (non-finite, sign change, zeros, wide gaps, outside
-//     the window, tolerance ties) is deferred to a per-warp buffer and
-//     evaluated exactly, 32 at a time, with float32 error-free transforms and
-//     integer digits added to a CTA-wide carry-save fixed-point accumulator.
-// Binary64 arithmetic is avoided in stage 1 (GB300 runs it at a small
-// fraction of float32 rate); binary64 values appear only as containers.
-// Stage 2 (compare_stage2): one CTA per segment merges the maxima of that
-// segment's pieces in CTA order, rounds the exact sums once and clears the
-// accumulator; all merged quantities are integers or exact values, so the
-// result does not depend on the grid or on the order of the atomics.
+//     the window, tolerance ties) is listed and evaluated exactly after the
+//     piece, with float32 error-free transforms and integer digits added to a
+//     CTA-wide carry-save fixed-point accumulator.
+// Binary64 arithmetic is avoided per element (GB300 runs it at a small
+// fraction of float32 rate); binary64 values appear only as containers and
+// in the once-per-segment rounding.
 #include <cuda_fp16.h>
 
 #include <cstdint>
@@ -348,6 +349,14 @@ struct WinRec {
 // Per-warp staging ring for the bulk copies: NSTAGE stages, each one warp
 // tile of CHV 16-byte vectors of each tensor (two vectors per lane).
 constexpr int NW = BLOCK / 32;
+
+// scratch of a segment's finalization
+struct FinScratch {
+  unsigned long long cnt[8];
+  long long limbs[NSUM * NLIMB];
+  Partial wbest[NW];
+  double sums[NSUM];
+};
 constexpr int NSTAGE = 3;
 constexpr int CHV = 64;
 
@@ -364,6 +373,8 @@ struct __align__(128) Smem {
   uint32_t* glist;                 // this CTA's list of general pairs (offsets), GCAP entries
   uint32_t gn;                     // entries appended in this piece (may exceed GCAP)
   uint32_t nfe;                    // bitwise-equal pairs holding NaN or Inf
+  int last;                        // this CTA finished the last piece of a one-segment call
+  FinScratch fin;
   int lb, ub;
   WinRec rec[BLOCK];
   uint32_t priv[NPB_MAX * HALF];   // per-thread 16-bit counters, two threads per word
@@ -1022,6 +1033,10 @@ template <int DT>
 __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p, int64_t pb, int64_t pe) {
   __syncthreads();
   const uint32_t n = sm.gn;
+  if (n == 0) {  // no general pair in this piece
+    if ((threadIdx.x & 31) == 0) part_none(sm.wbest[threadIdx.x >> 5]);
+    return;
+  }
   const int64_t lo = sm.lo;
   GenRec cd;
   gen_init(cd);
@@ -1071,7 +1086,13 @@ template <int DT>
 __device__ __noinline__ void first_pairs(Smem& sm, const CompareParams& p, int64_t pb, int64_t pe) {
   using Ty = Tr<DT>;
   constexpr long long NONE = 0x7FFFFFFFFFFFFFFFll;
-  if (threadIdx.x == 0) sm.ff = sm.fu = NONE;
+  if (threadIdx.x == 0) {
+    // the piece's first pair settles both unless it holds NaN or Inf
+    const uint32_t ag = load_scalar<DT>(p.g, pb) & Ty::MAG, ac = load_scalar<DT>(p.c, pb) & Ty::MAG;
+    const bool fin = ag < Ty::INF && ac < Ty::INF;
+    sm.ff = fin ? pb : NONE;
+    sm.fu = fin ? pb : NONE;
+  }
   for (int64_t base = pb;; base += BLOCK) {
     __syncthreads();
     if (base >= pe || (sm.ff != NONE && sm.fu != NONE)) break;
@@ -1120,11 +1141,17 @@ __device__ void fold_round(Lane& L, Smem& sm, int lexp) {
   __syncthreads();
 }
 
+__device__ void finalize_segment(const CompareParams& p, int64_t s, FinScratch& f);
+__device__ void write_empty_segments(const CompareParams& p);
+
 // End of one segment piece [pb, pe): the integer totals go to the segment's
-// accumulator (global atomics), the maxima to the CTA's partial slot.
+// accumulator (global atomics), the maxima to the CTA's partial slot.  The
+// CTA that finishes the segment's last piece then finalizes the segment.
 template <int DT>
 __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, int lexp, const CompareParams& p,
-                                             int64_t pb, int64_t pe, Partial* out, SegAcc* acc) {
+                                             int64_t seg, int64_t pb, int64_t pe) {
+  Partial* out = p.partials + seg + blockIdx.x;
+  SegAcc* acc = p.acc + seg;
   run_general<DT>(W, sm, p, pb, pe);
   fold_round<DT>(L, sm, lexp);
   first_pairs<DT>(sm, p, pb, pe);
@@ -1195,7 +1222,17 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, in
     const unsigned long long v = (&sm.sacc[0][0])[j];
     if (v) atomicAdd(reinterpret_cast<unsigned long long*>(&acc->limbs[0][0]) + j, v);
   }
+  // publish, then count this piece: the segment's pieces are the CTAs whose
+  // ranges meet it
+  __threadfence();
   __syncthreads();
+  if (threadIdx.x == 0) {
+    sm.last = 0;
+    if (p.nseg == 1) {  // one segment: its last CTA finalizes it (else a second launch does, in parallel)
+      const unsigned int pieces = (unsigned int)(cta_of(p.n_total - 1, p) - cta_of(0, p) + 1);
+      sm.last = atomicAdd(&acc->done, 1u) == pieces - 1u;
+    }
+  }
   // reset the CTA totals for the next piece
   for (int b = threadIdx.x; b < HBINS; b += BLOCK) sm.hist[b] = 0;
   for (int j = threadIdx.x; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
@@ -1204,6 +1241,10 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, in
   rec_init(sm.rec[threadIdx.x]);
   lane_init(L);
   __syncthreads();
+  if (sm.last) {
+    __threadfence();
+    finalize_segment(p, seg, sm.fin);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1246,7 +1287,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
   Lane L;
   lane_init(L);
   __syncthreads();
-  if (lo >= hi) return;
+  if (blockIdx.x == 0 && p.has_empty) write_empty_segments(p);
   uint32_t seq = 0;      // this warp's bulk-copy stage uses so far (stage = seq % NSTAGE)
   bool failed = false;   // a pipeline wait expired: skip the data, keep the barriers
   int64_t s = seg_of(lo, p.offsets, p.nseg);
@@ -1366,7 +1407,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
     }
     // scalar tail (fewer than VEC elements), after the body
     if (vb < ve && ve < pe) scalar_range(ve, pe);
-    finish_piece<DT>(L, W, sm, lexp, p, pb, pe, p.partials + s + blockIdx.x, p.acc + s);
+    finish_piece<DT>(L, W, sm, lexp, p, s, pb, pe);
     pb = pe;
   }
 }
@@ -1468,49 +1509,59 @@ __device__ double limbs_to_double(const long long* src) {
   return neg ? -r : r;
 }
 
-__global__ void __launch_bounds__(BLOCK) compare_stage2(CompareParams p) {
-  const int64_t s = blockIdx.x;
+// Copy of a partial written by another CTA (read from L2, past this SM's L1).
+__device__ __forceinline__ Partial load_partial(const Partial* src) {
+  Partial x;
+  const unsigned long long* w = reinterpret_cast<const unsigned long long*>(src);
+  unsigned long long* d = reinterpret_cast<unsigned long long*>(&x);
+#pragma unroll
+  for (int k = 0; k < (int)(sizeof(Partial) / 8); k++) d[k] = __ldcg(w + k);
+  return x;
+}
+
+// The whole CTA, once every piece of segment s is in: merge the pieces'
+// maxima in CTA order, round the exact sums once, write the outputs and clear
+// the accumulator for the next call.  Uses the CTA's totals in shared memory
+// as scratch (they are zero on entry and on exit).
+__device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s, FinScratch& f) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t s0 = p.offsets[s], s1 = p.offsets[s + 1];
   SegAcc* acc = p.acc + s;
-  __shared__ unsigned long long cnt[8];
-  __shared__ long long limbs[NSUM][NLIMB];
-  __shared__ double sums[NSUM];
-  __shared__ Partial wbest[BLOCK / 32];
-  // integer totals, then clear them for the next call
+  long long* limbs = f.limbs;
   unsigned long long hv = 0;
   if (tid < HBINS) {
-    hv = acc->hist[tid];
+    hv = __ldcg(&acc->hist[tid]);
     acc->hist[tid] = 0;
   }
   if (tid >= HBINS && tid < HBINS + 8) {
-    cnt[tid - HBINS] = acc->cnt[tid - HBINS];
+    f.cnt[tid - HBINS] = __ldcg(&acc->cnt[tid - HBINS]);
     acc->cnt[tid - HBINS] = 0;
   }
   if (tid >= 160 && tid < 160 + NSUM * NLIMB) {
     const int j = tid - 160;
-    (&limbs[0][0])[j] = (&acc->limbs[0][0])[j];
+    limbs[j] = __ldcg(&acc->limbs[0][0] + j);
     (&acc->limbs[0][0])[j] = 0;
   }
+  if (tid == 0) acc->done = 0;
   // maxima over the segment's pieces
   Partial x;
   part_none(x);
-  if (s1 > s0) {
+  {
     const int b0 = cta_of(s0, p), b1 = cta_of(s1 - 1, p);
-    for (int b = b0 + tid; b <= b1; b += BLOCK)
-      if (p.bounds[b] < p.bounds[b + 1]) part_merge(x, p.partials[s + b]);
+    for (int b = b0 + tid; b <= b1; b += BLOCK) part_merge(x, load_partial(p.partials + s + b));
   }
   part_warp_reduce(x);
-  if (lane == 0) wbest[warp] = x;
+  if (lane == 0) f.wbest[warp] = x;
   __syncthreads();
-  if (warp == 1 && lane < NSUM) sums[lane] = limbs_to_double(limbs[lane]);
+  if (warp == 1 && lane < NSUM) f.sums[lane] = limbs_to_double(limbs + lane * NLIMB);
   if (warp == 0) {
-    if (lane < BLOCK / 32) x = wbest[lane];
+    if (lane < NW) x = f.wbest[lane];
     else part_none(x);
     part_warp_reduce(x);
   }
   __syncthreads();
   if (tid == 0) {
+    const unsigned long long* cnt = f.cnt;
     peat_stats_t r;
     const uint64_t n = (uint64_t)(s1 - s0);
     r.n = n;
@@ -1541,22 +1592,44 @@ __global__ void __launch_bounds__(BLOCK) compare_stage2(CompareParams p) {
       r.max_ulp = 0;
       r.argmax_ulp = x.first_ulp >= 0 ? x.first_ulp - s0 : -1;
     }
-    r.sum_signed = sums[0];
-    r.sum_abs = sums[1];
-    r.sum_sq = sums[2];
+    r.sum_signed = f.sums[0];
+    r.sum_abs = f.sums[1];
+    r.sum_sq = f.sums[2];
     r.rtol_eff = p.rtol;
     r.atol_eff = p.atol;
     p.stats[s] = r;
   }
-  if (p.hist && tid < HBINS) p.hist[s * HBINS + tid] = hv + ((tid == 0 || tid == 64) ? cnt[0] : 0ull);
+  if (p.hist && tid < HBINS) p.hist[s * HBINS + tid] = hv + ((tid == 0 || tid == 64) ? f.cnt[0] : 0ull);
+  __syncthreads();
+}
+
+// Segments of a multi-segment call, one CTA each, after stage 1.
+__global__ void __launch_bounds__(BLOCK) compare_finalize(CompareParams p) {
+  __shared__ FinScratch f;
+  if (p.offsets[blockIdx.x] < p.offsets[blockIdx.x + 1]) finalize_segment(p, blockIdx.x, f);
+}
+
+// The outputs of every empty segment (no pairs): zero counts and sums, argmax -1.
+__device__ __noinline__ void write_empty_segments(const CompareParams& p) {
+  for (int64_t s = threadIdx.x; s < p.nseg; s += BLOCK) {
+    if (p.offsets[s] != p.offsets[s + 1]) continue;
+    peat_stats_t r;
+    memset(&r, 0, sizeof(r));
+    r.argmax_abs = r.argmax_rel = r.argmax_ulp = -1;
+    r.rtol_eff = p.rtol;
+    r.atol_eff = p.atol;
+    p.stats[s] = r;
+    if (p.hist)
+      for (int b = 0; b < HBINS; b++) p.hist[s * HBINS + b] = 0;
+  }
 }
 
 template <int DT>
 cudaError_t launch_t(const CompareParams& p, cudaStream_t st) {
   compare_stage1<DT><<<p.nctas, BLOCK, sizeof(Smem), st>>>(p);
   cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  if (p.nseg > 0) compare_stage2<<<(unsigned)p.nseg, BLOCK, 0, st>>>(p);
+  if (e != cudaSuccess || p.nseg <= 1) return e;
+  compare_finalize<<<(unsigned)p.nseg, BLOCK, 0, st>>>(p);
   return cudaGetLastError();
 }
 

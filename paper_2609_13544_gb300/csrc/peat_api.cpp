@@ -145,6 +145,8 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   p.acc = h->acc;
   p.partials = h->partials;
   p.glist = h->glist;
+  p.has_empty = 0;
+  for (int64_t s = 0; s < nseg && !p.has_empty; s++) p.has_empty = offsets[s + 1] == offsets[s];
   p.status = h->status_dev;
   p.wait_limit = h->wait_limit;
   p.rtol = rtol;

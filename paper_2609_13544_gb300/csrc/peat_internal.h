@@ -39,15 +39,18 @@ struct Partial {
   int64_t first_ulp;  // lowest index of a pair without NaN (-1 none)
 };
 
-// Integer totals of one segment: stage 1 adds into them with atomics (all
-// integers, so the order does not matter), stage 2 reads and clears them.
-// cnt: 0 EXACT, 1 window lanes, 2 window lanes within tol, 3 non-finite
-// pairs, 4 general within, 5 general mismatch, 6 NaN/Inf asymmetric,
-// 7 sign flip.  limbs: carry-save digits of the three exact sums.
+// Integer totals of one segment: every CTA piece of the segment adds into
+// them with atomics (all integers, so the order does not matter); the CTA that
+// finishes the segment's last piece reads and clears them.  cnt: 0 EXACT,
+// 1 window pairs, 2 window pairs within tol, 3 non-finite pairs, 4 general
+// within, 5 general mismatch, 6 NaN/Inf asymmetric, 7 sign flip.  limbs:
+// carry-save digits of the three exact sums.  done: pieces finished so far.
 struct SegAcc {
   unsigned long long hist[HBINS];
   unsigned long long cnt[8];
   long long limbs[NSUM][NLIMB];
+  unsigned int done;
+  unsigned int pad;
 };
 
 struct CompareParams {
@@ -62,6 +65,7 @@ struct CompareParams {
   Partial* partials;       // nseg + nctas slots; slot s + b holds CTA b's part of segment s
   SegAcc* acc;             // nseg accumulators, all zero between calls
   uint32_t* glist;         // nctas * GCAP offsets: each CTA's general pairs of the current piece
+  int has_empty;           // some segment is empty (CTA 0 writes the outputs of the empty segments)
   unsigned int* status;    // device-visible error word (bit 0: a bounded wait expired)
   unsigned int wait_limit; // iteration bound of a pipeline wait (0: give up at once, for tests)
   float rtol, atol;        // float32 tolerances

@@ -1,7 +1,9 @@
 """Throughput of the golden-vs-candidate error signature (peat_compare) on GB300.
 
-One step = one full pass of the compare (stage 1 stream over both tensors +
-stage 2 per-segment merge) over one synthetic workload resident in HBM.
+One step = one full call of the compare over one synthetic workload resident
+in HBM: both tensors streamed once, every segment's signature finalized (in
+the same kernel for a single-segment call, by a second small launch for a
+segmented one).
 Default workload: the [8,2048,4096] bf16 activation (67,108,864 pairs,
 RNE vs RTZ candidate).  Prints ONE JSON line (rank 0).
 
@@ -351,10 +353,14 @@ def run_gpu(args) -> None:
             "hbm_gbs": gbs, "frac_of_8tbs": gbs / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
                          "traffic": recorded_traffic(args.workload),
-                         "kernel": "compare_stage1 + compare_stage2 per call (event-timed on the launch stream)",
+                         "kernel": ("compare_stage1<%s>, the one launch of each call (finalization in the same "
+                                    "kernel), event-timed on the launch stream" % w.dtype) if nseg == 1 else
+                                   ("compare_stage1<%s> + compare_finalize per call, event-timed together on the "
+                                    "launch stream" % w.dtype),
+                         "algorithmic_bytes_per_launch": bytes_per_step,
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy)" if not peaks.get("fallback")
                          else "fallback 6.8 TB/s"},
-            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": 2 * args.steps, "clocks": clocks,
+            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": (1 if nseg == 1 else 2) * args.steps, "clocks": clocks,
             "wall_s_timed": wall,
         }
         print(json.dumps(line), flush=True)

@@ -216,8 +216,44 @@ peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* s
                                        uint64_t seed, uint64_t* counts_out, peat_stream_t stream);
 
 /* Text of the last error reported on h (never NULL; "" if none).  With
- * h == NULL, the last error of a failed peat_signature_create on this thread. */
+ * h == NULL, the last error on this thread of peat_signature_create or of
+ * peat_compare_noalloc, whichever failed last. */
 const char* peat_last_error(peat_handle_t h);
+
+/* peat_compare without a handle and without any allocation.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate at
+ * the moment they compare, for instance
+ *   - code whose device memory is wholly owned by a pool or caching allocator
+ *     (a framework at its memory limit, or a handler comparing tensors after
+ *     an out-of-memory error), where a new cudaMalloc fails or evicts;
+ *   - timing-sensitive loops, where cudaMalloc/cudaFree would synchronise the
+ *     device and stall every stream;
+ * and it does not need a handle (creating one allocates its workspace).
+ *
+ * Arguments, outputs and errors are those of peat_compare (one tensor, no
+ * segments).  Instead of a handle's workspace it uses one fixed block of
+ * device memory per device, reserved when the library's device code is
+ * loaded (about 21 MB: per-CTA lists of general-path pairs for up to 320
+ * CTAs, their partial results, the CTA bounds and one accumulator).  Nothing
+ * is allocated by a call, on the device or on the host.
+ *   - n above 320 * (2^31 - 65) elements is rejected with PEAT_ERR_UNSUPPORTED.
+ *   - The block's accumulator must be zero when a call starts.  It is zero
+ *     when the code loads and every call that runs to completion leaves it
+ *     zero; a call that fails to launch clears it with cudaMemsetAsync.
+ *   - All calls on one device share the block: two calls that overlap on the
+ *     GPU (different streams without ordering, or different host threads)
+ *     race and both results are invalid.  Order them on one stream.
+ *   - The first call on each device does a one-time setup (it looks up the
+ *     block's address with cudaGetSymbolAddress and sets kernel attributes);
+ *     make it before any stream capture.
+ *   - It launches two kernels on `stream` (the CTA bounds, then the compare).
+ *   - A bounded device-side wait that expires leaves the outputs invalid;
+ *     without a handle this entry point has no place to report it later.
+ * Errors: as peat_compare, plus PEAT_ERR_UNSUPPORTED (n or device ordinal
+ * beyond the limits); the text is in peat_last_error(NULL). */
+peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, int64_t n, peat_dtype_t dtype,
+                                   peat_tol_t tol, peat_stats_t* stats_out, uint64_t* hist_out,
+                                   peat_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -62,7 +62,7 @@ class InjectModel(ctypes.Structure):
 
 
 EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
-           "peat_pseudo_error_inject", "peat_last_error")
+           "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -91,6 +91,8 @@ def load(path: Optional[Path] = None) -> ctypes.CDLL:
     L.peat_pseudo_error_inject.restype = i32
     L.peat_last_error.argtypes = [vp]
     L.peat_last_error.restype = ctypes.c_char_p
+    L.peat_compare_noalloc.argtypes = [vp, vp, i64, i32, Tol, vp, vp, vp]
+    L.peat_compare_noalloc.restype = i32
     _lib = L
     return L
 
@@ -174,6 +176,18 @@ def peat_compare_raw(h: Handle, golden, candidate, rtol: float, atol: float, sta
     _check(rc, h)
 
 
+def peat_compare_noalloc_raw(golden, candidate, rtol: float, atol: float, stats_out, hist_out=None,
+                             stream=None) -> None:
+    """peat_compare_noalloc (no handle, no allocation) on preallocated device outputs."""
+    _dev_tensor_check(golden, candidate)
+    if golden.numel() != candidate.numel() or golden.dtype != candidate.dtype:
+        raise ValueError("golden and candidate differ in size or dtype")
+    rc = load().peat_compare_noalloc(golden.data_ptr(), candidate.data_ptr(), golden.numel(), dtype_code(golden),
+                                     Tol(rtol, atol), stats_out.data_ptr(),
+                                     hist_out.data_ptr() if hist_out is not None else None, _stream_ptr(stream))
+    _check(rc, None)
+
+
 def peat_compare_segmented_raw(h: Handle, golden, candidate, offsets, rtol: float, atol: float, stats_out,
                                hist_out=None, stream=None) -> None:
     _dev_tensor_check(golden, candidate)
@@ -208,6 +222,18 @@ def peat_compare(h: Handle, golden, candidate, rtol: float, atol: float = 0.0, s
     stats = torch.empty(STATS_BYTES, dtype=torch.uint8, device=dev)
     hist = torch.empty(HIST_BINS, dtype=torch.int64, device=dev)
     peat_compare_raw(h, golden, candidate, rtol, atol, stats, hist, stream)
+    s = stats_to_dicts(stats.cpu().numpy())[0]
+    return s, hist.cpu().numpy().view(np.uint64).reshape(2, 64)
+
+
+def peat_compare_noalloc(golden, candidate, rtol: float, atol: float = 0.0, stream=None):
+    """peat_compare_noalloc of one tensor pair: (stats dict, hist numpy uint64[2, 64]); synchronises.
+    (This convenience wrapper allocates its output tensors; the C entry point itself allocates nothing.)"""
+    import torch
+    dev = golden.device
+    stats = torch.empty(STATS_BYTES, dtype=torch.uint8, device=dev)
+    hist = torch.empty(HIST_BINS, dtype=torch.int64, device=dev)
+    peat_compare_noalloc_raw(golden, candidate, rtol, atol, stats, hist, stream)
     s = stats_to_dicts(stats.cpu().numpy())[0]
     return s, hist.cpu().numpy().view(np.uint64).reshape(2, 64)
 

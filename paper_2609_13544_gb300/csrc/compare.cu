@@ -1634,7 +1634,7 @@ cudaError_t launch_t(const CompareParams& p, cudaStream_t st) {
 }
 
 template <int DT>
-int64_t bound_t(int64_t b, int nctas, int64_t n, int64_t p0) {
+__host__ __device__ int64_t bound_t(int64_t b, int nctas, int64_t n, int64_t p0) {
   if (b <= 0) return 0;
   if (b >= nctas) return n;
   constexpr int VEC = Tr<DT>::VEC;
@@ -1644,7 +1644,28 @@ int64_t bound_t(int64_t b, int nctas, int64_t n, int64_t p0) {
   return lo < n ? lo : n;
 }
 
+// offsets {0, n} and the CTA bounds of a one-tensor call, written on the device
+template <int DT>
+__global__ void compare_bounds(int64_t* offsets, int64_t* bounds, int nctas, int64_t n, int64_t p0) {
+  for (int b = threadIdx.x; b <= nctas; b += blockDim.x) bounds[b] = bound_t<DT>(b, nctas, n, p0);
+  if (threadIdx.x == 0) {
+    offsets[0] = 0;
+    offsets[1] = n;
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_bounds_on_device(int dtype, int64_t* offsets, int64_t* bounds, int nctas, int64_t n, int64_t p0,
+                                    cudaStream_t s) {
+  switch (dtype) {
+    case PEAT_F32: compare_bounds<PEAT_F32><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0); break;
+    case PEAT_F16: compare_bounds<PEAT_F16><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0); break;
+    case PEAT_BF16: compare_bounds<PEAT_BF16><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
 
 cudaError_t launch_compare(int dtype, const CompareParams& p, cudaStream_t s) {
   switch (dtype) {

@@ -3,9 +3,12 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdint>
+#include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <unordered_set>
 #include <vector>
@@ -39,6 +42,10 @@ struct peat_handle_s {
 namespace {
 
 thread_local std::string g_create_error;
+// text of the last peat_compare_noalloc error on this thread (fixed storage:
+// that entry point allocates nothing, host memory included)
+thread_local char g_noalloc_error[192];
+thread_local bool g_null_error_is_noalloc = false;
 
 struct DeviceGuard {
   int prev = -1;
@@ -205,11 +212,49 @@ peat_status_t grow_inject(peat_handle_t h, size_t need) {
   return PEAT_OK;
 }
 
+// ---- scratch of the allocation-free compare ----------------------------------
+// One fixed block of device memory per device, reserved when the module
+// loads: no call of peat_compare_noalloc allocates.  Its accumulator (acc)
+// must be zero when a call starts: static device memory starts at zero, and
+// every call that completes leaves it zero (the finalizing CTA clears it).
+constexpr int NOALLOC_MAX_CTAS = 320;     // grid cap of the allocation-free compare
+constexpr int NOALLOC_MAX_DEVICES = 64;
+struct NoallocScratch {
+  peat::SegAcc acc;                                  // zero between calls
+  unsigned int status;                               // set by an expired device-side wait
+  unsigned int pad;
+  int64_t offsets[2];                                // {0, n}, written by the bounds kernel
+  int64_t bounds[NOALLOC_MAX_CTAS + 1];
+  peat::Partial partials[1 + NOALLOC_MAX_CTAS];
+  uint32_t glist[(size_t)NOALLOC_MAX_CTAS * peat::GCAP];
+};
+
+struct NoallocDevice {
+  std::atomic<int> ready{0};
+  NoallocScratch* scratch = nullptr;
+  int nsm = 0;
+};
+NoallocDevice g_noalloc_dev[NOALLOC_MAX_DEVICES];
+std::mutex g_noalloc_setup;
+
+peat_status_t noalloc_fail(peat_status_t st, const char* msg) {
+  std::snprintf(g_noalloc_error, sizeof(g_noalloc_error), "%s", msg);
+  return st;
+}
+peat_status_t noalloc_cuda_fail(cudaError_t e, const char* what) {
+  cudaGetLastError();
+  std::snprintf(g_noalloc_error, sizeof(g_noalloc_error), "%s: %s", what, cudaGetErrorString(e));
+  return PEAT_ERR_CUDA;
+}
+
 }  // namespace
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[sizeof(NoallocScratch)];
 
 extern "C" {
 
 peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg) {
+  g_null_error_is_noalloc = false;
   g_create_error.clear();
   if (!out) {
     g_create_error = "out is NULL";
@@ -441,8 +486,83 @@ peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* s
   return PEAT_OK;
 }
 
+peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, int64_t n, peat_dtype_t dtype,
+                                   peat_tol_t tol, peat_stats_t* stats_out, uint64_t* hist_out,
+                                   peat_stream_t stream) {
+  g_null_error_is_noalloc = true;
+  g_noalloc_error[0] = 0;
+  const int B = dtype_bytes(dtype);
+  if (!B) return noalloc_fail(PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
+  float rtol, atol;
+  if (!round_tol(tol, &rtol, &atol))
+    return noalloc_fail(PEAT_ERR_INVALID_ARG, "rtol and atol must be finite and >= 0 after rounding to float32");
+  if (n < 0) return noalloc_fail(PEAT_ERR_INVALID_ARG, "n < 0");
+  if (n > 0 && (!golden || !candidate)) return noalloc_fail(PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
+  if (!stats_out) return noalloc_fail(PEAT_ERR_INVALID_ARG, "stats_out is NULL");
+  // the per-CTA offsets of stage 1 are 32-bit: n / nctas must stay below 2^31 - 64
+  const int64_t max_n = (int64_t)NOALLOC_MAX_CTAS * (((int64_t)1 << 31) - 65);
+  if (n > max_n) return noalloc_fail(PEAT_ERR_UNSUPPORTED, "n exceeds the allocation-free limit (320 * (2^31 - 65))");
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return noalloc_cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= NOALLOC_MAX_DEVICES) return noalloc_fail(PEAT_ERR_UNSUPPORTED, "device ordinal above 63");
+  NoallocDevice& D = g_noalloc_dev[dev];
+  if (!D.ready.load(std::memory_order_acquire)) {
+    // first call on this device: find the scratch and configure the kernels
+    std::lock_guard<std::mutex> lk(g_noalloc_setup);
+    if (!D.ready.load(std::memory_order_relaxed)) {
+      void* ptr = nullptr;
+      e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+      if (e != cudaSuccess || !ptr) return noalloc_cuda_fail(e, "cudaGetSymbolAddress(scratch)");
+      e = peat::compare_prepare();
+      if (e != cudaSuccess) return noalloc_cuda_fail(e, "could not configure the compare kernels");
+      int nsm = 0;
+      e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess || nsm <= 0) return noalloc_cuda_fail(e, "cudaDeviceGetAttribute(SM count)");
+      D.scratch = static_cast<NoallocScratch*>(ptr);
+      D.nsm = nsm;
+      D.ready.store(1, std::memory_order_release);
+    }
+  }
+  NoallocScratch* S = D.scratch;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  peat::CompareParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.g = golden;
+  p.c = candidate;
+  p.n_total = n;
+  p.nseg = 1;
+  const uintptr_t ag = reinterpret_cast<uintptr_t>(golden), ac = reinterpret_cast<uintptr_t>(candidate);
+  if (n > 0 && ag % B == 0 && ac % B == 0 && ag % 16 == ac % 16)
+    p.p0 = (int64_t)(((16 - ag % 16) % 16) / B);
+  else
+    p.p0 = -1;
+  const int max_ctas = std::min(NOALLOC_MAX_CTAS, D.nsm * peat::compare_ctas_per_sm());
+  p.nctas = (int)std::max<int64_t>(1, std::min<int64_t>(max_ctas, (n + 4095) / 4096));
+  p.offsets = S->offsets;
+  p.bounds = S->bounds;
+  p.partials = S->partials;
+  p.acc = &S->acc;
+  p.glist = S->glist;
+  p.has_empty = n == 0;
+  p.status = &S->status;
+  p.wait_limit = 1u << 24;
+  p.rtol = rtol;
+  p.atol = atol;
+  p.stats = stats_out;
+  p.hist = hist_out;
+  e = peat::launch_bounds_on_device(dtype, S->offsets, S->bounds, p.nctas, n, p.p0, st);
+  if (e != cudaSuccess) return noalloc_cuda_fail(e, "bounds launch");
+  e = peat::launch_compare(dtype, p, st);
+  if (e != cudaSuccess) {
+    cudaMemsetAsync(&S->acc, 0, sizeof(S->acc), st);  // no partial totals may survive into the next call
+    return noalloc_cuda_fail(e, "compare launch");
+  }
+  return PEAT_OK;
+}
+
 const char* peat_last_error(peat_handle_t h) {
-  if (!h) return g_create_error.c_str();
+  if (!h) return g_null_error_is_noalloc ? g_noalloc_error : g_create_error.c_str();
   return h->err.c_str();
 }
 

@@ -82,6 +82,10 @@ cudaError_t compare_prepare();
 int64_t compare_cta_bound(int dtype, int64_t b, int nctas, int64_t n, int64_t p0);
 size_t compare_partial_bytes();
 size_t compare_segacc_bytes();
+// offsets {0, n} and the nctas + 1 CTA bounds of a one-tensor call, computed
+// by a one-CTA kernel (for the caller that has no host staging buffer)
+cudaError_t launch_bounds_on_device(int dtype, int64_t* offsets, int64_t* bounds, int nctas, int64_t n, int64_t p0,
+                                    cudaStream_t s);
 
 struct InjectElemParams {
   void* dst;

@@ -15,8 +15,8 @@ def declared_functions():
 
 def test_header_declares_the_boundary():
     assert declared_functions() == sorted([
-        "peat_compare", "peat_compare_segmented", "peat_last_error", "peat_pseudo_error_inject",
-        "peat_signature_create", "peat_signature_destroy"])
+        "peat_compare", "peat_compare_noalloc", "peat_compare_segmented", "peat_last_error",
+        "peat_pseudo_error_inject", "peat_signature_create", "peat_signature_destroy"])
 
 
 def test_library_builds_and_exports_every_declared_symbol():

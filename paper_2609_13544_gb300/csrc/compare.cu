@@ -357,7 +357,7 @@ struct FinScratch {
   Partial wbest[NW];
   double sums[NSUM];
 };
-constexpr int NSTAGE = 3;
+constexpr int NSTAGE = 2;  // a power of two: stage and phase are bit fields of the use count
 constexpr int CHV = 64;
 
 struct __align__(128) Smem {
@@ -770,9 +770,11 @@ __device__ __forceinline__ void count_equal(const uint4& g, uint32_t eqm, Smem& 
 
 // One warp tile of CHV vectors staged in shared memory: lane L owns vectors L
 // and L + 32; tile element e sits at offset tli + e from the CTA's first
-// element.  Equal pairs are counted in place; unequal pairs are queued (in
-// element order) and processed 32 at a time, so every thread does useful
-// work.  Pairs above the warp's maxima are then evaluated exactly.
+// element.  Equal pairs are counted in place.  When at most a quarter of the
+// pairs differ, each lane works through its own unequal pairs (cheaper than
+// compacting a few); otherwise they are queued (in element order) and
+// processed 32 at a time, so every thread does useful work.  Pairs above the
+// thread's maxima are then evaluated exactly.
 template <int DT>
 __device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nvalid, uint32_t tli, const Win& W,
                                         Smem& sm) {
@@ -783,9 +785,19 @@ __device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nv
   constexpr uint32_t FULL = (1u << VEC) - 1u;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const bool okA = lane < nvalid, okB = lane + 32 < nvalid;
-  const uint4 z = make_uint4(0, 0, 0, 0);
-  const uint4 gA = okA ? gt[lane] : z, cA = okA ? ct[lane] : z;
-  const uint4 gB = okB ? gt[lane + 32] : z, cB = okB ? ct[lane + 32] : z;
+  uint4 gA, cA, gB, cB;
+  if (nvalid == CHV) {  // a full tile (all but the last of a piece)
+    gA = gt[lane];
+    cA = ct[lane];
+    gB = gt[lane + 32];
+    cB = ct[lane + 32];
+  } else {
+    const uint4 z = make_uint4(0, 0, 0, 0);
+    gA = okA ? gt[lane] : z;
+    cA = okA ? ct[lane] : z;
+    gB = okB ? gt[lane + 32] : z;
+    cB = okB ? ct[lane + 32] : z;
+  }
   const bool diff = ((gA.x ^ cA.x) | (gA.y ^ cA.y) | (gA.z ^ cA.z) | (gA.w ^ cA.w) | (gB.x ^ cB.x) | (gB.y ^ cB.y) |
                      (gB.z ^ cB.z) | (gB.w ^ cB.w)) != 0u;
   if (!__any_sync(0xFFFFFFFFu, diff)) {  // the whole warp tile is bitwise equal
@@ -808,19 +820,46 @@ __device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nv
   const uint32_t tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
   const uint32_t totA = tot & 0xFFFFu, total = totA + (tot >> 16);
   L.uneq += __popc(nA) + __popc(nB);
+  if (total * 4u <= 64u * VEC) {
+    // sparse tile: each lane visits its own unequal pairs (slot s < VEC:
+    // element s of vector A, else element s - VEC of vector B; increasing index)
+    uint32_t m = nA | (nB << VEC), cm = 0;
+    while (m) {
+      const uint32_t sl = __ffs(m) - 1;
+      m &= m - 1u;
+      const uint32_t pos = sl < (uint32_t)VEC ? lane * VEC + sl : (lane + 32) * VEC + sl - VEC;
+      uint32_t gr, cr;
+      float gf, cf;
+      elem_at<DT>(gt, pos, gr, gf);
+      elem_at<DT>(ct, pos, cr, cf);
+      if (pair_proc<DT>(L, T, gr, cr, gf, cf, tli + pos, W, sm)) cm |= 1u << sl;
+    }
+    L.A += L.sa;
+    L.N += L.sn;
+    L.sa = L.sn = 0;
+    if (cm) {
+      WinRec& r = sm.rec[threadIdx.x];
+      do {
+        const uint32_t sl = __ffs(cm) - 1;
+        cm &= cm - 1u;
+        const uint32_t pos = sl < (uint32_t)VEC ? lane * VEC + sl : (lane + 32) * VEC + sl - VEC;
+        uint32_t gr, cr;
+        float gf, cf;
+        elem_at<DT>(gt, pos, gr, gf);
+        elem_at<DT>(ct, pos, cr, cf);
+        rescan_pair<DT>(gr, cr, gf, cf, tli + pos, W, r, T);
+      } while (cm);
+    }
+    __syncwarp();
+    return;
+  }
   uint32_t posA = (incl & 0xFFFFu) - (packed & 0xFFFFu);
   uint32_t posB = totA + (incl >> 16) - (packed >> 16);
   unsigned short* q = sm.qp[warp];
-  if (total * 4u <= 64u * VEC) {
-    // sparse tile: visit only the set bits
-    for (uint32_t m = nA; m; m &= m - 1u) q[posA++] = (unsigned short)(lane * VEC + __ffs(m) - 1);
-    for (uint32_t m = nB; m; m &= m - 1u) q[posB++] = (unsigned short)((lane + 32) * VEC + __ffs(m) - 1);
-  } else {
 #pragma unroll
-    for (int j = 0; j < VEC; j++) {
-      if ((nA >> j) & 1u) q[posA++] = (unsigned short)(lane * VEC + j);
-      if ((nB >> j) & 1u) q[posB++] = (unsigned short)((lane + 32) * VEC + j);
-    }
+  for (int j = 0; j < VEC; j++) {
+    if ((nA >> j) & 1u) q[posA++] = (unsigned short)(lane * VEC + j);
+    if ((nB >> j) & 1u) q[posB++] = (unsigned short)((lane + 32) * VEC + j);
   }
   __syncwarp();
   // two queue entries per iteration (e, e + 32: in index order per lane);

@@ -379,22 +379,31 @@ struct __align__(128) Smem {
   WinRec rec[BLOCK];
   uint32_t priv[NPB_MAX * HALF];   // per-thread 16-bit counters, two threads per word
   unsigned short qp[NW][CHV * 8];  // per-warp queue: tile positions of the unequal pairs
+  // the general path's totals, one copy per warp (fewer threads contend for an
+  // address), folded into hist and sacc at the end of each piece
+  unsigned long long ghist[NW][HBINS];
+  unsigned long long gsacc[NW][NSUM][NLIMB];
 };
 
 __device__ __forceinline__ void sacc_add(Smem& sm, int which, unsigned __int128 m, int e, bool neg) {
   for_digits(m, e, neg, [&](int j, int64_t v) { atomicAdd(&sm.sacc[which][j], (unsigned long long)v); });
 }
+// general-path terms: into this warp's copy of the sum digits
+__device__ __forceinline__ void gsacc_add(Smem& sm, int which, unsigned __int128 m, int e, bool neg) {
+  unsigned long long* d = sm.gsacc[threadIdx.x >> 5][which];
+  for_digits(m, e, neg, [&](int j, int64_t v) { atomicAdd(d + j, (unsigned long long)v); });
+}
 __device__ __forceinline__ void sacc_add_f(Smem& sm, int which, float x, bool neg, int sc) {
   if (x == 0.0f) return;
   int e;
   uint32_t m = split_float(x, e);
-  sacc_add(sm, which, m, e + sc, neg ^ (x < 0));
+  gsacc_add(sm, which, m, e + sc, neg ^ (x < 0));
 }
 __device__ __forceinline__ void sacc_add_prod_f(Smem& sm, int which, float x, float y, int sc) {
   if (x == 0.0f || y == 0.0f) return;
   int ex, ey;
   uint32_t mx = split_float(x, ex), my = split_float(y, ey);
-  sacc_add(sm, which, (unsigned __int128)((uint64_t)mx * my), ex + ey + sc, (x < 0) ^ (y < 0));
+  gsacc_add(sm, which, (unsigned __int128)((uint64_t)mx * my), ex + ey + sc, (x < 0) ^ (y < 0));
 }
 
 // floor(log2(a / g)) for a = (hi + lo) 2^sc > 0 and g > 0 (float32 pair, any range)
@@ -435,8 +444,8 @@ __device__ __forceinline__ void general_lane(Smem& sm, GenRec& cd, uint32_t G, u
       return;
     }
     cd.n_ga++;
-    atomicAdd(&sm.hist[63], 1ull);
-    atomicAdd(&sm.hist[64 + (ulpdef ? (u < 63 ? (int)u : 63) : 63)], 1ull);
+    atomicAdd(&sm.ghist[threadIdx.x >> 5][63], 1ull);
+    atomicAdd(&sm.ghist[threadIdx.x >> 5][64 + (ulpdef ? (u < 63 ? (int)u : 63) : 63)], 1ull);
     return;
   }
   float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
@@ -481,8 +490,8 @@ __device__ __forceinline__ void general_lane(Smem& sm, GenRec& cd, uint32_t G, u
     int k = log2_ratio(hi, lo, sc, ag) + 48;
     rb = k < 1 ? 1 : (k > 62 ? 62 : k);
   }
-  atomicAdd(&sm.hist[rb], 1ull);
-  atomicAdd(&sm.hist[64 + (u < 63 ? (int)u : 63)], 1ull);
+  atomicAdd(&sm.ghist[threadIdx.x >> 5][rb], 1ull);
+  atomicAdd(&sm.ghist[threadIdx.x >> 5][64 + (u < 63 ? (int)u : 63)], 1ull);
   // maxima, full (value, index) order
   {
     int c = cd.abs_idx < 0 ? 1 : cmp_mag(hi, lo, sc, cd.abs_hi, cd.abs_lo, cd.abs_sc);
@@ -1192,7 +1201,25 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, in
   Partial* out = p.partials + seg + blockIdx.x;
   SegAcc* acc = p.acc + seg;
   run_general<DT>(W, sm, p, pb, pe);
-  fold_round<DT>(L, sm, lexp);
+  fold_round<DT>(L, sm, lexp);  // ends with a barrier: the general path's per-warp totals are complete
+  for (int b = threadIdx.x; b < HBINS; b += BLOCK) {
+    unsigned long long v = 0;
+#pragma unroll
+    for (int w = 0; w < NW; w++) {
+      v += sm.ghist[w][b];
+      sm.ghist[w][b] = 0;
+    }
+    sm.hist[b] += v;
+  }
+  for (int j = threadIdx.x; j < NSUM * NLIMB; j += BLOCK) {
+    unsigned long long v = 0;
+#pragma unroll
+    for (int w = 0; w < NW; w++) {
+      v += (&sm.gsacc[w][0][0])[j];
+      (&sm.gsacc[w][0][0])[j] = 0;
+    }
+    (&sm.sacc[0][0])[j] += v;
+  }
   first_pairs<DT>(sm, p, pb, pe);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t lo = sm.lo;
@@ -1305,6 +1332,8 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
   for (int b = tid; b < HBINS; b += BLOCK) sm.hist[b] = 0;
   for (int j = tid; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
   for (int j = tid; j < R::NPB * HALF; j += BLOCK) sm.priv[j] = 0;
+  for (int j = tid; j < NW * HBINS; j += BLOCK) (&sm.ghist[0][0])[j] = 0;
+  for (int j = tid; j < NW * NSUM * NLIMB; j += BLOCK) (&sm.gsacc[0][0][0])[j] = 0;
   if (tid < 8) sm.cnt[tid] = 0;
   rec_init(sm.rec[tid]);
   const int64_t lo = p.bounds[blockIdx.x], hi = p.bounds[blockIdx.x + 1];

@@ -79,6 +79,54 @@ bool round_tol(peat_tol_t tol, float* r, float* a) {
   return std::isfinite(*r) && std::isfinite(*a);
 }
 
+// CTA ranges of a segmented call.  A CTA pays for its elements and, per
+// segment piece it meets, a fixed CTA-wide merge worth about PIECE_COST
+// elements.  For a capacity C, a greedy walk over the segments gives the
+// fewest CTAs with cost <= C each (cutting a segment where a CTA fills up);
+// a bisection on C finds the smallest capacity that fits in max_ctas CTAs,
+// i.e. one wave.  Writes out[0..nctas] and returns nctas (0: no split fits).
+constexpr int64_t PIECE_COST = 8192;
+
+int greedy_split(const int64_t* off, int64_t nseg, int64_t n, int64_t C, int cap, int64_t* out) {
+  int nct = 0;
+  out[0] = 0;
+  int64_t cost = 0;
+  for (int64_t s = 0; s < nseg; s++) {
+    int64_t pos = off[s];
+    const int64_t s1 = off[s + 1];
+    while (pos < s1) {
+      if (cost > 0 && cost + PIECE_COST >= C) {  // no room for another piece: close the CTA
+        if (nct == cap) return 0;
+        out[++nct] = pos;
+        cost = 0;
+      }
+      const int64_t take = std::min(s1 - pos, std::max<int64_t>(1, C - cost - PIECE_COST));
+      cost += PIECE_COST + take;
+      pos += take;
+      if (pos < s1) {  // the segment goes on in the next CTA
+        if (nct == cap) return 0;
+        out[++nct] = pos;
+        cost = 0;
+      }
+    }
+  }
+  if (out[nct] < n) {
+    if (nct == cap) return 0;
+    out[++nct] = n;
+  }
+  return nct;
+}
+
+int segment_split(const int64_t* off, int64_t nseg, int64_t n, int max_ctas, int64_t* out) {
+  int64_t lo = n / max_ctas, hi = n + (nseg + 1) * PIECE_COST;  // hi always fits in one CTA
+  for (int it = 0; it < 40 && lo + 1 < hi; it++) {
+    const int64_t mid = lo + (hi - lo) / 2;
+    if (greedy_split(off, nseg, n, mid, max_ctas, out) > 0) hi = mid;
+    else lo = mid;
+  }
+  return greedy_split(off, nseg, n, hi, max_ctas, out);
+}
+
 // wait until the pinned staging buffers may be rewritten
 peat_status_t wait_staging(peat_handle_t h) {
   if (h->staged_pending) {
@@ -140,7 +188,11 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   if (ps != PEAT_OK) return ps;
   std::memcpy(h->h_offsets, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
   int64_t* hb = h->h_offsets + nseg + 1;
-  for (int b = 0; b <= p.nctas; b++) hb[b] = peat::compare_cta_bound(dtype, b, p.nctas, n, p.p0);
+  const int nsplit = nseg > 1 && n > 0 ? segment_split(offsets, nseg, n, p.nctas, hb) : 0;
+  if (nsplit > 0)
+    p.nctas = nsplit;
+  else
+    for (int b = 0; b <= p.nctas; b++) hb[b] = peat::compare_cta_bound(dtype, b, p.nctas, n, p.p0);
   cudaError_t e = cudaMemcpyAsync(h->d_offsets, h->h_offsets, sizeof(int64_t) * (size_t)(nseg + 2 + p.nctas),
                                   cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(offsets)");
@@ -293,12 +345,13 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
     return PEAT_ERR_CUDA;
   }
   h->max_ctas = std::max(1, h->nsm * peat::compare_ctas_per_sm());
-  size_t slots = (size_t)h->max_segments + (size_t)h->max_ctas;
-  size_t staging = (size_t)h->max_segments + 2 + (size_t)h->max_ctas;
+  // segmented calls may use up to 2 * max_ctas CTAs (see segment_split)
+  size_t slots = (size_t)h->max_segments + 2 * (size_t)h->max_ctas;
+  size_t staging = (size_t)h->max_segments + 2 + 2 * (size_t)h->max_ctas;
   size_t acc_bytes = (size_t)h->max_segments * peat::compare_segacc_bytes();
   bool ok = cudaMalloc(&h->partials, slots * peat::compare_partial_bytes()) == cudaSuccess &&
             cudaMalloc(&h->acc, acc_bytes) == cudaSuccess &&
-            cudaMalloc(&h->glist, sizeof(uint32_t) * (size_t)peat::GCAP * (size_t)h->max_ctas) == cudaSuccess &&
+            cudaMalloc(&h->glist, sizeof(uint32_t) * (size_t)peat::GCAP * 2 * (size_t)h->max_ctas) == cudaSuccess &&
             cudaHostAlloc((void**)&h->status_host, sizeof(unsigned int), cudaHostAllocMapped) == cudaSuccess &&
             cudaHostGetDevicePointer((void**)&h->status_dev, h->status_host, 0) == cudaSuccess &&
             cudaMemset(h->acc, 0, acc_bytes) == cudaSuccess &&

@@ -49,10 +49,10 @@ namespace {
 // ---------------------------------------------------------------------------
 // element types
 // ---------------------------------------------------------------------------
-// UBMAX: the largest window ULP bound (u < 2^UB keeps c within a factor 2 of
-// g; the per-piece UB is sampled from the data and capped here).  LBMIN and
-// LBMAX bound the window's floor binade Lb so that 2^Lexp is a normal float32
-// (Lexp = Lb - BIAS - MB) and 1.5 * 2^(Lexp+23) is finite.
+// UBMAX: the largest ULP-distance bit length the window's position allows
+// for (the window sits 20 - UB binades deep below the largest golden seen).
+// LBMIN and LBMAX bound the window's floor binade Lb so that 2^Lexp is a
+// normal float32 (Lexp = Lb - BIAS - MB) and 1.5 * 2^(Lexp+23) is finite.
 template <int DT>
 struct Tr;
 template <>
@@ -82,12 +82,14 @@ constexpr int NUR = 63;  // ULP rows
 template <int DT>
 struct Rows {
   static constexpr int KLO = -(Tr<DT>::MB + 1);
-  static constexpr int KHI = DT == PEAT_F16 ? Tr<DT>::MB - 1 : Tr<DT>::UBMAX - Tr<DT>::MB;
+  // a window pair has c within a factor 2 of g, so |d| < |g| (k <= -1) unless
+  // g is an fp16 subnormal (|d| up to 2^MB - 1 steps of it)
+  static constexpr int KHI = DT == PEAT_F16 ? Tr<DT>::MB - 1 : -1;
   static constexpr int NPB = NUR + KHI - KLO + 1;
 };
 constexpr int HALF = BLOCK / 2;
 constexpr int ROWB = HALF * 4;  // bytes per private row
-constexpr int NPB_MAX = NUR + 9 + 11 + 1;
+constexpr int NPB_MAX = NUR + 24;  // float32: k in [-24, -1]
 
 template <int DT>
 __device__ __forceinline__ float to_f32(uint32_t b) {
@@ -358,6 +360,7 @@ struct FinScratch {
   double sums[NSUM];
 };
 constexpr int NSTAGE = 2;  // a power of two: stage and phase are bit fields of the use count
+constexpr int RWMAX = 6;   // window moves per warp and piece
 constexpr int CHV = 64;
 
 struct __align__(128) Smem {
@@ -376,6 +379,11 @@ struct __align__(128) Smem {
   int last;                        // this CTA finished the last piece of a one-segment call
   FinScratch fin;
   int lb, ub;
+  // each warp's windows in the current piece: window r applies from the warp's
+  // chunk wstart[w][r] on (r = 0: the piece's initial window, also for the head)
+  uint32_t nwin[NW];
+  uint32_t wstart[NW][RWMAX + 1];
+  int wlb[NW][RWMAX + 1];
   WinRec rec[BLOCK];
   uint32_t priv[NPB_MAX * HALF];   // per-thread 16-bit counters, two threads per word
   unsigned short qp[NW][CHV * 8];  // per-warp queue: tile positions of the unequal pairs
@@ -534,6 +542,7 @@ struct Lane {
   uint32_t sa, sn;   // this tile's sum of V, and of V over negative d
   uint32_t within;   // window pairs within tolerance
   uint32_t uneq;     // unequal pairs seen (the rest of the piece is bitwise equal)
+  uint32_t ndef;     // pairs sent to the general path in the current tile
   uint64_t A, N, Q;  // this round's sums of V, of V over negative d, of V^2
 };
 
@@ -546,19 +555,48 @@ struct Thr {
   float tra, trm; // ratio tra / trm
 };
 
+// The window (warp-uniform; a warp moves it when too many of a tile's pairs
+// fall outside): Lb is the floor binade, Lexp = Lb - BIAS - MB the weight of
+// V's unit.
 struct Win {
   float rtol, atol;
   float gmin;       // smallest |g| of a window pair: 2^(Lb + 1 - BIAS)
   float lim;        // |d| < 2^(Lexp + 22)
   float M;          // 1.5 * 2^(Lexp + 23): bits(|d| + M) - bits(M) = |d| / 2^Lexp
-  uint32_t udmax;   // window bound on ud (u < 2^UB)
+  int lb;           // Lb
   uint32_t base;    // shared address of this thread's counter in private row 0
   uint32_t inc;     // 1 (low half of the word) or 65536 (high half)
 };
 
+// the window with floor binade lb
+template <int DT>
+__device__ __forceinline__ void set_window_lb(Win& W, int lb) {
+  using Ty = Tr<DT>;
+  const int lexp = lb - Ty::BIAS - Ty::MB;
+  W.lb = lb;
+  W.gmin = (DT == PEAT_F16 && lb == Ty::LBMIN) ? __uint_as_float((uint32_t)(127 - 24) << 23)
+                                                 : __uint_as_float((uint32_t)(lb + 1 - Ty::BIAS + 127) << 23);
+  W.lim = __uint_as_float((uint32_t)(lexp + 22 + 127) << 23);
+  W.M = __uint_as_float(((uint32_t)(lexp + 23 + 127) << 23) | 0x400000u);
+}
+// The window placed for data whose largest finite golden exponent is emax and
+// whose ULP distances have ubits bits: V = |d| / 2^Lexp < 2^22 for such pairs
+// with goldens up to 2 binades above emax (one bit to spare on u).
+template <int DT>
+__device__ __forceinline__ int window_floor(int emax, int ubits) {
+  using Ty = Tr<DT>;
+  const int UB = min(ubits + 1, Ty::UBMAX);
+  const int lb = emax + UB - 20;
+  return lb < Ty::LBMIN ? Ty::LBMIN : (lb > Ty::LBMAX ? Ty::LBMAX : lb);
+}
+template <int DT>
+__device__ __forceinline__ int win_lexp(const Win& W) {
+  return W.lb - Tr<DT>::BIAS - Tr<DT>::MB;
+}
+
 __device__ __forceinline__ void lane_init(Lane& L) {
   L.sa = L.sn = 0;
-  L.within = L.uneq = 0;
+  L.within = L.uneq = L.ndef = 0;
   L.A = L.N = L.Q = 0;
 }
 __device__ __forceinline__ void thr_init(Thr& T) {
@@ -610,9 +648,15 @@ __device__ __forceinline__ bool rel_greater(float an1, float m1, float an2, floa
 
 // The window test.  gr, cr: raw bits (bf16: the float32 bits, i.e. raw << 16);
 // gf, cf: the values.  Also returns ud (the ULP distance, bf16: scaled by
-// 2^16), s = c - g, a = |s| and thr.  No sign test is needed: a pair of
-// opposite signs has ud >= 2^23 (bf16 scaled, float32) or >= 2^10 (fp16),
-// beyond every window bound.
+// 2^16), s = c - g, a = |s| and thr.  u < 2^MB keeps c within a factor 2 of
+// g (so c - g is exact in float32, Sterbenz); |g| >= gmin makes g and c
+// multiples of 2^Lexp; |d| < lim bounds V below 2^22; a tolerance tie goes to
+// the general path.  No sign test is needed: a pair of opposite signs has
+// ud > 2^23 (float32, bf16 scaled) or > 2^10 (fp16), beyond the bound.
+template <int DT>
+__device__ __forceinline__ uint32_t ud_bound() {
+  return DT == PEAT_BF16 ? (1u << Tr<DT>::MB) << 16 : 1u << Tr<DT>::MB;
+}
 template <int DT>
 __device__ __forceinline__ bool in_window(uint32_t gr, uint32_t cr, float gf, float cf, const Win& W, uint32_t& ud,
                                           float& s, float& a, float& thr) {
@@ -624,7 +668,7 @@ __device__ __forceinline__ bool in_window(uint32_t gr, uint32_t cr, float gf, fl
   a = fabsf(s);
   const float ag = fabsf(gf);
   thr = __fmaf_rn(W.rtol, ag, W.atol);
-  return ud < W.udmax && ag >= W.gmin && a < W.lim && a != thr;
+  return ud < ud_bound<DT>() && ag >= W.gmin && a < W.lim && a != thr;
 }
 
 // normalised ratio |d| / |g| = an / mg, mg in [1, 2)
@@ -652,6 +696,7 @@ __device__ __forceinline__ bool pair_proc(Lane& L, const Thr& T, uint32_t gr, ui
   float s, a, thr;
   if (!in_window<DT>(gr, cr, gf, cf, W, ud, s, a, thr)) {
     defer_pair(li, sm);
+    L.ndef++;
     return false;
   }
   L.within += a < thr ? 1u : 0u;
@@ -777,6 +822,79 @@ __device__ __forceinline__ void count_equal(const uint4& g, uint32_t eqm, Smem& 
   if (eqm && any_nonfinite<DT>(g)) atomicAdd(&sm.nfe, (uint32_t)__popc(nonfinite_lanes<DT>(g) & eqm));
 }
 
+__device__ __forceinline__ uint64_t wsum64(uint64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+  return v;
+}
+
+// This warp's window sums (in units of 2^lexp) into the CTA's exact
+// accumulator: A, N < 2^38 and Q < 2^60 per thread between flushes; warp sums
+// in 128 bits.
+__device__ __forceinline__ void flush_sums(Lane& L, Smem& sm, int lexp) {
+  const uint64_t A = wsum64(L.A), N = wsum64(L.N);
+  const uint64_t qlo = wsum64(L.Q & 0xFFFFFFFFull), qhi = wsum64(L.Q >> 32);
+  if ((threadIdx.x & 31) == 0) {
+    const uint64_t P = A - N;  // sum of V over positive d
+    if (P >= N) sacc_add(sm, 0, (unsigned __int128)(P - N), lexp, false);
+    else sacc_add(sm, 0, (unsigned __int128)(N - P), lexp, true);
+    sacc_add(sm, 1, (unsigned __int128)A, lexp, false);
+    sacc_add(sm, 2, (unsigned __int128)qlo + ((unsigned __int128)qhi << 32), 2 * lexp, false);
+  }
+  L.A = L.N = L.Q = 0;
+}
+
+// When a tile sent many pairs (at least 32, and a quarter of its unequal
+// ones) to the general path, the warp moves its window to the tile's own data
+// -- largest finite golden exponent, largest same-sign ULP distance -- after
+// flushing the sums kept in the old window's units, and logs the move so that
+// a rescan of the piece applies to every pair the window it saw.  At most
+// RWMAX moves per warp and piece.
+// the window floor for the data of a staged tile (out of line: rarely run)
+template <int DT>
+__device__ __noinline__ int tile_window_floor(const uint4* gt, const uint4* ct, int nvalid) {
+  using Ty = Tr<DT>;
+  const int lane = threadIdx.x & 31;
+  uint32_t emax = 0, umax = 0;
+#pragma unroll
+  for (int v = 0; v < 2; v++) {
+    if (lane + 32 * v >= nvalid) continue;
+    const uint4 gv = gt[lane + 32 * v], cv = ct[lane + 32 * v];
+#pragma unroll
+    for (int j = 0; j < Ty::VEC; j++) {
+      const uint32_t G = lane_bits<DT>(gv, j), C = lane_bits<DT>(cv, j);
+      const uint32_t e = (G & Ty::MAG) >> Ty::MB;
+      if (e < (uint32_t)Ty::EMAX && e > emax) emax = e;
+      if (((G ^ C) & Ty::SIGN) == 0u && (G & Ty::MAG) < Ty::INF && (C & Ty::MAG) < Ty::INF)
+        umax = max(umax, G > C ? G - C : C - G);
+    }
+  }
+  emax = __reduce_max_sync(0xFFFFFFFFu, emax);
+  umax = __reduce_max_sync(0xFFFFFFFFu, umax);
+  return window_floor<DT>((int)emax, 32 - __clz(umax));
+}
+
+// nd: the warp's general pairs of this tile, total: its unequal pairs
+template <int DT>
+__device__ __forceinline__ void maybe_rewindow(Lane& L, Win& W, const uint4* gt, const uint4* ct, int nvalid,
+                                               uint32_t nd, uint32_t total, uint32_t ichunk, Smem& sm) {
+  if (nd < 32u || nd * 4u < total) return;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t r = sm.nwin[warp];
+  if (r >= (uint32_t)RWMAX) return;
+  const int lb = tile_window_floor<DT>(gt, ct, nvalid);
+  if (lb == W.lb) return;
+  flush_sums(L, sm, win_lexp<DT>(W));
+  set_window_lb<DT>(W, lb);
+  __syncwarp();
+  if (lane == 0) {
+    sm.wstart[warp][r + 1] = ichunk + 1;
+    sm.wlb[warp][r + 1] = lb;
+    sm.nwin[warp] = r + 1;
+  }
+  __syncwarp();
+}
+
 // One warp tile of CHV vectors staged in shared memory: lane L owns vectors L
 // and L + 32; tile element e sits at offset tli + e from the CTA's first
 // element.  Equal pairs are counted in place.  When at most a quarter of the
@@ -785,8 +903,8 @@ __device__ __forceinline__ void count_equal(const uint4& g, uint32_t eqm, Smem& 
 // processed 32 at a time, so every thread does useful work.  Pairs above the
 // thread's maxima are then evaluated exactly.
 template <int DT>
-__device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nvalid, uint32_t tli, const Win& W,
-                                        Smem& sm) {
+__device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nvalid, uint32_t tli, Win& W,
+                                        uint32_t ichunk, Smem& sm) {
   // the candidate ring sits a fixed distance after the golden ring
   const uint4* ct = gt + (offsetof(Smem, ring_c) - offsetof(Smem, ring_g)) / sizeof(uint4);
   using Ty = Tr<DT>;
@@ -817,9 +935,9 @@ __device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nv
   const uint32_t nA = okA ? unequal_mask<DT>(gA, cA) : 0u, nB = okB ? unequal_mask<DT>(gB, cB) : 0u;
   if (okA) count_equal<DT>(gA, FULL & ~nA, sm);
   if (okB) count_equal<DT>(gB, FULL & ~nB, sm);
-  // queue the unequal positions; one scan of the packed counts gives the
-  // A-queue and B-queue offsets
-  const uint32_t packed = __popc(nA) | (__popc(nB) << 16);
+  // one scan of the packed counts gives the A-queue and B-queue offsets (10-bit
+  // fields: a warp tile has at most 512 pairs)
+  const uint32_t packed = __popc(nA) | (__popc(nB) << 10);
   uint32_t incl = packed;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -827,7 +945,7 @@ __device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nv
     if (lane >= o) incl += t;
   }
   const uint32_t tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
-  const uint32_t totA = tot & 0xFFFFu, total = totA + (tot >> 16);
+  const uint32_t totA = tot & 0x3FFu, total = totA + ((tot >> 10) & 0x3FFu);
   L.uneq += __popc(nA) + __popc(nB);
   if (total * 4u <= 64u * VEC) {
     // sparse tile: each lane visits its own unequal pairs (slot s < VEC:
@@ -859,11 +977,12 @@ __device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nv
         rescan_pair<DT>(gr, cr, gf, cf, tli + pos, W, r, T);
       } while (cm);
     }
+    L.ndef = 0;  // sparse tiles never move the window (a quarter of their pairs at most differ)
     __syncwarp();
     return;
   }
-  uint32_t posA = (incl & 0xFFFFu) - (packed & 0xFFFFu);
-  uint32_t posB = totA + (incl >> 16) - (packed >> 16);
+  uint32_t posA = (incl & 0x3FFu) - (packed & 0x3FFu);
+  uint32_t posB = totA + ((incl >> 10) & 0x3FFu) - ((packed >> 10) & 0x3FFu);
   unsigned short* q = sm.qp[warp];
 #pragma unroll
   for (int j = 0; j < VEC; j++) {
@@ -903,6 +1022,11 @@ __device__ __forceinline__ void do_tile(Lane& L, Thr& T, const uint4* gt, int nv
       elem_at<DT>(ct, pos, cr, cf);
       rescan_pair<DT>(gr, cr, gf, cf, tli + pos, W, r, T);
     } while (cm);
+  }
+  {
+    const uint32_t nd = __reduce_add_sync(0xFFFFFFFFu, L.ndef);
+    L.ndef = 0;
+    maybe_rewindow<DT>(L, W, gt, ct, nvalid, nd, total, ichunk, sm);
   }
   __syncwarp();
 }
@@ -1049,10 +1173,6 @@ __device__ __forceinline__ void part_warp_reduce(Partial& x) {
   }
 }
 
-__device__ __forceinline__ uint64_t warp_sum64(uint64_t v) {
-  for (int o = 16; o > 0; o >>= 1) v += (uint64_t)shfl_i64((int64_t)v, o);
-  return v;
-}
 
 // warp sums of the general path's class counters into the CTA counters
 __device__ __forceinline__ void gen_counts(const GenRec& g, Smem& sm) {
@@ -1078,7 +1198,8 @@ __device__ __forceinline__ void gen_counts(const GenRec& g, Smem& sm) {
 // of the piece with the same window test.  Out of line, so that the hot loop
 // carries no call.  Leaves each warp's general maxima in sm.wbest[warp].
 template <int DT>
-__device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p, int64_t pb, int64_t pe) {
+__device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p, int64_t pb, int64_t pe,
+                                         int64_t vb, int64_t ve) {
   __syncthreads();
   const uint32_t n = sm.gn;
   if (n == 0) {  // no general pair in this piece
@@ -1102,9 +1223,28 @@ __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p
         gr = G << 16;
         cr = C << 16;
       }
+      // the window this pair was tested with: the head ran with the initial
+      // window, a body chunk with its warp's window of that time, the tail
+      // with its thread's warp's last window
+      int w = 0;
+      uint32_t ik = 0;
+      if (vb < ve && i >= vb) {
+        if (i >= ve) {
+          w = (int)(((i - ve) % BLOCK) >> 5);
+          ik = 0xFFFFFFFFu;
+        } else {
+          const int64_t k = (i - vb) / (CHV * Tr<DT>::VEC);
+          w = (int)(k % NW);
+          ik = (uint32_t)(k / NW);
+        }
+      }
+      int r = (int)sm.nwin[w];
+      while (r > 0 && sm.wstart[w][r] > ik) r--;
+      Win Wi = W;
+      set_window_lb<DT>(Wi, sm.wlb[w][r]);
       uint32_t ud;
       float s, a, thr;
-      if (!in_window<DT>(gr, cr, to_f32<DT>(G), to_f32<DT>(C), W, ud, s, a, thr))
+      if (!in_window<DT>(gr, cr, to_f32<DT>(G), to_f32<DT>(C), Wi, ud, s, a, thr))
         general_lane<DT>(sm, cd, G, C, i, W.rtol, W.atol);
     }
   }
@@ -1160,17 +1300,7 @@ template <int DT>
 __device__ void fold_round(Lane& L, Smem& sm, int lexp) {
   constexpr int NPB = Rows<DT>::NPB;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  // window sums: A, N < 2^38 and Q < 2^60 per thread per round; warp sums in 128 bits
-  const uint64_t A = warp_sum64(L.A), N = warp_sum64(L.N);
-  const uint64_t qlo = warp_sum64(L.Q & 0xFFFFFFFFull), qhi = warp_sum64(L.Q >> 32);
-  if (lane == 0) {
-    const uint64_t P = A - N;  // sum of V over positive d
-    if (P >= N) sacc_add(sm, 0, (unsigned __int128)(P - N), lexp, false);
-    else sacc_add(sm, 0, (unsigned __int128)(N - P), lexp, true);
-    sacc_add(sm, 1, (unsigned __int128)A, lexp, false);
-    sacc_add(sm, 2, (unsigned __int128)qlo + ((unsigned __int128)qhi << 32), 2 * lexp, false);
-  }
-  L.A = L.N = L.Q = 0;
+  flush_sums(L, sm, lexp);  // lexp: this warp's window
   __syncthreads();
   // private rows: one warp per row
   for (int r = warp; r < NPB; r += NW) {
@@ -1196,12 +1326,12 @@ __device__ void write_empty_segments(const CompareParams& p);
 // accumulator (global atomics), the maxima to the CTA's partial slot.  The
 // CTA that finishes the segment's last piece then finalizes the segment.
 template <int DT>
-__device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, int lexp, const CompareParams& p,
-                                             int64_t seg, int64_t pb, int64_t pe) {
+__device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, const CompareParams& p,
+                                             int64_t seg, int64_t pb, int64_t pe, int64_t vb, int64_t ve) {
   Partial* out = p.partials + seg + blockIdx.x;
   SegAcc* acc = p.acc + seg;
-  run_general<DT>(W, sm, p, pb, pe);
-  fold_round<DT>(L, sm, lexp);  // ends with a barrier: the general path's per-warp totals are complete
+  run_general<DT>(W, sm, p, pb, pe, vb, ve);
+  fold_round<DT>(L, sm, win_lexp<DT>(W));  // ends with a barrier: the general path's per-warp totals are complete
   for (int b = threadIdx.x; b < HBINS; b += BLOCK) {
     unsigned long long v = 0;
 #pragma unroll
@@ -1410,18 +1540,16 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
       atomicMax(&sm.ub, (int)(32 - __clz(umax)));
     }
     __syncthreads();
-    // u < 2^UB with one bit to spare over the sample; V = |d| / 2^Lexp < 2^22
-    // for such pairs with goldens up to 2 binades above the largest seen
-    int UB = sm.ub + 1;
-    UB = UB > Ty::UBMAX ? Ty::UBMAX : UB;
-    int lb = sm.lb + UB - 20;
-    lb = lb < Ty::LBMIN ? Ty::LBMIN : (lb > Ty::LBMAX ? Ty::LBMAX : lb);
-    const int lexp = lb - Ty::BIAS - Ty::MB;  // weight of V's unit
-    W.gmin = (DT == PEAT_F16 && lb == Ty::LBMIN) ? __uint_as_float((uint32_t)(127 - 24) << 23)
-                                                   : __uint_as_float((uint32_t)(lb + 1 - Ty::BIAS + 127) << 23);
-    W.lim = __uint_as_float((uint32_t)(lexp + 22 + 127) << 23);
-    W.M = __uint_as_float(((uint32_t)(lexp + 23 + 127) << 23) | 0x400000u);
-    W.udmax = (1u << UB) << (DT == PEAT_BF16 ? 16 : 0);
+    // the piece's initial window, the first entry of every warp's window log
+    {
+      const int lb0 = window_floor<DT>(sm.lb, sm.ub);
+      set_window_lb<DT>(W, lb0);
+      if (lane == 0) {
+        sm.nwin[warp] = 0;
+        sm.wstart[warp][0] = 0;
+        sm.wlb[warp][0] = lb0;
+      }
+    }
     Thr T;
     thr_init(T);
     auto scalar_range = [&](int64_t b0, int64_t b1) {
@@ -1436,7 +1564,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
       for (int64_t r0 = pb; r0 < h_end; r0 += ROUND_ELEMS) {
         const int64_t r1 = min(h_end, r0 + ROUND_ELEMS);
         scalar_range(r0, r1);
-        if (r1 < h_end) fold_round<DT>(L, sm, lexp);
+        if (r1 < h_end) fold_round<DT>(L, sm, win_lexp<DT>(W));
       }
     }
     // vector body: warp w takes chunks w, w + NW, ... of CHV vectors from its
@@ -1458,12 +1586,12 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
         if (!failed) {
           const int64_t v0 = k * CHV;
           const int nvalid = (int)min((int64_t)CHV, nvec - v0);
-          do_tile<DT>(L, T, sm.ring_g[warp][st], nvalid, (uint32_t)(vb + v0 * VEC - lo), W, sm);
+          do_tile<DT>(L, T, sm.ring_g[warp][st], nvalid, (uint32_t)(vb + v0 * VEC - lo), W, (uint32_t)i, sm);
           if (lane == 0 && i + NSTAGE < my_chunks) issue(seq + NSTAGE, warp + NW * (i + NSTAGE));
         }
         seq++;
       }
-      if (r1 < nchunk) fold_round<DT>(L, sm, lexp);
+      if (r1 < nchunk) fold_round<DT>(L, sm, win_lexp<DT>(W));
     }
     if (fail_i >= 0) {
       // copies this warp issued but never consumed: wait for them before the
@@ -1475,7 +1603,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
     }
     // scalar tail (fewer than VEC elements), after the body
     if (vb < ve && ve < pe) scalar_range(ve, pe);
-    finish_piece<DT>(L, W, sm, lexp, p, s, pb, pe);
+    finish_piece<DT>(L, W, sm, p, s, pb, pe, vb, ve);
     pb = pe;
   }
 }

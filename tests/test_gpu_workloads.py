@@ -66,6 +66,17 @@ def test_c3_resnet50_full(peat_gpu, oracle, h):
     assert len(st) == 161
 
 
+def test_c3_resnet50_flattened_one_segment(peat_gpu, oracle, h):
+    """All 161 parameter tensors as one flat buffer: the error statistics change
+    from tensor to tensor inside every CTA's range, so warps move their windows
+    (and CTAs holding many general pairs rescan with the logged windows)."""
+    from paper_2609_13544_gb300 import workloads as W
+    w = W.c3_resnet50(device="cuda")
+    w.offsets = None
+    st = compare_workload(peat_gpu, oracle, h, w, "c3-flat")
+    assert st["n"] == 25_557_032
+
+
 def small_gpt_shapes():
     d, vocab, layers = 256, 4000, 3
     shapes = [(vocab, d), (512, d)]

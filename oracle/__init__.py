@@ -47,6 +47,16 @@ class Stats(ctypes.Structure):
     ]
 
 
+class TopK(ctypes.Structure):
+    _fields_ = [
+        ("n_finite", ctypes.c_uint64),
+        ("k", ctypes.c_uint64),
+        ("threshold", ctypes.c_double),
+        ("sum", ctypes.c_double),
+        ("mean", ctypes.c_double),
+    ]
+
+
 class InjectModel(ctypes.Structure):
     _fields_ = [
         ("kind", ctypes.c_int32),
@@ -70,6 +80,8 @@ def lib() -> ctypes.CDLL:
         L.orc_compare.restype = i32
         L.orc_compare_segmented.argtypes = [vp, vp, vp, i64, i32, dbl, dbl, ctypes.POINTER(Stats), vp]
         L.orc_compare_segmented.restype = i32
+        L.orc_topk_mean.argtypes = [vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, ctypes.POINTER(TopK)]
+        L.orc_topk_mean.restype = i32
         L.orc_ulp_key.argtypes = [ctypes.c_uint32, i32]
         L.orc_ulp_key.restype = i64
         L.orc_exact_sum.argtypes = [vp, i64]
@@ -122,6 +134,19 @@ def compare(g, c, dtype: str, rtol: float, atol: float = 0.0):
     if rc:
         raise ValueError(f"oracle rejected the arguments (code {rc})")
     return _stats_dict(st), hist
+
+
+def topk_mean(g, c, dtype: str, num: int = 1, den: int = 10) -> dict:
+    """Mean of the ceil(n_finite * num / den) largest |c - g| (Section IV-B-3,
+    "Mean of Top 10% Errors"): dict of n_finite, k, threshold, sum, mean."""
+    gb, cb = _bits(g, dtype), _bits(c, dtype)
+    if gb.size != cb.size:
+        raise ValueError("golden and candidate differ in length")
+    out = TopK()
+    rc = lib().orc_topk_mean(gb.ctypes.data, cb.ctypes.data, gb.size, DTYPES[dtype], num, den, ctypes.byref(out))
+    if rc:
+        raise ValueError(f"oracle rejected the arguments (code {rc})")
+    return {f: getattr(out, f) for f, _ in TopK._fields_}
 
 
 def compare_segmented(g, c, offsets: Sequence[int], dtype: str, rtol: float, atol: float = 0.0):

@@ -517,6 +517,83 @@ int orc_compare_segmented(const void* g, const void* c, const int64_t* offsets, 
 }
 
 /* ------------------------------------------------------------------------ */
+/* Mean of the top errors (Section IV-B-3, "Mean of Top 10% Errors").  Every  */
+/* finite |d| is kept exactly as s + t (s = RN64(|d|)); sorting on (s, t)   */
+/* orders the exact values (RN64 is monotone, and equal s leave t1 - t2 as  */
+/* the exact difference); the k largest are added in the exact accumulator. */
+/* ------------------------------------------------------------------------ */
+static int cmp_mag2_desc(const void* x, const void* y) {
+  const mag2_t* a = (const mag2_t*)x;
+  const mag2_t* b = (const mag2_t*)y;
+  if (a->s != b->s) return a->s > b->s ? -1 : 1;
+  if (a->t != b->t) return a->t > b->t ? -1 : 1;
+  return 0;
+}
+
+/* RN-even double of (value of a) / k for a >= 0 and k >= 1: the value is
+ * shifted up 128 bits before an exact long division, so the quotient carries
+ * at least 64 significant bits and the remainder only sets the sticky bit. */
+static double acc_div_rn(const acc_t* in, uint64_t k) {
+  acc_t a = *in, q;
+  for (int j = ACC_W - 1; j >= 2; j--) a.w[j] = a.w[j - 2];
+  a.w[1] = a.w[0] = 0;
+  u128 rem = 0;
+  for (int j = ACC_W - 1; j >= 0; j--) {
+    u128 cur = (rem << 64) | a.w[j];
+    q.w[j] = (uint64_t)(cur / k);
+    rem = cur % k;
+  }
+  int top = -1;
+  for (int j = ACC_W - 1; j >= 0 && top < 0; j--)
+    if (q.w[j]) top = j * 64 + 63 - __builtin_clzll(q.w[j]);
+  if (top < 0) return 0.0;
+  uint64_t mant = 0;
+  for (int b = top; b > top - 53; b--) mant = (mant << 1) | (uint64_t)acc_bit(&q, b);
+  int round = acc_bit(&q, top - 53);
+  int sticky = rem != 0;
+  for (int b = top - 54; b >= 0 && !sticky; b--) sticky = acc_bit(&q, b);
+  if (round && (sticky || (mant & 1u))) mant++;
+  return ldexp((double)mant, top - 52 + ACC_LSB - 128);
+}
+
+int orc_topk_mean(const void* g, const void* c, int64_t n, int dtype, uint64_t num, uint64_t den, orc_topk* out) {
+  if (!dtype_ok(dtype) || n < 0 || !out || (n > 0 && (!g || !c)) || den == 0 || num == 0 || num > den)
+    return ORC_BAD_ARG;
+  memset(out, 0, sizeof(*out));
+  mag2_t* m = (mag2_t*)malloc(sizeof(mag2_t) * (size_t)(n > 0 ? n : 1));
+  if (!m) abort();
+  uint64_t nf = 0;
+  for (int64_t i = 0; i < n; i++) {
+    val_t vg = decode(raw_bits(g, i, dtype), dtype), vc = decode(raw_bits(c, i, dtype), dtype);
+    if (vg.nan || vg.inf || vc.nan || vc.inf) continue;
+    double s, t;
+    two_sum(vc.v, -vg.v, &s, &t); /* d = s + t exactly */
+    m[nf].s = fabs(s);
+    m[nf].t = s < 0 ? -t : t;     /* |d| = |s| + (sign of s) t */
+    nf++;
+  }
+  out->n_finite = nf;
+  /* k = ceil(nf * num / den), exact */
+  u128 prod = (u128)nf * num;
+  uint64_t k = (uint64_t)((prod + den - 1) / den);
+  out->k = k;
+  if (k > 0) {
+    qsort(m, (size_t)nf, sizeof(mag2_t), cmp_mag2_desc);
+    acc_t a;
+    acc_zero(&a);
+    for (uint64_t i = 0; i < k; i++) {
+      acc_add_double(&a, m[i].s, 0);
+      acc_add_double(&a, m[i].t, 0);
+    }
+    out->threshold = m[k - 1].s;
+    out->sum = acc_to_double(&a);
+    out->mean = acc_div_rn(&a, k);
+  }
+  free(m);
+  return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Pseudo-error injector.                                                    */
 /* Randomness: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random  */
 /* numbers: as easy as 1, 2, 3", SC'11), key = the 64-bit seed, counter =    */

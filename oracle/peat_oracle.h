@@ -62,6 +62,20 @@ int orc_compare(const void* g, const void* c, int64_t n, int dtype, double rtol,
 int orc_compare_segmented(const void* g, const void* c, const int64_t* offsets, int64_t nseg,
                           int dtype, double rtol, double atol, orc_stats* st, uint64_t* hist);
 
+/* Mean of the top errors (Section IV-B-3, "Mean of Top 10% Errors"): over
+ * the pairs with both operands finite, the k = ceil(n_finite * num / den)
+ * largest |c - g| (0 < num <= den; the paper's score is num/den = 1/10).
+ * Ties do not change the value.  All quantities exact, then RN64. */
+typedef struct {
+  uint64_t n_finite;  /* pairs with both operands finite */
+  uint64_t k;         /* pairs taken */
+  double threshold;   /* RN64 of the k-th largest |c - g| (0 if k = 0) */
+  double sum;         /* RN64 of the exact sum of the k largest |c - g| */
+  double mean;        /* RN64 of that exact sum divided by k (0 if k = 0) */
+} orc_topk;
+
+int orc_topk_mean(const void* g, const void* c, int64_t n, int dtype, uint64_t num, uint64_t den, orc_topk* out);
+
 /* ULP key of one raw bit pattern: +magnitude bits, negated when the sign
  * bit is set (so both zeros map to 0).  Exposed for the tests. */
 int64_t orc_ulp_key(uint32_t bits, int dtype);

@@ -472,3 +472,53 @@ def test_inject_rate_and_noise_models(oracle):
     y = dst.view(np.float32).astype(np.float16)
     up = np.nextafter(y, np.where(src >= 0, np.float16(np.inf), np.float16(-np.inf)))
     assert np.all(np.abs(y.astype(np.float64)) <= np.abs(src)) and np.all(np.abs(up.astype(np.float64)) > np.abs(src))
+
+
+# ---------------------------------------------------------------- mean of the top errors
+def ref_topk(g, c, dtype, num, den):
+    """Mean of the top errors from exact rationals: sort every finite |c - g|,
+    take the ceil(n_finite * num / den) largest, add and divide exactly."""
+    a = []
+    for gb, cb in zip(g.tolist(), c.tolist()):
+        gv, cv = decode(int(gb), dtype), decode(int(cb), dtype)
+        if math.isfinite(gv) and math.isfinite(cv):
+            a.append(abs(Fraction(cv) - Fraction(gv)))
+    a.sort(reverse=True)
+    k = -(-len(a) * num // den)
+    if k == 0:
+        return {"n_finite": len(a), "k": 0, "threshold": 0.0, "sum": 0.0, "mean": 0.0}
+    S = sum(a[:k], Fraction(0))
+    return {"n_finite": len(a), "k": k, "threshold": float(a[k - 1]), "sum": float(S), "mean": float(S / k)}
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16"])
+@pytest.mark.parametrize("frac", [(1, 10), (1, 1), (3, 7), (1, 1000)])
+def test_topk_against_exact_rationals(oracle, dtype, frac):
+    rng = np.random.default_rng({"f32": 31, "f16": 32, "bf16": 33}[dtype] + frac[1])
+    g, c = _random_pairs(dtype, 2000, rng)
+    got = oracle.topk_mean(g, c, dtype, *frac)
+    assert got == ref_topk(g, c, dtype, *frac)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16"])
+def test_topk_whole_population_is_the_mean_error(oracle, dtype):
+    # num = den takes every finite pair: the sum is the signature's sum |d|
+    rng = np.random.default_rng(41)
+    g, c = _random_pairs(dtype, 3000, rng)
+    st, _ = oracle.compare(g, c, dtype, 1e-3, 0.0)
+    got = oracle.topk_mean(g, c, dtype, 1, 1)
+    assert got["k"] == got["n_finite"] == st["n_finite"]
+    assert got["sum"] == st["sum_abs"]
+
+
+def test_topk_ties_zeros_and_arguments(oracle):
+    x = np.full(1000, 0x3F80, np.uint16)            # bf16 1.0
+    y = np.full(1000, 0x3F81, np.uint16)            # one step above: every |d| = 2^-7
+    got = oracle.topk_mean(x, y, "bf16", 1, 10)
+    assert got == {"n_finite": 1000, "k": 100, "threshold": 2.0 ** -7, "sum": 100 * 2.0 ** -7, "mean": 2.0 ** -7}
+    assert oracle.topk_mean(x, x, "bf16", 1, 10)["mean"] == 0.0      # self-compare
+    nan = np.full(10, 0x7FC0, np.uint16)
+    assert oracle.topk_mean(nan, nan, "bf16", 1, 10)["k"] == 0       # no finite pair
+    for num, den in ((0, 10), (11, 10), (1, 0)):
+        with pytest.raises(ValueError):
+            oracle.topk_mean(x, y, "bf16", num, den)

@@ -215,6 +215,38 @@ peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* s
                                        peat_dtype_t dtype, const peat_inject_t* models, int nmodels,
                                        uint64_t seed, uint64_t* counts_out, peat_stream_t stream);
 
+/* Mean of the top errors of one tensor pair (Section IV-B-3, "Mean of Top
+ * 10% Errors").  48 bytes. */
+typedef struct {
+  uint64_t n_finite;  /* pairs with both operands finite */
+  uint64_t k;         /* pairs taken: ceil(n_finite * num / den) */
+  double threshold;   /* RN64 of the k-th largest |c - g| (0 if k = 0) */
+  double sum;         /* RN64 of the exact sum of the k largest |c - g| */
+  double mean;        /* RN64 of that exact sum divided by k (0 if k = 0) */
+  uint32_t exact;     /* 1: every field exact as defined.  0: more than 4096 pairs whose
+                         |c - g| is not a float32 value (float32 or float16 operands of
+                         different magnitudes) share the float32 rounding of the k-th
+                         largest; they were then ordered by that rounding alone, so sum
+                         and mean may be off by their rounding errors */
+  uint32_t reserved;
+} peat_topk_t;
+
+/* Mean of the top errors: over the pairs with both operands finite, the
+ * k = ceil(n_finite * num / den) largest |c - g| (0 < num <= den; the paper's
+ * score is num/den = 1/10), their exact sum and its exact mean, each rounded
+ * once to nearest-even binary64.  Ties do not change the value.
+ *   golden, candidate  as for peat_compare (device, any alignment).
+ *   out                device pointer to one peat_topk_t.
+ * Streams both tensors four times (three digit-histogram passes of a radix
+ * select, then the exact sum), asynchronously on `stream`; the handle's
+ * workspace is shared with its other calls (do not overlap them).
+ * Errors: INVALID_ARG (null pointer with n > 0, n < 0, bad dtype, num = 0,
+ * num > den, out NULL), UNSUPPORTED (more than 2^24 elements per thread of the
+ * grid: n above about 2^42 on a 152-SM GPU), CUDA. */
+peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* candidate, int64_t n,
+                             peat_dtype_t dtype, uint64_t num, uint64_t den, peat_topk_t* out,
+                             peat_stream_t stream);
+
 /* Text of the last error reported on h (never NULL; "" if none).  With
  * h == NULL, the last error on this thread of peat_signature_create or of
  * peat_compare_noalloc, whichever failed last. */

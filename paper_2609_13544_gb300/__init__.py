@@ -31,6 +31,13 @@ PEAT_FLAG_TEST_EXPIRE_WAITS = 0x80000000
 STATUS = {0: "PEAT_OK", 1: "PEAT_ERR_INVALID_ARG", 2: "PEAT_ERR_UNSUPPORTED", 3: "PEAT_ERR_ALLOC",
           4: "PEAT_ERR_CUDA", 5: "PEAT_ERR_TIMEOUT", 6: "PEAT_ERR_INTERNAL"}
 
+TOPK_BYTES = 48
+
+# numpy view of peat_topk_t
+TOPK_DTYPE = np.dtype([("n_finite", "<u8"), ("k", "<u8"), ("threshold", "<f8"), ("sum", "<f8"), ("mean", "<f8"),
+                       ("exact", "<u4"), ("reserved", "<u4")])
+assert TOPK_DTYPE.itemsize == TOPK_BYTES
+
 # numpy view of peat_stats_t
 STATS_DTYPE = np.dtype([
     ("n", "<u8"), ("count", "<u8", (5,)), ("n_finite", "<u8"),
@@ -62,7 +69,7 @@ class InjectModel(ctypes.Structure):
 
 
 EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
-           "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc")
+           "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc", "peat_topk_mean")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -93,6 +100,8 @@ def load(path: Optional[Path] = None) -> ctypes.CDLL:
     L.peat_last_error.restype = ctypes.c_char_p
     L.peat_compare_noalloc.argtypes = [vp, vp, i64, i32, Tol, vp, vp, vp]
     L.peat_compare_noalloc.restype = i32
+    L.peat_topk_mean.argtypes = [vp, vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, vp, vp]
+    L.peat_topk_mean.restype = i32
     _lib = L
     return L
 
@@ -251,6 +260,26 @@ def peat_compare_segmented(h: Handle, golden, candidate, offsets: Sequence[int],
         return [], np.zeros((0, 2, 64), np.uint64)
     s = stats_to_dicts(stats.cpu().numpy()[: nseg * STATS_BYTES])
     return s, hist.cpu().numpy()[: nseg * HIST_BINS].view(np.uint64).reshape(nseg, 2, 64)
+
+
+def peat_topk_mean_raw(h: Handle, golden, candidate, num: int, den: int, out, stream=None) -> None:
+    """peat_topk_mean on a preallocated device output (out: uint8[48])."""
+    _dev_tensor_check(golden, candidate)
+    if golden.numel() != candidate.numel() or golden.dtype != candidate.dtype:
+        raise ValueError("golden and candidate differ in size or dtype")
+    rc = load().peat_topk_mean(h.ptr, golden.data_ptr(), candidate.data_ptr(), golden.numel(), dtype_code(golden),
+                               ctypes.c_uint64(num), ctypes.c_uint64(den), out.data_ptr(), _stream_ptr(stream))
+    _check(rc, h)
+
+
+def peat_topk_mean(h: Handle, golden, candidate, num: int = 1, den: int = 10, stream=None) -> dict:
+    """Mean of the top num/den of the errors of one tensor pair: dict of n_finite, k,
+    threshold, sum, mean, exact; synchronises."""
+    import torch
+    out = torch.empty(TOPK_BYTES, dtype=torch.uint8, device=golden.device)
+    peat_topk_mean_raw(h, golden, candidate, num, den, out, stream)
+    r = np.frombuffer(out.cpu().numpy().tobytes(), dtype=TOPK_DTYPE)[0]
+    return {k: r[k].item() for k in TOPK_DTYPE.names if k != "reserved"}
 
 
 def inject_model(kind: str, k: int = 0, bit_lo: int = 0, bit_hi: int = 0, x: float = 0.0) -> dict:

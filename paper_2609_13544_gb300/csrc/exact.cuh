@@ -1,0 +1,151 @@
+// Exact integer digits shared by the library's kernels: values split into
+// integer significands, signed 32-bit digits of a fixed-point accumulator
+// (digit j weighs 2^(32 j + LIMB_LSB)), and the one rounding of such an
+// accumulator to binary64.
+#pragma once
+#include <cstdint>
+
+#include "peat_internal.h"
+
+namespace peat {
+
+// x = m * 2^e with m an integer (x finite, nonzero); float32 and binary64
+__device__ __forceinline__ uint32_t split_float(float x, int& e) {
+  uint32_t b = __float_as_uint(x) & 0x7FFFFFFFu;
+  uint32_t be = b >> 23, m = b & 0x7FFFFFu;
+  if (be == 0) {
+    e = -149;
+    return m;
+  }
+  e = (int)be - 150;
+  return m | 0x800000u;
+}
+__device__ __forceinline__ uint64_t split_double(double x, int& e) {
+  uint64_t b = (uint64_t)__double_as_longlong(x) & 0x7FFFFFFFFFFFFFFFull;
+  int be = (int)(b >> 52);
+  uint64_t m = b & 0xFFFFFFFFFFFFFull;
+  if (be == 0) {
+    e = -1074;
+    return m;
+  }
+  e = be - 1075;
+  return m | (1ull << 52);
+}
+
+// Signed 32-bit digits of +-m * 2^e (m < 2^128), delivered to f(digit, value).
+// Every value that occurs is a multiple of 2^LIMB_LSB and below 2^352.
+template <class F>
+__device__ __forceinline__ void for_digits(unsigned __int128 m, int e, bool neg, F&& f) {
+  if (m == 0) return;
+  int p = e - LIMB_LSB;
+  int j = p >> 5, r = p & 31;
+  uint32_t md[4] = {(uint32_t)m, (uint32_t)(m >> 32), (uint32_t)(m >> 64), (uint32_t)(m >> 96)};
+  uint32_t out[5];
+  out[0] = md[0] << r;
+#pragma unroll
+  for (int k = 1; k < 4; k++) out[k] = (md[k] << r) | (r ? (md[k - 1] >> (32 - r)) : 0u);
+  out[4] = r ? (md[3] >> (32 - r)) : 0u;
+#pragma unroll
+  for (int k = 0; k < 5; k++)
+    if (out[k] && j + k < NLIMB) f(j + k, neg ? -(int64_t)out[k] : (int64_t)out[k]);
+}
+
+// RN-even binary64 of the exact value of NLIMB carry-save digits (digit j
+// weighs 2^(32 j + LIMB_LSB)).  Loops are unrolled with constant indices so
+// the digits stay in registers.
+__device__ inline double limbs_to_double(const long long* src) {
+  int64_t d[NLIMB];
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++) d[j] = src[j];
+  // carry-propagate: digits 0..NLIMB-2 into [0, 2^32), the top digit signed
+  int64_t carry = 0;
+#pragma unroll
+  for (int j = 0; j < NLIMB - 1; j++) {
+    const int64_t v = d[j] + carry;
+    carry = v >> 32;
+    d[j] = v & 0xFFFFFFFFll;
+  }
+  d[NLIMB - 1] += carry;
+  const bool neg = d[NLIMB - 1] < 0;
+  if (neg) {
+    carry = 0;
+#pragma unroll
+    for (int j = 0; j < NLIMB - 1; j++) {
+      const int64_t v = -d[j] + carry;
+      carry = v >> 32;
+      d[j] = v & 0xFFFFFFFFll;
+    }
+    d[NLIMB - 1] = -d[NLIMB - 1] + carry;
+  }
+  // the top nonzero digit, the two below it, and a sticky bit for the rest
+  int top = -1;
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++)
+    if (d[j] != 0) top = j;
+  if (top < 0) return 0.0;
+  uint64_t w2 = 0, w1 = 0, w0 = 0;
+  bool sticky = false;
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++) {
+    if (j == top) w2 = (uint64_t)d[j];
+    if (j == top - 1) w1 = (uint64_t)d[j];
+    if (j == top - 2) w0 = (uint64_t)d[j];
+    if (j < top - 2 && d[j] != 0) sticky = true;
+  }
+  // after normalisation every digit is below 2^32 (the sums stay below 2^352):
+  // W = w2 2^64 + w1 2^32 + w0 < 2^96, value = W 2^(32 (top - 2) + LIMB_LSB)
+  const int b = 31 - __clz((uint32_t)w2);  // leading one of w2
+  const unsigned __int128 W = ((unsigned __int128)w2 << 64) | ((unsigned __int128)w1 << 32) | w0;
+  const int shift = b + 1;                 // W >> shift has its leading one at bit 63
+  const uint64_t m = (uint64_t)(W >> shift);
+  if ((W & (((unsigned __int128)1 << shift) - 1)) != 0) sticky = true;
+  uint64_t mant = m >> 11;
+  const uint64_t rbits = m & 0x7FFull;
+  if (rbits > 0x400ull || (rbits == 0x400ull && (sticky || (mant & 1ull)))) mant++;
+  const int e = 11 + shift + 32 * (top - 2) + LIMB_LSB;
+  const double r = ldexp((double)mant, e);
+  return neg ? -r : r;
+}
+
+// RN-even binary64 of (exact value of the digits) / k, for a non-negative
+// value and k >= 1.  The value is shifted up 128 bits before an exact long
+// division (base 2^32), so the quotient carries at least 64 significant bits
+// and the remainder only decides the sticky bit.
+__device__ inline double limbs_div_rn(const long long* src, uint64_t k) {
+  constexpr int ND = NLIMB + 4;
+  uint32_t d[ND];
+  int64_t carry = 0;
+#pragma unroll
+  for (int j = 0; j < 4; j++) d[j] = 0;
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++) {  // carry-propagate into base-2^32 digits (the value is >= 0)
+    const int64_t v = src[j] + carry;
+    carry = v >> 32;
+    d[j + 4] = (uint32_t)(v & 0xFFFFFFFFll);
+  }
+  uint32_t q[ND];
+  unsigned __int128 rem = 0;
+  for (int j = ND - 1; j >= 0; j--) {
+    const unsigned __int128 cur = (rem << 32) | d[j];
+    q[j] = (uint32_t)(cur / k);
+    rem = cur % k;
+  }
+  int top = -1;
+  for (int j = ND - 1; j >= 0 && top < 0; j--)
+    if (q[j]) top = j;
+  if (top < 0) return 0.0;
+  const uint64_t w2 = q[top], w1 = top >= 1 ? q[top - 1] : 0, w0 = top >= 2 ? q[top - 2] : 0;
+  bool sticky = rem != 0;
+  for (int j = 0; j < top - 2 && !sticky; j++) sticky = q[j] != 0;
+  const int b = 31 - __clz((uint32_t)w2);
+  const unsigned __int128 W = ((unsigned __int128)w2 << 64) | ((unsigned __int128)w1 << 32) | w0;
+  const int shift = b + 1;
+  const uint64_t m = (uint64_t)(W >> shift);
+  if ((W & (((unsigned __int128)1 << shift) - 1)) != 0) sticky = true;
+  uint64_t mant = m >> 11;
+  const uint64_t rbits = m & 0x7FFull;
+  if (rbits > 0x400ull || (rbits == 0x400ull && (sticky || (mant & 1ull)))) mant++;
+  return ldexp((double)mant, 11 + shift + 32 * (top - 2) + LIMB_LSB - 128);
+}
+
+}  // namespace peat

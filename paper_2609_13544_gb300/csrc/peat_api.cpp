@@ -32,6 +32,9 @@ struct peat_handle_s {
   int64_t* h_offsets = nullptr;  // pinned staging of the same
   cudaEvent_t staged = nullptr;  // the last staging copy has been consumed
   bool staged_pending = false;
+  // mean-of-top-errors workspace, zero between calls
+  peat::TopkState* topk = nullptr;
+  peat::TopkListEntry* topk_list = nullptr;
   // injector staging (grown on demand)
   int64_t* d_inj = nullptr;
   int64_t* h_inj = nullptr;
@@ -358,6 +361,9 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
             cudaMalloc(&h->d_offsets, sizeof(int64_t) * staging) == cudaSuccess &&
             cudaMallocHost(&h->h_offsets, sizeof(int64_t) * staging) == cudaSuccess &&
             cudaEventCreateWithFlags(&h->staged, cudaEventDisableTiming) == cudaSuccess &&
+            cudaMalloc(&h->topk, sizeof(peat::TopkState)) == cudaSuccess &&
+            cudaMemset(h->topk, 0, sizeof(peat::TopkState)) == cudaSuccess &&
+            cudaMalloc(&h->topk_list, sizeof(peat::TopkListEntry) * peat::TK_LCAP) == cudaSuccess &&
             cudaDeviceSynchronize() == cudaSuccess;
   if (!ok) {
     cudaGetLastError();
@@ -383,6 +389,8 @@ peat_status_t peat_signature_destroy(peat_handle_t h) {
     if (h->h_offsets) cudaFreeHost(h->h_offsets);
     if (h->d_inj) cudaFree(h->d_inj);
     if (h->h_inj) cudaFreeHost(h->h_inj);
+    if (h->topk) cudaFree(h->topk);
+    if (h->topk_list) cudaFree(h->topk_list);
     if (h->staged) cudaEventDestroy(h->staged);
     cudaGetLastError();
   }
@@ -404,6 +412,52 @@ peat_status_t peat_compare_segmented(peat_handle_t h, const void* golden, const 
                                      peat_tol_t tol, peat_stats_t* stats_out, uint64_t* hist_out,
                                      peat_stream_t stream) {
   return compare_impl(h, golden, candidate, offsets, nseg, dtype, tol, stats_out, hist_out, stream);
+}
+
+peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* candidate, int64_t n,
+                             peat_dtype_t dtype, uint64_t num, uint64_t den, peat_topk_t* out,
+                             peat_stream_t stream) {
+  if (!h) return PEAT_ERR_INVALID_ARG;
+  const int B = dtype_bytes(dtype);
+  if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
+  if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
+  if (n > 0 && (!golden || !candidate)) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
+  if (num == 0 || num > den) return fail(h, PEAT_ERR_INVALID_ARG, "need 0 < num <= den");
+  if (!out) return fail(h, PEAT_ERR_INVALID_ARG, "out is NULL");
+  DeviceGuard dg(h->device);
+  if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
+  peat::TopkParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.g = golden;
+  p.c = candidate;
+  p.n = n;
+  const uintptr_t ag = reinterpret_cast<uintptr_t>(golden), ac = reinterpret_cast<uintptr_t>(candidate);
+  const int64_t vec = 16 / B;
+  p.p0 = -1;
+  if (n > 0 && ag % B == 0 && ac % B == 0 && ag % 16 == ac % 16) {
+    const int64_t p0 = (int64_t)(((16 - ag % 16) % 16) / B);
+    if (p0 < n) {
+      p.p0 = p0;
+      p.nvec = (n - p0) / vec;
+    }
+  }
+  p.num = num;
+  p.den = den;
+  p.st = h->topk;
+  p.list = h->topk_list;
+  p.out = out;
+  // streaming passes: up to 8 resident CTAs of 256 threads per SM, about one per 16K elements
+  const int64_t want = (n + 16383) / 16384;
+  const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)h->nsm * 8, want));
+  // per-thread integer sums in the sum pass stay below 2^64
+  if (n / ((int64_t)nctas * 256) >= ((int64_t)1 << 24) - 16)
+    return fail(h, PEAT_ERR_UNSUPPORTED, "n is too large for one call (more than 2^24 elements per thread)");
+  cudaError_t e = peat::launch_topk(dtype, p, nctas, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    cudaMemsetAsync(h->topk, 0, sizeof(peat::TopkState), reinterpret_cast<cudaStream_t>(stream));
+    return cuda_fail(h, e, "top-k launch");
+  }
+  return PEAT_OK;
 }
 
 peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* src, int64_t n,

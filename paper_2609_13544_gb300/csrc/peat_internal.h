@@ -87,6 +87,40 @@ size_t compare_segacc_bytes();
 cudaError_t launch_bounds_on_device(int dtype, int64_t* offsets, int64_t* bounds, int nctas, int64_t n, int64_t p0,
                                     cudaStream_t s);
 
+// ---- mean of the top errors (topk.cu) ----
+constexpr int TK_BINS = 2048;   // digit histogram bins (11-bit digits)
+constexpr unsigned TK_LCAP = 4096;  // threshold-bucket pairs with an inexact float32 |d| kept for the final order
+
+// Device state of one peat_topk_mean call, zero between calls.  key(|d|) is an
+// order-preserving 32-bit key; three digit passes (11, 11, 10 bits) resolve the
+// key T of the k-th largest |d|; krem is then how many pairs with key T belong
+// to the top k.
+struct TopkState {
+  unsigned long long hist[3][TK_BINS];
+  unsigned long long nfin;      // finite pairs
+  unsigned long long k, krem;
+  unsigned long long nbucket;   // pairs with key T
+  unsigned int prefix;          // resolved high bits of T (all 32 after the third pass)
+  unsigned int nlist;           // bucket pairs whose |d| is not a float32 (may exceed TK_LCAP)
+  long long limbs[NLIMB];       // exact sum of the |d| above T
+};
+struct TopkListEntry {
+  float lo;  // |d| = (T's float + lo) * 2^sc
+  int sc;
+};
+struct TopkParams {
+  const void* g;
+  const void* c;
+  int64_t n;
+  int64_t p0;     // first element of the 16-byte vector grid; -1: none
+  int64_t nvec;   // vectors on the grid
+  uint64_t num, den;
+  TopkState* st;
+  TopkListEntry* list;
+  peat_topk_t* out;
+};
+cudaError_t launch_topk(int dtype, const TopkParams& p, int nctas, cudaStream_t s);
+
 struct InjectElemParams {
   void* dst;
   const void* src;

@@ -223,11 +223,11 @@ typedef struct {
   double threshold;   /* RN64 of the k-th largest |c - g| (0 if k = 0) */
   double sum;         /* RN64 of the exact sum of the k largest |c - g| */
   double mean;        /* RN64 of that exact sum divided by k (0 if k = 0) */
-  uint32_t exact;     /* 1: every field exact as defined.  0: more than 4096 pairs whose
+  uint32_t exact;     /* 1: every field exact as defined.  0: more than 65536 pairs whose
                          |c - g| is not a float32 value (float32 or float16 operands of
                          different magnitudes) share the float32 rounding of the k-th
-                         largest; they were then ordered by that rounding alone, so sum
-                         and mean may be off by their rounding errors */
+                         largest; the excess were taken at that rounding, so sum, mean
+                         and threshold may be off by their rounding errors */
   uint32_t reserved;
 } peat_topk_t;
 
@@ -237,9 +237,12 @@ typedef struct {
  * once to nearest-even binary64.  Ties do not change the value.
  *   golden, candidate  as for peat_compare (device, any alignment).
  *   out                device pointer to one peat_topk_t.
- * Streams both tensors four times (three digit-histogram passes of a radix
- * select, then the exact sum), asynchronously on `stream`; the handle's
- * workspace is shared with its other calls (do not overlap them).
+ * Streams both tensors three times (a radix select over an order-preserving
+ * key of |c - g|, 10 + 11 + 10 bits, that sums exactly what it has resolved
+ * as it goes), a fourth time only when more than 65536 pairs whose |c - g| is
+ * not a float32 value lie within 1024 float32 steps of the k-th largest;
+ * asynchronously on `stream`.  The handle's workspace is shared with its
+ * other calls (do not overlap them).
  * Errors: INVALID_ARG (null pointer with n > 0, n < 0, bad dtype, num = 0,
  * num > den, out NULL), UNSUPPORTED (more than 2^24 elements per thread of the
  * grid: n above about 2^42 on a 152-SM GPU), CUDA. */

@@ -108,44 +108,54 @@ __device__ inline double limbs_to_double(const long long* src) {
 }
 
 // RN-even binary64 of (exact value of the digits) / k, for a non-negative
-// value and k >= 1.  The value is shifted up 128 bits before an exact long
-// division (base 2^32), so the quotient carries at least 64 significant bits
-// and the remainder only decides the sticky bit.
+// value and k >= 1.  The value's leading 128 bits W (the rest only decides
+// whether anything below is nonzero) divided by k give a quotient of at least
+// 64 bits; with the remainder and the dropped bits as the sticky bit, that
+// quotient rounds exactly as the full quotient does.
 __device__ inline double limbs_div_rn(const long long* src, uint64_t k) {
-  constexpr int ND = NLIMB + 4;
-  uint32_t d[ND];
+  uint32_t d[NLIMB];
   int64_t carry = 0;
 #pragma unroll
-  for (int j = 0; j < 4; j++) d[j] = 0;
-#pragma unroll
-  for (int j = 0; j < NLIMB; j++) {  // carry-propagate into base-2^32 digits (the value is >= 0)
+  for (int j = 0; j < NLIMB; j++) {  // carry-propagate into base-2^32 digits
     const int64_t v = src[j] + carry;
     carry = v >> 32;
-    d[j + 4] = (uint32_t)(v & 0xFFFFFFFFll);
-  }
-  uint32_t q[ND];
-  unsigned __int128 rem = 0;
-  for (int j = ND - 1; j >= 0; j--) {
-    const unsigned __int128 cur = (rem << 32) | d[j];
-    q[j] = (uint32_t)(cur / k);
-    rem = cur % k;
+    d[j] = (uint32_t)(v & 0xFFFFFFFFll);
   }
   int top = -1;
-  for (int j = ND - 1; j >= 0 && top < 0; j--)
-    if (q[j]) top = j;
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++)
+    if (d[j] != 0) top = j;
   if (top < 0) return 0.0;
-  const uint64_t w2 = q[top], w1 = top >= 1 ? q[top - 1] : 0, w0 = top >= 2 ? q[top - 2] : 0;
-  bool sticky = rem != 0;
-  for (int j = 0; j < top - 2 && !sticky; j++) sticky = q[j] != 0;
-  const int b = 31 - __clz((uint32_t)w2);
-  const unsigned __int128 W = ((unsigned __int128)w2 << 64) | ((unsigned __int128)w1 << 32) | w0;
-  const int shift = b + 1;
-  const uint64_t m = (uint64_t)(W >> shift);
-  if ((W & (((unsigned __int128)1 << shift) - 1)) != 0) sticky = true;
+  uint32_t w4 = 0, w3 = 0, w2 = 0, w1 = 0, w0 = 0;
+  bool sticky = false;
+#pragma unroll
+  for (int j = 0; j < NLIMB; j++) {
+    if (j == top) w4 = d[j];
+    if (j == top - 1) w3 = d[j];
+    if (j == top - 2) w2 = d[j];
+    if (j == top - 3) w1 = d[j];
+    if (j == top - 4) w0 = d[j];
+    if (j < top - 4 && d[j] != 0) sticky = true;
+  }
+  // the 160-bit window w4..w0 shifted so that its leading one is bit 127 of W
+  const int lz = __clz(w4);
+  const unsigned __int128 win = ((unsigned __int128)w4 << 96) | ((unsigned __int128)w3 << 64) |
+                                ((unsigned __int128)w2 << 32) | w1;
+  const unsigned __int128 W = lz ? ((win << lz) | (w0 >> (32 - lz))) : win;
+  if ((lz ? (uint32_t)(w0 << lz) : w0) != 0) sticky = true;
+  // value = W 2^E + (below), E the weight of W's last bit
+  const int E = 32 * (top - 3) - lz + LIMB_LSB;
+  const unsigned __int128 q = W / k;
+  if (W - q * k != 0) sticky = true;
+  const uint64_t qh = (uint64_t)(q >> 64);
+  const int qlz = qh ? __clzll(qh) : 64 + __clzll((uint64_t)q);
+  const int shift = 64 - qlz;  // q >= 2^63: bits of q below its leading 64
+  const uint64_t m = (uint64_t)(q >> shift);
+  if (shift > 0 && (q & (((unsigned __int128)1 << shift) - 1)) != 0) sticky = true;
   uint64_t mant = m >> 11;
   const uint64_t rbits = m & 0x7FFull;
   if (rbits > 0x400ull || (rbits == 0x400ull && (sticky || (mant & 1ull)))) mant++;
-  return ldexp((double)mant, 11 + shift + 32 * (top - 2) + LIMB_LSB - 128);
+  return ldexp((double)mant, 11 + shift + E);
 }
 
 }  // namespace peat

@@ -446,9 +446,9 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
   p.st = h->topk;
   p.list = h->topk_list;
   p.out = out;
-  // streaming passes: up to 8 resident CTAs of 256 threads per SM, about one per 16K elements
-  const int64_t want = (n + 16383) / 16384;
-  const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)h->nsm * 8, want));
+  // streaming passes: one wave of resident CTAs, about one CTA per 1K elements
+  const int64_t want = (n + 1023) / 1024;
+  const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>(peat::topk_max_ctas(h->nsm), want));
   // per-thread integer sums in the sum pass stay below 2^64
   if (n / ((int64_t)nctas * 256) >= ((int64_t)1 << 24) - 16)
     return fail(h, PEAT_ERR_UNSUPPORTED, "n is too large for one call (more than 2^24 elements per thread)");

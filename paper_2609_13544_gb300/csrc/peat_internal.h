@@ -88,25 +88,33 @@ cudaError_t launch_bounds_on_device(int dtype, int64_t* offsets, int64_t* bounds
                                     cudaStream_t s);
 
 // ---- mean of the top errors (topk.cu) ----
-constexpr int TK_BINS = 2048;   // digit histogram bins (11-bit digits)
-constexpr unsigned TK_LCAP = 4096;  // threshold-bucket pairs with an inexact float32 |d| kept for the final order
+// key(|d|) is an order-preserving 31-bit key of |c - g|.  A sample picks a
+// window of TK_WIN digits of key >> 21 (TK_NB0 values); a streaming pass
+// counts exactly and resolves key >> 10 inside the window (TK_NB1 = 2048
+// values per digit); a second one resolves the last 10 bits (TK_NB2).  Should
+// the window miss, an exact pass over key >> 21 replaces the sample.
+constexpr int TK_NB0 = 1024, TK_NB1 = 2048, TK_NB2 = 1024, TK_WIN = 3;
+constexpr int64_t TK_SAMPLE = 1 << 18;  // pairs in the sample
+constexpr unsigned TK_LCAP = 65536;     // listed pairs whose |d| is not a float32 value
 
-// Device state of one peat_topk_mean call, zero between calls.  key(|d|) is an
-// order-preserving 32-bit key; three digit passes (11, 11, 10 bits) resolve the
-// key T of the k-th largest |d|; krem is then how many pairs with key T belong
-// to the top k.
+// Device state of one peat_topk_mean call, zero between calls.
 struct TopkState {
-  unsigned long long hist[3][TK_BINS];
+  unsigned long long hist0[TK_NB0], hist1[TK_WIN * TK_NB1], hist2[TK_NB2];
+  unsigned long long nonfin;    // pairs with a NaN or an infinity
+  unsigned long long above;     // pairs with key >> 21 above the window
   unsigned long long nfin;      // finite pairs
-  unsigned long long k, krem;
-  unsigned long long nbucket;   // pairs with key T
-  unsigned int prefix;          // resolved high bits of T (all 32 after the third pass)
-  unsigned int nlist;           // bucket pairs whose |d| is not a float32 (may exceed TK_LCAP)
-  long long limbs[NLIMB];       // exact sum of the |d| above T
+  unsigned long long k;         // pairs taken
+  unsigned long long krem;      // of them, still to place inside the resolved prefix
+  unsigned int Plo, Phi;        // the window of key >> 21
+  unsigned int P0, P1, T;       // key >> 21, key >> 10, and the key of the k-th largest |d|
+  unsigned int ok;              // the window held the k-th largest
+  unsigned int done[3];         // CTAs finished, per pass
+  unsigned int nlist, nlist2;   // list entries from the last pass and the optional extra one
+  long long limbs[NLIMB];       // exact sum of the |d| resolved above the prefix
 };
 struct TopkListEntry {
-  float lo;  // |d| = (T's float + lo) * 2^sc
-  int sc;
+  float lo;      // |d| = (value of key + lo), the value of key taken as in the key's definition
+  unsigned key;
 };
 struct TopkParams {
   const void* g;
@@ -119,6 +127,8 @@ struct TopkParams {
   TopkListEntry* list;
   peat_topk_t* out;
 };
+// CTAs of the streaming passes that fit on the device at once
+int topk_max_ctas(int nsm);
 cudaError_t launch_topk(int dtype, const TopkParams& p, int nctas, cudaStream_t s);
 
 struct InjectElemParams {

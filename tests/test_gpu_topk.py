@@ -167,3 +167,62 @@ def test_c2_full_size_against_torch(peat_gpu, h):
     assert math.isclose(r["sum"], s, rel_tol=1e-12)
     assert math.isclose(r["mean"], s / k, rel_tol=1e-12)
     assert r["exact"] == 1
+
+
+def test_inexact_pairs_beyond_the_list(peat_gpu, oracle, h):
+    """More than 65536 pairs whose |d| is not a float32 value within 1024
+    float32 steps of the k-th largest: the fourth pass sums that range again."""
+    rng = np.random.default_rng(31)
+    n_near = 100_000
+    j = rng.integers(0, 500, n_near)
+    c = (np.float32(2 ** 24) + 2 * j).astype(np.float32)           # spacing 2 above 2^24
+    g = -(rng.random(n_near).astype(np.float32) * np.float32(0.99) + np.float32(0.005))
+    g_rest = np.zeros(400_000, np.float32)
+    c_rest = rng.random(400_000).astype(np.float32)
+    gb = f32_bits(np.concatenate([g, g_rest]))
+    cb = f32_bits(np.concatenate([c, c_rest]))
+    perm = rng.permutation(gb.size)
+    gb, cb = gb[perm], cb[perm]
+    for num, den in [(1, 10), (1, 7), (1, 5), (1, 1)]:
+        check(peat_gpu, oracle, h, gb, cb, "f32", num, den, ctx="list overflow")
+
+
+def test_bucket_beyond_the_list_is_flagged(peat_gpu, oracle, h):
+    """More than 65536 inexact pairs tied in float32 with the k-th largest: the
+    result is flagged inexact and stays within their rounding errors."""
+    rng = np.random.default_rng(32)
+    m = 70_000
+    g = -(rng.random(m).astype(np.float32) * np.float32(0.99) + np.float32(0.005))
+    c = np.full(m, np.float32(2 ** 24 + 2), np.float32)
+    gb = f32_bits(np.concatenate([g, np.zeros(630_000, np.float32)]))
+    cb = f32_bits(np.concatenate([c, rng.random(630_000).astype(np.float32)]))
+    gt, ct = to_device(gb, "f32"), to_device(cb, "f32")
+    gr = peat_gpu.peat_topk_mean(h, gt, ct, 1, 20)   # k = 35000, inside the tie
+    orr = oracle.topk_mean(gb, cb, "f32", 1, 20)
+    assert gr["exact"] == 0
+    assert gr["n_finite"] == orr["n_finite"] and gr["k"] == orr["k"]
+    assert math.isclose(gr["sum"], orr["sum"], rel_tol=1e-6)
+    assert math.isclose(gr["threshold"], orr["threshold"], rel_tol=1e-6)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("pattern", ["every16", "runs"])
+def test_sampled_window_misses(peat_gpu, oracle, h, dtype, pattern):
+    """Small errors on evenly spaced pairs (every 16th, or the first 256 of
+    every 2048) and large ones elsewhere: a sample drawn from such positions
+    picks a window that misses the k-th largest, and the exact passes take
+    over; either way the result is the oracle's."""
+    import torch
+    n = 1 << 22
+    rng = np.random.default_rng(40)
+    g = rng.standard_normal(n).astype(np.float32)
+    pos = np.arange(n)
+    small = (pos % 16 == 0) if pattern == "every16" else (pos % 2048 < 256)
+    rel = np.where(small, 1e-6, 0.3).astype(np.float32)
+    c = (g * (1 + rel * rng.standard_normal(n).astype(np.float32))).astype(np.float32)
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    iv = torch.int32 if dtype == "f32" else torch.int16
+    gb = torch.from_numpy(g).to(tdt).view(iv).numpy().view(NP_BITS[dtype])
+    cb = torch.from_numpy(c).to(tdt).view(iv).numpy().view(NP_BITS[dtype])
+    for num, den in [(1, 10), (1, 1000)]:
+        check(peat_gpu, oracle, h, gb, cb, dtype, num, den, ctx="sample misses")

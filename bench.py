@@ -50,7 +50,7 @@ def measured_peaks() -> dict:
 
 def kernel_source_sha() -> str:
     h = hashlib.sha256()
-    for f in ("compare.cu", "peat_internal.h"):
+    for f in ("compare.cu", "exact.cuh", "peat_internal.h"):
         h.update((ROOT / "paper_2609_13544_gb300" / "csrc" / f).read_bytes())
     return h.hexdigest()[:16]
 
@@ -296,6 +296,33 @@ def run_gpu(args) -> None:
     peaks = measured_peaks()
     peak = float(peaks.get("hbm_gbs", 6800.0))
 
+    # the mean of the top 10 % of the errors (Section IV-B-3) on the same
+    # tensor: its own timing, reported beside the compare's line
+    topk = None
+    if w.offsets is None and not args.no_topk:
+        tk_out = torch.empty(peat.TOPK_BYTES, dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            peat.peat_topk_mean_raw(h, g, c, 1, 10, tk_out, stream)
+        barrier()
+        tk_calls = max(3, min(200, args.steps // 20))
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(tk_calls):
+            peat.peat_topk_mean_raw(h, g, c, 1, 10, tk_out, stream)
+        t1.record(stream)
+        barrier()
+        tk_ms = max_over_ranks(t0.elapsed_time(t1), dev) / tk_calls
+        r = np.frombuffer(tk_out.cpu().numpy().tobytes(), dtype=peat.TOPK_DTYPE)[0]
+        read_gbs = bytes_per_step / (tk_ms * 1e-3) / 1e9
+        topk = {"op": "peat_topk_mean, num/den = 1/10", "calls": tk_calls, "us_per_call": tk_ms * 1e3,
+                "pairs_per_s": w.n / (tk_ms * 1e-3), "k": int(r["k"]), "exact": int(r["exact"]),
+                "full_reads_per_call": 2,
+                "roofline": {"bound": "hbm", "achieved": 2 * read_gbs, "peak": peak, "unit": "GB/s",
+                             "frac": 2 * read_gbs / peak,
+                             "algorithmic_bytes_per_call": 2 * bytes_per_step,
+                             "note": "two streaming reads of both tensors per call (the counting pass and the "
+                                     "last-digit pass) plus a sample and one-CTA selects"}}
+
     # end to end through the C ABI with host buffers: H2D of both tensors from
     # pinned memory, the compare, D2H of the stats and histograms, every step
     e2e = None
@@ -361,6 +388,7 @@ def run_gpu(args) -> None:
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy)" if not peaks.get("fallback")
                          else "fallback 6.8 TB/s"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": (1 if nseg == 1 else 2) * args.steps, "clocks": clocks,
+            "next_rows": {"f1_top10_mean": topk},
             "wall_s_timed": wall,
         }
         print(json.dumps(line), flush=True)
@@ -378,6 +406,7 @@ def main():
     ap.add_argument("--workload", default="c2", choices=sorted(WORKLOAD_NAMES))
     ap.add_argument("--impl", default="peat", choices=["peat", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-topk", action="store_true", help="skip the timing of the top-10 %% mean")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -323,6 +323,30 @@ def run_gpu(args) -> None:
                              "note": "two streaming reads of both tensors per call (the counting pass and the "
                                      "last-digit pass) plus a sample and one-CTA selects"}}
 
+    # the context statistics of the golden tensor(s) (Section IV-C-2): one read
+    tstats = None
+    if not args.no_topk:
+        off = [0, w.n] if w.offsets is None else list(w.offsets)
+        ts_out = torch.empty((len(off) - 1) * peat.TSTATS_BYTES, dtype=torch.uint8, device=dev)
+        for _ in range(3):
+            peat.peat_tensor_stats_raw(h, g, off, ts_out, stream)
+        barrier()
+        ts_calls = max(3, min(200, args.steps // 20))
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(ts_calls):
+            peat.peat_tensor_stats_raw(h, g, off, ts_out, stream)
+        t1.record(stream)
+        barrier()
+        ts_ms = max_over_ranks(t0.elapsed_time(t1), dev) / ts_calls
+        one = bytes_per_step // 2
+        ts_gbs = one / (ts_ms * 1e-3) / 1e9
+        tstats = {"op": "peat_tensor_stats of the golden tensor(s)", "calls": ts_calls, "segments": len(off) - 1,
+                  "us_per_call": ts_ms * 1e3, "elements_per_s": w.n / (ts_ms * 1e-3),
+                  "roofline": {"bound": "hbm", "achieved": ts_gbs, "peak": peak, "unit": "GB/s",
+                               "frac": ts_gbs / peak, "algorithmic_bytes_per_call": one,
+                               "note": "one read of the tensor; stage 1 plus a per-segment finalize"}}
+
     # end to end through the C ABI with host buffers: H2D of both tensors from
     # pinned memory, the compare, D2H of the stats and histograms, every step
     e2e = None
@@ -388,7 +412,7 @@ def run_gpu(args) -> None:
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy)" if not peaks.get("fallback")
                          else "fallback 6.8 TB/s"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": (1 if nseg == 1 else 2) * args.steps, "clocks": clocks,
-            "next_rows": {"f1_top10_mean": topk},
+            "next_rows": {"f1_top10_mean": topk, "f3_context_stats": tstats},
             "wall_s_timed": wall,
         }
         print(json.dumps(line), flush=True)
@@ -406,7 +430,8 @@ def main():
     ap.add_argument("--workload", default="c2", choices=sorted(WORKLOAD_NAMES))
     ap.add_argument("--impl", default="peat", choices=["peat", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-topk", action="store_true", help="skip the timing of the top-10 %% mean")
+    ap.add_argument("--no-topk", action="store_true",
+                    help="skip the timings of the next rows (top-10 %% mean, context statistics)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

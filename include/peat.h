@@ -250,9 +250,59 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
                              peat_dtype_t dtype, uint64_t num, uint64_t den, peat_topk_t* out,
                              peat_stream_t stream);
 
+/* Context statistics of one recorded tensor (Section IV-C-2: the means and
+ * variances of the weight and activation tensors that the error scores are
+ * correlated with).  80 bytes.  Every double is the exact value rounded once
+ * to nearest-even. */
+typedef struct {
+  uint64_t n;         /* elements */
+  uint64_t n_finite;  /* finite elements */
+  uint64_t n_nan;     /* NaN elements */
+  uint64_t n_inf;     /* infinite elements */
+  double sum;         /* sum of the finite elements */
+  double sum_sq;      /* sum of their squares */
+  double mean;        /* sum / n_finite (0 if n_finite = 0) */
+  double var;         /* population variance: (n_finite sum_sq - sum^2) / n_finite^2, exact
+                         before its one rounding (0 if n_finite = 0) */
+  double min, max;    /* smallest and largest finite element (0 if none) */
+} peat_tstats_t;
+
+/* Context statistics of each segment s = [offsets[s], offsets[s+1]) of x
+ * (a single tensor: offsets = {0, n}, nseg = 1).
+ *   x           device pointer, dtype elements, any alignment.
+ *   offsets     HOST array of nseg + 1 non-decreasing int64, offsets[0] = 0;
+ *               copied before return.
+ *   stats_out   device pointer to nseg peat_tstats_t.
+ * Streams x once (about 25 integer operations per element), then one thread
+ * per segment forms the mean and the variance from the exact sums.
+ * Asynchronous on `stream`; shares the handle's workspace with its other
+ * calls (do not overlap them).
+ * Errors: INVALID_ARG (bad dtype, offsets, null pointers), UNSUPPORTED (nseg
+ * above the handle's max_segments, a segment of 2^36 elements or more), CUDA. */
+peat_status_t peat_tensor_stats(peat_handle_t h, const void* x, const int64_t* offsets, int64_t nseg,
+                                peat_dtype_t dtype, peat_tstats_t* stats_out, peat_stream_t stream);
+
+/* Host-side Analyzer steps (Section IV-C).  No GPU work; x and y are HOST
+ * arrays of finite doubles.
+ *
+ * peat_spearman: Spearman rank correlation of x and y (Section IV-C-2): the
+ *   Pearson correlation of their ranks, tied values taking the mean of the
+ *   ranks they span.  *rho_out = NaN when n < 2 or either ranking is constant.
+ *   The rank sums are exact integers; rho is their exact ratio up to the one
+ *   square root and division (a few ulps).
+ * peat_mean_std: the model-wise error range of one layer (Section IV-C-1): the
+ *   mean and the standard deviation of its scores across epochs, with ddof 0
+ *   (population) or 1 (sample); std = NaN when n <= ddof, mean = NaN when
+ *   n = 0.
+ * Errors: INVALID_ARG (null pointer, n < 0, a non-finite value, ddof not 0 or
+ *   1); text in peat_last_error(NULL). */
+peat_status_t peat_spearman(const double* x, const double* y, int64_t n, double* rho_out);
+peat_status_t peat_mean_std(const double* x, int64_t n, int ddof, double* mean_out, double* std_out);
+
 /* Text of the last error reported on h (never NULL; "" if none).  With
- * h == NULL, the last error on this thread of peat_signature_create or of
- * peat_compare_noalloc, whichever failed last. */
+ * h == NULL, the last error on this thread of the calls that take no handle
+ * (peat_signature_create, peat_compare_noalloc, peat_spearman,
+ * peat_mean_std), whichever failed last. */
 const char* peat_last_error(peat_handle_t h);
 
 /* peat_compare without a handle and without any allocation.  The paper has no

@@ -57,6 +57,22 @@ class TopK(ctypes.Structure):
     ]
 
 
+ACC_WORDS, ACC_LSB = 24, -768
+
+
+class TStats(ctypes.Structure):
+    _fields_ = [
+        ("n", ctypes.c_uint64),
+        ("n_finite", ctypes.c_uint64),
+        ("n_nan", ctypes.c_uint64),
+        ("n_inf", ctypes.c_uint64),
+        ("min", ctypes.c_double),
+        ("max", ctypes.c_double),
+        ("sum_words", ctypes.c_uint64 * ACC_WORDS),
+        ("sum_sq_words", ctypes.c_uint64 * ACC_WORDS),
+    ]
+
+
 class InjectModel(ctypes.Structure):
     _fields_ = [
         ("kind", ctypes.c_int32),
@@ -82,6 +98,8 @@ def lib() -> ctypes.CDLL:
         L.orc_compare_segmented.restype = i32
         L.orc_topk_mean.argtypes = [vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, ctypes.POINTER(TopK)]
         L.orc_topk_mean.restype = i32
+        L.orc_tensor_stats.argtypes = [vp, i64, i32, ctypes.POINTER(TStats)]
+        L.orc_tensor_stats.restype = i32
         L.orc_ulp_key.argtypes = [ctypes.c_uint32, i32]
         L.orc_ulp_key.restype = i64
         L.orc_exact_sum.argtypes = [vp, i64]
@@ -147,6 +165,104 @@ def topk_mean(g, c, dtype: str, num: int = 1, den: int = 10) -> dict:
     if rc:
         raise ValueError(f"oracle rejected the arguments (code {rc})")
     return {f: getattr(out, f) for f, _ in TopK._fields_}
+
+
+def _acc_int(words) -> int:
+    """The fixed-point words as a Python integer (value = integer * 2^ACC_LSB)."""
+    v = 0
+    for j, w in enumerate(words):
+        v |= int(w) << (64 * j)
+    if v >> (64 * ACC_WORDS - 1):
+        v -= 1 << (64 * ACC_WORDS)
+    return v
+
+
+def tensor_stats(x, dtype: str) -> dict:
+    """Context statistics of one tensor (Section IV-C-2): counts, finite min and
+    max, and sum, sum of squares, mean and population variance of the finite
+    elements, each the exact value rounded once (Python integers and
+    correctly rounded integer division carry the last steps)."""
+    from fractions import Fraction
+    xb = _bits(x, dtype)
+    out = TStats()
+    rc = lib().orc_tensor_stats(xb.ctypes.data, xb.size, DTYPES[dtype], ctypes.byref(out))
+    if rc:
+        raise ValueError(f"oracle rejected the arguments (code {rc})")
+    s1, s2, nf = _acc_int(out.sum_words), _acc_int(out.sum_sq_words), out.n_finite
+    unit = 1 << (-ACC_LSB)
+    d = {"n": out.n, "n_finite": nf, "n_nan": out.n_nan, "n_inf": out.n_inf,
+         "sum": float(Fraction(s1, unit)), "sum_sq": float(Fraction(s2, unit)),
+         "mean": float(Fraction(s1, nf * unit)) if nf else 0.0,
+         "var": float(Fraction(nf * s2 * unit - s1 * s1, nf * nf * unit * unit)) if nf else 0.0,
+         "min": out.min, "max": out.max}
+    return d
+
+
+def tensor_stats_segmented(x, offsets: Sequence[int], dtype: str) -> list:
+    xb = _bits(x, dtype)
+    return [tensor_stats(xb[int(offsets[s]):int(offsets[s + 1])], dtype) for s in range(len(offsets) - 1)]
+
+
+def _exact_ranks(v):
+    """Ranks 1..n of the values, ties taking the mean of the ranks they span."""
+    from fractions import Fraction
+    n = len(v)
+    order = sorted(range(n), key=lambda i: v[i])
+    r = [Fraction(0)] * n
+    i = 0
+    while i < n:
+        j = i
+        while j + 1 < n and v[order[j + 1]] == v[order[i]]:
+            j += 1
+        for k in range(i, j + 1):
+            r[order[k]] = Fraction(i + j + 2, 2)
+        i = j + 1
+    return r
+
+
+def spearman(x, y) -> float:
+    """Spearman rank correlation (Section IV-C-2): Pearson correlation of the
+    ranks (mean ranks for ties), exact up to one square root taken at 60
+    significant digits; NaN when n < 2 or a ranking is constant."""
+    from decimal import Decimal, localcontext
+    x, y = [float(a) for a in x], [float(b) for b in y]
+    n = len(x)
+    if n != len(y):
+        raise ValueError("x and y differ in length")
+    if n < 2:
+        return float("nan")
+    rx, ry = _exact_ranks(x), _exact_ranks(y)
+    mx, my = sum(rx) / n, sum(ry) / n
+    cxy = sum((a - mx) * (b - my) for a, b in zip(rx, ry))
+    cxx = sum((a - mx) ** 2 for a in rx)
+    cyy = sum((b - my) ** 2 for b in ry)
+    if cxx == 0 or cyy == 0:
+        return float("nan")
+    with localcontext() as ctx:
+        ctx.prec = 60
+        q = (Decimal(cxy.numerator) / Decimal(cxy.denominator)) / (
+            (Decimal(cxx.numerator) / Decimal(cxx.denominator)) * (Decimal(cyy.numerator) / Decimal(cyy.denominator))).sqrt()
+        return float(q)
+
+
+def mean_std(x, ddof: int = 0):
+    """Model-wise error range of one layer (Section IV-C-1): mean and standard
+    deviation of its scores across epochs (ddof 0: population, 1: sample),
+    exact up to one square root at 60 significant digits."""
+    from decimal import Decimal, localcontext
+    from fractions import Fraction
+    v = [Fraction(float(a)) for a in x]
+    n = len(v)
+    if n == 0:
+        return float("nan"), float("nan")
+    m = sum(v) / n
+    if n <= ddof:
+        return float(m), float("nan")
+    var = sum((a - m) ** 2 for a in v) / (n - ddof)
+    with localcontext() as ctx:
+        ctx.prec = 60
+        sd = (Decimal(var.numerator) / Decimal(var.denominator)).sqrt()
+    return float(m), float(sd)
 
 
 def compare_segmented(g, c, offsets: Sequence[int], dtype: str, rtol: float, atol: float = 0.0):

@@ -594,6 +594,41 @@ int orc_topk_mean(const void* g, const void* c, int64_t n, int dtype, uint64_t n
 }
 
 /* ------------------------------------------------------------------------ */
+/* Context statistics (Section IV-C-2): every finite element decoded exactly */
+/* and added, and its square added, in the fixed-point accumulator.          */
+/* ------------------------------------------------------------------------ */
+int orc_tensor_stats(const void* x, int64_t n, int dtype, orc_tstats* out) {
+  if (!dtype_ok(dtype) || n < 0 || !out || (n > 0 && !x)) return ORC_BAD_ARG;
+  memset(out, 0, sizeof(*out));
+  out->n = (uint64_t)n;
+  acc_t s1, s2;
+  acc_zero(&s1);
+  acc_zero(&s2);
+  for (int64_t i = 0; i < n; i++) {
+    val_t v = decode(raw_bits(x, i, dtype), dtype);
+    if (v.nan) {
+      out->n_nan++;
+      continue;
+    }
+    if (v.inf) {
+      out->n_inf++;
+      continue;
+    }
+    /* extremes by value, -0 below +0 */
+    if (out->n_finite == 0 || v.v < out->min || (v.v == out->min && signbit(v.v) && !signbit(out->min)))
+      out->min = v.v;
+    if (out->n_finite == 0 || v.v > out->max || (v.v == out->max && !signbit(v.v) && signbit(out->max)))
+      out->max = v.v;
+    out->n_finite++;
+    acc_add_double(&s1, fabs(v.v), v.v < 0);
+    acc_add_product(&s2, v.v, v.v, 0);
+  }
+  memcpy(out->sum_words, s1.w, sizeof(s1.w));
+  memcpy(out->sum_sq_words, s2.w, sizeof(s2.w));
+  return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Pseudo-error injector.                                                    */
 /* Randomness: Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random  */
 /* numbers: as easy as 1, 2, 3", SC'11), key = the 64-bit seed, counter =    */

@@ -76,6 +76,24 @@ typedef struct {
 
 int orc_topk_mean(const void* g, const void* c, int64_t n, int dtype, uint64_t num, uint64_t den, orc_topk* out);
 
+/* Context statistics of one tensor (Section IV-C-2: the means and variances
+ * of the weight and activation tensors the error scores are correlated
+ * with): counts, the finite minimum and maximum, and the exact sum and sum
+ * of squares of the finite elements as fixed-point words (two's complement,
+ * ORC_ACC_WORDS little-endian 64-bit words, least significant bit
+ * 2^ORC_ACC_LSB), from which the caller forms the mean and the variance
+ * exactly. */
+#define ORC_ACC_WORDS 24
+#define ORC_ACC_LSB (-768)
+typedef struct {
+  uint64_t n, n_finite, n_nan, n_inf;
+  double min, max;  /* finite extremes (0 if none) */
+  uint64_t sum_words[ORC_ACC_WORDS];
+  uint64_t sum_sq_words[ORC_ACC_WORDS];
+} orc_tstats;
+
+int orc_tensor_stats(const void* x, int64_t n, int dtype, orc_tstats* out);
+
 /* ULP key of one raw bit pattern: +magnitude bits, negated when the sign
  * bit is set (so both zeros map to 0).  Exposed for the tests. */
 int64_t orc_ulp_key(uint32_t bits, int dtype);

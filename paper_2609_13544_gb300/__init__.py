@@ -38,6 +38,13 @@ TOPK_DTYPE = np.dtype([("n_finite", "<u8"), ("k", "<u8"), ("threshold", "<f8"), 
                        ("exact", "<u4"), ("reserved", "<u4")])
 assert TOPK_DTYPE.itemsize == TOPK_BYTES
 
+TSTATS_BYTES = 80
+
+# numpy view of peat_tstats_t
+TSTATS_DTYPE = np.dtype([("n", "<u8"), ("n_finite", "<u8"), ("n_nan", "<u8"), ("n_inf", "<u8"), ("sum", "<f8"),
+                         ("sum_sq", "<f8"), ("mean", "<f8"), ("var", "<f8"), ("min", "<f8"), ("max", "<f8")])
+assert TSTATS_DTYPE.itemsize == TSTATS_BYTES
+
 # numpy view of peat_stats_t
 STATS_DTYPE = np.dtype([
     ("n", "<u8"), ("count", "<u8", (5,)), ("n_finite", "<u8"),
@@ -69,7 +76,8 @@ class InjectModel(ctypes.Structure):
 
 
 EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
-           "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc", "peat_topk_mean")
+           "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc", "peat_topk_mean",
+           "peat_tensor_stats", "peat_spearman", "peat_mean_std")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -102,6 +110,13 @@ def load(path: Optional[Path] = None) -> ctypes.CDLL:
     L.peat_compare_noalloc.restype = i32
     L.peat_topk_mean.argtypes = [vp, vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, vp, vp]
     L.peat_topk_mean.restype = i32
+    L.peat_tensor_stats.argtypes = [vp, vp, vp, i64, i32, vp, vp]
+    L.peat_tensor_stats.restype = i32
+    dp = ctypes.POINTER(ctypes.c_double)
+    L.peat_spearman.argtypes = [dp, dp, i64, dp]
+    L.peat_spearman.restype = i32
+    L.peat_mean_std.argtypes = [dp, i64, i32, dp, dp]
+    L.peat_mean_std.restype = i32
     _lib = L
     return L
 
@@ -280,6 +295,55 @@ def peat_topk_mean(h: Handle, golden, candidate, num: int = 1, den: int = 10, st
     peat_topk_mean_raw(h, golden, candidate, num, den, out, stream)
     r = np.frombuffer(out.cpu().numpy().tobytes(), dtype=TOPK_DTYPE)[0]
     return {k: r[k].item() for k in TOPK_DTYPE.names if k != "reserved"}
+
+
+def peat_tensor_stats_raw(h: Handle, x, offsets, stats_out, stream=None) -> None:
+    """peat_tensor_stats on a preallocated device output (stats_out: uint8[80 * nseg])."""
+    _dev_tensor_check(x)
+    off = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    if off.size < 1 or off[-1] > x.numel():
+        raise ValueError("offsets exceed the tensor")
+    rc = load().peat_tensor_stats(h.ptr, x.data_ptr(), off.ctypes.data, off.size - 1, dtype_code(x),
+                                  stats_out.data_ptr(), _stream_ptr(stream))
+    _check(rc, h)
+
+
+def peat_tensor_stats(h: Handle, x, offsets: Optional[Sequence[int]] = None, stream=None):
+    """Context statistics of x (one dict) or of each segment (a list of dicts); synchronises."""
+    import torch
+    off = [0, x.numel()] if offsets is None else list(offsets)
+    nseg = len(off) - 1
+    out = torch.empty(max(nseg, 1) * TSTATS_BYTES, dtype=torch.uint8, device=x.device)
+    peat_tensor_stats_raw(h, x, off, out, stream)
+    arr = np.frombuffer(out.cpu().numpy()[: nseg * TSTATS_BYTES].tobytes(), dtype=TSTATS_DTYPE)
+    res = [{k: r[k].item() for k in TSTATS_DTYPE.names} for r in arr]
+    return res[0] if offsets is None else res
+
+
+def _host_doubles(v) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(v, dtype=np.float64))
+
+
+def peat_spearman(x, y) -> float:
+    """Spearman rank correlation of two host sequences (mean ranks for ties)."""
+    a, b = _host_doubles(x), _host_doubles(y)
+    if a.size != b.size:
+        raise ValueError("x and y differ in length")
+    dp = ctypes.POINTER(ctypes.c_double)
+    rho = ctypes.c_double()
+    rc = load().peat_spearman(a.ctypes.data_as(dp), b.ctypes.data_as(dp), a.size, ctypes.byref(rho))
+    _check(rc, None)
+    return rho.value
+
+
+def peat_mean_std(x, ddof: int = 0):
+    """(mean, std) of a host sequence of scores (ddof 0: population, 1: sample)."""
+    a = _host_doubles(x)
+    dp = ctypes.POINTER(ctypes.c_double)
+    m, sd = ctypes.c_double(), ctypes.c_double()
+    rc = load().peat_mean_std(a.ctypes.data_as(dp), a.size, ddof, ctypes.byref(m), ctypes.byref(sd))
+    _check(rc, None)
+    return m.value, sd.value
 
 
 def inject_model(kind: str, k: int = 0, bit_lo: int = 0, bit_hi: int = 0, x: float = 0.0) -> dict:

@@ -30,11 +30,14 @@ struct peat_handle_s {
   unsigned int wait_limit = 1u << 24;   // polls before a pipeline wait gives up
   int64_t* d_offsets = nullptr;  // offsets (nseg + 1) then CTA bounds (nctas + 1)
   int64_t* h_offsets = nullptr;  // pinned staging of the same
+  int64_t* d_single = nullptr;   // one-tensor calls: {0, n} then CTA bounds, written on the device
   cudaEvent_t staged = nullptr;  // the last staging copy has been consumed
   bool staged_pending = false;
   // mean-of-top-errors workspace, zero between calls
   peat::TopkState* topk = nullptr;
   peat::TopkListEntry* topk_list = nullptr;
+  // context-statistics accumulators (one per segment), zero between calls
+  peat::TsAcc* tsacc = nullptr;
   // injector staging (grown on demand)
   int64_t* d_inj = nullptr;
   int64_t* h_inj = nullptr;
@@ -187,23 +190,33 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   if (n / p.nctas >= ((int64_t)1 << 31) - 64)
     return fail(h, PEAT_ERR_UNSUPPORTED, "n is too large for one call (more than 2^31 elements per CTA)");
 
-  peat_status_t ps = wait_staging(h);
-  if (ps != PEAT_OK) return ps;
-  std::memcpy(h->h_offsets, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
-  int64_t* hb = h->h_offsets + nseg + 1;
-  const int nsplit = nseg > 1 && n > 0 ? segment_split(offsets, nseg, n, p.nctas, hb) : 0;
-  if (nsplit > 0)
-    p.nctas = nsplit;
-  else
-    for (int b = 0; b <= p.nctas; b++) hb[b] = peat::compare_cta_bound(dtype, b, p.nctas, n, p.p0);
-  cudaError_t e = cudaMemcpyAsync(h->d_offsets, h->h_offsets, sizeof(int64_t) * (size_t)(nseg + 2 + p.nctas),
-                                  cudaMemcpyHostToDevice, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(offsets)");
-  e = cudaEventRecord(h->staged, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
-  h->staged_pending = true;
-  p.offsets = h->d_offsets;
-  p.bounds = h->d_offsets + nseg + 1;
+  cudaError_t e;
+  if (nseg == 1) {
+    // one tensor: offsets and CTA bounds written on the device, no host staging
+    // (so back-to-back calls do not wait for each other on the host)
+    e = peat::launch_bounds_on_device(dtype, h->d_single, h->d_single + 2, p.nctas, n, p.p0, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "bounds launch");
+    p.offsets = h->d_single;
+    p.bounds = h->d_single + 2;
+  } else {
+    peat_status_t ps = wait_staging(h);
+    if (ps != PEAT_OK) return ps;
+    std::memcpy(h->h_offsets, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
+    int64_t* hb = h->h_offsets + nseg + 1;
+    const int nsplit = n > 0 ? segment_split(offsets, nseg, n, p.nctas, hb) : 0;
+    if (nsplit > 0)
+      p.nctas = nsplit;
+    else
+      for (int b = 0; b <= p.nctas; b++) hb[b] = peat::compare_cta_bound(dtype, b, p.nctas, n, p.p0);
+    e = cudaMemcpyAsync(h->d_offsets, h->h_offsets, sizeof(int64_t) * (size_t)(nseg + 2 + p.nctas),
+                        cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(offsets)");
+    e = cudaEventRecord(h->staged, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
+    h->staged_pending = true;
+    p.offsets = h->d_offsets;
+    p.bounds = h->d_offsets + nseg + 1;
+  }
   p.acc = h->acc;
   p.partials = h->partials;
   p.glist = h->glist;
@@ -360,10 +373,13 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
             cudaMemset(h->acc, 0, acc_bytes) == cudaSuccess &&
             cudaMalloc(&h->d_offsets, sizeof(int64_t) * staging) == cudaSuccess &&
             cudaMallocHost(&h->h_offsets, sizeof(int64_t) * staging) == cudaSuccess &&
+            cudaMalloc(&h->d_single, sizeof(int64_t) * (3 + 2 * (size_t)h->max_ctas)) == cudaSuccess &&
             cudaEventCreateWithFlags(&h->staged, cudaEventDisableTiming) == cudaSuccess &&
             cudaMalloc(&h->topk, sizeof(peat::TopkState)) == cudaSuccess &&
             cudaMemset(h->topk, 0, sizeof(peat::TopkState)) == cudaSuccess &&
             cudaMalloc(&h->topk_list, sizeof(peat::TopkListEntry) * peat::TK_LCAP) == cudaSuccess &&
+            cudaMalloc(&h->tsacc, sizeof(peat::TsAcc) * (size_t)h->max_segments) == cudaSuccess &&
+            cudaMemset(h->tsacc, 0, sizeof(peat::TsAcc) * (size_t)h->max_segments) == cudaSuccess &&
             cudaDeviceSynchronize() == cudaSuccess;
   if (!ok) {
     cudaGetLastError();
@@ -387,10 +403,12 @@ peat_status_t peat_signature_destroy(peat_handle_t h) {
     if (h->status_host) cudaFreeHost(h->status_host);
     if (h->d_offsets) cudaFree(h->d_offsets);
     if (h->h_offsets) cudaFreeHost(h->h_offsets);
+    if (h->d_single) cudaFree(h->d_single);
     if (h->d_inj) cudaFree(h->d_inj);
     if (h->h_inj) cudaFreeHost(h->h_inj);
     if (h->topk) cudaFree(h->topk);
     if (h->topk_list) cudaFree(h->topk_list);
+    if (h->tsacc) cudaFree(h->tsacc);
     if (h->staged) cudaEventDestroy(h->staged);
     cudaGetLastError();
   }
@@ -457,6 +475,150 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
     cudaMemsetAsync(h->topk, 0, sizeof(peat::TopkState), reinterpret_cast<cudaStream_t>(stream));
     return cuda_fail(h, e, "top-k launch");
   }
+  return PEAT_OK;
+}
+
+peat_status_t peat_tensor_stats(peat_handle_t h, const void* x, const int64_t* offsets, int64_t nseg,
+                                peat_dtype_t dtype, peat_tstats_t* stats_out, peat_stream_t stream) {
+  if (!h) return PEAT_ERR_INVALID_ARG;
+  const int B = dtype_bytes(dtype);
+  if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
+  if (nseg < 0) return fail(h, PEAT_ERR_INVALID_ARG, "nseg < 0");
+  if (nseg > h->max_segments) return fail(h, PEAT_ERR_UNSUPPORTED, "nseg exceeds the handle's max_segments");
+  if (!offsets) return fail(h, PEAT_ERR_INVALID_ARG, "offsets is NULL");
+  if (offsets[0] != 0) return fail(h, PEAT_ERR_INVALID_ARG, "offsets[0] must be 0");
+  for (int64_t s = 0; s < nseg; s++) {
+    if (offsets[s + 1] < offsets[s]) return fail(h, PEAT_ERR_INVALID_ARG, "offsets must be non-decreasing");
+    if (offsets[s + 1] - offsets[s] >= ((int64_t)1 << 36))
+      return fail(h, PEAT_ERR_UNSUPPORTED, "a segment of 2^36 elements or more");
+  }
+  const int64_t n = offsets[nseg];
+  if (n > 0 && !x) return fail(h, PEAT_ERR_INVALID_ARG, "x is NULL");
+  if (nseg > 0 && !stats_out) return fail(h, PEAT_ERR_INVALID_ARG, "stats_out is NULL");
+  if (nseg == 0) return PEAT_OK;
+  DeviceGuard dg(h->device);
+  if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  peat::TsParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.x = x;
+  p.n_total = n;
+  p.nseg = nseg;
+  const uintptr_t ax = reinterpret_cast<uintptr_t>(x);
+  p.p0 = (n > 0 && ax % B == 0) ? (int64_t)(((16 - ax % 16) % 16) / B) : -1;
+  // one wave of resident CTAs, about one CTA per 8K elements, within the staging area
+  const int64_t want = (n + 8191) / 8192;
+  const int64_t cap = std::min<int64_t>((int64_t)peat::tstats_ctas_per_sm() * h->nsm, 2 * (int64_t)h->max_ctas);
+  p.nctas = (int)std::max<int64_t>(1, std::min<int64_t>(cap, want));
+  cudaError_t e;
+  if (nseg == 1) {  // one tensor: no host staging (see compare_impl)
+    e = peat::launch_bounds_on_device(dtype, h->d_single, h->d_single + 2, p.nctas, n, p.p0, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "bounds launch");
+    p.offsets = h->d_single;
+    p.bounds = h->d_single + 2;
+  } else {
+    peat_status_t ps = wait_staging(h);
+    if (ps != PEAT_OK) return ps;
+    std::memcpy(h->h_offsets, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
+    int64_t* hb = h->h_offsets + nseg + 1;
+    for (int b = 0; b <= p.nctas; b++) hb[b] = peat::compare_cta_bound(dtype, b, p.nctas, n, p.p0);
+    e = cudaMemcpyAsync(h->d_offsets, h->h_offsets, sizeof(int64_t) * (size_t)(nseg + 2 + p.nctas),
+                        cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(offsets)");
+    e = cudaEventRecord(h->staged, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
+    h->staged_pending = true;
+    p.offsets = h->d_offsets;
+    p.bounds = h->d_offsets + nseg + 1;
+  }
+  p.acc = h->tsacc;
+  p.out = stats_out;
+  e = peat::launch_tstats(dtype, p, st);
+  if (e != cudaSuccess) {
+    cudaMemsetAsync(h->tsacc, 0, sizeof(peat::TsAcc) * (size_t)nseg, st);
+    return cuda_fail(h, e, "tensor-stats launch");
+  }
+  return PEAT_OK;
+}
+
+namespace {
+peat_status_t host_fail(const char* msg) {
+  g_null_error_is_noalloc = false;
+  g_create_error = msg;
+  return PEAT_ERR_INVALID_ARG;
+}
+}  // namespace
+
+peat_status_t peat_spearman(const double* x, const double* y, int64_t n, double* rho_out) {
+  if (!rho_out || n < 0 || (n > 0 && (!x || !y))) return host_fail("null pointer or n < 0");
+  for (int64_t i = 0; i < n; i++)
+    if (!std::isfinite(x[i]) || !std::isfinite(y[i])) return host_fail("a value is not finite");
+  if (n < 2) {
+    *rho_out = std::nan("");
+    return PEAT_OK;
+  }
+  // doubled ranks (integers): a tie group spanning ranks r..r+c-1 takes r + (c - 1) / 2 each
+  auto doubled_ranks = [n](const double* v) {
+    std::vector<int64_t> idx((size_t)n), r2((size_t)n);
+    for (int64_t i = 0; i < n; i++) idx[(size_t)i] = i;
+    std::stable_sort(idx.begin(), idx.end(), [v](int64_t a, int64_t b) { return v[a] < v[b]; });
+    for (int64_t i = 0; i < n;) {
+      int64_t j = i;
+      while (j + 1 < n && v[idx[(size_t)(j + 1)]] == v[idx[(size_t)i]]) j++;
+      for (int64_t k = i; k <= j; k++) r2[(size_t)idx[(size_t)k]] = (i + 1) + (j + 1);  // 2 * mean rank
+      i = j + 1;
+    }
+    return r2;
+  };
+  const std::vector<int64_t> rx = doubled_ranks(x), ry = doubled_ranks(y);
+  // exact integer moments of the doubled ranks
+  __int128 sx = 0, sy = 0, sxx = 0, syy = 0, sxy = 0;
+  for (int64_t i = 0; i < n; i++) {
+    const __int128 a = rx[(size_t)i], b = ry[(size_t)i];
+    sx += a;
+    sy += b;
+    sxx += a * a;
+    syy += b * b;
+    sxy += a * b;
+  }
+  const __int128 N = n;
+  const __int128 cxy = N * sxy - sx * sy, cxx = N * sxx - sx * sx, cyy = N * syy - sy * sy;
+  if (cxx == 0 || cyy == 0) {
+    *rho_out = std::nan("");
+    return PEAT_OK;
+  }
+  const long double num = (long double)cxy, den = sqrtl((long double)cxx) * sqrtl((long double)cyy);
+  *rho_out = (double)(num / den);
+  return PEAT_OK;
+}
+
+peat_status_t peat_mean_std(const double* x, int64_t n, int ddof, double* mean_out, double* std_out) {
+  if (!mean_out || !std_out || n < 0 || (n > 0 && !x)) return host_fail("null pointer or n < 0");
+  if (ddof != 0 && ddof != 1) return host_fail("ddof must be 0 or 1");
+  for (int64_t i = 0; i < n; i++)
+    if (!std::isfinite(x[i])) return host_fail("a value is not finite");
+  if (n == 0) {
+    *mean_out = *std_out = std::nan("");
+    return PEAT_OK;
+  }
+  // two passes with compensated (Neumaier) sums
+  auto csum = [n](auto f) {
+    double s = 0.0, c = 0.0;
+    for (int64_t i = 0; i < n; i++) {
+      const double v = f(i), t = s + v;
+      c += std::fabs(s) >= std::fabs(v) ? (s - t) + v : (v - t) + s;
+      s = t;
+    }
+    return s + c;
+  };
+  const double mean = csum([x](int64_t i) { return x[i]; }) / (double)n;
+  *mean_out = mean;
+  if (n <= ddof) {
+    *std_out = std::nan("");
+    return PEAT_OK;
+  }
+  const double ss = csum([x, mean](int64_t i) { return (x[i] - mean) * (x[i] - mean); });
+  *std_out = std::sqrt(ss / (double)(n - ddof));
   return PEAT_OK;
 }
 

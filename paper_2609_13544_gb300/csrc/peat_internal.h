@@ -131,6 +131,26 @@ struct TopkParams {
 int topk_max_ctas(int nsm);
 cudaError_t launch_topk(int dtype, const TopkParams& p, int nctas, cudaStream_t s);
 
+// ---- context statistics (tstats.cu) ----
+struct TsAcc {  // per segment, zero between calls
+  long long limbs[2][NLIMB];      // exact sum and sum of squares of the finite elements
+  unsigned long long nfin, nnan, ninf;
+  unsigned int kmin_inv, kmax;    // order keys: ~(smallest finite), largest finite
+};
+struct TsParams {
+  const void* x;
+  int64_t n_total;
+  int64_t p0;               // first element of the 16-byte vector grid; -1: none
+  int64_t nseg;
+  const int64_t* offsets;   // device, nseg + 1
+  const int64_t* bounds;    // device, nctas + 1
+  int nctas;
+  TsAcc* acc;               // nseg accumulators
+  peat_tstats_t* out;       // device, nseg records
+};
+int tstats_ctas_per_sm();
+cudaError_t launch_tstats(int dtype, const TsParams& p, cudaStream_t s);
+
 struct InjectElemParams {
   void* dst;
   const void* src;

@@ -16,7 +16,8 @@ def declared_functions():
 def test_header_declares_the_boundary():
     assert declared_functions() == sorted([
         "peat_compare", "peat_compare_noalloc", "peat_compare_segmented", "peat_last_error",
-        "peat_pseudo_error_inject", "peat_signature_create", "peat_signature_destroy", "peat_topk_mean"])
+        "peat_mean_std", "peat_pseudo_error_inject", "peat_signature_create", "peat_signature_destroy",
+        "peat_spearman", "peat_tensor_stats", "peat_topk_mean"])
 
 
 def test_library_builds_and_exports_every_declared_symbol():
@@ -33,6 +34,7 @@ def test_binding_names_match_the_abi():
         assert hasattr(peat, name), name
     assert peat.STATS_DTYPE.itemsize == 144
     assert peat.TOPK_DTYPE.itemsize == 48
+    assert peat.TSTATS_DTYPE.itemsize == 80
 
 
 def test_last_error_without_handle_is_empty_string():

@@ -522,3 +522,66 @@ def test_topk_ties_zeros_and_arguments(oracle):
     for num, den in ((0, 10), (11, 10), (1, 0)):
         with pytest.raises(ValueError):
             oracle.topk_mean(x, y, "bf16", num, den)
+
+
+# ---------------------------------------------------------------------------
+# context statistics (Section IV-C-2): pinned to exact rational arithmetic on
+# the decoded values and to Python's statistics module
+# ---------------------------------------------------------------------------
+def _decoded(bits, dtype):
+    import torch
+    tdt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}[dtype]
+    iv = torch.int32 if dtype == "f32" else torch.int16
+    t = torch.from_numpy(np.ascontiguousarray(bits).view(np.int32 if dtype == "f32" else np.int16)).view(tdt)
+    return [float(v) for v in t.to(torch.float64).tolist()]
+
+
+def ref_tstats(vals):
+    from fractions import Fraction
+    fin = [v for v in vals if math.isfinite(v)]
+    nf = len(fin)
+    s1 = sum(Fraction(v) for v in fin)
+    s2 = sum(Fraction(v) * Fraction(v) for v in fin)
+    out = {"n": len(vals), "n_finite": nf, "n_nan": sum(1 for v in vals if math.isnan(v)),
+           "n_inf": sum(1 for v in vals if math.isinf(v)), "sum": float(s1), "sum_sq": float(s2),
+           "mean": float(s1 / nf) if nf else 0.0, "var": float(s2 / nf - (s1 / nf) ** 2) if nf else 0.0}
+    if nf:
+        key = lambda v: (v, math.copysign(1.0, v))  # -0 below +0
+        out["min"], out["max"] = min(fin, key=key), max(fin, key=key)
+    else:
+        out["min"] = out["max"] = 0.0
+    return out
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f16", "bf16"])
+def test_tensor_stats_against_exact_rationals(oracle, dtype):
+    from parity_util import random_pairs
+    for seed, n in [(1, 0), (2, 1), (3, 17), (4, 3000)]:
+        g, c = random_pairs(dtype, n, seed)
+        bits = np.concatenate([g, c])
+        got = oracle.tensor_stats(bits, dtype)
+        want = ref_tstats(_decoded(bits, dtype))
+        for k, v in want.items():
+            a = got[k]
+            assert a == v and (not isinstance(v, float) or math.copysign(1, a) == math.copysign(1, v)), \
+                (dtype, seed, k, a, v)
+
+
+def test_tensor_stats_closed_forms(oracle):
+    import statistics
+    # a constant tensor has variance exactly 0; two values a, b have (a - b)^2 / 4
+    c = np.full(1000, 0.1, np.float32).view(np.uint32)
+    r = oracle.tensor_stats(c, "f32")
+    assert r["var"] == 0.0 and r["mean"] == float(np.float32(0.1))
+    ab = np.array([3.0, -1.0] * 50, np.float32).view(np.uint32)
+    assert oracle.tensor_stats(ab, "f32")["var"] == 4.0
+    # statistics.pvariance / fmean work in exact fractions on these doubles
+    rng = np.random.default_rng(9)
+    x = (rng.standard_normal(5000) * 3 + 100).astype(np.float32)
+    r = oracle.tensor_stats(x.view(np.uint32), "f32")
+    assert r["var"] == statistics.pvariance([float(v) for v in x])
+    assert r["mean"] == statistics.mean([float(v) for v in x])
+    # -0 sorts below +0 in min/max
+    z = np.array([0.0, -0.0, 0.0], np.float32).view(np.uint32)
+    rz = oracle.tensor_stats(z, "f32")
+    assert math.copysign(1, rz["min"]) < 0 and math.copysign(1, rz["max"]) > 0

@@ -33,7 +33,8 @@ __device__ __forceinline__ uint64_t split_double(double x, int& e) {
 }
 
 // Signed 32-bit digits of +-m * 2^e (m < 2^128), delivered to f(digit, value).
-// Every value that occurs is a multiple of 2^LIMB_LSB and below 2^352.
+// Every value that occurs is a multiple of 2^LIMB_LSB and below 2^352; a digit
+// outside [0, NLIMB) is dropped rather than written out of bounds.
 template <class F>
 __device__ __forceinline__ void for_digits(unsigned __int128 m, int e, bool neg, F&& f) {
   if (m == 0) return;
@@ -47,7 +48,7 @@ __device__ __forceinline__ void for_digits(unsigned __int128 m, int e, bool neg,
   out[4] = r ? (md[3] >> (32 - r)) : 0u;
 #pragma unroll
   for (int k = 0; k < 5; k++)
-    if (out[k] && j + k < NLIMB) f(j + k, neg ? -(int64_t)out[k] : (int64_t)out[k]);
+    if (out[k] && (unsigned)(j + k) < (unsigned)NLIMB) f(j + k, neg ? -(int64_t)out[k] : (int64_t)out[k]);
 }
 
 // RN-even binary64 of the exact value of NLIMB carry-save digits (digit j

@@ -181,3 +181,25 @@ def test_forced_wait_expiry_reports_timeout_and_context_survives(peat_gpu, oracl
     torch.cuda.synchronize()
     bad.close()
     check_pair(peat_gpu, oracle, h, gb, cb, "bf16", 1e-3, 0.0, ctx="after forced expiry")
+
+
+@pytest.mark.parametrize("rtol", [2.0 ** -7, 2.0 ** -3, 1e-3])
+@pytest.mark.parametrize("atol", [0.0, 1e-7])
+def test_tolerance_ties_float32(peat_gpu, oracle, h, rtol, atol):
+    """Pairs whose |c - g| is the float32 rounding of rtol |g| exactly, and their
+    one-step neighbours: the tolerance decided at and around the tie (with
+    atol = 0 by the sign of rtol |g| - |d| in the window path)."""
+    rng = np.random.default_rng(61)
+    n = 200_000
+    mag = (rng.standard_normal(n) * np.exp2(rng.integers(-30, 30, n))).astype(np.float32)
+    g = (mag.view(np.uint32) & np.uint32(0xFFFFF000)).view(np.float32)  # low mantissa bits clear
+    r32 = np.float32(rtol)
+    a = (np.abs(g).astype(np.float64) * np.float64(r32)).astype(np.float32)  # RN32(rtol |g|)
+    c0 = (g + np.where(rng.random(n) < 0.5, a, -a)).astype(np.float32)
+    up = np.nextafter(c0, np.float32(np.inf))
+    dn = np.nextafter(c0, np.float32(-np.inf))
+    gb = np.concatenate([g, g, g]).view(np.uint32)
+    cb = np.concatenate([c0, up, dn]).view(np.uint32)
+    perm = rng.permutation(gb.size)
+    gs = check_pair(peat_gpu, oracle, h, gb[perm], cb[perm], "f32", rtol, atol, ctx=f"ties rtol={rtol} atol={atol}")
+    assert gs["within_tol"] > 0 and gs["mismatch"] > 0

@@ -1160,12 +1160,8 @@ __device__ __forceinline__ void gen_counts(const GenRec& g, Smem& sm) {
 template <int DT>
 __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p, int64_t pb, int64_t pe,
                                          int64_t vb, int64_t ve) {
-  __syncthreads();
+  // entered only after a barrier and with at least one general pair (finish_piece)
   const uint32_t n = sm.gn;
-  if (n == 0) {  // no general pair in this piece
-    if ((threadIdx.x & 31) == 0) part_none(sm.wbest[threadIdx.x >> 5]);
-    return;
-  }
   const int64_t lo = sm.lo;
   GenRec cd;
   gen_init(cd);
@@ -1290,7 +1286,14 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
                                              int64_t seg, int64_t pb, int64_t pe, int64_t vb, int64_t ve) {
   Partial* out = p.partials + seg + blockIdx.x;
   SegAcc* acc = p.acc + seg;
-  run_general<DT>(W, sm, p, pb, pe, vb, ve);
+  // the piece's general pairs, if any: the out-of-line call (and its register
+  // traffic) only when there is one
+  __syncthreads();
+  if (sm.gn != 0) {
+    run_general<DT>(W, sm, p, pb, pe, vb, ve);
+  } else if ((threadIdx.x & 31) == 0) {
+    part_none(sm.wbest[threadIdx.x >> 5]);
+  }
   fold_round<DT>(L, sm, win_lexp<DT>(W));  // ends with a barrier: the general path's per-warp totals are complete
   for (int b = threadIdx.x; b < HBINS; b += BLOCK) {
     unsigned long long v = 0;

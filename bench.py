@@ -347,6 +347,30 @@ def run_gpu(args) -> None:
                                "frac": ts_gbs / peak, "algorithmic_bytes_per_call": one,
                                "note": "one read of the tensor; stage 1 plus a per-segment finalize"}}
 
+    # isclose pass counts over an 8 x 8 tolerance grid (Section III-A, Fig. 5): one read of both tensors
+    isc = None
+    if not args.no_topk:
+        rts = [0.0, 1e-5, 1e-4, 1e-3, 2.0 ** -7, 1e-2, 0.1, 1.0]
+        ats = [0.0, 1e-8, 1e-6, 1e-4, 1e-2, 1.0, 1e3, 1e30]
+        ic_out = torch.empty(64, dtype=torch.int64, device=dev)
+        for _ in range(3):
+            peat.peat_isclose_grid_raw(h, g, c, rts, ats, ic_out, stream)
+        barrier()
+        ic_calls = max(3, min(50, args.steps // 100))
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(ic_calls):
+            peat.peat_isclose_grid_raw(h, g, c, rts, ats, ic_out, stream)
+        t1.record(stream)
+        barrier()
+        ic_ms = max_over_ranks(t0.elapsed_time(t1), dev) / ic_calls
+        ic_gbs = bytes_per_step / (ic_ms * 1e-3) / 1e9
+        isc = {"op": "peat_isclose_grid, 8 rtols x 8 atols", "calls": ic_calls, "us_per_call": ic_ms * 1e3,
+               "pairs_per_s": w.n / (ic_ms * 1e-3),
+               "roofline": {"bound": "alu", "achieved": ic_gbs, "peak": peak, "unit": "GB/s", "frac": ic_gbs / peak,
+                            "algorithmic_bytes_per_call": bytes_per_step,
+                            "note": "one read of both tensors; 64 exact tolerance decisions per differing pair"}}
+
     # end to end through the C ABI with host buffers: H2D of both tensors from
     # pinned memory, the compare, D2H of the stats and histograms, every step
     e2e = None
@@ -412,7 +436,7 @@ def run_gpu(args) -> None:
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy)" if not peaks.get("fallback")
                          else "fallback 6.8 TB/s"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": (1 if nseg == 1 else 2) * args.steps, "clocks": clocks,
-            "next_rows": {"f1_top10_mean": topk, "f3_context_stats": tstats},
+            "next_rows": {"f1_top10_mean": topk, "f3_context_stats": tstats, "f4_isclose_grid": isc},
             "wall_s_timed": wall,
         }
         print(json.dumps(line), flush=True)

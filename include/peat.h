@@ -250,6 +250,26 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
                              peat_dtype_t dtype, uint64_t num, uint64_t den, peat_topk_t* out,
                              peat_stream_t stream);
 
+/* torch.isclose pass counts over a grid of tolerances (Section III-A; its
+ * Fig. 5 plots the share of output elements isclose accepts for FP16-FP32
+ * and FP32-FP64 pairs as rtol and atol vary), in one read of both tensors:
+ * counts_out[i * na + j] = the pairs peat_compare with tolerance
+ * (rtols[i], atols[j]) would class EXACT or WITHIN_TOL, i.e. both operands
+ * NaN, or the same infinity, or finite with |c - g| <= atols[j] + rtols[i] |g|
+ * exactly.
+ *   golden, candidate  as for peat_compare (device, any alignment).
+ *   rtols, atols       HOST arrays (read before return); every value finite
+ *                      and >= 0, rounded to float32 as peat_compare does;
+ *                      rtols non-decreasing after the rounding.
+ *   nr, na             1 <= nr, na and nr * na <= 64.
+ *   counts_out         device pointer to nr * na uint64 (overwritten).
+ * About 4 nr na + 10 na log2(nr) operations per differing pair (bitwise-equal
+ * warp slots cost a vote).  Asynchronous on `stream`.
+ * Errors: INVALID_ARG (bad dtype, pointers, tolerances or grid size), CUDA. */
+peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void* candidate, int64_t n,
+                                peat_dtype_t dtype, const double* rtols, int nr, const double* atols, int na,
+                                uint64_t* counts_out, peat_stream_t stream);
+
 /* Context statistics of one recorded tensor (Section IV-C-2: the means and
  * variances of the weight and activation tensors that the error scores are
  * correlated with).  80 bytes.  Every double is the exact value rounded once

@@ -167,6 +167,17 @@ def topk_mean(g, c, dtype: str, num: int = 1, den: int = 10) -> dict:
     return {f: getattr(out, f) for f, _ in TopK._fields_}
 
 
+def isclose_grid(g, c, dtype: str, rtols, atols) -> np.ndarray:
+    """torch.isclose pass counts over a tolerance grid (Section III-A, Fig. 5):
+    cell (i, j) = EXACT + WITHIN_TOL of the compare with (rtols[i], atols[j])."""
+    out = np.zeros((len(rtols), len(atols)), np.uint64)
+    for i, r in enumerate(rtols):
+        for j, a in enumerate(atols):
+            st, _ = compare(g, c, dtype, float(r), float(a))
+            out[i, j] = st["exact"] + st["within_tol"]
+    return out
+
+
 def _acc_int(words) -> int:
     """The fixed-point words as a Python integer (value = integer * 2^ACC_LSB)."""
     v = 0

@@ -77,7 +77,7 @@ class InjectModel(ctypes.Structure):
 
 EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
            "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc", "peat_topk_mean",
-           "peat_tensor_stats", "peat_spearman", "peat_mean_std")
+           "peat_tensor_stats", "peat_spearman", "peat_mean_std", "peat_isclose_grid")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -110,6 +110,8 @@ def load(path: Optional[Path] = None) -> ctypes.CDLL:
     L.peat_compare_noalloc.restype = i32
     L.peat_topk_mean.argtypes = [vp, vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, vp, vp]
     L.peat_topk_mean.restype = i32
+    L.peat_isclose_grid.argtypes = [vp, vp, vp, i64, i32, vp, i32, vp, i32, vp, vp]
+    L.peat_isclose_grid.restype = i32
     L.peat_tensor_stats.argtypes = [vp, vp, vp, i64, i32, vp, vp]
     L.peat_tensor_stats.restype = i32
     dp = ctypes.POINTER(ctypes.c_double)
@@ -318,6 +320,26 @@ def peat_tensor_stats(h: Handle, x, offsets: Optional[Sequence[int]] = None, str
     arr = np.frombuffer(out.cpu().numpy()[: nseg * TSTATS_BYTES].tobytes(), dtype=TSTATS_DTYPE)
     res = [{k: r[k].item() for k in TSTATS_DTYPE.names} for r in arr]
     return res[0] if offsets is None else res
+
+
+def peat_isclose_grid_raw(h: Handle, golden, candidate, rtols, atols, counts_out, stream=None) -> None:
+    """peat_isclose_grid on a preallocated device output (counts_out: int64[len(rtols) * len(atols)])."""
+    _dev_tensor_check(golden, candidate)
+    if golden.numel() != candidate.numel() or golden.dtype != candidate.dtype:
+        raise ValueError("golden and candidate differ in size or dtype")
+    r, a = _host_doubles(rtols), _host_doubles(atols)
+    rc = load().peat_isclose_grid(h.ptr, golden.data_ptr(), candidate.data_ptr(), golden.numel(),
+                                  dtype_code(golden), r.ctypes.data, r.size, a.ctypes.data, a.size,
+                                  counts_out.data_ptr(), _stream_ptr(stream))
+    _check(rc, h)
+
+
+def peat_isclose_grid(h: Handle, golden, candidate, rtols, atols, stream=None) -> np.ndarray:
+    """isclose pass counts, uint64 [len(rtols), len(atols)]; synchronises."""
+    import torch
+    out = torch.empty(len(rtols) * len(atols), dtype=torch.int64, device=golden.device)
+    peat_isclose_grid_raw(h, golden, candidate, rtols, atols, out, stream)
+    return out.cpu().numpy().view(np.uint64).reshape(len(rtols), len(atols))
 
 
 def _host_doubles(v) -> np.ndarray:

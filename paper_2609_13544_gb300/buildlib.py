@@ -17,7 +17,7 @@ ROOT = PKG.parent
 CSRC = PKG / "csrc"
 OUT_DIR = PKG / "_build"
 LIB = OUT_DIR / "libpeat.so"
-SOURCES = ["compare.cu", "topk.cu", "tstats.cu", "inject.cu", "peat_api.cpp"]
+SOURCES = ["compare.cu", "topk.cu", "tstats.cu", "isclose.cu", "inject.cu", "peat_api.cpp"]
 HEADERS = [CSRC / "peat_internal.h", CSRC / "exact.cuh", ROOT / "include" / "peat.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",

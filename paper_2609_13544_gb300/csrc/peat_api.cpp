@@ -478,6 +478,62 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
   return PEAT_OK;
 }
 
+peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void* candidate, int64_t n,
+                                peat_dtype_t dtype, const double* rtols, int nr, const double* atols, int na,
+                                uint64_t* counts_out, peat_stream_t stream) {
+  if (!h) return PEAT_ERR_INVALID_ARG;
+  const int B = dtype_bytes(dtype);
+  if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
+  if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
+  if (n > 0 && (!golden || !candidate)) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
+  if (!rtols || !atols || !counts_out) return fail(h, PEAT_ERR_INVALID_ARG, "rtols/atols/counts_out is NULL");
+  if (nr < 1 || na < 1 || nr * na > peat::ISC_MAX)
+    return fail(h, PEAT_ERR_INVALID_ARG, "need 1 <= nr, na and nr * na <= 64");
+  peat::IscParams p;
+  std::memset(&p, 0, sizeof(p));
+  for (int i = 0; i < nr; i++) {
+    float r, a;
+    if (!round_tol(peat_tol_t{rtols[i], 0.0}, &r, &a))
+      return fail(h, PEAT_ERR_INVALID_ARG, "rtols must be finite and >= 0 after rounding to float32");
+    if (i > 0 && r < p.rtol[i - 1]) return fail(h, PEAT_ERR_INVALID_ARG, "rtols must be non-decreasing");
+    p.rtol[i] = r;
+  }
+  for (int j = 0; j < na; j++) {
+    float r, a;
+    if (!round_tol(peat_tol_t{0.0, atols[j]}, &r, &a))
+      return fail(h, PEAT_ERR_INVALID_ARG, "atols must be finite and >= 0 after rounding to float32");
+    p.atol[j] = a;
+  }
+  DeviceGuard dg(h->device);
+  if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  p.g = golden;
+  p.c = candidate;
+  p.n = n;
+  p.nr = nr;
+  p.na = na;
+  p.ncells = nr * na;
+  p.counts = reinterpret_cast<unsigned long long*>(counts_out);
+  const uintptr_t ag = reinterpret_cast<uintptr_t>(golden), ac = reinterpret_cast<uintptr_t>(candidate);
+  const int64_t vec = 16 / B;
+  p.p0 = -1;
+  if (n > 0 && ag % B == 0 && ac % B == 0 && ag % 16 == ac % 16) {
+    const int64_t p0 = (int64_t)(((16 - ag % 16) % 16) / B);
+    if (p0 < n) {
+      p.p0 = p0;
+      p.nvec = (n - p0) / vec;
+    }
+  }
+  cudaError_t e = cudaMemsetAsync(counts_out, 0, sizeof(uint64_t) * (size_t)p.ncells, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemsetAsync(counts)");
+  if (n == 0) return PEAT_OK;
+  const int64_t want = (n + 4095) / 4096;
+  const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)h->nsm * 8, want));
+  e = peat::launch_isclose(dtype, p, nctas, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "isclose launch");
+  return PEAT_OK;
+}
+
 peat_status_t peat_tensor_stats(peat_handle_t h, const void* x, const int64_t* offsets, int64_t nseg,
                                 peat_dtype_t dtype, peat_tstats_t* stats_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;

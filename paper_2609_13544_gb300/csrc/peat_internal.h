@@ -151,6 +151,20 @@ struct TsParams {
 int tstats_ctas_per_sm();
 cudaError_t launch_tstats(int dtype, const TsParams& p, cudaStream_t s);
 
+// ---- isclose pass counts over a tolerance grid (isclose.cu) ----
+constexpr int ISC_MAX = 64;  // cells (nr * na) at most; nr, na at most as many
+struct IscParams {
+  const void* g;
+  const void* c;
+  int64_t n;
+  int64_t p0;     // first element of the 16-byte vector grid; -1: none
+  int64_t nvec;   // vectors on the grid
+  int nr, na, ncells;
+  float rtol[ISC_MAX], atol[ISC_MAX];  // float32 tolerances, rtol ascending
+  unsigned long long* counts;          // device, ncells (cell i * na + j), zero before the launch
+};
+cudaError_t launch_isclose(int dtype, const IscParams& p, int nctas, cudaStream_t s);
+
 struct InjectElemParams {
   void* dst;
   const void* src;

@@ -215,6 +215,26 @@ peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* s
                                        peat_dtype_t dtype, const peat_inject_t* models, int nmodels,
                                        uint64_t seed, uint64_t* counts_out, peat_stream_t stream);
 
+/* Fused pseudo-error assessment of one tensor (the Inject and Compare steps
+ * of the playback loop, Alg. 1, in one read of the golden tensor): the
+ * candidate is golden with models[0..nmodels) applied in array order, each
+ * element generated in registers and never written to memory, and the result
+ * is that of peat_compare(golden, candidate) with the candidate
+ * peat_pseudo_error_inject(golden, models, seed) would write, bit for bit.
+ *   golden        device array of n elements (any alignment).
+ *   models        HOST array, 1 <= nmodels <= 8, element-wise kinds only
+ *                 (NAN_INF, SIGNFLIP, REL_GAUSS, ADD_GAUSS, BIAS, the casts);
+ *                 parameters as for peat_pseudo_error_inject.
+ *   seed          the injector's seed (same Philox counters).
+ *   tol, stats_out, hist_out  as for peat_compare.
+ * No per-model fire counts are produced.
+ * Errors: INVALID_ARG (as for the two calls it fuses), UNSUPPORTED (a
+ * fixed-count model: RZ, RV, BITFLIP draw their positions on the host and
+ * are applied by peat_pseudo_error_inject), CUDA, ALLOC. */
+peat_status_t peat_inject_compare(peat_handle_t h, const void* golden, int64_t n, peat_dtype_t dtype,
+                                  const peat_inject_t* models, int nmodels, uint64_t seed, peat_tol_t tol,
+                                  peat_stats_t* stats_out, uint64_t* hist_out, peat_stream_t stream);
+
 /* Mean of the top errors of one tensor pair (Section IV-B-3, "Mean of Top
  * 10% Errors").  48 bytes. */
 typedef struct {

@@ -6,7 +6,7 @@ ABI through ctypes, and unpacks the result records.  It raises if the
 library has not been built (there is no CPU fallback).
 
 Names follow the C ABI: ``peat_signature_create``, ``peat_compare``,
-``peat_compare_segmented``, ``peat_pseudo_error_inject``, ``peat_last_error``.
+``peat_compare_segmented``, ``peat_pseudo_error_inject``, ``peat_inject_compare``, ``peat_last_error``.
 """
 from __future__ import annotations
 
@@ -77,7 +77,7 @@ class InjectModel(ctypes.Structure):
 
 EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
            "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc", "peat_topk_mean",
-           "peat_tensor_stats", "peat_spearman", "peat_mean_std", "peat_isclose_grid")
+           "peat_tensor_stats", "peat_spearman", "peat_mean_std", "peat_isclose_grid", "peat_inject_compare")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -104,6 +104,9 @@ def load(path: Optional[Path] = None) -> ctypes.CDLL:
     L.peat_pseudo_error_inject.argtypes = [vp, vp, vp, i64, i32, ctypes.POINTER(InjectModel), i32,
                                            ctypes.c_uint64, vp, vp]
     L.peat_pseudo_error_inject.restype = i32
+    L.peat_inject_compare.argtypes = [vp, vp, i64, i32, ctypes.POINTER(InjectModel), i32, ctypes.c_uint64, Tol,
+                                      vp, vp, vp]
+    L.peat_inject_compare.restype = i32
     L.peat_last_error.argtypes = [vp]
     L.peat_last_error.restype = ctypes.c_char_p
     L.peat_compare_noalloc.argtypes = [vp, vp, i64, i32, Tol, vp, vp, vp]
@@ -378,16 +381,45 @@ def peat_pseudo_error_inject(h: Handle, src, models: Sequence[dict], seed: int, 
     _dev_tensor_check(src)
     if dst is None:
         dst = torch.empty_like(src)
-    arr = (InjectModel * max(len(models), 1))()
-    for i, m in enumerate(models):
-        arr[i] = InjectModel(INJECT_KINDS[m["kind"]], m.get("k", 0), m.get("bit_lo", 0), m.get("bit_hi", 0),
-                             float(m.get("x", 0.0)))
+    arr = _model_array(models)
     counts = torch.zeros(max(len(models), 1), dtype=torch.int64, device=src.device)
     rc = load().peat_pseudo_error_inject(h.ptr, dst.data_ptr(), src.data_ptr(), src.numel(), dtype_code(src), arr,
                                          len(models), ctypes.c_uint64(seed), counts.data_ptr(),
                                          _stream_ptr(stream))
     _check(rc, h)
     return dst, counts[: len(models)].cpu().numpy().view(np.uint64)
+
+
+def _model_array(models: Sequence[dict]):
+    arr = (InjectModel * max(len(models), 1))()
+    for i, m in enumerate(models):
+        arr[i] = InjectModel(INJECT_KINDS[m["kind"]], m.get("k", 0), m.get("bit_lo", 0), m.get("bit_hi", 0),
+                             float(m.get("x", 0.0)))
+    return arr
+
+
+def peat_inject_compare_raw(h: Handle, golden, models: Sequence[dict], seed: int, rtol: float, atol: float,
+                            stats_out, hist_out=None, stream=None) -> None:
+    """peat_inject_compare on preallocated device outputs (stats_out: uint8[144], hist_out: int64[128])."""
+    _dev_tensor_check(golden)
+    rc = load().peat_inject_compare(h.ptr, golden.data_ptr(), golden.numel(), dtype_code(golden),
+                                    _model_array(models), len(models), ctypes.c_uint64(seed), Tol(rtol, atol),
+                                    stats_out.data_ptr(), hist_out.data_ptr() if hist_out is not None else None,
+                                    _stream_ptr(stream))
+    _check(rc, h)
+
+
+def peat_inject_compare(h: Handle, golden, models: Sequence[dict], seed: int, rtol: float, atol: float = 0.0,
+                        stream=None):
+    """Signature of golden against its injected copy (generated in the kernel, never stored):
+    (stats dict, hist numpy uint64[2, 64]); synchronises."""
+    import torch
+    dev = golden.device
+    stats = torch.empty(STATS_BYTES, dtype=torch.uint8, device=dev)
+    hist = torch.empty(HIST_BINS, dtype=torch.int64, device=dev)
+    peat_inject_compare_raw(h, golden, models, seed, rtol, atol, stats, hist, stream)
+    s = stats_to_dicts(stats.cpu().numpy())[0]
+    return s, hist.cpu().numpy().view(np.uint64).reshape(2, 64)
 
 
 def derived_scores(st: dict) -> dict:

@@ -42,6 +42,7 @@
 #include <cstdint>
 
 #include "exact.cuh"
+#include "inject_models.cuh"
 #include "peat_internal.h"
 
 namespace peat {
@@ -110,6 +111,41 @@ template <int DT>
 __device__ __forceinline__ uint32_t load_scalar(const void* base, int64_t i) {
   if constexpr (Tr<DT>::BYTES == 4) return __ldg(reinterpret_cast<const uint32_t*>(base) + i);
   else return (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(base) + i);
+}
+
+// The candidate of a fused call: the golden after the call's element-wise
+// models, in order (the same arithmetic as the injector's passes).
+template <int DT>
+__device__ __forceinline__ uint32_t inj_chain(const CompareParams& p, uint32_t b, int64_t i) {
+  for (int m = 0; m < p.inj_n; m++) {
+    bool fired;
+    b = inj::apply_model<DT>(b, i, p.inj[m].kind, p.inj[m].model, p.inj[m].threshold, p.inj[m].x, p.inj_k0,
+                             p.inj_k1, fired);
+  }
+  return b;
+}
+// candidate element i (golden bits G): generated (fused) or read
+template <int DT, bool INJ>
+__device__ __forceinline__ uint32_t cand_at(const CompareParams& p, int64_t i, uint32_t G) {
+  if constexpr (INJ) return inj_chain<DT>(p, G, i);
+  else return load_scalar<DT>(p.c, i);
+}
+// the candidate vector of golden vector gv whose first element is i0
+template <int DT>
+__device__ __forceinline__ uint4 inj_vec(const CompareParams& p, const uint4& gv, int64_t i0) {
+  uint32_t w[4] = {gv.x, gv.y, gv.z, gv.w};
+  if constexpr (Tr<DT>::BYTES == 4) {
+#pragma unroll
+    for (int j = 0; j < 4; j++) w[j] = inj_chain<DT>(p, w[j], i0 + j);
+  } else {
+#pragma unroll
+    for (int k = 0; k < 4; k++) {
+      const uint32_t lo = inj_chain<DT>(p, w[k] & 0xFFFFu, i0 + 2 * k);
+      const uint32_t hi = inj_chain<DT>(p, w[k] >> 16, i0 + 2 * k + 1);
+      w[k] = (lo & 0xFFFFu) | (hi << 16);
+    }
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
 __device__ __forceinline__ uint4 load_vec(const void* base, int64_t byte_off) {
@@ -1157,7 +1193,7 @@ __device__ __forceinline__ void gen_counts(const GenRec& g, Smem& sm) {
 // the CTA: from the list when it held them all, else found again by a rescan
 // of the piece with the same window test.  Out of line, so that the hot loop
 // carries no call.  Leaves each warp's general maxima in sm.wbest[warp].
-template <int DT>
+template <int DT, bool INJ>
 __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p, int64_t pb, int64_t pe,
                                          int64_t vb, int64_t ve) {
   // entered only after a barrier and with at least one general pair (finish_piece)
@@ -1168,11 +1204,12 @@ __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p
   if (n <= (uint32_t)GCAP) {
     for (uint32_t e = threadIdx.x; e < n; e += BLOCK) {
       const int64_t i = lo + sm.glist[e];
-      general_lane<DT>(sm, cd, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), i, W.rtol, W.atol);
+      const uint32_t G = load_scalar<DT>(p.g, i);
+      general_lane<DT>(sm, cd, G, cand_at<DT, INJ>(p, i, G), i, W.rtol, W.atol);
     }
   } else {
     for (int64_t i = pb + threadIdx.x; i < pe; i += BLOCK) {
-      const uint32_t G = load_scalar<DT>(p.g, i), C = load_scalar<DT>(p.c, i);
+      const uint32_t G = load_scalar<DT>(p.g, i), C = cand_at<DT, INJ>(p, i, G);
       if (G == C) continue;
       uint32_t gr = G, cr = C;
       if constexpr (DT == PEAT_BF16) {
@@ -1226,13 +1263,14 @@ __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p
 
 // [pb, pe): the lowest index of a finite pair and of a pair without NaN
 // (the argmax when every error is zero), searched BLOCK elements at a time
-template <int DT>
+template <int DT, bool INJ>
 __device__ __noinline__ void first_pairs(Smem& sm, const CompareParams& p, int64_t pb, int64_t pe) {
   using Ty = Tr<DT>;
   constexpr long long NONE = 0x7FFFFFFFFFFFFFFFll;
   if (threadIdx.x == 0) {
     // the piece's first pair settles both unless it holds NaN or Inf
-    const uint32_t ag = load_scalar<DT>(p.g, pb) & Ty::MAG, ac = load_scalar<DT>(p.c, pb) & Ty::MAG;
+    const uint32_t G0 = load_scalar<DT>(p.g, pb);
+    const uint32_t ag = G0 & Ty::MAG, ac = cand_at<DT, INJ>(p, pb, G0) & Ty::MAG;
     const bool fin = ag < Ty::INF && ac < Ty::INF;
     sm.ff = fin ? pb : NONE;
     sm.fu = fin ? pb : NONE;
@@ -1242,7 +1280,8 @@ __device__ __noinline__ void first_pairs(Smem& sm, const CompareParams& p, int64
     if (base >= pe || (sm.ff != NONE && sm.fu != NONE)) break;
     const int64_t i = base + threadIdx.x;
     if (i < pe) {
-      const uint32_t ag = load_scalar<DT>(p.g, i) & Ty::MAG, ac = load_scalar<DT>(p.c, i) & Ty::MAG;
+      const uint32_t Gi = load_scalar<DT>(p.g, i);
+      const uint32_t ag = Gi & Ty::MAG, ac = cand_at<DT, INJ>(p, i, Gi) & Ty::MAG;
       if (ag < Ty::INF && ac < Ty::INF) atomicMin(&sm.ff, (long long)i);
       if (ag <= Ty::INF && ac <= Ty::INF) atomicMin(&sm.fu, (long long)i);
     }
@@ -1281,7 +1320,7 @@ __device__ void write_empty_segments(const CompareParams& p);
 // End of one segment piece [pb, pe): the integer totals go to the segment's
 // accumulator (global atomics), the maxima to the CTA's partial slot.  The
 // CTA that finishes the segment's last piece then finalizes the segment.
-template <int DT>
+template <int DT, bool INJ>
 __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, const CompareParams& p,
                                              int64_t seg, int64_t pb, int64_t pe, int64_t vb, int64_t ve) {
   Partial* out = p.partials + seg + blockIdx.x;
@@ -1290,7 +1329,7 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
   // traffic) only when there is one
   __syncthreads();
   if (sm.gn != 0) {
-    run_general<DT>(W, sm, p, pb, pe, vb, ve);
+    run_general<DT, INJ>(W, sm, p, pb, pe, vb, ve);
   } else if ((threadIdx.x & 31) == 0) {
     part_none(sm.wbest[threadIdx.x >> 5]);
   }
@@ -1313,7 +1352,7 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
     }
     (&sm.sacc[0][0])[j] += v;
   }
-  first_pairs<DT>(sm, p, pb, pe);
+  first_pairs<DT, INJ>(sm, p, pb, pe);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t lo = sm.lo;
   // window pairs = unequal pairs - general pairs; EXACT = the piece length -
@@ -1345,7 +1384,8 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
     }
     if (r.ra > 0.0f) {
       const int64_t i = lo + r.ridx;
-      const float gf = to_f32<DT>(load_scalar<DT>(p.g, i)), cf = to_f32<DT>(load_scalar<DT>(p.c, i));
+      const uint32_t Gi = load_scalar<DT>(p.g, i);
+      const float gf = to_f32<DT>(Gi), cf = to_f32<DT>(cand_at<DT, INJ>(p, i, Gi));
       w.rel_hi = fabsf(__fsub_rn(cf, gf));
       w.rel_g = fabsf(gf);
       w.rel_idx = i;
@@ -1411,7 +1451,7 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
 // ---------------------------------------------------------------------------
 constexpr int CTAS_PER_SM = 2;
 
-template <int DT>
+template <int DT, bool INJ>
 __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(CompareParams p) {
   using Ty = Tr<DT>;
   using R = Rows<DT>;
@@ -1474,9 +1514,9 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
       const uint32_t bytes = (uint32_t)(min((int64_t)CHV, nvec - v0) * 16);
       const int64_t off = (vb + v0 * VEC) * Ty::BYTES;
       fence_proxy_async();
-      mbar_expect_tx(&sm.bar[warp][st], 2 * bytes);
+      mbar_expect_tx(&sm.bar[warp][st], INJ ? bytes : 2 * bytes);
       bulk_load(&sm.ring_g[warp][st][0], gbase + off, bytes, &sm.bar[warp][st]);
-      bulk_load(&sm.ring_c[warp][st][0], cbase + off, bytes, &sm.bar[warp][st]);
+      if (!INJ) bulk_load(&sm.ring_c[warp][st][0], cbase + off, bytes, &sm.bar[warp][st]);
     };
     const int64_t my_chunks = nchunk > warp ? (nchunk - warp + NW - 1) / NW : 0;
     if (lane == 0 && !failed)
@@ -1487,7 +1527,8 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
     __syncthreads();
     if (tid < nvec) {
       const uint4 gv = load_vec(p.g, (vb + (int64_t)tid * VEC) * Ty::BYTES);
-      const uint4 cv = load_vec(p.c, (vb + (int64_t)tid * VEC) * Ty::BYTES);
+      const uint4 cv = INJ ? inj_vec<DT>(p, gv, vb + (int64_t)tid * VEC)
+                           : load_vec(p.c, (vb + (int64_t)tid * VEC) * Ty::BYTES);
       uint32_t emax = 0, umax = 0;
 #pragma unroll
       for (int j = 0; j < VEC; j++) {
@@ -1516,8 +1557,10 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
     Thr T;
     thr_init(T);
     auto scalar_range = [&](int64_t b0, int64_t b1) {
-      for (int64_t i = b0 + tid; i < b1; i += BLOCK)
-        do_scalar<DT>(L, T, load_scalar<DT>(p.g, i), load_scalar<DT>(p.c, i), (uint32_t)(i - lo), W, sm);
+      for (int64_t i = b0 + tid; i < b1; i += BLOCK) {
+        const uint32_t G = load_scalar<DT>(p.g, i);
+        do_scalar<DT>(L, T, G, cand_at<DT, INJ>(p, i, G), (uint32_t)(i - lo), W, sm);
+      }
     };
     // scalar head: fewer than VEC elements, or the whole piece in scalar mode
     // (then in rounds of at most 65535 elements per thread)
@@ -1549,6 +1592,12 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
         if (!failed) {
           const int64_t v0 = k * CHV;
           const int nvalid = (int)min((int64_t)CHV, nvec - v0);
+          if constexpr (INJ) {
+            // the candidate tile, generated from the golden tile into the candidate ring
+            for (int v = lane; v < nvalid; v += 32)
+              sm.ring_c[warp][st][v] = inj_vec<DT>(p, sm.ring_g[warp][st][v], vb + (v0 + v) * VEC);
+            __syncwarp();
+          }
           do_tile<DT>(L, T, sm.ring_g[warp][st], nvalid, (uint32_t)(vb + v0 * VEC - lo), W, (uint32_t)i, sm);
           if (lane == 0 && i + NSTAGE < my_chunks) issue(seq + NSTAGE, warp + NW * (i + NSTAGE));
         }
@@ -1566,7 +1615,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
     }
     // scalar tail (fewer than VEC elements), after the body
     if (vb < ve && ve < pe) scalar_range(ve, pe);
-    finish_piece<DT>(L, W, sm, p, s, pb, pe, vb, ve);
+    finish_piece<DT, INJ>(L, W, sm, p, s, pb, pe, vb, ve);
     pb = pe;
   }
 }
@@ -1729,7 +1778,8 @@ __device__ __noinline__ void write_empty_segments(const CompareParams& p) {
 
 template <int DT>
 cudaError_t launch_t(const CompareParams& p, cudaStream_t st) {
-  compare_stage1<DT><<<p.nctas, BLOCK, sizeof(Smem), st>>>(p);
+  if (p.inj_n > 0) compare_stage1<DT, true><<<p.nctas, BLOCK, sizeof(Smem), st>>>(p);
+  else compare_stage1<DT, false><<<p.nctas, BLOCK, sizeof(Smem), st>>>(p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || p.nseg <= 1) return e;
   compare_finalize<<<(unsigned)p.nseg, BLOCK, 0, st>>>(p);
@@ -1788,13 +1838,18 @@ int64_t compare_cta_bound(int dtype, int64_t b, int nctas, int64_t n, int64_t p0
 }
 
 // once per device, before the first launch
+template <int DT, bool INJ>
+cudaError_t prepare_one() {
+  cudaError_t e =
+      cudaFuncSetAttribute(compare_stage1<DT, INJ>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(Smem));
+  if (e == cudaSuccess)  // as much shared memory as the SM offers: CTAS_PER_SM CTAs of sizeof(Smem) each
+    e = cudaFuncSetAttribute(compare_stage1<DT, INJ>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  return e;
+}
 template <int DT>
 cudaError_t prepare_t() {
-  cudaError_t e =
-      cudaFuncSetAttribute(compare_stage1<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(Smem));
-  if (e == cudaSuccess)  // as much shared memory as the SM offers: CTAS_PER_SM CTAs of sizeof(Smem) each
-    e = cudaFuncSetAttribute(compare_stage1<DT>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-  return e;
+  cudaError_t e = prepare_one<DT, false>();
+  return e == cudaSuccess ? prepare_one<DT, true>() : e;
 }
 
 cudaError_t compare_prepare() {

@@ -143,9 +143,16 @@ peat_status_t wait_staging(peat_handle_t h) {
   return PEAT_OK;
 }
 
+// element-wise models of a fused call, already validated
+struct InjSpec {
+  int n = 0;
+  uint64_t seed = 0;
+  peat::InjStep step[peat::INJ_MAX];
+};
+
 peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const int64_t* offsets,
                            int64_t nseg, peat_dtype_t dtype, peat_tol_t tol, peat_stats_t* stats,
-                           uint64_t* hist, peat_stream_t stream) {
+                           uint64_t* hist, peat_stream_t stream, const InjSpec* inj = nullptr) {
   if (!h) return PEAT_ERR_INVALID_ARG;
   int B = dtype_bytes(dtype);
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
@@ -160,7 +167,7 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   for (int64_t s = 0; s < nseg; s++)
     if (offsets[s + 1] < offsets[s]) return fail(h, PEAT_ERR_INVALID_ARG, "offsets must be non-decreasing");
   const int64_t n = offsets[nseg];
-  if (n > 0 && (!g || !c)) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
+  if (n > 0 && (!g || (!c && !inj))) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
   if (nseg > 0 && !stats) return fail(h, PEAT_ERR_INVALID_ARG, "stats_out is NULL");
   if (h->status_host && *(volatile unsigned int*)h->status_host) {
     *(volatile unsigned int*)h->status_host = 0;
@@ -178,6 +185,13 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   p.c = c;
   p.n_total = n;
   p.nseg = nseg;
+  if (inj) {  // the candidate is generated from the golden: align on the golden alone
+    p.inj_n = inj->n;
+    p.inj_k0 = (uint32_t)inj->seed;
+    p.inj_k1 = (uint32_t)(inj->seed >> 32);
+    for (int m = 0; m < inj->n; m++) p.inj[m] = inj->step[m];
+    c = g;
+  }
   uintptr_t ag = reinterpret_cast<uintptr_t>(g), ac = reinterpret_cast<uintptr_t>(c);
   if (n > 0 && ag % B == 0 && ac % B == 0 && ag % 16 == ac % 16)
     p.p0 = (int64_t)(((16 - ag % 16) % 16) / B);
@@ -676,6 +690,40 @@ peat_status_t peat_mean_std(const double* x, int64_t n, int ddof, double* mean_o
   const double ss = csum([x, mean](int64_t i) { return (x[i] - mean) * (x[i] - mean); });
   *std_out = std::sqrt(ss / (double)(n - ddof));
   return PEAT_OK;
+}
+
+peat_status_t peat_inject_compare(peat_handle_t h, const void* golden, int64_t n, peat_dtype_t dtype,
+                                  const peat_inject_t* models, int nmodels, uint64_t seed, peat_tol_t tol,
+                                  peat_stats_t* stats_out, uint64_t* hist_out, peat_stream_t stream) {
+  if (!h) return PEAT_ERR_INVALID_ARG;
+  if (!dtype_bytes(dtype)) return fail(h, PEAT_ERR_INVALID_ARG, "bad dtype");
+  if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
+  if (nmodels < 1 || nmodels > peat::INJ_MAX) return fail(h, PEAT_ERR_INVALID_ARG, "nmodels outside [1, 8]");
+  if (!models) return fail(h, PEAT_ERR_INVALID_ARG, "models is NULL");
+  InjSpec spec;
+  spec.n = nmodels;
+  spec.seed = seed;
+  for (int m = 0; m < nmodels; m++) {
+    const peat_inject_t& md = models[m];
+    if (md.kind < PEAT_INJ_RZ || md.kind > PEAT_INJ_CAST_BF16_RTZ) return fail(h, PEAT_ERR_INVALID_ARG, "bad model kind");
+    if (!peat::inj_elementwise(md.kind))
+      return fail(h, PEAT_ERR_UNSUPPORTED, "fixed-count models (RZ, RV, BITFLIP) cannot be fused: inject, then compare");
+    if (md.kind <= PEAT_INJ_SIGNFLIP) {
+      if (!(md.x >= 0.0 && md.x <= 1.0)) return fail(h, PEAT_ERR_INVALID_ARG, "rate outside [0, 1]");
+    } else if (md.kind <= PEAT_INJ_BIAS) {
+      if (!std::isfinite(md.x) || !std::isfinite((float)md.x)) return fail(h, PEAT_ERR_INVALID_ARG, "parameter not finite");
+    } else if (dtype != PEAT_F32) {
+      return fail(h, PEAT_ERR_INVALID_ARG, "cast models apply to float32 tensors only");
+    }
+    peat::InjStep& st = spec.step[m];
+    st.kind = md.kind;
+    st.model = (uint32_t)m;
+    const double t = std::floor(md.x * 4294967296.0);
+    st.threshold = (uint64_t)std::min(std::max(t, 0.0), 4294967296.0);
+    st.x = (float)md.x;
+  }
+  int64_t off[2] = {0, n};
+  return compare_impl(h, golden, nullptr, off, 1, dtype, tol, stats_out, hist_out, stream, &spec);
 }
 
 peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* src, int64_t n,

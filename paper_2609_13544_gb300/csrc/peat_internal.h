@@ -53,9 +53,30 @@ struct SegAcc {
   unsigned int pad;
 };
 
+// One element-wise pseudo-error model of a fused inject-and-compare call.
+constexpr int INJ_MAX = 8;
+struct InjStep {
+  int kind;            // PEAT_INJ_* (element-wise kinds only)
+  uint32_t model;      // its index in the caller's list (Philox counter word)
+  uint64_t threshold;  // Bernoulli threshold on a 32-bit word (rates)
+  float x;             // sigma, alpha or rate parameter in float32
+};
+
+// the element-wise model kinds (those a fused call can generate per element)
+inline bool inj_elementwise(int kind) {
+  return kind == PEAT_INJ_NAN_INF || kind == PEAT_INJ_SIGNFLIP || kind == PEAT_INJ_REL_GAUSS ||
+         kind == PEAT_INJ_ADD_GAUSS || kind == PEAT_INJ_BIAS || kind == PEAT_INJ_CAST_F16_RNE ||
+         kind == PEAT_INJ_CAST_F16_RTZ || kind == PEAT_INJ_CAST_BF16_RNE || kind == PEAT_INJ_CAST_BF16_RTZ;
+}
+
 struct CompareParams {
   const void* g;
-  const void* c;
+  const void* c;           // unused when inj_n > 0
+  // fused injection: the candidate is the golden after inj[0..inj_n) applied
+  // in order, generated in the tiles and never stored (inj_n = 0: c is read)
+  int inj_n;
+  uint32_t inj_k0, inj_k1;  // the seed
+  InjStep inj[INJ_MAX];
   int64_t n_total;
   const int64_t* offsets;  // device copy, nseg + 1 entries
   const int64_t* bounds;   // device copy, nctas + 1 CTA range boundaries

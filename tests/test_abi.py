@@ -15,7 +15,7 @@ def declared_functions():
 
 def test_header_declares_the_boundary():
     assert declared_functions() == sorted([
-        "peat_compare", "peat_compare_noalloc", "peat_compare_segmented", "peat_last_error",
+        "peat_compare", "peat_compare_noalloc", "peat_compare_segmented", "peat_inject_compare", "peat_last_error",
         "peat_isclose_grid", "peat_mean_std", "peat_pseudo_error_inject", "peat_signature_create",
         "peat_signature_destroy",
         "peat_spearman", "peat_tensor_stats", "peat_topk_mean"])

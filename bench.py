@@ -50,7 +50,7 @@ def measured_peaks() -> dict:
 
 def kernel_source_sha() -> str:
     h = hashlib.sha256()
-    for f in ("compare.cu", "exact.cuh", "peat_internal.h"):
+    for f in ("compare.cu", "exact.cuh", "inject_models.cuh", "peat_internal.h"):
         h.update((ROOT / "paper_2609_13544_gb300" / "csrc" / f).read_bytes())
     return h.hexdigest()[:16]
 
@@ -371,6 +371,48 @@ def run_gpu(args) -> None:
                             "algorithmic_bytes_per_call": bytes_per_step,
                             "note": "one read of both tensors; 64 exact tolerance decisions per differing pair"}}
 
+    # fused inject + compare (Alg. 1's Inject and Compare in one read of the golden): the
+    # candidate g (1 + 1e-3 z) generated in the kernel, against the injector writing it
+    # followed by the compare reading both
+    fused = None
+    if w.offsets is None and not args.no_topk:
+        scratch = torch.empty_like(g)
+        cnt = torch.zeros(1, dtype=torch.int64, device=dev)
+        fu_calls = max(3, min(100, args.steps // 50))
+
+        def timed(fn):
+            for _ in range(3):
+                fn()
+            barrier()
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record(stream)
+            for _ in range(fu_calls):
+                fn()
+            t1.record(stream)
+            barrier()
+            return max_over_ranks(t0.elapsed_time(t1), dev) / fu_calls
+
+        per_model = {}
+        for name, x in (("rel_gauss", 1e-3), ("bias", 1e-3)):
+            models = [peat.inject_model(name, x=x)]
+            ms_inj = timed(lambda: peat.peat_pseudo_error_inject_raw(h, scratch, g, models, 9, cnt, stream))
+            ms_cmp = timed(lambda: peat.peat_compare_raw(h, g, scratch, w.rtol, w.atol, stats, hist, stream))
+            ms_fu = timed(lambda: peat.peat_inject_compare_raw(h, g, models, 9, w.rtol, w.atol, stats, hist, stream))
+            per_model[f"{name} {x:g}"] = {"fused_us": ms_fu * 1e3, "inject_us": ms_inj * 1e3,
+                                          "compare_us": ms_cmp * 1e3, "speedup": (ms_inj + ms_cmp) / ms_fu}
+        head = per_model["rel_gauss 0.001"]
+        one = bytes_per_step // 2
+        fu_gbs = one / (head["fused_us"] * 1e-6) / 1e9
+        fused = {"op": "peat_inject_compare on the golden, against peat_pseudo_error_inject into a scratch "
+                       "tensor followed by peat_compare", "calls": fu_calls,
+                 "us_per_call": head["fused_us"], "pairs_per_s": w.n / (head["fused_us"] * 1e-6),
+                 "per_model": per_model,
+                 "roofline": {"bound": "alu", "achieved": fu_gbs, "peak": peak, "unit": "GB/s",
+                              "frac": fu_gbs / peak, "algorithmic_bytes_per_call": one,
+                              "note": "rel_gauss: one read of the golden; per four elements one Philox4x32-10 "
+                                      "draw and two Box-Muller pairs, then the compare"}}
+        del scratch
+
     # end to end through the C ABI with host buffers: every step copies both
     # tensors from pinned host memory, compares them and reads the stats and
     # histograms back.  Two device buffer sets: step i's copies (copy stream)
@@ -458,7 +500,8 @@ def run_gpu(args) -> None:
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy)" if not peaks.get("fallback")
                          else "fallback 6.8 TB/s"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": (1 if nseg == 1 else 2) * args.steps, "clocks": clocks,
-            "next_rows": {"f1_top10_mean": topk, "f3_context_stats": tstats, "f4_isclose_grid": isc},
+            "next_rows": {"f1_top10_mean": topk, "f2_fused_inject_compare": fused, "f3_context_stats": tstats,
+                          "f4_isclose_grid": isc},
             "wall_s_timed": wall,
         }
         print(json.dumps(line), flush=True)
@@ -477,7 +520,8 @@ def main():
     ap.add_argument("--impl", default="peat", choices=["peat", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-topk", action="store_true",
-                    help="skip the timings of the next rows (top-10 %% mean, context statistics)")
+                    help="skip the timings of the next rows (top-10 %% mean, fused inject + compare, "
+                         "context statistics, isclose grid)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

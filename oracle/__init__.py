@@ -110,8 +110,10 @@ def lib() -> ctypes.CDLL:
         L.orc_inject.restype = i32
         L.orc_philox4x32_10.argtypes = [vp, vp, vp]
         L.orc_philox4x32_10.restype = None
-        L.orc_normal_from_words.argtypes = [ctypes.c_uint32, ctypes.c_uint32]
-        L.orc_normal_from_words.restype = ctypes.c_float
+        L.orc_normal_pair_from_words.argtypes = [ctypes.c_uint32, ctypes.c_uint32, vp]
+        L.orc_normal_pair_from_words.restype = None
+        L.orc_sin2pi.argtypes = [ctypes.c_float]
+        L.orc_sin2pi.restype = ctypes.c_float
         L.orc_logf.argtypes = [ctypes.c_float]
         L.orc_logf.restype = ctypes.c_float
         L.orc_cos2pi.argtypes = [ctypes.c_float]
@@ -335,8 +337,11 @@ def philox(ctr: Sequence[int], key: Sequence[int]) -> list:
     return [int(v) for v in out]
 
 
-def normal_from_words(w0: int, w1: int) -> float:
-    return float(lib().orc_normal_from_words(w0, w1))
+def normal_pair_from_words(w0: int, w1: int) -> tuple:
+    """The Box-Muller pair (r cos 2 pi u2, r sin 2 pi u2) of two Philox words."""
+    z = np.zeros(2, np.float32)
+    lib().orc_normal_pair_from_words(w0, w1, z.ctypes.data)
+    return float(z[0]), float(z[1])
 
 
 def logf(x: float) -> float:
@@ -345,3 +350,7 @@ def logf(x: float) -> float:
 
 def cos2pi(u: float) -> float:
     return float(lib().orc_cos2pi(u))
+
+
+def sin2pi(u: float) -> float:
+    return float(lib().orc_sin2pi(u))

@@ -640,6 +640,7 @@ int orc_tensor_stats(const void* x, int64_t n, int dtype, orc_tstats* out) {
 #define PHILOX_W1 0xBB67AE85u
 #define TAG_ELEM 0x454C454Du /* per-element draws */
 #define TAG_POS 0x504F5331u  /* position draws of the fixed-count models */
+#define TAG_CLASS 0x434C5353u /* NaN/Inf class of a fired element */
 
 void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]) {
   uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
@@ -712,9 +713,11 @@ float orc_logf(float x) {
   return fmaf(ef, LN2_HI, fmaf(ef, LN2_LO, lm));
 }
 
-/* cos(2*pi*u) for u in [0, 1): quadrant reduction on u (exact), then the
- * Taylor series of cos and sin on |x| <= pi/4. */
-float orc_cos2pi(float u) {
+/* cos(2*pi*u) and sin(2*pi*u) for u in [0, 1): quadrant reduction on u
+ * (exact: u = q/4 + r), then the Taylor series of cos and sin of x = 2 pi r,
+ * |x| <= pi/4, and the quadrant's signs and swap:
+ * cos(x + q pi/2), sin(x + q pi/2) for q = 0..3. */
+static void sincos2pi(float u, float* s_out, float* c_out) {
   const float TWO_PI = 0x1.921fb6p+2f;
   const float I2 = 0x1p-1f, I4 = 0x1.555556p-5f, I6 = 0x1.6c16c2p-10f, I8 = 0x1.a01a02p-16f,
               I10 = 0x1.27e4fcp-22f;
@@ -733,21 +736,38 @@ float orc_cos2pi(float u) {
   sp = fmaf(x2, sp, -I3);
   float x3 = x * x2;
   float sinx = fmaf(x3, sp, x);
-  int j = (int)q & 3;
-  if (j == 0) return cosx;
-  if (j == 1) return -sinx;
-  if (j == 2) return -cosx;
-  return sinx;
+  switch ((int)q & 3) {
+    case 0: *c_out = cosx; *s_out = sinx; break;
+    case 1: *c_out = -sinx; *s_out = cosx; break;
+    case 2: *c_out = -cosx; *s_out = -sinx; break;
+    default: *c_out = sinx; *s_out = -cosx; break;
+  }
 }
 
-/* Box-Muller: z = sqrt(-2 ln u1) cos(2 pi u2), u1 in (0, 1], u2 in [0, 1),
- * each from the top 24 bits of a Philox word. */
-float orc_normal_from_words(uint32_t w0, uint32_t w1) {
+float orc_cos2pi(float u) {
+  float s, c;
+  sincos2pi(u, &s, &c);
+  return c;
+}
+
+float orc_sin2pi(float u) {
+  float s, c;
+  sincos2pi(u, &s, &c);
+  return s;
+}
+
+/* Box-Muller: from u1 in (0, 1] and u2 in [0, 1), each the top 24 bits of a
+ * Philox word, the two independent normals r cos(2 pi u2) and
+ * r sin(2 pi u2), r = sqrt(-2 ln u1). */
+void orc_normal_pair_from_words(uint32_t w0, uint32_t w1, float z[2]) {
   float u1 = (float)((w0 >> 8) + 1u) * 0x1p-24f;
   float u2 = (float)(w1 >> 8) * 0x1p-24f;
   float l = orc_logf(u1);
   float r = sqrtf(-2.0f * l);
-  return r * orc_cos2pi(u2);
+  float s, c;
+  sincos2pi(u2, &s, &c);
+  z[0] = r * c;
+  z[1] = r * s;
 }
 
 /* float32 -> binary16 bit pattern, round to nearest even or toward zero */
@@ -879,17 +899,23 @@ int orc_inject(void* dst, const void* src, int64_t n, int dtype, const orc_injec
       uint64_t thr = bernoulli_threshold(md->x);
       float x32 = (float)md->x;
       for (int64_t i = 0; i < n; i++) {
+        /* one draw serves the block of four elements 4d .. 4d+3: element i
+         * takes word i mod 4, or the normal its word pair gives (r cos for
+         * the first element of the pair, r sin for the second) */
         uint32_t w[4];
-        draw(seed, (uint64_t)i, (uint32_t)m, TAG_ELEM, w);
+        draw(seed, (uint64_t)i >> 2, (uint32_t)m, TAG_ELEM, w);
+        int j = (int)(i & 3);
         uint32_t b = raw_bits(dst, i, dtype);
         if (md->kind == ORC_INJ_NAN_INF || md->kind == ORC_INJ_SIGNFLIP) {
-          if ((uint64_t)w[0] >= thr) continue;
+          if ((uint64_t)w[j] >= thr) continue;
           fired++;
           uint32_t nb;
           if (md->kind == ORC_INJ_SIGNFLIP) {
             nb = b ^ (dtype == ORC_F32 ? 0x80000000u : 0x8000u);
           } else {
-            uint32_t sel = w[1] >> 30; /* 0,1: NaN; 2: +Inf; 3: -Inf */
+            uint32_t cw[4];
+            draw(seed, (uint64_t)i, (uint32_t)m, TAG_CLASS, cw);
+            uint32_t sel = cw[0] >> 30; /* 0,1: NaN; 2: +Inf; 3: -Inf */
             if (dtype == ORC_F32)
               nb = sel < 2 ? 0x7FC00000u : (sel == 2 ? 0x7F800000u : 0xFF800000u);
             else if (dtype == ORC_F16)
@@ -909,12 +935,14 @@ int orc_inject(void* dst, const void* src, int64_t n, int dtype, const orc_injec
         fired++;
         float x = load_f32(dst, i, dtype);
         float y;
+        float zp[2] = {0.0f, 0.0f};
+        if (md->kind == ORC_INJ_REL_GAUSS || md->kind == ORC_INJ_ADD_GAUSS)
+          orc_normal_pair_from_words(w[j & 2], w[(j & 2) + 1], zp);
+        float z = zp[j & 1];
         if (md->kind == ORC_INJ_REL_GAUSS) {
-          float z = orc_normal_from_words(w[0], w[1]);
           float scale = fmaf(x32, z, 1.0f); /* RN32(1 + sigma*z) */
           y = x * scale;
         } else if (md->kind == ORC_INJ_ADD_GAUSS) {
-          float z = orc_normal_from_words(w[0], w[1]);
           y = fmaf(x32, z, x); /* RN32(x + sigma*z) */
         } else if (md->kind == ORC_INJ_BIAS) {
           y = fmaf(x32, fabsf(x), x); /* RN32(x + alpha*|x|) */

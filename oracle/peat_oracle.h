@@ -132,9 +132,10 @@ int orc_inject(void* dst, const void* src, int64_t n, int dtype, const orc_injec
 
 /* Building blocks exposed for their own pins. */
 void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]);
-float orc_normal_from_words(uint32_t w0, uint32_t w1);
+void orc_normal_pair_from_words(uint32_t w0, uint32_t w1, float z[2]);
 float orc_logf(float x);
 float orc_cos2pi(float u);
+float orc_sin2pi(float u);
 
 #ifdef __cplusplus
 }

@@ -185,6 +185,12 @@ def _stream_ptr(stream) -> Optional[int]:
     return stream.cuda_stream
 
 
+def _sync(stream) -> None:
+    """The dict wrappers read their outputs back: wait for the stream the call ran on."""
+    if stream is not None:
+        stream.synchronize()
+
+
 def _dev_tensor_check(*ts):
     for t in ts:
         if not t.is_cuda:
@@ -251,6 +257,7 @@ def peat_compare(h: Handle, golden, candidate, rtol: float, atol: float = 0.0, s
     stats = torch.empty(STATS_BYTES, dtype=torch.uint8, device=dev)
     hist = torch.empty(HIST_BINS, dtype=torch.int64, device=dev)
     peat_compare_raw(h, golden, candidate, rtol, atol, stats, hist, stream)
+    _sync(stream)
     s = stats_to_dicts(stats.cpu().numpy())[0]
     return s, hist.cpu().numpy().view(np.uint64).reshape(2, 64)
 
@@ -263,6 +270,7 @@ def peat_compare_noalloc(golden, candidate, rtol: float, atol: float = 0.0, stre
     stats = torch.empty(STATS_BYTES, dtype=torch.uint8, device=dev)
     hist = torch.empty(HIST_BINS, dtype=torch.int64, device=dev)
     peat_compare_noalloc_raw(golden, candidate, rtol, atol, stats, hist, stream)
+    _sync(stream)
     s = stats_to_dicts(stats.cpu().numpy())[0]
     return s, hist.cpu().numpy().view(np.uint64).reshape(2, 64)
 
@@ -276,6 +284,7 @@ def peat_compare_segmented(h: Handle, golden, candidate, offsets: Sequence[int],
     stats = torch.empty(max(nseg, 1) * STATS_BYTES, dtype=torch.uint8, device=dev)
     hist = torch.empty(max(nseg, 1) * HIST_BINS, dtype=torch.int64, device=dev)
     peat_compare_segmented_raw(h, golden, candidate, offsets, rtol, atol, stats, hist, stream)
+    _sync(stream)
     if nseg == 0:
         return [], np.zeros((0, 2, 64), np.uint64)
     s = stats_to_dicts(stats.cpu().numpy()[: nseg * STATS_BYTES])
@@ -298,6 +307,7 @@ def peat_topk_mean(h: Handle, golden, candidate, num: int = 1, den: int = 10, st
     import torch
     out = torch.empty(TOPK_BYTES, dtype=torch.uint8, device=golden.device)
     peat_topk_mean_raw(h, golden, candidate, num, den, out, stream)
+    _sync(stream)
     r = np.frombuffer(out.cpu().numpy().tobytes(), dtype=TOPK_DTYPE)[0]
     return {k: r[k].item() for k in TOPK_DTYPE.names if k != "reserved"}
 
@@ -320,6 +330,7 @@ def peat_tensor_stats(h: Handle, x, offsets: Optional[Sequence[int]] = None, str
     nseg = len(off) - 1
     out = torch.empty(max(nseg, 1) * TSTATS_BYTES, dtype=torch.uint8, device=x.device)
     peat_tensor_stats_raw(h, x, off, out, stream)
+    _sync(stream)
     arr = np.frombuffer(out.cpu().numpy()[: nseg * TSTATS_BYTES].tobytes(), dtype=TSTATS_DTYPE)
     res = [{k: r[k].item() for k in TSTATS_DTYPE.names} for r in arr]
     return res[0] if offsets is None else res
@@ -342,6 +353,7 @@ def peat_isclose_grid(h: Handle, golden, candidate, rtols, atols, stream=None) -
     import torch
     out = torch.empty(len(rtols) * len(atols), dtype=torch.int64, device=golden.device)
     peat_isclose_grid_raw(h, golden, candidate, rtols, atols, out, stream)
+    _sync(stream)
     return out.cpu().numpy().view(np.uint64).reshape(len(rtols), len(atols))
 
 
@@ -375,6 +387,18 @@ def inject_model(kind: str, k: int = 0, bit_lo: int = 0, bit_hi: int = 0, x: flo
     return {"kind": kind, "k": k, "bit_lo": bit_lo, "bit_hi": bit_hi, "x": x}
 
 
+def peat_pseudo_error_inject_raw(h: Handle, dst, src, models: Sequence[dict], seed: int, counts_out,
+                                 stream=None) -> None:
+    """peat_pseudo_error_inject on preallocated device tensors (counts_out: int64[len(models)])."""
+    _dev_tensor_check(dst, src)
+    if dst.numel() != src.numel() or dst.dtype != src.dtype:
+        raise ValueError("dst and src differ in size or dtype")
+    rc = load().peat_pseudo_error_inject(h.ptr, dst.data_ptr(), src.data_ptr(), src.numel(), dtype_code(src),
+                                         _model_array(models), len(models), ctypes.c_uint64(seed),
+                                         counts_out.data_ptr(), _stream_ptr(stream))
+    _check(rc, h)
+
+
 def peat_pseudo_error_inject(h: Handle, src, models: Sequence[dict], seed: int, dst=None, stream=None):
     """Apply error models to src on the GPU; returns (dst tensor, counts numpy uint64)."""
     import torch
@@ -387,6 +411,7 @@ def peat_pseudo_error_inject(h: Handle, src, models: Sequence[dict], seed: int, 
                                          len(models), ctypes.c_uint64(seed), counts.data_ptr(),
                                          _stream_ptr(stream))
     _check(rc, h)
+    _sync(stream)
     return dst, counts[: len(models)].cpu().numpy().view(np.uint64)
 
 
@@ -418,6 +443,7 @@ def peat_inject_compare(h: Handle, golden, models: Sequence[dict], seed: int, rt
     stats = torch.empty(STATS_BYTES, dtype=torch.uint8, device=dev)
     hist = torch.empty(HIST_BINS, dtype=torch.int64, device=dev)
     peat_inject_compare_raw(h, golden, models, seed, rtol, atol, stats, hist, stream)
+    _sync(stream)
     s = stats_to_dicts(stats.cpu().numpy())[0]
     return s, hist.cpu().numpy().view(np.uint64).reshape(2, 64)
 

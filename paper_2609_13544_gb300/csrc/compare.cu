@@ -115,8 +115,10 @@ __device__ __forceinline__ uint32_t load_scalar(const void* base, int64_t i) {
 
 // The candidate of a fused call: the golden after the call's element-wise
 // models, in order (the same arithmetic as the injector's passes).
+// (out of line: the scalar paths that call it are rare, and one copy keeps
+// the generation code out of their inlined bodies)
 template <int DT>
-__device__ __forceinline__ uint32_t inj_chain(const CompareParams& p, uint32_t b, int64_t i) {
+__device__ __noinline__ uint32_t inj_chain(const CompareParams& p, uint32_t b, int64_t i) {
   for (int m = 0; m < p.inj_n; m++) {
     bool fired;
     b = inj::apply_model<DT>(b, i, p.inj[m].kind, p.inj[m].model, p.inj[m].threshold, p.inj[m].x, p.inj_k0,
@@ -130,22 +132,72 @@ __device__ __forceinline__ uint32_t cand_at(const CompareParams& p, int64_t i, u
   if constexpr (INJ) return inj_chain<DT>(p, G, i);
   else return load_scalar<DT>(p.c, i);
 }
-// the candidate vector of golden vector gv whose first element is i0
+template <int DT>
+__device__ __forceinline__ void unpack_vec(const uint4& v, uint32_t (&e)[16 / Tr<DT>::BYTES]) {
+#pragma unroll
+  for (int j = 0; j < 16 / Tr<DT>::BYTES; j++) e[j] = lane_bits<DT>(v, j);
+}
+template <int DT>
+__device__ __forceinline__ uint4 pack_vec(const uint32_t (&e)[16 / Tr<DT>::BYTES]) {
+  if constexpr (Tr<DT>::BYTES == 4) return make_uint4(e[0], e[1], e[2], e[3]);
+  else
+    return make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16), e[6] | (e[7] << 16));
+}
+
+// the candidate vector of golden vector gv whose first element is i0: whole
+// blocks of four (one draw each) when i0 is on the block grid, else element
+// by element
 template <int DT>
 __device__ __forceinline__ uint4 inj_vec(const CompareParams& p, const uint4& gv, int64_t i0) {
-  uint32_t w[4] = {gv.x, gv.y, gv.z, gv.w};
-  if constexpr (Tr<DT>::BYTES == 4) {
-#pragma unroll
-    for (int j = 0; j < 4; j++) w[j] = inj_chain<DT>(p, w[j], i0 + j);
+  constexpr int VEC = 16 / Tr<DT>::BYTES, NB = VEC / 4;
+  uint32_t e[VEC];
+  unpack_vec<DT>(gv, e);
+  if ((i0 & 3) == 0) {
+    for (int m = 0; m < p.inj_n; m++) {
+      const InjStep st = p.inj[m];
+      inj::with_kind(st.kind, [&](auto k) {
+        inj::apply_blocks<DT, decltype(k)::value, NB>(e, i0, st.model, st.threshold, st.x, p.inj_k0, p.inj_k1);
+      });
+    }
   } else {
 #pragma unroll
-    for (int k = 0; k < 4; k++) {
-      const uint32_t lo = inj_chain<DT>(p, w[k] & 0xFFFFu, i0 + 2 * k);
-      const uint32_t hi = inj_chain<DT>(p, w[k] >> 16, i0 + 2 * k + 1);
-      w[k] = (lo & 0xFFFFu) | (hi << 16);
-    }
+    for (int j = 0; j < VEC; j++) e[j] = inj_chain<DT>(p, e[j], i0 + j);
   }
-  return make_uint4(w[0], w[1], w[2], w[3]);
+  return pack_vec<DT>(e);
+}
+
+// The candidate chunk of a fused call, ct[v] for golden gt[v], v = lane,
+// lane + 32, ... < nvalid, vector v starting at element i0 + v VEC: model by
+// model over the chunk (one branch on the kind per model, then code without
+// branches), each lane rewriting its own vectors in place.  Out of line,
+// called once per chunk.
+template <int DT>
+__device__ __noinline__ void inj_chunk(const CompareParams& p, const uint4* gt, uint4* ct, int nvalid, int64_t i0) {
+  constexpr int VEC = 16 / Tr<DT>::BYTES, NB = VEC / 4;
+  const int lane = threadIdx.x & 31;
+  if ((i0 & 3) != 0) {  // off the block grid
+    for (int v = lane; v < nvalid; v += 32) ct[v] = inj_vec<DT>(p, gt[v], i0 + (int64_t)v * VEC);
+    return;
+  }
+  for (int m = 0; m < p.inj_n; m++) {
+    const InjStep st = p.inj[m];
+    const uint4* src = m == 0 ? gt : ct;
+    inj::with_kind(st.kind, [&](auto k) {
+      for (int v = lane; v < nvalid; v += 32) {
+        uint32_t e[VEC];
+        unpack_vec<DT>(src[v], e);
+        inj::apply_blocks<DT, decltype(k)::value, NB>(e, i0 + (int64_t)v * VEC, st.model, st.threshold, st.x,
+                                                       p.inj_k0, p.inj_k1);
+        ct[v] = pack_vec<DT>(e);
+      }
+    });
+  }
+}
+
+// one candidate vector, out of line (the window sample of a piece)
+template <int DT>
+__device__ __noinline__ uint4 inj_one(const CompareParams& p, uint4 gv, int64_t i0) {
+  return inj_vec<DT>(p, gv, i0);
 }
 
 __device__ __forceinline__ uint4 load_vec(const void* base, int64_t byte_off) {
@@ -1527,7 +1579,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
     __syncthreads();
     if (tid < nvec) {
       const uint4 gv = load_vec(p.g, (vb + (int64_t)tid * VEC) * Ty::BYTES);
-      const uint4 cv = INJ ? inj_vec<DT>(p, gv, vb + (int64_t)tid * VEC)
+      const uint4 cv = INJ ? inj_one<DT>(p, gv, vb + (int64_t)tid * VEC)
                            : load_vec(p.c, (vb + (int64_t)tid * VEC) * Ty::BYTES);
       uint32_t emax = 0, umax = 0;
 #pragma unroll
@@ -1594,8 +1646,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
           const int nvalid = (int)min((int64_t)CHV, nvec - v0);
           if constexpr (INJ) {
             // the candidate tile, generated from the golden tile into the candidate ring
-            for (int v = lane; v < nvalid; v += 32)
-              sm.ring_c[warp][st][v] = inj_vec<DT>(p, sm.ring_g[warp][st][v], vb + (v0 + v) * VEC);
+            inj_chunk<DT>(p, sm.ring_g[warp][st], sm.ring_c[warp][st], nvalid, vb + v0 * VEC);
             __syncwarp();
           }
           do_tile<DT>(L, T, sm.ring_g[warp][st], nvalid, (uint32_t)(vb + v0 * VEC - lo), W, (uint32_t)i, sm);

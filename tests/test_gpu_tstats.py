@@ -126,3 +126,30 @@ def test_workload_c2_full_against_torch(peat_gpu, h):
     assert math.isclose(r["sum_sq"], float((x * x).sum()), rel_tol=1e-12)
     assert math.isclose(r["var"], float(x.var(unbiased=False)), rel_tol=1e-10)
     assert r["min"] == float(x.min()) and r["max"] == float(x.max())
+
+
+def test_one_tensor_bounds_reused_across_calls(peat_gpu, oracle, h):
+    """One-tensor calls keep their CTA bounds on the device and rewrite them
+    only when the size, alignment, CTA count or stream changes: interleave
+    compares and statistics (different CTA counts for the same n), a second
+    stream and a misaligned view on one handle."""
+    from parity_util import assert_hist_equal, assert_stats_equal
+    n = 300_007
+    gb, cb = noise_pairs("bf16", n, seed=91)
+    g, c = to_device(gb, "bf16"), to_device(cb, "bf16")
+    ost, ohist = oracle.compare(gb, cb, "bf16", 1e-3, 0.0)
+    ots = oracle.tensor_stats(gb, "bf16")
+    side = torch.cuda.Stream()
+    for rep in range(2):
+        st, hist = peat_gpu.peat_compare(h, g, c, 1e-3)
+        assert_stats_equal(st, ost, f"compare {rep}")
+        assert_hist_equal(hist, ohist, f"compare {rep}")
+        check_one(peat_gpu.peat_tensor_stats(h, g), ots, f"stats {rep}")
+        st, hist = peat_gpu.peat_compare(h, g, c, 1e-3, stream=side)
+        side.synchronize()
+        assert_stats_equal(st, ost, f"side stream {rep}")
+        st, hist = peat_gpu.peat_compare(h, to_device(gb, "bf16", 3), to_device(cb, "bf16", 3), 1e-3)
+        assert_stats_equal(st, ost, f"misaligned {rep}")
+        st, hist = peat_gpu.peat_compare(h, g[:n - 5], c[:n - 5], 1e-3)
+        o5, _ = oracle.compare(gb[:n - 5], cb[:n - 5], "bf16", 1e-3, 0.0)
+        assert_stats_equal(st, o5, f"shorter {rep}")

@@ -416,17 +416,63 @@ def test_logf_and_cos2pi_against_libm(oracle):
         assert abs(oracle.logf(x32) - ref) <= 3e-7 * max(1.0, abs(ref)), x32
     for u in np.arange(0, 1 << 24, 3001) * 2.0 ** -24:
         assert abs(oracle.cos2pi(float(u)) - math.cos(2 * math.pi * u)) < 4e-7, u
+        assert abs(oracle.sin2pi(float(u)) - math.sin(2 * math.pi * u)) < 4e-7, u
+    # the quadrant boundaries, where the reduction swaps cos and sin
+    for u, c, s_ in ((0.0, 1.0, 0.0), (0.25, 0.0, 1.0), (0.5, -1.0, 0.0), (0.75, 0.0, -1.0)):
+        assert abs(oracle.cos2pi(u) - c) < 1e-7 and abs(oracle.sin2pi(u) - s_) < 1e-7, u
 
 
-def test_box_muller_moments(oracle):
+def test_box_muller_pair_moments(oracle):
+    """Both components of a Box-Muller pair are N(0, 1) and independent: the
+    squared radius z0^2 + z1^2 is exponential with mean 2 (P(> 2) = 1/e)."""
     n = 100000
     w = [oracle.philox([i, 0, 7, 1], [5, 0]) for i in range(n)]
-    z = np.array([oracle.normal_from_words(a[0], a[1]) for a in w])
-    assert abs(z.mean()) < 5 / math.sqrt(n)
-    assert abs(z.var() - 1) < 5 * math.sqrt(2 / n)
-    kurt = ((z - z.mean()) ** 4).mean() / z.var() ** 2
-    assert abs(kurt - 3) < 5 * math.sqrt(24 / n)
-    assert abs((np.abs(z) < 1).mean() - 0.6826894921) < 5 * math.sqrt(0.22 / n)
+    zz = np.array([oracle.normal_pair_from_words(a[0], a[1]) for a in w])
+    for z in (zz[:, 0], zz[:, 1]):
+        assert abs(z.mean()) < 5 / math.sqrt(n)
+        assert abs(z.var() - 1) < 5 * math.sqrt(2 / n)
+        kurt = ((z - z.mean()) ** 4).mean() / z.var() ** 2
+        assert abs(kurt - 3) < 5 * math.sqrt(24 / n)
+        assert abs((np.abs(z) < 1).mean() - 0.6826894921) < 5 * math.sqrt(0.22 / n)
+    r2 = zz[:, 0].astype(np.float64) ** 2 + zz[:, 1].astype(np.float64) ** 2
+    assert abs(r2.mean() - 2) < 5 * 2 / math.sqrt(n)
+    assert abs((r2 > 2).mean() - math.exp(-1)) < 5 * math.sqrt(0.24 / n)
+    assert abs(np.corrcoef(zz[:, 0], zz[:, 1])[0, 1]) < 5 / math.sqrt(n)
+    assert abs(np.corrcoef(zz[:, 0] ** 2, zz[:, 1] ** 2)[0, 1]) < 5 / math.sqrt(n)
+
+
+def test_inject_draw_blocks_are_independent(oracle):
+    """One draw serves four neighbouring elements: every position in the
+    block still fires at the model's rate, independently of its neighbours,
+    and the noise of neighbours is independent N(0, 1) (the Box-Muller pair
+    of positions 2k, 2k+1 has squared radius of mean 2, P(> 2) = 1/e)."""
+    n = 400000
+    src = np.full(n, 1.0, np.float32)
+    rate = 0.1
+    dst, cnt = oracle.inject(src, "f32", [oracle.model("signflip", x=rate)], seed=3)
+    f = (dst != src.view(np.uint32)).reshape(-1, 4)
+    for j in range(4):
+        assert abs(f[:, j].mean() - rate) < 5 * math.sqrt(rate * (1 - rate) / (n // 4)), j
+    for a, b in ((0, 1), (1, 2), (2, 3), (0, 3)):
+        both = (f[:, a] & f[:, b]).mean()
+        assert abs(both - rate * rate) < 5 * math.sqrt(rate * rate / (n // 4)), (a, b)
+    # NaN / +Inf / -Inf in the shares 1/2, 1/4, 1/4
+    dst, cnt = oracle.inject(src, "f32", [oracle.model("nan_inf", x=0.05)], seed=4)
+    v = dst.view(np.float32)
+    k = int(cnt[0])
+    for share, hit in ((0.5, np.isnan(v)), (0.25, v == np.inf), (0.25, v == -np.inf)):
+        assert abs(hit.sum() / k - share) < 5 * math.sqrt(share * (1 - share) / k)
+    sigma = 2.0 ** -10
+    dst, _ = oracle.inject(src, "f32", [oracle.model("add_gauss", x=sigma)], seed=5)
+    e = ((dst.view(np.float32).astype(np.float64) - 1.0) / sigma).reshape(-1, 4)
+    for j in range(4):
+        assert abs(e[:, j].mean()) < 5 / math.sqrt(n // 4) and abs(e[:, j].var() - 1) < 0.03, j
+    for a, b in ((0, 1), (2, 3)):
+        r2 = e[:, a] ** 2 + e[:, b] ** 2
+        assert abs(r2.mean() - 2) < 0.06 and abs((r2 > 2).mean() - math.exp(-1)) < 0.01
+    for a, b in ((0, 1), (1, 2), (0, 2), (2, 3)):
+        assert abs(np.corrcoef(e[:, a], e[:, b])[0, 1]) < 0.01, (a, b)
+        assert abs(np.corrcoef(e[:, a] ** 2, e[:, b] ** 2)[0, 1]) < 0.015, (a, b)
 
 
 def test_inject_fixed_count_models(oracle):

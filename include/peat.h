@@ -283,8 +283,9 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
  *                      rtols non-decreasing after the rounding.
  *   nr, na             1 <= nr, na and nr * na <= 64.
  *   counts_out         device pointer to nr * na uint64 (overwritten).
- * About 4 nr na + 10 na log2(nr) operations per differing pair (bitwise-equal
- * warp slots cost a vote).  Asynchronous on `stream`.
+ * About 15 na log2(nr) operations per differing pair (a binary search per
+ * atol, bounded by the previous atol's result; bitwise-equal warp slots cost
+ * a vote).  Asynchronous on `stream`.
  * Errors: INVALID_ARG (bad dtype, pointers, tolerances or grid size), CUDA. */
 peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void* candidate, int64_t n,
                                 peat_dtype_t dtype, const double* rtols, int nr, const double* atols, int na,

@@ -5,12 +5,16 @@
 // under that tolerance, i.e. both operands the same NaN/infinity class or
 // |c - g| <= atol_j + rtol_i |g| exactly.  One read of both tensors.
 //
-// Per pair and atol_j, the first rtol index i* that accepts the pair (0 for
-// an EXACT pair, nr for one no tolerance accepts) comes from a binary search
-// (acceptance grows with rtol); each test is one fma with a float32 margin,
-// and the integer digits of a - atol - rtol |g| decide the rare close calls.
-// A warp counts cell (i, j) as the population of the ballot i*_j <= i; lane
-// c % 32 keeps cell c's count in a register.
+// Acceptance grows with rtol and with atol, so a pair is described by
+// f(j) = the first rtol index accepting it at atol_j (0 for an EXACT pair,
+// nr for none), and f does not increase along the atols sorted ascending.
+// Exact pairs are counted per thread.  A warp queues its differing finite
+// pairs in shared memory and takes them 32 at a time: each lane finds f(j)
+// for the atols in ascending order by a binary search bounded by f(j - 1)
+// (each test one fma with a float32 margin; the integer digits of
+// a - atol - rtol |g| decide the close calls), and the warp adds each atol's
+// f values to a shared histogram, one atomic per distinct value.  Cell
+// (i, j) is the histogram's prefix over f <= i.
 #include <cuda_fp16.h>
 
 #include <cstdint>
@@ -137,77 +141,106 @@ __device__ __forceinline__ void abs_diff(float gf, float cf, float& hi, float& l
   lo = s < 0.0f ? -t : t;
 }
 
-// One pair slot of a warp (every lane calls it; ok: this lane holds a pair):
-// the first accepting rtol index per atol, then one ballot per cell.
+constexpr int NW = TB / 32;
+constexpr int QCAP = 64;  // a warp's queue: at most 31 left over plus 32 new pairs
+constexpr int NBIN = 2 * ISC_MAX;  // na (nr + 1) <= nr na + na <= 128
+
+struct QEntry {
+  float hi, lo, ag;
+  int sc;
+};
+
+struct IscSmem {
+  float R[ISC_MAX], A[ISC_MAX];  // rtols ascending, atols ascending
+  unsigned H[NBIN];              // H[j (nr + 1) + f]: pairs whose first accepting rtol at atol j is f
+  QEntry q[NW][QCAP];
+};
+
+// The lane's pair: kind 0 accepted by every tolerance (EXACT), 1 by none,
+// 2 finite and different: |c - g| = (hi + lo) 2^sc, ag = |g|.
 template <int DT>
-__device__ __forceinline__ void ic_pair(const IscParams& p, const float* R, const float* A, uint32_t G, uint32_t C,
-                                        bool ok, uint32_t& c0, uint32_t& c1) {
+__device__ __forceinline__ int classify(uint32_t G, uint32_t C, float& hi, float& lo, int& sc, float& ag) {
   using T = IC<DT>;
-  const int lane = threadIdx.x & 31;
-  // kind 0: accepted by every tolerance; 1: by none; 2: search
-  int kind = 1;
-  float hi = 0.0f, lo = 0.0f, ag = 0.0f;
-  int sc = 0;
-  if (ok) {
-    if (G == C) {
-      kind = 0;
-    } else {
-      const uint32_t mg = G & T::MAG, mc = C & T::MAG;
-      if (mg >= T::INF || mc >= T::INF) {
-        // both NaN, or the same infinity (G == C handled above): EXACT
-        kind = (mg > T::INF && mc > T::INF) ? 0 : 1;
-      } else {
-        const float gf = ic_f32<DT>(G), cf = ic_f32<DT>(C);
-        if (gf == cf) {
-          kind = 0;  // +0 and -0
-        } else {
-          abs_diff(gf, cf, hi, lo, sc);
-          ag = fabsf(gf);
-          kind = 2;
-        }
-      }
-    }
-  }
-  if (__all_sync(0xFFFFFFFFu, kind == 0)) {  // a whole slot of EXACT pairs: every cell
-    if (lane < p.ncells) c0 += 32u;
-    if (lane + 32 < p.ncells) c1 += 32u;
-    return;
-  }
+  if (G == C) return 0;
+  const uint32_t mg = G & T::MAG, mc = C & T::MAG;
+  if (mg >= T::INF || mc >= T::INF) return (mg > T::INF && mc > T::INF) ? 0 : 1;  // both NaN: EXACT
+  const float gf = ic_f32<DT>(G), cf = ic_f32<DT>(C);
+  if (gf == cf) return 0;  // +0 and -0
+  abs_diff(gf, cf, hi, lo, sc);
+  ag = fabsf(gf);
+  return 2;
+}
+
+// One batch of the warp's queue: lane takes entry e (valid: it holds one).
+__device__ __forceinline__ void run_batch(const IscParams& p, IscSmem& sm, const QEntry& e, bool valid) {
+  const int nb = p.nr + 1;
+  int prev = valid ? p.nr : 0;  // f(j - 1); invalid lanes carry 0 and add nothing
   for (int j = 0; j < p.na; j++) {
-    int first = kind == 0 ? 0 : p.nr;
-    if (kind == 2) {
-      int a = 0, b = p.nr;
+    const unsigned vmask = __ballot_sync(0xFFFFFFFFu, valid && prev > 0);
+    if (vmask == 0u) {
+      // every valid lane is accepted at rtol_0 from here on: f = 0 for the remaining atols
+      const int nvalid = __popc(__ballot_sync(0xFFFFFFFFu, valid));
+      if ((threadIdx.x & 31) == 0)
+        for (int jj = j; jj < p.na; jj++) atomicAdd(&sm.H[jj * nb], (unsigned)nvalid);
+      return;
+    }
+    int f = prev;
+    if (valid && prev > 0) {
+      int a = 0, b = prev;
+      const float at = sm.A[j];
       while (a < b) {
         const int mid = (a + b) >> 1;
-        if (close_test(hi, lo, sc, ag, R[mid], A[j])) b = mid;
+        if (close_test(e.hi, e.lo, e.sc, e.ag, sm.R[mid], at)) b = mid;
         else a = mid + 1;
       }
-      first = a;
+      f = a;
     }
-    for (int i = 0; i < p.nr; i++) {
-      const int cell = i * p.na + j;
-      const uint32_t cnt = __popc(__ballot_sync(0xFFFFFFFFu, first <= i));
-      if (lane == (cell & 31)) {
-        if (cell < 32) c0 += cnt;
-        else c1 += cnt;
-      }
-    }
+    prev = f;
+    const int key = valid ? f : -1;
+    const unsigned grp = __match_any_sync(0xFFFFFFFFu, key);
+    if (valid && (threadIdx.x & 31) == __ffs(grp) - 1) atomicAdd(&sm.H[j * nb + f], (unsigned)__popc(grp));
   }
+}
+
+// Queue the lane's pair if it needs a search; take a batch once 32 wait.
+// Every lane of the warp calls it (ok: this lane holds a pair).
+template <int DT>
+__device__ __forceinline__ void ic_pair(const IscParams& p, IscSmem& sm, uint32_t G, uint32_t C, bool ok, int& qn,
+                                        uint32_t& nexact) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float hi = 0.0f, lo = 0.0f, ag = 0.0f;
+  int sc = 0;
+  const int kind = ok ? classify<DT>(G, C, hi, lo, sc, ag) : 1;
+  nexact += kind == 0;
+  const unsigned m = __ballot_sync(0xFFFFFFFFu, kind == 2);
+  if (m == 0u) return;
+  if (kind == 2) sm.q[warp][qn + __popc(m & ((1u << lane) - 1u))] = QEntry{hi, lo, ag, sc};
+  qn += __popc(m);
+  if (qn < 32) return;
+  __syncwarp();
+  const QEntry e = sm.q[warp][lane];
+  __syncwarp();
+  if (lane < qn - 32) sm.q[warp][lane] = sm.q[warp][32 + lane];
+  qn -= 32;
+  __syncwarp();
+  run_batch(p, sm, e, true);
 }
 
 template <int DT>
 __global__ void __launch_bounds__(TB) isclose_grid(IscParams p) {
   constexpr int VEC = IC<DT>::VEC, B = IC<DT>::BYTES;
-  __shared__ float R[ISC_MAX], A[ISC_MAX];
-  const int lane = threadIdx.x & 31;
+  __shared__ IscSmem sm;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int i = threadIdx.x; i < ISC_MAX; i += TB) {
-    R[i] = i < p.nr ? p.rtol[i] : 0.0f;
-    A[i] = i < p.na ? p.atol[i] : 0.0f;
+    sm.R[i] = i < p.nr ? p.rtol[i] : 0.0f;
+    sm.A[i] = i < p.na ? p.atol[i] : 0.0f;
   }
+  for (int i = threadIdx.x; i < NBIN; i += TB) sm.H[i] = 0u;
   __syncthreads();
   const int64_t stride = (int64_t)gridDim.x * TB;
   const int64_t gt = (int64_t)blockIdx.x * TB + threadIdx.x;
-  uint32_t c0 = 0, c1 = 0;  // cells lane and lane + 32 (those below ncells)
+  int qn = 0;            // this warp's queue length (the same in every lane)
+  uint32_t nexact = 0;   // this thread's EXACT pairs (below 2^32: the host bounds the elements per CTA)
   // rounds of one vector per thread, whole warps in every round
   for (int64_t v = gt; __any_sync(0xFFFFFFFFu, v < p.nvec); v += stride) {
     const bool ok = v < p.nvec;
@@ -217,8 +250,12 @@ __global__ void __launch_bounds__(TB) isclose_grid(IscParams p) {
       gv = ic_vec(p.g, off);
       cv = ic_vec(p.c, off);
     }
+    if (__all_sync(0xFFFFFFFFu, !ok || (gv.x == cv.x && gv.y == cv.y && gv.z == cv.z && gv.w == cv.w))) {
+      nexact += ok ? VEC : 0;  // a warp slot of bitwise-equal vectors
+      continue;
+    }
 #pragma unroll
-    for (int j = 0; j < VEC; j++) ic_pair<DT>(p, R, A, ic_lane<DT>(gv, j), ic_lane<DT>(cv, j), ok, c0, c1);
+    for (int j = 0; j < VEC; j++) ic_pair<DT>(p, sm, ic_lane<DT>(gv, j), ic_lane<DT>(cv, j), ok, qn, nexact);
   }
   // elements outside the vector grid, in whole-warp rounds as well
   const int64_t head = p.p0 >= 0 ? p.p0 : p.n, tail = p.p0 >= 0 ? p.p0 + p.nvec * VEC : p.n;
@@ -233,10 +270,26 @@ __global__ void __launch_bounds__(TB) isclose_grid(IscParams p) {
       G = ic_load<DT>(p.g, i);
       C = ic_load<DT>(p.c, i);
     }
-    ic_pair<DT>(p, R, A, G, C, ok, c0, c1);
+    ic_pair<DT>(p, sm, G, C, ok, qn, nexact);
   }
-  if (c0 && lane < p.ncells) atomicAdd(p.counts + lane, (unsigned long long)c0);
-  if (c1 && lane + 32 < p.ncells) atomicAdd(p.counts + 32 + lane, (unsigned long long)c1);
+  // the rest of the queue
+  if (qn > 0) {
+    __syncwarp();
+    const QEntry e = sm.q[warp][lane < qn ? lane : 0];
+    run_batch(p, sm, e, lane < qn);
+  }
+  // exact pairs: f = 0 at every atol
+  const uint32_t ne = __reduce_add_sync(0xFFFFFFFFu, nexact);
+  if (lane == 0 && ne)
+    for (int j = 0; j < p.na; j++) atomicAdd(&sm.H[j * (p.nr + 1)], ne);
+  __syncthreads();
+  // cell (i, j) = pairs with f(j) <= i, into the caller's cell order
+  for (int c = threadIdx.x; c < p.ncells; c += TB) {
+    const int i = c / p.na, j = c - i * p.na;
+    unsigned long long cnt = 0;
+    for (int f = 0; f <= i; f++) cnt += sm.H[j * (p.nr + 1) + f];
+    if (cnt) atomicAdd(p.counts + i * p.na + p.aperm[j], cnt);
+  }
 }
 
 template <int DT>

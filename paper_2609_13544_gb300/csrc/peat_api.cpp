@@ -537,12 +537,16 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
     if (i > 0 && r < p.rtol[i - 1]) return fail(h, PEAT_ERR_INVALID_ARG, "rtols must be non-decreasing");
     p.rtol[i] = r;
   }
+  float at[peat::ISC_MAX];
   for (int j = 0; j < na; j++) {
-    float r, a;
-    if (!round_tol(peat_tol_t{0.0, atols[j]}, &r, &a))
+    float r;
+    if (!round_tol(peat_tol_t{0.0, atols[j]}, &r, &at[j]))
       return fail(h, PEAT_ERR_INVALID_ARG, "atols must be finite and >= 0 after rounding to float32");
-    p.atol[j] = a;
+    p.aperm[j] = j;
   }
+  // the kernel walks the atols in ascending order (stable: equal atols keep their order)
+  std::stable_sort(p.aperm, p.aperm + na, [&](int x, int y) { return at[x] < at[y]; });
+  for (int j = 0; j < na; j++) p.atol[j] = at[p.aperm[j]];
   DeviceGuard dg(h->device);
   if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -568,6 +572,8 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
   if (n == 0) return PEAT_OK;
   const int64_t want = (n + 4095) / 4096;
   const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)h->nsm * 8, want));
+  // per-CTA counts are 32-bit
+  if (n / nctas >= ((int64_t)1 << 31)) return fail(h, PEAT_ERR_UNSUPPORTED, "more than 2^31 elements per CTA");
   e = peat::launch_isclose(dtype, p, nctas, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "isclose launch");
   return PEAT_OK;

@@ -181,8 +181,9 @@ struct IscParams {
   int64_t p0;     // first element of the 16-byte vector grid; -1: none
   int64_t nvec;   // vectors on the grid
   int nr, na, ncells;
-  float rtol[ISC_MAX], atol[ISC_MAX];  // float32 tolerances, rtol ascending
-  unsigned long long* counts;          // device, ncells (cell i * na + j), zero before the launch
+  float rtol[ISC_MAX], atol[ISC_MAX];  // float32 tolerances, both ascending
+  int aperm[ISC_MAX];                  // the caller's index of the j-th smallest atol
+  unsigned long long* counts;          // device, ncells (cell i * na + caller's j), zero before the launch
 };
 cudaError_t launch_isclose(int dtype, const IscParams& p, int nctas, cudaStream_t s);
 

@@ -104,3 +104,25 @@ def test_invalid_arguments(peat_gpu, h):
         peat_gpu.peat_isclose_grid(h, g, g, [0.1] * 9, [0.0] * 8)      # 72 cells
     with pytest.raises(peat_gpu.PeatError):
         peat_gpu.peat_isclose_grid(h, g, g, [float("nan")], [0.0])
+
+
+@pytest.mark.parametrize("dtype", DTYPES)
+def test_repeated_and_descending_tolerances(peat_gpu, oracle, h, dtype):
+    """Repeated rtols, repeated atols and atols in descending order: the kernel
+    walks the atols sorted, the counts come back in the caller's order."""
+    gb, cb = noise_pairs(dtype, 50_003, seed=33, rel=2e-3)
+    check(peat_gpu, oracle, h, gb, cb, dtype, [0.0, 0.0, 1e-3, 1e-3, 1e-2], [1e-2, 0.0, 1e-4, 1e-2, 0.0, 1e30],
+          ctx="repeated")
+    check(peat_gpu, oracle, h, gb, cb, dtype, RTOLS, ATOLS[::-1], ctx="descending atols")
+
+
+def test_half_the_pairs_differ(peat_gpu, oracle, h):
+    """bf16 round-to-nearest against round-toward-zero of the same float32
+    values (about half the pairs differ by one ulp): many full queue batches,
+    vector rounds with and without an all-equal warp slot, a ragged tail."""
+    n = (1 << 20) + 7
+    x = torch.from_numpy(np.random.default_rng(8).standard_normal(n).astype(np.float32) * 2)
+    gb = x.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16).copy()
+    cb = (x.view(torch.int32).numpy().view(np.uint32) >> 16).astype(np.uint16)
+    got = check(peat_gpu, oracle, h, gb, cb, "bf16", ctx="rne vs rtz")
+    assert got[0, 0] < n * 0.6 and got[-1, -1] == n

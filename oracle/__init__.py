@@ -18,8 +18,8 @@ import numpy as np
 
 from .build import LIB, build
 
-DTYPES = {"f32": 0, "f16": 1, "bf16": 2}
-ITEMSIZE = {"f32": 4, "f16": 2, "bf16": 2}
+DTYPES = {"f32": 0, "f16": 1, "bf16": 2, "f8e4m3": 3, "f8e5m2": 4}
+ITEMSIZE = {"f32": 4, "f16": 2, "bf16": 2, "f8e4m3": 1, "f8e5m2": 1}
 CLASSES = ("exact", "within_tol", "mismatch", "nan_inf_asym", "sign_flip")
 INJECT_KINDS = {
     "rz": 0, "rv": 1, "bitflip": 2, "nan_inf": 3, "signflip": 4, "rel_gauss": 5,
@@ -123,15 +123,16 @@ def lib() -> ctypes.CDLL:
 
 
 def _bits(x, dtype: str) -> np.ndarray:
-    """Raw bit patterns of x as a contiguous uint16/uint32 array."""
-    if hasattr(x, "detach"):  # a CPU torch tensor (bf16 has no numpy dtype)
+    """Raw bit patterns of x as a contiguous uint8/uint16/uint32 array."""
+    size = ITEMSIZE[dtype]
+    if hasattr(x, "detach"):  # a CPU torch tensor (bf16 and fp8 have no numpy dtype)
         import torch
         x = x.detach().cpu().contiguous()
-        x = x.view(torch.int32 if ITEMSIZE[dtype] == 4 else torch.int16).numpy()
+        x = x.view({4: torch.int32, 2: torch.int16, 1: torch.uint8}[size]).numpy()
     x = np.ascontiguousarray(x)
-    if x.dtype.itemsize != ITEMSIZE[dtype]:
-        raise ValueError(f"{dtype} needs {ITEMSIZE[dtype]}-byte elements, got {x.dtype}")
-    return x.reshape(-1).view(np.uint32 if ITEMSIZE[dtype] == 4 else np.uint16)
+    if x.dtype.itemsize != size:
+        raise ValueError(f"{dtype} needs {size}-byte elements, got {x.dtype}")
+    return x.reshape(-1).view({4: np.uint32, 2: np.uint16, 1: np.uint8}[size])
 
 
 def _stats_dict(s: Stats) -> dict:

@@ -190,8 +190,11 @@ double orc_exact_dot(const double* x, const double* y, int64_t n) {
 }
 
 /* ------------------------------------------------------------------------ */
-/* Decoding of the three element types, straight from IEEE 754 binary16,    */
-/* binary32 and the bfloat16 layout (top half of a binary32).               */
+/* Decoding of the element types, straight from IEEE 754 binary16 and      */
+/* binary32, the bfloat16 layout (top half of a binary32) and the two 8-bit */
+/* formats of the OCP FP8 specification: E5M2 (IEEE-like: exponent bias 15, */
+/* infinities and NaNs at the all-ones exponent) and E4M3 "fn" (bias 7, no  */
+/* infinities, the only NaN is S.1111.111, so S.1111.110 = 448 is finite).  */
 /* ------------------------------------------------------------------------ */
 typedef struct {
   int nan, inf, sign;
@@ -205,6 +208,7 @@ static uint32_t raw_bits(const void* base, int64_t i, int dtype) {
     memcpy(&b, (const char*)base + 4 * i, 4);
     return b;
   }
+  if (dtype == ORC_F8E4M3 || dtype == ORC_F8E5M2) return ((const uint8_t*)base)[i];
   uint16_t h;
   memcpy(&h, (const char*)base + 2 * i, 2);
   return h;
@@ -218,14 +222,23 @@ static val_t decode(uint32_t b, int dtype) {
     sbit = 31, ebits = 8, mbits = 23, bias = 127;
   } else if (dtype == ORC_F16) {
     sbit = 15, ebits = 5, mbits = 10, bias = 15;
-  } else {
+  } else if (dtype == ORC_BF16) {
     sbit = 15, ebits = 8, mbits = 7, bias = 127;
+  } else if (dtype == ORC_F8E5M2) {
+    sbit = 7, ebits = 5, mbits = 2, bias = 15;
+  } else {
+    sbit = 7, ebits = 4, mbits = 3, bias = 7;
   }
   r.sign = (int)((b >> sbit) & 1u);
   r.mag = b & ((1u << sbit) - 1u);
   uint32_t e = r.mag >> mbits, m = r.mag & ((1u << mbits) - 1u);
   uint32_t emax = (1u << ebits) - 1u;
-  if (e == emax) {
+  if (dtype == ORC_F8E4M3) {
+    if (r.mag == 0x7Fu) { /* the only NaN; the rest of the top binade is finite */
+      r.nan = 1;
+      return r;
+    }
+  } else if (e == emax) {
     r.nan = (m != 0);
     r.inf = (m == 0);
     return r;
@@ -487,12 +500,16 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
 }
 
 static int dtype_ok(int dtype) { return dtype == ORC_F32 || dtype == ORC_F16 || dtype == ORC_BF16; }
-static int dtype_size(int dtype) { return dtype == ORC_F32 ? 4 : 2; }
+/* the compare (and the isclose grid built on it) also takes the 8-bit formats */
+static int dtype_ok_cmp(int dtype) { return dtype_ok(dtype) || dtype == ORC_F8E4M3 || dtype == ORC_F8E5M2; }
+static int dtype_size(int dtype) {
+  return dtype == ORC_F32 ? 4 : (dtype == ORC_F16 || dtype == ORC_BF16 ? 2 : 1);
+}
 
 int orc_compare(const void* g, const void* c, int64_t n, int dtype, double rtol, double atol,
                 orc_stats* st, uint64_t* hist) {
   double r, a;
-  if (!dtype_ok(dtype) || n < 0 || !st || !hist || (n > 0 && (!g || !c))) return ORC_BAD_ARG;
+  if (!dtype_ok_cmp(dtype) || n < 0 || !st || !hist || (n > 0 && (!g || !c))) return ORC_BAD_ARG;
   if (!tol_ok(rtol, atol, &r, &a)) return ORC_BAD_ARG;
   compare_range(g, c, n, dtype, r, a, st, hist);
   return ORC_OK;
@@ -501,7 +518,7 @@ int orc_compare(const void* g, const void* c, int64_t n, int dtype, double rtol,
 int orc_compare_segmented(const void* g, const void* c, const int64_t* offsets, int64_t nseg,
                           int dtype, double rtol, double atol, orc_stats* st, uint64_t* hist) {
   double r, a;
-  if (!dtype_ok(dtype) || nseg < 0 || !offsets || (nseg > 0 && (!st || !hist))) return ORC_BAD_ARG;
+  if (!dtype_ok_cmp(dtype) || nseg < 0 || !offsets || (nseg > 0 && (!st || !hist))) return ORC_BAD_ARG;
   if (!tol_ok(rtol, atol, &r, &a)) return ORC_BAD_ARG;
   if (offsets[0] != 0) return ORC_BAD_ARG;
   for (int64_t s = 0; s < nseg; s++)

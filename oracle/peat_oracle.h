@@ -24,7 +24,7 @@ extern "C" {
 #endif
 
 /* element types (codes agree with the library's dtype codes) */
-enum { ORC_F32 = 0, ORC_F16 = 1, ORC_BF16 = 2 };
+enum { ORC_F32 = 0, ORC_F16 = 1, ORC_BF16 = 2, ORC_F8E4M3 = 3, ORC_F8E5M2 = 4 };
 
 /* classes, in the order of the library's class counters */
 enum { ORC_EXACT = 0, ORC_WITHIN_TOL = 1, ORC_MISMATCH = 2, ORC_NAN_INF_ASYM = 3,

@@ -8,8 +8,10 @@ import multiprocessing as mp
 
 import numpy as np
 
-NP_BITS = {"f32": np.uint32, "f16": np.uint16, "bf16": np.uint16}
-TORCH_DT = {"f32": "float32", "f16": "float16", "bf16": "bfloat16"}
+NP_BITS = {"f32": np.uint32, "f16": np.uint16, "bf16": np.uint16, "f8e4m3": np.uint8, "f8e5m2": np.uint8}
+TORCH_DT = {"f32": "float32", "f16": "float16", "bf16": "bfloat16", "f8e4m3": "float8_e4m3fn",
+            "f8e5m2": "float8_e5m2"}
+WIDTH = {"f32": 32, "f16": 16, "bf16": 16, "f8e4m3": 8, "f8e5m2": 8}
 INT_KEYS = ("n", "count", "n_finite", "argmax_abs", "argmax_rel", "max_ulp", "argmax_ulp")
 EXACT_FLOAT_KEYS = ("max_abs", "max_rel", "rtol_eff", "atol_eff")
 SUM_KEYS = ("sum_abs", "sum_sq", "sum_signed")

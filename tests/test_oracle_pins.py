@@ -20,7 +20,17 @@ import torch
 
 GOLD = json.loads((Path(__file__).parent / "golden" / "hand_cases.json").read_text())
 CLASS_IDX = {"exact": 0, "within_tol": 1, "mismatch": 2, "nan_inf_asym": 3, "sign_flip": 4}
-NP_BITS = {"f32": np.uint32, "f16": np.uint16, "bf16": np.uint16}
+NP_BITS = {"f32": np.uint32, "f16": np.uint16, "bf16": np.uint16, "f8e4m3": np.uint8, "f8e5m2": np.uint8}
+FP8 = {"f8e4m3": "float8_e4m3fn", "f8e5m2": "float8_e5m2"}
+_FP8_TABLE = {}
+
+
+def fp8_table(dtype):
+    """Every 8-bit pattern's value, from torch's own float8 conversions (OCP FP8)."""
+    if dtype not in _FP8_TABLE:
+        t = torch.arange(256, dtype=torch.int32).to(torch.uint8).view(getattr(torch, FP8[dtype]))
+        _FP8_TABLE[dtype] = t.to(torch.float32).tolist()
+    return _FP8_TABLE[dtype]
 
 
 # ---------------------------------------------------------------- helpers
@@ -30,11 +40,13 @@ def decode(bits: int, dtype: str) -> float:
         return float(np.array([bits], np.uint32).view(np.float32)[0])
     if dtype == "f16":
         return float(np.array([bits], np.uint16).view(np.float16)[0])
+    if dtype in FP8:
+        return fp8_table(dtype)[bits]
     return float(np.array([bits << 16], np.uint32).view(np.float32)[0])
 
 
 def signbit(bits: int, dtype: str) -> int:
-    return (bits >> (31 if dtype == "f32" else 15)) & 1
+    return (bits >> {"f32": 31, "f8e4m3": 7, "f8e5m2": 7}.get(dtype, 15)) & 1
 
 
 def rn32(x: float) -> float:
@@ -138,6 +150,58 @@ def test_ulp_key_f32_successor(oracle):
     for a, b in zip(x.view(np.uint32)[:5000], up.view(np.uint32)[:5000]):
         assert oracle.ulp_key(int(b), "f32") == oracle.ulp_key(int(a), "f32") + 1
     assert oracle.ulp_key(0, "f32") == oracle.ulp_key(0x80000000, "f32") == 0
+
+
+# ---------------------------------------------------------------- 8-bit types, every pair
+def test_fp8_formats_against_the_specification(oracle):
+    """OCP FP8: E4M3 has no infinities, its only NaNs are 0x7F / 0xFF and
+    0x7E = 448 is its largest value; E5M2 is IEEE-like (0x7C = +Inf, 0x7B =
+    57344); subnormal steps 2^-9 and 2^-16."""
+    e4, e5 = fp8_table("f8e4m3"), fp8_table("f8e5m2")
+    assert e4[0x7E] == 448.0 and math.isnan(e4[0x7F]) and math.isnan(e4[0xFF]) and e4[0x01] == 2.0 ** -9
+    assert sum(math.isnan(v) for v in e4) == 2 and not any(math.isinf(v) for v in e4)
+    assert e5[0x7B] == 57344.0 and e5[0x7C] == math.inf and e5[0xFC] == -math.inf and e5[0x01] == 2.0 ** -16
+    assert sum(math.isnan(v) for v in e5) == 6
+    # the oracle decodes the same values: compare each pattern with +0 (d = the value)
+    for dt, tab in (("f8e4m3", e4), ("f8e5m2", e5)):
+        c = np.arange(256, dtype=np.uint8)
+        stats, _ = oracle.compare_segmented(np.zeros(256, np.uint8), c, np.arange(257), dt, 0.0, 0.0)
+        for b in range(256):
+            if math.isfinite(tab[b]):
+                assert stats[b]["sum_signed"] == tab[b] and stats[b]["n_finite"] == 1, (dt, b)
+            else:
+                assert stats[b]["n_finite"] == 0 and stats[b]["count"][3] == 1, (dt, b)
+
+
+@pytest.mark.parametrize("dtype", ["f8e4m3", "f8e5m2"])
+@pytest.mark.parametrize("tol", [(0.0, 0.0), (0.125, 2.0 ** -7)])
+def test_fp8_every_pair_against_exact_rationals(oracle, dtype, tol):
+    """All 65,536 (golden, candidate) pairs of the type: class, both bins, the
+    ULP distance as the distance of signed ranks among the distinct non-NaN
+    values, and the exact error terms."""
+    rtol, atol = tol
+    tab = fp8_table(dtype)
+    distinct = sorted({v for v in tab if not math.isnan(v)})
+    pos = {v: i for i, v in enumerate(distinct)}
+    rank = [None if math.isnan(v) else pos[v] - pos[0.0] for v in tab]
+    g = np.repeat(np.arange(256, dtype=np.uint8), 256)
+    c = np.tile(np.arange(256, dtype=np.uint8), 256)
+    stats, hist = oracle.compare_segmented(g, c, np.arange(g.size + 1), dtype, rtol, atol)
+    for i in range(g.size):
+        gb, cb = int(g[i]), int(c[i])
+        ref = ref_pair(gb, cb, dtype, rtol, atol)
+        st = stats[i]
+        assert st["count"][ref["cls"]] == 1, (hex(gb), hex(cb), ref, st["count"])
+        assert hist[i][0][ref["relbin"]] == 1, (hex(gb), hex(cb), ref["relbin"])
+        rg, rc = rank[gb], rank[cb]
+        if rg is None or rc is None:
+            assert st["argmax_ulp"] == -1 and hist[i][1][0 if (rg is None and rc is None) else 63] == 1
+        else:
+            assert st["max_ulp"] == abs(rc - rg) and hist[i][1][min(abs(rc - rg), 63)] == 1
+        if ref["finite"]:
+            assert st["sum_signed"] == float(ref["d"]) and st["sum_abs"] == float(ref["a"])
+            assert st["sum_sq"] == float(ref["d"] ** 2) and st["max_abs"] == float(ref["a"])
+            assert st["max_rel"] == (math.inf if ref["rel"] is None else float(ref["rel"]))
 
 
 # ---------------------------------------------------------------- exact rationals on random pairs

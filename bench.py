@@ -413,6 +413,36 @@ def run_gpu(args) -> None:
                                       "draw and two Box-Muller pairs, then the compare"}}
         del scratch
 
+    # the 8-bit formats (OCP FP8): the golden's values rounded to E4M3 / E5M2 against the same
+    # values with relative noise 2^-4, rounded the same way; one read of both 1-byte tensors
+    fp8 = None
+    if w.offsets is None and not args.no_topk:
+        fp8 = {}
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(17)
+        x = g.float()
+        y = x * (1.0 + 0.0625 * torch.randn(x.shape, generator=gen, device=dev))
+        for name, tdt in (("e4m3", torch.float8_e4m3fn), ("e5m2", torch.float8_e5m2)):
+            g8, c8 = x.to(tdt), y.to(tdt)
+            for _ in range(3):
+                peat.peat_compare_raw(h, g8, c8, 0.125, 0.0, stats, hist, stream)
+            barrier()
+            calls = max(3, min(100, args.steps // 50))
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record(stream)
+            for _ in range(calls):
+                peat.peat_compare_raw(h, g8, c8, 0.125, 0.0, stats, hist, stream)
+            t1.record(stream)
+            barrier()
+            ms = max_over_ranks(t0.elapsed_time(t1), dev) / calls
+            gbs8 = 2 * w.n / (ms * 1e-3) / 1e9
+            fp8[name] = {"us_per_call": ms * 1e3, "pairs_per_s": w.n / (ms * 1e-3),
+                         "roofline": {"bound": "alu", "achieved": gbs8, "peak": peak, "unit": "GB/s",
+                                      "frac": gbs8 / peak, "algorithmic_bytes_per_call": 2 * w.n}}
+            del g8, c8
+        del x, y
+        fp8 = {"op": "peat_compare on 8-bit golden and candidate (rtol 1/8)", "calls": calls, **fp8}
+
     # end to end through the C ABI with host buffers: every step copies both
     # tensors from pinned host memory, compares them and reads the stats and
     # histograms back.  Two device buffer sets: step i's copies (copy stream)
@@ -501,7 +531,7 @@ def run_gpu(args) -> None:
                          else "fallback 6.8 TB/s"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": (1 if nseg == 1 else 2) * args.steps, "clocks": clocks,
             "next_rows": {"f1_top10_mean": topk, "f2_fused_inject_compare": fused, "f3_context_stats": tstats,
-                          "f4_isclose_grid": isc},
+                          "f4_isclose_grid": isc, "f4_fp8_compare": fp8},
             "wall_s_timed": wall,
         }
         print(json.dumps(line), flush=True)

@@ -59,7 +59,12 @@ extern "C" {
 /* A CUDA stream (layout-compatible with cudaStream_t / CUstream). */
 typedef struct CUstream_st* peat_stream_t;
 
-typedef enum { PEAT_F32 = 0, PEAT_F16 = 1, PEAT_BF16 = 2 } peat_dtype_t;
+/* Element types.  The 8-bit ones are the OCP FP8 formats: E4M3 ("fn": exponent
+ * bias 7, no infinities, S.1111.111 the only NaN, 448 the largest value) and
+ * E5M2 (bias 15, IEEE-like infinities and NaNs); peat_compare,
+ * peat_compare_segmented and peat_isclose_grid take them, the other entry
+ * points return PEAT_ERR_UNSUPPORTED. */
+typedef enum { PEAT_F32 = 0, PEAT_F16 = 1, PEAT_BF16 = 2, PEAT_F8E4M3 = 3, PEAT_F8E5M2 = 4 } peat_dtype_t;
 
 typedef enum {
   PEAT_OK = 0,

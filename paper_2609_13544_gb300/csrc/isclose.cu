@@ -21,9 +21,12 @@
 
 #include "exact.cuh"
 #include "peat_internal.h"
+#include "tol_exact.cuh"
 
 namespace peat {
 namespace {
+
+using namespace tolx;
 
 constexpr int TB = 256;
 
@@ -44,25 +47,58 @@ struct IC<PEAT_BF16> {
   static constexpr int BYTES = 2, VEC = 8;
   static constexpr uint32_t MAG = 0x7FFFu, INF = 0x7F80u;
 };
+template <>
+struct IC<PEAT_F8E5M2> {  // IEEE-like: infinities and NaNs at the all-ones exponent
+  static constexpr int BYTES = 1, VEC = 16;
+  static constexpr uint32_t MAG = 0x7Fu, INF = 0x7Cu;
+};
+template <>
+struct IC<PEAT_F8E4M3> {  // no infinities: 0x7F (either sign) is the only NaN
+  static constexpr int BYTES = 1, VEC = 16;
+  static constexpr uint32_t MAG = 0x7Fu, INF = 0x7Fu;
+};
 
+// magnitude bits: not finite / NaN
+template <int DT>
+__device__ __forceinline__ bool ic_nonfinite(uint32_t m) { return m >= IC<DT>::INF; }
+template <int DT>
+__device__ __forceinline__ bool ic_nan(uint32_t m) {
+  if constexpr (DT == PEAT_F8E4M3) return m == 0x7Fu;
+  else return m > IC<DT>::INF;
+}
+
+// the value of a finite pattern (exact in float32)
 template <int DT>
 __device__ __forceinline__ float ic_f32(uint32_t r) {
-  if constexpr (DT == PEAT_F32) return __uint_as_float(r);
-  else if constexpr (DT == PEAT_BF16) return __uint_as_float(r << 16);
-  else return __half2float(__ushort_as_half((unsigned short)r));
+  if constexpr (DT == PEAT_F32) {
+    return __uint_as_float(r);
+  } else if constexpr (DT == PEAT_BF16) {
+    return __uint_as_float(r << 16);
+  } else if constexpr (DT == PEAT_F16) {
+    return __half2float(__ushort_as_half((unsigned short)r));
+  } else if constexpr (DT == PEAT_F8E5M2) {
+    return __half2float(__ushort_as_half((unsigned short)(r << 8)));  // the top byte of a binary16
+  } else {
+    // E4M3: exponent bias 7, 3 fraction bits; subnormals m 2^-9
+    const uint32_t e = (r >> 3) & 0xFu, m = r & 7u;
+    const float v = e ? __uint_as_float(((e + 120u) << 23) | (m << 20)) : __fmul_rn(__uint2float_rn(m), 0x1p-9f);
+    return (r & 0x80u) ? -v : v;
+  }
 }
 
 template <int DT>
 __device__ __forceinline__ uint32_t ic_lane(const uint4& v, int j) {
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
   if constexpr (IC<DT>::BYTES == 4) return w[j];
-  else return (w[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+  else if constexpr (IC<DT>::BYTES == 2) return (w[j >> 1] >> (16 * (j & 1))) & 0xFFFFu;
+  else return (w[j >> 2] >> (8 * (j & 3))) & 0xFFu;
 }
 
 template <int DT>
 __device__ __forceinline__ uint32_t ic_load(const void* base, int64_t i) {
   if constexpr (IC<DT>::BYTES == 4) return __ldg(reinterpret_cast<const uint32_t*>(base) + i);
-  else return (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(base) + i);
+  else if constexpr (IC<DT>::BYTES == 2) return (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(base) + i);
+  else return (uint32_t)__ldg(reinterpret_cast<const unsigned char*>(base) + i);
 }
 
 __device__ __forceinline__ uint4 ic_vec(const void* base, int64_t byte_off) {
@@ -72,73 +108,6 @@ __device__ __forceinline__ uint4 ic_vec(const void* base, int64_t byte_off) {
                : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                : "l"(q));
   return v;
-}
-
-// sign of (hi + lo) 2^sc - atol - rtol ag, exactly (integer digits)
-__device__ __noinline__ int excess_sign(float hi, float lo, int sc, float ag, float rtol, float atol) {
-  int64_t d[NLIMB];
-#pragma unroll
-  for (int j = 0; j < NLIMB; j++) d[j] = 0;
-  auto add = [&](int j, int64_t v) { d[j] += v; };
-  int e;
-  if (hi != 0.0f) {
-    const uint32_t m = split_float(hi, e);
-    for_digits(m, e + sc, false, add);
-  }
-  if (lo != 0.0f) {
-    const uint32_t m = split_float(lo, e);
-    for_digits(m, e + sc, lo < 0.0f, add);
-  }
-  if (atol != 0.0f) {
-    const uint32_t m = split_float(atol, e);
-    for_digits(m, e, true, add);
-  }
-  if (rtol != 0.0f && ag != 0.0f) {
-    int er, eg;
-    const uint32_t mr = split_float(rtol, er), mg = split_float(ag, eg);
-    for_digits((uint64_t)mr * mg, er + eg, true, add);
-  }
-  int64_t carry = 0;
-#pragma unroll
-  for (int j = 0; j < NLIMB - 1; j++) {
-    const int64_t v = d[j] + carry;
-    carry = v >> 32;
-    d[j] = v & 0xFFFFFFFFll;
-  }
-  d[NLIMB - 1] += carry;
-  if (d[NLIMB - 1] != 0) return d[NLIMB - 1] < 0 ? -1 : 1;
-  bool nz = false;
-#pragma unroll
-  for (int j = 0; j < NLIMB - 1; j++) nz |= d[j] != 0;
-  return nz ? 1 : 0;
-}
-
-// a = (hi + lo) 2^sc <= atol + rtol ag, exactly
-__device__ __forceinline__ bool close_test(float hi, float lo, int sc, float ag, float rtol, float atol) {
-  const float thr = __fmaf_rn(rtol, ag, atol);
-  if (sc == 0 && hi >= 1e-30f && thr >= 1e-30f) {
-    // |lo| <= 2^-24 hi and thr is within 2^-24 of the exact bound: margins of 2^-21
-    if (__fmul_rn(hi, 1.0000005f) < __fmul_rn(thr, 0.9999995f)) return true;
-    if (__fmul_rn(hi, 0.9999995f) > __fmul_rn(thr, 1.0000005f)) return false;
-  }
-  return excess_sign(hi, lo, sc, ag, rtol, atol) <= 0;
-}
-
-// |d| = (hi + lo) 2^sc exactly (float32 TwoSum, halved when c - g overflows)
-__device__ __forceinline__ void abs_diff(float gf, float cf, float& hi, float& lo, int& sc) {
-  float x = cf, y = -gf;
-  sc = 0;
-  float s = __fadd_rn(x, y);
-  if (!(fabsf(s) < __int_as_float(0x7F800000))) {
-    x = __fmul_rn(x, 0.5f);
-    y = __fmul_rn(y, 0.5f);
-    s = __fadd_rn(x, y);
-    sc = 1;
-  }
-  const float yv = __fsub_rn(s, x), xv = __fsub_rn(s, yv);
-  const float t = __fadd_rn(__fsub_rn(x, xv), __fsub_rn(y, yv));
-  hi = fabsf(s);
-  lo = s < 0.0f ? -t : t;
 }
 
 constexpr int NW = TB / 32;
@@ -163,7 +132,7 @@ __device__ __forceinline__ int classify(uint32_t G, uint32_t C, float& hi, float
   using T = IC<DT>;
   if (G == C) return 0;
   const uint32_t mg = G & T::MAG, mc = C & T::MAG;
-  if (mg >= T::INF || mc >= T::INF) return (mg > T::INF && mc > T::INF) ? 0 : 1;  // both NaN: EXACT
+  if (ic_nonfinite<DT>(mg) || ic_nonfinite<DT>(mc)) return (ic_nan<DT>(mg) && ic_nan<DT>(mc)) ? 0 : 1;  // both NaN: EXACT
   const float gf = ic_f32<DT>(G), cf = ic_f32<DT>(C);
   if (gf == cf) return 0;  // +0 and -0
   abs_diff(gf, cf, hi, lo, sc);
@@ -305,6 +274,8 @@ cudaError_t launch_isclose(int dtype, const IscParams& p, int nctas, cudaStream_
     case PEAT_F32: return launch_t<PEAT_F32>(p, nctas, s);
     case PEAT_F16: return launch_t<PEAT_F16>(p, nctas, s);
     case PEAT_BF16: return launch_t<PEAT_BF16>(p, nctas, s);
+    case PEAT_F8E4M3: return launch_t<PEAT_F8E4M3>(p, nctas, s);
+    case PEAT_F8E5M2: return launch_t<PEAT_F8E5M2>(p, nctas, s);
   }
   return cudaErrorInvalidValue;
 }

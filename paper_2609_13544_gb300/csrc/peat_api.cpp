@@ -47,6 +47,10 @@ struct peat_handle_s {
   int64_t* d_inj = nullptr;
   int64_t* h_inj = nullptr;
   size_t inj_cap = 0;  // in int64 elements
+  // 8-bit compare: pinned staging of offsets and work items, device copy plus item records
+  int64_t* h_f8 = nullptr;
+  void* d_f8 = nullptr;
+  size_t f8_hcap = 0, f8_dcap = 0;  // bytes
   std::string err;
 };
 
@@ -81,7 +85,10 @@ peat_status_t cuda_fail(peat_handle_t h, cudaError_t e, const char* what) {
   return fail(h, PEAT_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }
 
+// the element types of the main kernels (the 8-bit formats have their own compare)
 int dtype_bytes(int dt) { return dt == PEAT_F32 ? 4 : (dt == PEAT_F16 || dt == PEAT_BF16 ? 2 : 0); }
+bool is_fp8(int dt) { return dt == PEAT_F8E4M3 || dt == PEAT_F8E5M2; }
+const char* const FP8_ONLY = "8-bit formats: peat_compare, peat_compare_segmented and peat_isclose_grid only";
 
 bool round_tol(peat_tol_t tol, float* r, float* a) {
   if (!(tol.rtol >= 0.0) || !(tol.atol >= 0.0)) return false;  // rejects NaN too
@@ -168,6 +175,143 @@ static cudaError_t single_bounds(peat_handle_t h, int dtype, int nctas, int64_t 
   return cudaSuccess;
 }
 
+// floor(mx 2^ex + my 2^ey) for mx, my < 2^57, saturated at 2^40.  The
+// fractional parts are added in 128-bit fixed point with unit 2^-120, exact
+// for exponents down to -120; a term below that is under 2^-64 and cannot
+// complete a carry, since the other term's fraction is then at most
+// 1 - 2^-57.
+static uint64_t floor_dyadic_sum(uint64_t mx, int ex, uint64_t my, int ey) {
+  const uint64_t CAP = 1ull << 40;
+  uint64_t fl = 0;
+  unsigned __int128 fr = 0;
+  const uint64_t ms[2] = {mx, my};
+  const int es[2] = {ex, ey};
+  for (int t = 0; t < 2; t++) {
+    const uint64_t m = ms[t];
+    const int e = es[t];
+    if (m == 0 || e < -120) continue;
+    if (e >= 0) {
+      if (e >= 40 || (m >> (40 - e)) != 0) return CAP;
+      fl += m << e;
+    } else {
+      const int k = -e;
+      if (k < 64) {
+        fl += m >> k;
+        fr += (unsigned __int128)(m & ((1ull << k) - 1)) << (120 - k);
+      } else {
+        fr += (unsigned __int128)m << (120 - k);
+      }
+    }
+  }
+  if (fr >> 120) fl += 1;
+  return std::min(fl, CAP);
+}
+
+// x = m 2^e with m a 24-bit integer (x a finite float32 >= 0; m = 0 for 0)
+static void split_f32(float x, uint64_t* m, int* e) {
+  if (x == 0.0f) {
+    *m = 0;
+    *e = 0;
+    return;
+  }
+  int ex;
+  const float fr = std::frexp(x, &ex);  // x = fr 2^ex, fr in [0.5, 1)
+  *m = (uint64_t)std::ldexp(fr, 24);    // exact: 24 significant bits
+  *e = ex - 24;
+}
+
+// The 8-bit formats: work items of at most `ch` elements within one segment
+// (about four per SM for one tensor), one record each, merged per segment.
+static peat_status_t compare8_impl(peat_handle_t h, const void* g, const void* c, const int64_t* offsets,
+                                   int64_t nseg, int dtype, float rtol, float atol, peat_stats_t* stats,
+                                   uint64_t* hist, cudaStream_t st) {
+  const int64_t n = offsets[nseg];
+  int64_t ch = (n + 4 * (int64_t)h->nsm - 1) / (4 * (int64_t)h->nsm);
+  ch = std::min<int64_t>(std::max<int64_t>((ch + 15) / 16 * 16, 4096), (int64_t)1 << 22);
+  int64_t nitems = 0;
+  for (int64_t s = 0; s < nseg; s++) nitems += (offsets[s + 1] - offsets[s] + ch - 1) / ch;
+  // staging: offsets (nseg + 1), item_b, item_e, item_seg (nitems each), seg_first (nseg + 1)
+  const size_t nwords = (size_t)(nseg + 1) * 2 + 3 * (size_t)nitems;
+  const size_t hbytes = nwords * sizeof(int64_t);
+  const size_t dbytes = hbytes + (size_t)std::max<int64_t>(nitems, 1) * sizeof(peat::Part8);
+  peat_status_t ps = wait_staging(h);  // the pinned staging is free
+  if (ps != PEAT_OK) return ps;
+  if (hbytes > h->f8_hcap || dbytes > h->f8_dcap) {
+    if (h->h_f8) cudaFreeHost(h->h_f8);
+    if (h->d_f8) cudaFree(h->d_f8);
+    h->h_f8 = nullptr;
+    h->d_f8 = nullptr;
+    h->f8_hcap = h->f8_dcap = 0;
+    const size_t hc = std::max(hbytes, (size_t)65536), dc = std::max(dbytes, (size_t)1 << 20);
+    if (cudaMallocHost(&h->h_f8, hc) != cudaSuccess || cudaMalloc(&h->d_f8, dc) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(h, PEAT_ERR_ALLOC, "8-bit compare workspace allocation failed");
+    }
+    h->f8_hcap = hc;
+    h->f8_dcap = dc;
+  }
+  int64_t* ho = h->h_f8;
+  int64_t* hb = ho + (nseg + 1);
+  int64_t* he = hb + nitems;
+  int64_t* hs = he + nitems;
+  int64_t* hf = hs + nitems;
+  std::memcpy(ho, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
+  int64_t it = 0;
+  for (int64_t s = 0; s < nseg; s++) {
+    hf[s] = it;
+    for (int64_t x = offsets[s]; x < offsets[s + 1]; x += ch, it++) {
+      hb[it] = x;
+      he[it] = std::min(offsets[s + 1], x + ch);
+      hs[it] = s;
+    }
+  }
+  hf[nseg] = it;
+  int64_t* d = static_cast<int64_t*>(h->d_f8);
+  cudaError_t e = cudaMemcpyAsync(d, ho, hbytes, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(8-bit items)");
+  e = cudaEventRecord(h->staged, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
+  h->staged_pending = true;
+  if (hist) {
+    e = cudaMemsetAsync(hist, 0, sizeof(uint64_t) * PEAT_HIST_BINS * (size_t)nseg, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemsetAsync(hist)");
+  }
+  peat::Cmp8Params p;
+  std::memset(&p, 0, sizeof(p));
+  p.g = g;
+  p.c = c;
+  p.offsets = d;
+  p.item_b = d + (nseg + 1);
+  p.item_e = p.item_b + nitems;
+  p.item_seg = p.item_e + nitems;
+  p.seg_first = p.item_seg + nitems;
+  p.nitems = nitems;
+  p.nseg = nseg;
+  p.rtol = rtol;
+  p.atol = atol;
+  {
+    // the tolerance as one integer bound per golden magnitude: |d| 2^S <= rtol K + atol 2^S
+    const int S = dtype == PEAT_F8E4M3 ? 9 : 16, MB = dtype == PEAT_F8E4M3 ? 3 : 2;
+    uint64_t mr, ma;
+    int er, ea;
+    split_f32(rtol, &mr, &er);
+    split_f32(atol, &ma, &ea);
+    for (uint32_t mag = 0; mag < 128; mag++) {
+      const uint32_t ee = mag >> MB, mm = mag & ((1u << MB) - 1u);
+      const uint64_t K = ee == 0 ? mm : ((uint64_t)(mm | (1u << MB)) << (ee - 1));  // |g| 2^S (unused past the finite range)
+      p.amax[mag] = floor_dyadic_sum(mr * K, er, ma, ea + S);
+    }
+  }
+  p.vec = (reinterpret_cast<uintptr_t>(g) % 16 == 0 && reinterpret_cast<uintptr_t>(c) % 16 == 0) ? 1 : 0;
+  p.parts = reinterpret_cast<peat::Part8*>(reinterpret_cast<char*>(h->d_f8) + hbytes);
+  p.stats = stats;
+  p.hist = reinterpret_cast<unsigned long long*>(hist);
+  const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>(nitems, 2 * (int64_t)h->nsm));
+  e = peat::launch_compare8(dtype, p, nctas, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "8-bit compare launch");
+  return PEAT_OK;
+}
+
 // element-wise models of a fused call, already validated
 struct InjSpec {
   int n = 0;
@@ -180,7 +324,9 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
                            uint64_t* hist, peat_stream_t stream, const InjSpec* inj = nullptr) {
   if (!h) return PEAT_ERR_INVALID_ARG;
   int B = dtype_bytes(dtype);
-  if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
+  const bool f8 = is_fp8(dtype);
+  if (!B && !f8) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be one of peat_dtype_t");
+  if (f8 && inj) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   float rtol, atol;
   if (!round_tol(tol, &rtol, &atol))
     return fail(h, PEAT_ERR_INVALID_ARG, "rtol and atol must be finite and >= 0 after rounding to float32");
@@ -203,6 +349,7 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   DeviceGuard dg(h->device);
   if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (f8) return compare8_impl(h, g, c, offsets, nseg, dtype, rtol, atol, stats, hist, st);
 
   peat::CompareParams p;
   std::memset(&p, 0, sizeof(p));
@@ -445,6 +592,8 @@ peat_status_t peat_signature_destroy(peat_handle_t h) {
     if (h->d_single) cudaFree(h->d_single);
     if (h->d_inj) cudaFree(h->d_inj);
     if (h->h_inj) cudaFreeHost(h->h_inj);
+    if (h->d_f8) cudaFree(h->d_f8);
+    if (h->h_f8) cudaFreeHost(h->h_f8);
     if (h->topk) cudaFree(h->topk);
     if (h->topk_list) cudaFree(h->topk_list);
     if (h->tsacc) cudaFree(h->tsacc);
@@ -475,6 +624,7 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
                              peat_dtype_t dtype, uint64_t num, uint64_t den, peat_topk_t* out,
                              peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
+  if (is_fp8(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   const int B = dtype_bytes(dtype);
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
   if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
@@ -521,8 +671,8 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
                                 peat_dtype_t dtype, const double* rtols, int nr, const double* atols, int na,
                                 uint64_t* counts_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
-  const int B = dtype_bytes(dtype);
-  if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
+  const int B = is_fp8(dtype) ? 1 : dtype_bytes(dtype);
+  if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be one of peat_dtype_t");
   if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
   if (n > 0 && (!golden || !candidate)) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
   if (!rtols || !atols || !counts_out) return fail(h, PEAT_ERR_INVALID_ARG, "rtols/atols/counts_out is NULL");
@@ -582,6 +732,7 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
 peat_status_t peat_tensor_stats(peat_handle_t h, const void* x, const int64_t* offsets, int64_t nseg,
                                 peat_dtype_t dtype, peat_tstats_t* stats_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
+  if (is_fp8(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   const int B = dtype_bytes(dtype);
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
   if (nseg < 0) return fail(h, PEAT_ERR_INVALID_ARG, "nseg < 0");
@@ -727,6 +878,7 @@ peat_status_t peat_inject_compare(peat_handle_t h, const void* golden, int64_t n
                                   const peat_inject_t* models, int nmodels, uint64_t seed, peat_tol_t tol,
                                   peat_stats_t* stats_out, uint64_t* hist_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
+  if (is_fp8(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   if (!dtype_bytes(dtype)) return fail(h, PEAT_ERR_INVALID_ARG, "bad dtype");
   if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
   if (nmodels < 1 || nmodels > peat::INJ_MAX) return fail(h, PEAT_ERR_INVALID_ARG, "nmodels outside [1, 8]");
@@ -761,6 +913,7 @@ peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* s
                                        peat_dtype_t dtype, const peat_inject_t* models, int nmodels,
                                        uint64_t seed, uint64_t* counts_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
+  if (is_fp8(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   int B = dtype_bytes(dtype);
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "bad dtype");
   if (n < 0 || nmodels < 0 || nmodels > 64) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0 or nmodels outside [0, 64]");
@@ -895,6 +1048,7 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
                                    peat_stream_t stream) {
   g_null_error_is_noalloc = true;
   g_noalloc_error[0] = 0;
+  if (is_fp8(dtype)) return noalloc_fail(PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   const int B = dtype_bytes(dtype);
   if (!B) return noalloc_fail(PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
   float rtol, atol;

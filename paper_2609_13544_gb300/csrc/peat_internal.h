@@ -187,6 +187,37 @@ struct IscParams {
 };
 cudaError_t launch_isclose(int dtype, const IscParams& p, int nctas, cudaStream_t s);
 
+// 8-bit formats: one item's totals (sums in units of 2^-S, 2^-2S)
+struct Part8 {
+  unsigned long long cnt[PEAT_NCLASS], nfin;
+  unsigned long long s1lo, s1hi, s2lo, s2hi, sdlo, sdhi;
+  unsigned long long ma;
+  long long ia;
+  unsigned long long ra, rb;
+  long long ir;
+  unsigned long long mu;
+  long long iu;
+};
+struct Cmp8Params {
+  const void* g;
+  const void* c;
+  const int64_t* offsets;    // nseg + 1
+  const int64_t* item_b;     // work items: [item_b, item_e) within segment item_seg
+  const int64_t* item_e;
+  const int64_t* item_seg;
+  const int64_t* seg_first;  // items of segment s: [seg_first[s], seg_first[s + 1])
+  int64_t nitems, nseg;
+  float rtol, atol;
+  // amax[m]: the largest |c - g| 2^S the tolerance accepts for a golden of magnitude bits m,
+  // floor(rtol |g| 2^S + atol 2^S) (2^40 when it exceeds every possible difference)
+  unsigned long long amax[128];
+  int vec;                   // both bases 16-byte aligned
+  Part8* parts;              // nitems
+  peat_stats_t* stats;       // nseg
+  unsigned long long* hist;  // nseg x 128, zero before the launch; NULL: none
+};
+cudaError_t launch_compare8(int dtype, const Cmp8Params& p, int nctas, cudaStream_t s);
+
 struct InjectElemParams {
   void* dst;
   const void* src;

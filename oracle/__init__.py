@@ -18,8 +18,8 @@ import numpy as np
 
 from .build import LIB, build
 
-DTYPES = {"f32": 0, "f16": 1, "bf16": 2, "f8e4m3": 3, "f8e5m2": 4}
-ITEMSIZE = {"f32": 4, "f16": 2, "bf16": 2, "f8e4m3": 1, "f8e5m2": 1}
+DTYPES = {"f32": 0, "f16": 1, "bf16": 2, "f8e4m3": 3, "f8e5m2": 4, "f64": 5}
+ITEMSIZE = {"f32": 4, "f16": 2, "bf16": 2, "f8e4m3": 1, "f8e5m2": 1, "f64": 8}
 CLASSES = ("exact", "within_tol", "mismatch", "nan_inf_asym", "sign_flip")
 INJECT_KINDS = {
     "rz": 0, "rv": 1, "bitflip": 2, "nan_inf": 3, "signflip": 4, "rel_gauss": 5,
@@ -57,7 +57,7 @@ class TopK(ctypes.Structure):
     ]
 
 
-ACC_WORDS, ACC_LSB = 24, -768
+ACC_WORDS, ACC_LSB = 72, -2304
 
 
 class TStats(ctypes.Structure):
@@ -100,7 +100,7 @@ def lib() -> ctypes.CDLL:
         L.orc_topk_mean.restype = i32
         L.orc_tensor_stats.argtypes = [vp, i64, i32, ctypes.POINTER(TStats)]
         L.orc_tensor_stats.restype = i32
-        L.orc_ulp_key.argtypes = [ctypes.c_uint32, i32]
+        L.orc_ulp_key.argtypes = [ctypes.c_uint64, i32]
         L.orc_ulp_key.restype = i64
         L.orc_exact_sum.argtypes = [vp, i64]
         L.orc_exact_sum.restype = dbl
@@ -128,11 +128,11 @@ def _bits(x, dtype: str) -> np.ndarray:
     if hasattr(x, "detach"):  # a CPU torch tensor (bf16 and fp8 have no numpy dtype)
         import torch
         x = x.detach().cpu().contiguous()
-        x = x.view({4: torch.int32, 2: torch.int16, 1: torch.uint8}[size]).numpy()
+        x = x.view({8: torch.int64, 4: torch.int32, 2: torch.int16, 1: torch.uint8}[size]).numpy()
     x = np.ascontiguousarray(x)
     if x.dtype.itemsize != size:
         raise ValueError(f"{dtype} needs {size}-byte elements, got {x.dtype}")
-    return x.reshape(-1).view({4: np.uint32, 2: np.uint16, 1: np.uint8}[size])
+    return x.reshape(-1).view({8: np.uint64, 4: np.uint32, 2: np.uint16, 1: np.uint8}[size])
 
 
 def _stats_dict(s: Stats) -> dict:

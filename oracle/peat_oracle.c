@@ -43,6 +43,7 @@
  */
 #include "peat_oracle.h"
 
+#include <float.h>
 #include <math.h>
 #include <stdlib.h>
 #include <string.h>
@@ -50,11 +51,12 @@
 /* ------------------------------------------------------------------------ */
 /* Exact fixed-point accumulator (Kulisch's long accumulator): a two's       */
 /* complement integer of ACC_W 64-bit words whose bit 0 weighs 2^ACC_LSB.    */
-/* Every double, and every product of two doubles, that occurs here lies in  */
-/* [2^-700, 2^700], far inside the range.                                    */
+/* It holds every double (down to 2^-1074), every product of two doubles     */
+/* (down to 2^-2148, up to 2^2048 with the factor 4 of a scaled difference)  */
+/* and sums of up to 2^60 such products.                                     */
 /* ------------------------------------------------------------------------ */
-#define ACC_W 24
-#define ACC_LSB (-768)
+#define ACC_W ORC_ACC_WORDS
+#define ACC_LSB ORC_ACC_LSB
 
 typedef struct {
   uint64_t w[ACC_W];
@@ -154,13 +156,16 @@ static double acc_to_double(const acc_t* in) {
   for (int j = ACC_W - 1; j >= 0 && top < 0; j--)
     if (a.w[j]) top = j * 64 + 63 - __builtin_clzll(a.w[j]);
   if (top < 0) return 0.0;
+  /* the last kept bit: 53 significant bits, but none below 2^-1074 */
+  int low = top - 52;
+  if (low + ACC_LSB < -1074) low = -1074 - ACC_LSB;
   uint64_t mant = 0;
-  for (int k = top; k > top - 53; k--) mant = (mant << 1) | (uint64_t)acc_bit(&a, k);
-  int round = acc_bit(&a, top - 53);
+  for (int k = top; k >= low; k--) mant = (mant << 1) | (uint64_t)acc_bit(&a, k);
+  int round = acc_bit(&a, low - 1);
   int sticky = 0;
-  for (int k = top - 54; k >= 0 && !sticky; k--) sticky = acc_bit(&a, k);
+  for (int k = low - 2; k >= 0 && !sticky; k--) sticky = acc_bit(&a, k);
   if (round && (sticky || (mant & 1u))) mant++;
-  double r = ldexp((double)mant, top - 52 + ACC_LSB);
+  double r = ldexp((double)mant, low + ACC_LSB); /* +inf past the largest double */
   return neg ? -r : r;
 }
 
@@ -199,10 +204,15 @@ double orc_exact_dot(const double* x, const double* y, int64_t n) {
 typedef struct {
   int nan, inf, sign;
   double v;     /* exact value when finite (signed; -0.0 for negative zero) */
-  uint32_t mag; /* bit pattern without the sign bit */
+  uint64_t mag; /* bit pattern without the sign bit */
 } val_t;
 
-static uint32_t raw_bits(const void* base, int64_t i, int dtype) {
+static uint64_t raw_bits(const void* base, int64_t i, int dtype) {
+  if (dtype == ORC_F64) {
+    uint64_t b;
+    memcpy(&b, (const char*)base + 8 * i, 8);
+    return b;
+  }
   if (dtype == ORC_F32) {
     uint32_t b;
     memcpy(&b, (const char*)base + 4 * i, 4);
@@ -214,11 +224,13 @@ static uint32_t raw_bits(const void* base, int64_t i, int dtype) {
   return h;
 }
 
-static val_t decode(uint32_t b, int dtype) {
+static val_t decode(uint64_t b, int dtype) {
   val_t r;
   memset(&r, 0, sizeof(r));
   int sbit, ebits, mbits, bias;
-  if (dtype == ORC_F32) {
+  if (dtype == ORC_F64) {
+    sbit = 63, ebits = 11, mbits = 52, bias = 1023;
+  } else if (dtype == ORC_F32) {
     sbit = 31, ebits = 8, mbits = 23, bias = 127;
   } else if (dtype == ORC_F16) {
     sbit = 15, ebits = 5, mbits = 10, bias = 15;
@@ -230,9 +242,9 @@ static val_t decode(uint32_t b, int dtype) {
     sbit = 7, ebits = 4, mbits = 3, bias = 7;
   }
   r.sign = (int)((b >> sbit) & 1u);
-  r.mag = b & ((1u << sbit) - 1u);
-  uint32_t e = r.mag >> mbits, m = r.mag & ((1u << mbits) - 1u);
-  uint32_t emax = (1u << ebits) - 1u;
+  r.mag = b & ((1ull << sbit) - 1u);
+  uint64_t e = r.mag >> mbits, m = r.mag & ((1ull << mbits) - 1u);
+  uint64_t emax = (1ull << ebits) - 1u;
   if (dtype == ORC_F8E4M3) {
     if (r.mag == 0x7Fu) { /* the only NaN; the rest of the top binade is finite */
       r.nan = 1;
@@ -247,12 +259,12 @@ static val_t decode(uint32_t b, int dtype) {
   if (e == 0)
     x = ldexp((double)m, 1 - bias - mbits); /* subnormal */
   else
-    x = ldexp((double)(m | (1u << mbits)), (int)e - bias - mbits);
+    x = ldexp((double)(m | (1ull << mbits)), (int)e - bias - mbits);
   r.v = r.sign ? -x : x;
   return r;
 }
 
-int64_t orc_ulp_key(uint32_t bits, int dtype) {
+int64_t orc_ulp_key(uint64_t bits, int dtype) {
   val_t v = decode(bits, dtype);
   return v.sign ? -(int64_t)v.mag : (int64_t)v.mag;
 }
@@ -271,26 +283,42 @@ static void two_sum(double x, double y, double* s, double* t) {
 }
 
 typedef struct {
-  double s, t; /* |d| = s + t exactly, s = RN64(|d|) */
+  double s, t; /* |d| = (s + t) 2^sc exactly, s = RN64(|d| / 2^sc) */
+  int sc;      /* 1 when c - g overflows binary64 (then both were halved), else 0 */
 } mag2_t;
 
-/* sign(a - y) for an exact two-term a and a double y */
-static int cmp_mag_dbl(mag2_t a, double y) {
+/* a += (neg ? -1 : +1) * x * 2^sc and the same for a product */
+static void acc_add_double_sc(acc_t* a, double x, int sc, int neg) {
+  if (x == 0.0) return;
+  int e;
+  uint64_t m = dbl_split(x, &e);
+  acc_add_mag(a, (u128)m, e + sc, neg ^ (x < 0));
+}
+static void acc_add_product_sc(acc_t* a, double x, double y, int sc, int neg) {
+  if (x == 0.0 || y == 0.0) return;
+  int ex, ey;
+  uint64_t mx = dbl_split(x, &ex), my = dbl_split(y, &ey);
+  acc_add_mag(a, (u128)mx * (u128)my, ex + ey + sc, neg ^ (x < 0) ^ (y < 0));
+}
+static void acc_add_mag2(acc_t* x, mag2_t a, int neg) {
+  acc_add_double_sc(x, a.s, a.sc, neg);
+  acc_add_double_sc(x, a.t, a.sc, neg);
+}
+
+/* sign(a - y 2^k) for an exact two-term a and a double y >= 0 */
+static int cmp_mag_dbl_pow2(mag2_t a, double y, int k) {
   acc_t x;
   acc_zero(&x);
-  acc_add_double(&x, a.s, 0);
-  acc_add_double(&x, a.t, 0);
-  acc_add_double(&x, y, 1);
+  acc_add_mag2(&x, a, 0);
+  acc_add_double_sc(&x, y, k, 1);
   return acc_sign(&x);
 }
 
 static int cmp_mag(mag2_t a, mag2_t b) {
   acc_t x;
   acc_zero(&x);
-  acc_add_double(&x, a.s, 0);
-  acc_add_double(&x, a.t, 0);
-  acc_add_double(&x, b.s, 1);
-  acc_add_double(&x, b.t, 1);
+  acc_add_mag2(&x, a, 0);
+  acc_add_mag2(&x, b, 1);
   return acc_sign(&x);
 }
 
@@ -314,17 +342,18 @@ static int cmp_rel(rel_t r1, rel_t r2) {
   if (k1 != 1) return 0;
   acc_t x;
   acc_zero(&x);
-  acc_add_product(&x, r1.a.s, r2.absg, 0);
-  acc_add_product(&x, r1.a.t, r2.absg, 0);
-  acc_add_product(&x, r2.a.s, r1.absg, 1);
-  acc_add_product(&x, r2.a.t, r1.absg, 1);
+  acc_add_product_sc(&x, r1.a.s, r2.absg, r1.a.sc, 0);
+  acc_add_product_sc(&x, r1.a.t, r2.absg, r1.a.sc, 0);
+  acc_add_product_sc(&x, r2.a.s, r1.absg, r2.a.sc, 1);
+  acc_add_product_sc(&x, r2.a.t, r1.absg, r2.a.sc, 1);
   return acc_sign(&x);
 }
 
+/* the last bit of the stored significand (normal or subnormal) */
 static int mant_is_even(double q) {
-  int e;
-  uint64_t m = dbl_split(q, &e);
-  return (m & 1u) == 0;
+  uint64_t b;
+  memcpy(&b, &q, 8);
+  return (b & 1u) == 0;
 }
 
 /* RN64 of a finite positive quotient a/absg: the candidate double with the
@@ -335,17 +364,28 @@ static double rel_value(rel_t r) {
   int k = rel_kind(r);
   if (k == 0) return 0.0;
   if (k == 2) return INFINITY;
-  double q0 = r.a.s / r.absg;
+  /* past the rounding threshold of the largest double, (2^54 - 1) 2^970, the quotient rounds to +inf */
+  {
+    acc_t x;
+    acc_zero(&x);
+    acc_add_mag2(&x, r.a, 0);
+    int eg;
+    uint64_t mg = dbl_split(r.absg, &eg);
+    acc_add_mag(&x, (u128)mg * (((u128)1 << 54) - 1), eg + 970, 1);
+    if (acc_sign(&x) >= 0) return INFINITY;
+  }
+  double q0 = ldexp(r.a.s / r.absg, r.a.sc);
+  if (!(q0 <= DBL_MAX)) q0 = DBL_MAX;
   double best = 0.0;
   acc_t best_res;
   int have = 0;
   double q = q0;
   for (int i = 0; i < 4; i++) q = nextafter(q, 0.0);
   for (int step = 0; step < 9; step++, q = nextafter(q, INFINITY)) {
+    if (isinf(q)) break;
     acc_t res;
     acc_zero(&res);
-    acc_add_double(&res, r.a.s, 0);
-    acc_add_double(&res, r.a.t, 0);
+    acc_add_mag2(&res, r.a, 0);
     acc_add_product(&res, q, r.absg, 1);
     if (!have) {
       best = q, best_res = res, have = 1;
@@ -360,9 +400,9 @@ static double rel_value(rel_t r) {
 /* floor(log2(a/absg)) for a > 0, absg > 0: the integer k with
  * absg*2^k <= a < absg*2^(k+1), found from an estimate by exact comparisons */
 static int rel_log2_floor(mag2_t a, double absg) {
-  int k = ilogb(a.s) - ilogb(absg);
-  while (cmp_mag_dbl(a, ldexp(absg, k)) < 0) k--;
-  while (cmp_mag_dbl(a, ldexp(absg, k + 1)) >= 0) k++;
+  int k = ilogb(a.s) + a.sc - ilogb(absg);
+  while (cmp_mag_dbl_pow2(a, absg, k) < 0) k--;
+  while (cmp_mag_dbl_pow2(a, absg, k + 1) >= 0) k++;
   return k;
 }
 
@@ -393,8 +433,8 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
   acc_zero(&s_signed);
 
   int have_abs = 0, have_rel = 0, have_ulp = 0;
-  mag2_t best_abs = {0.0, 0.0};
-  rel_t best_rel = {{0.0, 0.0}, 0.0};
+  mag2_t best_abs = {0.0, 0.0, 0};
+  rel_t best_rel = {{0.0, 0.0, 0}, 0.0};
   uint64_t best_ulp = 0;
 
   for (int64_t i = 0; i < n; i++) {
@@ -405,7 +445,8 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
     int ulp_defined = !g.nan && !c.nan;
     int64_t kg = g.sign ? -(int64_t)g.mag : (int64_t)g.mag;
     int64_t kc = c.sign ? -(int64_t)c.mag : (int64_t)c.mag;
-    uint64_t u = (uint64_t)(kc > kg ? kc - kg : kg - kc);
+    /* |kc - kg| < 2^64: the unsigned difference is exact */
+    uint64_t u = kc >= kg ? (uint64_t)kc - (uint64_t)kg : (uint64_t)kg - (uint64_t)kc;
 
     if (!gfin || !cfin) {
       int equal = (g.nan && c.nan) || (g.inf && c.inf && g.sign == c.sign);
@@ -418,8 +459,13 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
     } else {
       st->n_finite++;
       double s, t;
+      int sc = 0;
       two_sum(c.v, -g.v, &s, &t); /* d = c - g = s + t exactly */
-      mag2_t a = (s < 0.0) ? (mag2_t){-s, -t} : (mag2_t){s, t};
+      if (!isfinite(s)) {           /* binary64 operands whose difference overflows: */
+        two_sum(0.5 * c.v, -0.5 * g.v, &s, &t); /* halving is exact at that size */
+        sc = 1;
+      }
+      mag2_t a = (s < 0.0) ? (mag2_t){-s, -t, sc} : (mag2_t){s, t, sc};
       double absg = fabs(g.v);
 
       /* classification, in precedence order */
@@ -428,8 +474,7 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
       } else {
         acc_t x; /* a - (atol + rtol*|g|) */
         acc_zero(&x);
-        acc_add_double(&x, a.s, 0);
-        acc_add_double(&x, a.t, 0);
+        acc_add_mag2(&x, a, 0);
         acc_add_double(&x, atol, 1);
         acc_add_product(&x, rtol, absg, 1);
         if (acc_sign(&x) <= 0)
@@ -464,15 +509,14 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
         have_rel = 1;
       }
 
-      /* exact sums: d, |d| and d^2 = s^2 + 2st + t^2 */
-      acc_add_double(&s_signed, s, 0);
-      acc_add_double(&s_signed, t, 0);
-      acc_add_double(&s_abs, a.s, 0);
-      acc_add_double(&s_abs, a.t, 0);
-      acc_add_product(&s_sq, s, s, 0);
-      acc_add_product(&s_sq, s, t, 0);
-      acc_add_product(&s_sq, s, t, 0);
-      acc_add_product(&s_sq, t, t, 0);
+      /* exact sums: d, |d| and d^2 = (s^2 + 2st + t^2) 4^sc */
+      acc_add_double_sc(&s_signed, s, sc, 0);
+      acc_add_double_sc(&s_signed, t, sc, 0);
+      acc_add_mag2(&s_abs, a, 0);
+      acc_add_product_sc(&s_sq, s, s, 2 * sc, 0);
+      acc_add_product_sc(&s_sq, s, t, 2 * sc, 0);
+      acc_add_product_sc(&s_sq, s, t, 2 * sc, 0);
+      acc_add_product_sc(&s_sq, t, t, 2 * sc, 0);
     }
 
     if (ulp_defined && (!have_ulp || u > best_ulp)) {
@@ -488,8 +532,7 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
   if (have_abs) {
     acc_t x;
     acc_zero(&x);
-    acc_add_double(&x, best_abs.s, 0);
-    acc_add_double(&x, best_abs.t, 0);
+    acc_add_mag2(&x, best_abs, 0);
     st->max_abs = acc_to_double(&x);
   }
   if (have_rel) st->max_rel = rel_value(best_rel);
@@ -501,9 +544,11 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
 
 static int dtype_ok(int dtype) { return dtype == ORC_F32 || dtype == ORC_F16 || dtype == ORC_BF16; }
 /* the compare (and the isclose grid built on it) also takes the 8-bit formats */
-static int dtype_ok_cmp(int dtype) { return dtype_ok(dtype) || dtype == ORC_F8E4M3 || dtype == ORC_F8E5M2; }
+static int dtype_ok_cmp(int dtype) {
+  return dtype_ok(dtype) || dtype == ORC_F8E4M3 || dtype == ORC_F8E5M2 || dtype == ORC_F64;
+}
 static int dtype_size(int dtype) {
-  return dtype == ORC_F32 ? 4 : (dtype == ORC_F16 || dtype == ORC_BF16 ? 2 : 1);
+  return dtype == ORC_F64 ? 8 : dtype == ORC_F32 ? 4 : (dtype == ORC_F16 || dtype == ORC_BF16 ? 2 : 1);
 }
 
 int orc_compare(const void* g, const void* c, int64_t n, int dtype, double rtol, double atol,
@@ -587,6 +632,7 @@ int orc_topk_mean(const void* g, const void* c, int64_t n, int dtype, uint64_t n
     two_sum(vc.v, -vg.v, &s, &t); /* d = s + t exactly */
     m[nf].s = fabs(s);
     m[nf].t = s < 0 ? -t : t;     /* |d| = |s| + (sign of s) t */
+    m[nf].sc = 0;                 /* these element types never overflow binary64 */
     nf++;
   }
   out->n_finite = nf;

@@ -24,7 +24,7 @@ extern "C" {
 #endif
 
 /* element types (codes agree with the library's dtype codes) */
-enum { ORC_F32 = 0, ORC_F16 = 1, ORC_BF16 = 2, ORC_F8E4M3 = 3, ORC_F8E5M2 = 4 };
+enum { ORC_F32 = 0, ORC_F16 = 1, ORC_BF16 = 2, ORC_F8E4M3 = 3, ORC_F8E5M2 = 4, ORC_F64 = 5 };
 
 /* classes, in the order of the library's class counters */
 enum { ORC_EXACT = 0, ORC_WITHIN_TOL = 1, ORC_MISMATCH = 2, ORC_NAN_INF_ASYM = 3,
@@ -83,8 +83,8 @@ int orc_topk_mean(const void* g, const void* c, int64_t n, int dtype, uint64_t n
  * ORC_ACC_WORDS little-endian 64-bit words, least significant bit
  * 2^ORC_ACC_LSB), from which the caller forms the mean and the variance
  * exactly. */
-#define ORC_ACC_WORDS 24
-#define ORC_ACC_LSB (-768)
+#define ORC_ACC_WORDS 72
+#define ORC_ACC_LSB (-2304)
 typedef struct {
   uint64_t n, n_finite, n_nan, n_inf;
   double min, max;  /* finite extremes (0 if none) */
@@ -96,7 +96,7 @@ int orc_tensor_stats(const void* x, int64_t n, int dtype, orc_tstats* out);
 
 /* ULP key of one raw bit pattern: +magnitude bits, negated when the sign
  * bit is set (so both zeros map to 0).  Exposed for the tests. */
-int64_t orc_ulp_key(uint32_t bits, int dtype);
+int64_t orc_ulp_key(uint64_t bits, int dtype);
 
 /* RN-even double of an exact rational sum of doubles, exposed so the tests
  * can check the exact accumulator against Python's exact integers:

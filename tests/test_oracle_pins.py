@@ -20,7 +20,8 @@ import torch
 
 GOLD = json.loads((Path(__file__).parent / "golden" / "hand_cases.json").read_text())
 CLASS_IDX = {"exact": 0, "within_tol": 1, "mismatch": 2, "nan_inf_asym": 3, "sign_flip": 4}
-NP_BITS = {"f32": np.uint32, "f16": np.uint16, "bf16": np.uint16, "f8e4m3": np.uint8, "f8e5m2": np.uint8}
+NP_BITS = {"f32": np.uint32, "f16": np.uint16, "bf16": np.uint16, "f8e4m3": np.uint8, "f8e5m2": np.uint8,
+           "f64": np.uint64}
 FP8 = {"f8e4m3": "float8_e4m3fn", "f8e5m2": "float8_e5m2"}
 _FP8_TABLE = {}
 
@@ -42,11 +43,13 @@ def decode(bits: int, dtype: str) -> float:
         return float(np.array([bits], np.uint16).view(np.float16)[0])
     if dtype in FP8:
         return fp8_table(dtype)[bits]
+    if dtype == "f64":
+        return float(np.array([bits], np.uint64).view(np.float64)[0])
     return float(np.array([bits << 16], np.uint32).view(np.float32)[0])
 
 
 def signbit(bits: int, dtype: str) -> int:
-    return (bits >> {"f32": 31, "f8e4m3": 7, "f8e5m2": 7}.get(dtype, 15)) & 1
+    return (bits >> {"f32": 31, "f8e4m3": 7, "f8e5m2": 7, "f64": 63}.get(dtype, 15)) & 1
 
 
 def rn32(x: float) -> float:
@@ -202,6 +205,112 @@ def test_fp8_every_pair_against_exact_rationals(oracle, dtype, tol):
             assert st["sum_signed"] == float(ref["d"]) and st["sum_abs"] == float(ref["a"])
             assert st["sum_sq"] == float(ref["d"] ** 2) and st["max_abs"] == float(ref["a"])
             assert st["max_rel"] == (math.inf if ref["rel"] is None else float(ref["rel"]))
+
+
+# ---------------------------------------------------------------- binary64
+def rn64(q: Fraction) -> float:
+    """Round-to-nearest binary64 of an exact rational, +-inf past the largest double."""
+    try:
+        return float(q)
+    except OverflowError:  # the rounded value is past the largest double
+        return math.inf if q > 0 else -math.inf
+
+
+def _random_f64_pairs(n, rng):
+    """Mixture: relative noise, one-ULP neighbours, arbitrary patterns, sign flips,
+    zeros, subnormals, and operands near the largest double (the difference overflows)."""
+    g = (rng.standard_normal(n) * np.exp2(rng.integers(-60, 60, n))).astype(np.float64)
+    c = g * (1 + 1e-12 * rng.standard_normal(n))
+    kind = rng.integers(0, 9, n)
+    gb, cb = g.view(np.uint64).copy(), c.view(np.uint64).copy()
+    cb = np.where(kind == 0, gb + rng.integers(-3, 4, n).astype(np.int64).astype(np.uint64), cb)
+    cb = np.where(kind == 1, rng.integers(0, 2 ** 63, n, dtype=np.uint64) * np.uint64(2)
+                  + rng.integers(0, 2, n, dtype=np.uint64), cb)
+    cb = np.where(kind == 2, gb ^ np.uint64(1 << 63), cb)
+    cb = np.where(kind == 3, np.uint64(0), cb)
+    sub = rng.integers(0, 1 << 52, n, dtype=np.uint64)
+    gb = np.where(kind == 4, sub, gb)
+    cb = np.where(kind == 4, sub + rng.integers(0, 5, n, dtype=np.uint64), cb)
+    big = np.float64(1.7e308)
+    gb = np.where(kind == 5, np.array([-big]).view(np.uint64)[0], gb)
+    cb = np.where(kind == 5, (big * (1 - 1e-3 * rng.random(n))).view(np.uint64), cb)
+    cb = np.where(kind == 6, gb, cb)
+    return gb.astype(np.uint64), cb.astype(np.uint64)
+
+
+def test_f64_ulp_key_successor(oracle):
+    rng = np.random.default_rng(64)
+    x = (rng.standard_normal(3000) * np.exp2(rng.integers(-1000, 1000, 3000))).astype(np.float64)
+    x = np.concatenate([x, [0.0, 5e-324, -5e-324, 2.2250738585072014e-308, 1.7976931348623157e308]])
+    with np.errstate(over="ignore"):  # the largest double steps to +inf, one key further
+        up = np.nextafter(x, np.inf)
+    for a, b in zip(x.view(np.uint64), up.view(np.uint64)):
+        assert oracle.ulp_key(int(b), "f64") == oracle.ulp_key(int(a), "f64") + 1, hex(int(a))
+    assert oracle.ulp_key(0, "f64") == oracle.ulp_key(1 << 63, "f64") == 0
+    inf = int(np.array([np.inf]).view(np.uint64)[0])
+    assert oracle.ulp_key(inf, "f64") == oracle.ulp_key(0x7FEFFFFFFFFFFFFF, "f64") + 1
+
+
+def test_f64_per_pair_against_exact_rationals(oracle):
+    rng = np.random.default_rng(641)
+    g, c = _random_f64_pairs(2500, rng)
+    rtol, atol = 1e-9, 1e-300
+    stats, hist = oracle.compare_segmented(g, c, np.arange(g.size + 1), "f64", rtol, atol)
+    for i in range(g.size):
+        ref = ref_pair(int(g[i]), int(c[i]), "f64", rtol, atol)
+        st = stats[i]
+        assert st["count"][ref["cls"]] == 1, (i, hex(g[i]), hex(c[i]), ref, st["count"])
+        assert hist[i][0][ref["relbin"]] == 1, (i, ref["relbin"], np.nonzero(hist[i][0]))
+        if ref["finite"]:
+            assert st["sum_signed"] == rn64(ref["d"]) and st["sum_abs"] == rn64(ref["a"])
+            assert st["sum_sq"] == rn64(ref["d"] ** 2) and st["max_abs"] == rn64(ref["a"])
+            assert st["max_rel"] == (math.inf if ref["rel"] is None else rn64(ref["rel"])), (hex(g[i]), hex(c[i]))
+
+
+def test_f64_aggregate_against_exact_rationals(oracle):
+    rng = np.random.default_rng(642)
+    g, c = _random_f64_pairs(1500, rng)
+    g[900], c[900] = g[400], c[400]  # a tie for the maxima
+    st, hist = oracle.compare(g, c, "f64", 1e-6, 0.0)
+    S0 = S1 = S2 = Fraction(0)
+    best_a = best_r = None
+    ia = ir = -1
+    for i in range(g.size):
+        ref = ref_pair(int(g[i]), int(c[i]), "f64", 1e-6, 0.0)
+        if not ref["finite"]:
+            continue
+        S0 += ref["d"]
+        S1 += ref["a"]
+        S2 += ref["d"] ** 2
+        if best_a is None or ref["a"] > best_a:
+            best_a, ia = ref["a"], i
+        r = ref["rel"] if ref["rel"] is not None else math.inf
+        if best_r is None or r > best_r:
+            best_r, ir = r, i
+    assert (st["sum_signed"], st["sum_abs"], st["sum_sq"]) == (rn64(S0), rn64(S1), rn64(S2))
+    assert st["argmax_abs"] == ia and st["max_abs"] == rn64(best_a)
+    assert st["argmax_rel"] == ir
+    assert st["max_rel"] == (math.inf if best_r == math.inf else rn64(best_r))
+
+
+def test_f64_range_edges(oracle):
+    """Differences past the largest double, subnormal sums that round, and a
+    quotient past the rounding threshold of the largest double."""
+    big, tiny = 1.7976931348623157e308, 5e-324
+    g = np.array([-big, 0.0, tiny, 2 * tiny, 1e-300], np.float64)
+    c = np.array([big, 3 * tiny, 0.0, 0.0, 1e10], np.float64)
+    st, _ = oracle.compare(g, c, "f64", 0.0, 0.0)
+    d = [Fraction(float(b)) - Fraction(float(a)) for a, b in zip(g, c)]
+    assert st["max_abs"] == math.inf and st["argmax_abs"] == 0     # 2 * big rounds past the largest double
+    assert st["sum_signed"] == rn64(sum(d)) == math.inf
+    assert st["sum_sq"] == rn64(sum(x * x for x in d)) == math.inf
+    st, _ = oracle.compare(g[1:4], c[1:4], "f64", 0.0, 0.0)
+    dd = [Fraction(float(b)) - Fraction(float(a)) for a, b in zip(g[1:4], c[1:4])]
+    assert st["sum_sq"] == rn64(sum(x * x for x in dd)) == 0.0       # squares far below the smallest subnormal
+    assert st["sum_abs"] == rn64(sum(abs(x) for x in dd)) == 6 * tiny
+    assert st["max_rel"] == math.inf                                # g = 0 < |d|
+    st, _ = oracle.compare(g[4:], c[4:], "f64", 0.0, 0.0)
+    assert st["max_rel"] == math.inf                                # 1e10 / 1e-300 rounds past the largest double
 
 
 # ---------------------------------------------------------------- exact rationals on random pairs

@@ -443,6 +443,33 @@ def run_gpu(args) -> None:
         del x, y
         fp8 = {"op": "peat_compare on 8-bit golden and candidate (rtol 1/8)", "calls": calls, **fp8}
 
+    # binary64 (Fig. 5's FP32-FP64 pairs): the golden's values plus noise 1e-3 in binary64, against
+    # their float32 rounding widened back to binary64; one read of both 8-byte tensors
+    f64 = None
+    if w.offsets is None and not args.no_topk:
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(19)
+        g64 = g.double() + 1e-3 * torch.randn(g.shape, generator=gen, device=dev, dtype=torch.float64)
+        c64 = g64.float().double()
+        for _ in range(3):
+            peat.peat_compare_raw(h, g64, c64, 1e-7, 0.0, stats, hist, stream)
+        barrier()
+        calls = max(3, min(20, args.steps // 200))
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(calls):
+            peat.peat_compare_raw(h, g64, c64, 1e-7, 0.0, stats, hist, stream)
+        t1.record(stream)
+        barrier()
+        ms = max_over_ranks(t0.elapsed_time(t1), dev) / calls
+        gbs64 = 16 * w.n / (ms * 1e-3) / 1e9
+        f64 = {"op": "peat_compare on binary64 golden and its float32 rounding (rtol 1e-7)", "calls": calls,
+               "us_per_call": ms * 1e3, "pairs_per_s": w.n / (ms * 1e-3),
+               "roofline": {"bound": "alu", "achieved": gbs64, "peak": peak, "unit": "GB/s", "frac": gbs64 / peak,
+                            "algorithmic_bytes_per_call": 16 * w.n,
+                            "note": "FP64 TwoSum per pair and the three sums as digit atomics in shared memory"}}
+        del g64, c64
+
     # end to end through the C ABI with host buffers: every step copies both
     # tensors from pinned host memory, compares them and reads the stats and
     # histograms back.  Two device buffer sets: step i's copies (copy stream)
@@ -531,7 +558,7 @@ def run_gpu(args) -> None:
                          else "fallback 6.8 TB/s"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": (1 if nseg == 1 else 2) * args.steps, "clocks": clocks,
             "next_rows": {"f1_top10_mean": topk, "f2_fused_inject_compare": fused, "f3_context_stats": tstats,
-                          "f4_isclose_grid": isc, "f4_fp8_compare": fp8},
+                          "f4_isclose_grid": isc, "f4_fp8_compare": fp8, "f4_f64_compare": f64},
             "wall_s_timed": wall,
         }
         print(json.dumps(line), flush=True)

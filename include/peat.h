@@ -62,9 +62,19 @@ typedef struct CUstream_st* peat_stream_t;
 /* Element types.  The 8-bit ones are the OCP FP8 formats: E4M3 ("fn": exponent
  * bias 7, no infinities, S.1111.111 the only NaN, 448 the largest value) and
  * E5M2 (bias 15, IEEE-like infinities and NaNs); peat_compare,
- * peat_compare_segmented and peat_isclose_grid take them, the other entry
- * points return PEAT_ERR_UNSUPPORTED. */
-typedef enum { PEAT_F32 = 0, PEAT_F16 = 1, PEAT_BF16 = 2, PEAT_F8E4M3 = 3, PEAT_F8E5M2 = 4 } peat_dtype_t;
+ * peat_compare_segmented and peat_isclose_grid take them.  PEAT_F64
+ * (IEEE binary64, e.g. a float32 output widened exactly to compare with a
+ * binary64 one) is taken by peat_compare and peat_compare_segmented; its
+ * ULP distance counts binary64 steps and its sums may round to +-inf.  The
+ * other entry points return PEAT_ERR_UNSUPPORTED for these types. */
+typedef enum {
+  PEAT_F32 = 0,
+  PEAT_F16 = 1,
+  PEAT_BF16 = 2,
+  PEAT_F8E4M3 = 3,
+  PEAT_F8E5M2 = 4,
+  PEAT_F64 = 5
+} peat_dtype_t;
 
 typedef enum {
   PEAT_OK = 0,

@@ -172,7 +172,8 @@ def peat_signature_destroy(h: Handle) -> None:
 
 def dtype_code(t) -> int:
     import torch
-    m = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2, torch.float8_e4m3fn: 3, torch.float8_e5m2: 4}
+    m = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2, torch.float8_e4m3fn: 3, torch.float8_e5m2: 4,
+         torch.float64: 5}
     if t.dtype not in m:
         raise TypeError(f"unsupported dtype {t.dtype}")
     return m[t.dtype]

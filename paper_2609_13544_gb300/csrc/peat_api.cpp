@@ -88,7 +88,10 @@ peat_status_t cuda_fail(peat_handle_t h, cudaError_t e, const char* what) {
 // the element types of the main kernels (the 8-bit formats have their own compare)
 int dtype_bytes(int dt) { return dt == PEAT_F32 ? 4 : (dt == PEAT_F16 || dt == PEAT_BF16 ? 2 : 0); }
 bool is_fp8(int dt) { return dt == PEAT_F8E4M3 || dt == PEAT_F8E5M2; }
-const char* const FP8_ONLY = "8-bit formats: peat_compare, peat_compare_segmented and peat_isclose_grid only";
+// the element types with a compare of their own (and no other entry point but the isclose grid for 8 bits)
+bool own_compare(int dt) { return is_fp8(dt) || dt == PEAT_F64; }
+const char* const FP8_ONLY =
+    "8-bit and binary64 operands: peat_compare and peat_compare_segmented (and peat_isclose_grid for 8 bits) only";
 
 bool round_tol(peat_tol_t tol, float* r, float* a) {
   if (!(tol.rtol >= 0.0) || !(tol.atol >= 0.0)) return false;  // rejects NaN too
@@ -175,6 +178,76 @@ static cudaError_t single_bounds(peat_handle_t h, int dtype, int nctas, int64_t 
   return cudaSuccess;
 }
 
+// Work items for the 8-bit and binary64 compares: runs of at most `ch`
+// elements within one segment (about four per SM for one tensor), staged
+// with the offsets into the handle's workspace, followed by one record of
+// `part_bytes` per item.  Fills the item fields of p (any of the two
+// parameter structs) and returns the device base of the records.
+struct Items {
+  const int64_t *offsets, *item_b, *item_e, *item_seg, *seg_first;
+  int64_t nitems;
+  void* parts;
+};
+static peat_status_t stage_items(peat_handle_t h, const int64_t* offsets, int64_t nseg, size_t part_bytes,
+                                 cudaStream_t st, Items* out) {
+  const int64_t n = offsets[nseg];
+  int64_t ch = (n + 4 * (int64_t)h->nsm - 1) / (4 * (int64_t)h->nsm);
+  ch = std::min<int64_t>(std::max<int64_t>((ch + 15) / 16 * 16, 4096), (int64_t)1 << 22);
+  int64_t nitems = 0;
+  for (int64_t s = 0; s < nseg; s++) nitems += (offsets[s + 1] - offsets[s] + ch - 1) / ch;
+  // staging: offsets (nseg + 1), item_b, item_e, item_seg (nitems each), seg_first (nseg + 1)
+  const size_t nwords = (size_t)(nseg + 1) * 2 + 3 * (size_t)nitems;
+  const size_t hbytes = nwords * sizeof(int64_t);
+  const size_t pbase = (hbytes + 255) / 256 * 256;
+  const size_t dbytes = pbase + (size_t)std::max<int64_t>(nitems, 1) * part_bytes;
+  peat_status_t ps = wait_staging(h);  // the pinned staging is free
+  if (ps != PEAT_OK) return ps;
+  if (hbytes > h->f8_hcap || dbytes > h->f8_dcap) {
+    if (h->h_f8) cudaFreeHost(h->h_f8);
+    if (h->d_f8) cudaFree(h->d_f8);
+    h->h_f8 = nullptr;
+    h->d_f8 = nullptr;
+    h->f8_hcap = h->f8_dcap = 0;
+    const size_t hc = std::max(hbytes, (size_t)65536), dc = std::max(dbytes, (size_t)1 << 20);
+    if (cudaMallocHost(&h->h_f8, hc) != cudaSuccess || cudaMalloc(&h->d_f8, dc) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(h, PEAT_ERR_ALLOC, "compare workspace allocation failed");
+    }
+    h->f8_hcap = hc;
+    h->f8_dcap = dc;
+  }
+  int64_t* ho = h->h_f8;
+  int64_t* hb = ho + (nseg + 1);
+  int64_t* he = hb + nitems;
+  int64_t* hs = he + nitems;
+  int64_t* hf = hs + nitems;
+  std::memcpy(ho, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
+  int64_t it = 0;
+  for (int64_t s = 0; s < nseg; s++) {
+    hf[s] = it;
+    for (int64_t x = offsets[s]; x < offsets[s + 1]; x += ch, it++) {
+      hb[it] = x;
+      he[it] = std::min(offsets[s + 1], x + ch);
+      hs[it] = s;
+    }
+  }
+  hf[nseg] = it;
+  int64_t* d = static_cast<int64_t*>(h->d_f8);
+  cudaError_t e = cudaMemcpyAsync(d, ho, hbytes, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(items)");
+  e = cudaEventRecord(h->staged, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
+  h->staged_pending = true;
+  out->offsets = d;
+  out->item_b = d + (nseg + 1);
+  out->item_e = out->item_b + nitems;
+  out->item_seg = out->item_e + nitems;
+  out->seg_first = out->item_seg + nitems;
+  out->nitems = nitems;
+  out->parts = reinterpret_cast<char*>(h->d_f8) + pbase;
+  return PEAT_OK;
+}
+
 // floor(mx 2^ex + my 2^ey) for mx, my < 2^57, saturated at 2^40.  The
 // fractional parts are added in 128-bit fixed point with unit 2^-120, exact
 // for exponents down to -120; a term below that is under 2^-64 and cannot
@@ -220,58 +293,14 @@ static void split_f32(float x, uint64_t* m, int* e) {
   *e = ex - 24;
 }
 
-// The 8-bit formats: work items of at most `ch` elements within one segment
-// (about four per SM for one tensor), one record each, merged per segment.
+// The 8-bit formats: items of one segment each, one record per item, merged per segment.
 static peat_status_t compare8_impl(peat_handle_t h, const void* g, const void* c, const int64_t* offsets,
                                    int64_t nseg, int dtype, float rtol, float atol, peat_stats_t* stats,
                                    uint64_t* hist, cudaStream_t st) {
-  const int64_t n = offsets[nseg];
-  int64_t ch = (n + 4 * (int64_t)h->nsm - 1) / (4 * (int64_t)h->nsm);
-  ch = std::min<int64_t>(std::max<int64_t>((ch + 15) / 16 * 16, 4096), (int64_t)1 << 22);
-  int64_t nitems = 0;
-  for (int64_t s = 0; s < nseg; s++) nitems += (offsets[s + 1] - offsets[s] + ch - 1) / ch;
-  // staging: offsets (nseg + 1), item_b, item_e, item_seg (nitems each), seg_first (nseg + 1)
-  const size_t nwords = (size_t)(nseg + 1) * 2 + 3 * (size_t)nitems;
-  const size_t hbytes = nwords * sizeof(int64_t);
-  const size_t dbytes = hbytes + (size_t)std::max<int64_t>(nitems, 1) * sizeof(peat::Part8);
-  peat_status_t ps = wait_staging(h);  // the pinned staging is free
+  Items it;
+  peat_status_t ps = stage_items(h, offsets, nseg, sizeof(peat::Part8), st, &it);
   if (ps != PEAT_OK) return ps;
-  if (hbytes > h->f8_hcap || dbytes > h->f8_dcap) {
-    if (h->h_f8) cudaFreeHost(h->h_f8);
-    if (h->d_f8) cudaFree(h->d_f8);
-    h->h_f8 = nullptr;
-    h->d_f8 = nullptr;
-    h->f8_hcap = h->f8_dcap = 0;
-    const size_t hc = std::max(hbytes, (size_t)65536), dc = std::max(dbytes, (size_t)1 << 20);
-    if (cudaMallocHost(&h->h_f8, hc) != cudaSuccess || cudaMalloc(&h->d_f8, dc) != cudaSuccess) {
-      cudaGetLastError();
-      return fail(h, PEAT_ERR_ALLOC, "8-bit compare workspace allocation failed");
-    }
-    h->f8_hcap = hc;
-    h->f8_dcap = dc;
-  }
-  int64_t* ho = h->h_f8;
-  int64_t* hb = ho + (nseg + 1);
-  int64_t* he = hb + nitems;
-  int64_t* hs = he + nitems;
-  int64_t* hf = hs + nitems;
-  std::memcpy(ho, offsets, sizeof(int64_t) * (size_t)(nseg + 1));
-  int64_t it = 0;
-  for (int64_t s = 0; s < nseg; s++) {
-    hf[s] = it;
-    for (int64_t x = offsets[s]; x < offsets[s + 1]; x += ch, it++) {
-      hb[it] = x;
-      he[it] = std::min(offsets[s + 1], x + ch);
-      hs[it] = s;
-    }
-  }
-  hf[nseg] = it;
-  int64_t* d = static_cast<int64_t*>(h->d_f8);
-  cudaError_t e = cudaMemcpyAsync(d, ho, hbytes, cudaMemcpyHostToDevice, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpyAsync(8-bit items)");
-  e = cudaEventRecord(h->staged, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventRecord");
-  h->staged_pending = true;
+  cudaError_t e;
   if (hist) {
     e = cudaMemsetAsync(hist, 0, sizeof(uint64_t) * PEAT_HIST_BINS * (size_t)nseg, st);
     if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemsetAsync(hist)");
@@ -280,12 +309,12 @@ static peat_status_t compare8_impl(peat_handle_t h, const void* g, const void* c
   std::memset(&p, 0, sizeof(p));
   p.g = g;
   p.c = c;
-  p.offsets = d;
-  p.item_b = d + (nseg + 1);
-  p.item_e = p.item_b + nitems;
-  p.item_seg = p.item_e + nitems;
-  p.seg_first = p.item_seg + nitems;
-  p.nitems = nitems;
+  p.offsets = it.offsets;
+  p.item_b = it.item_b;
+  p.item_e = it.item_e;
+  p.item_seg = it.item_seg;
+  p.seg_first = it.seg_first;
+  p.nitems = it.nitems;
   p.nseg = nseg;
   p.rtol = rtol;
   p.atol = atol;
@@ -303,12 +332,47 @@ static peat_status_t compare8_impl(peat_handle_t h, const void* g, const void* c
     }
   }
   p.vec = (reinterpret_cast<uintptr_t>(g) % 16 == 0 && reinterpret_cast<uintptr_t>(c) % 16 == 0) ? 1 : 0;
-  p.parts = reinterpret_cast<peat::Part8*>(reinterpret_cast<char*>(h->d_f8) + hbytes);
+  p.parts = static_cast<peat::Part8*>(it.parts);
   p.stats = stats;
   p.hist = reinterpret_cast<unsigned long long*>(hist);
-  const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>(nitems, 2 * (int64_t)h->nsm));
+  const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>(it.nitems, 2 * (int64_t)h->nsm));
   e = peat::launch_compare8(dtype, p, nctas, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "8-bit compare launch");
+  return PEAT_OK;
+}
+
+// binary64: the same item structure, records with the three sums as digits.
+static peat_status_t compare64_impl(peat_handle_t h, const void* g, const void* c, const int64_t* offsets,
+                                    int64_t nseg, float rtol, float atol, peat_stats_t* stats, uint64_t* hist,
+                                    cudaStream_t st) {
+  Items it;
+  peat_status_t ps = stage_items(h, offsets, nseg, sizeof(peat::Part64), st, &it);
+  if (ps != PEAT_OK) return ps;
+  cudaError_t e;
+  if (hist) {
+    e = cudaMemsetAsync(hist, 0, sizeof(uint64_t) * PEAT_HIST_BINS * (size_t)nseg, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemsetAsync(hist)");
+  }
+  peat::Cmp64Params p;
+  std::memset(&p, 0, sizeof(p));
+  p.g = g;
+  p.c = c;
+  p.offsets = it.offsets;
+  p.item_b = it.item_b;
+  p.item_e = it.item_e;
+  p.item_seg = it.item_seg;
+  p.seg_first = it.seg_first;
+  p.nitems = it.nitems;
+  p.nseg = nseg;
+  p.rtol = (double)rtol;
+  p.atol = (double)atol;
+  p.vec = (reinterpret_cast<uintptr_t>(g) % 16 == 0 && reinterpret_cast<uintptr_t>(c) % 16 == 0) ? 1 : 0;
+  p.parts = static_cast<peat::Part64*>(it.parts);
+  p.stats = stats;
+  p.hist = reinterpret_cast<unsigned long long*>(hist);
+  const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>(it.nitems, 2 * (int64_t)h->nsm));
+  e = peat::launch_compare64(p, nctas, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "binary64 compare launch");
   return PEAT_OK;
 }
 
@@ -324,9 +388,9 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
                            uint64_t* hist, peat_stream_t stream, const InjSpec* inj = nullptr) {
   if (!h) return PEAT_ERR_INVALID_ARG;
   int B = dtype_bytes(dtype);
-  const bool f8 = is_fp8(dtype);
-  if (!B && !f8) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be one of peat_dtype_t");
-  if (f8 && inj) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
+  const bool f8 = is_fp8(dtype), f64 = dtype == PEAT_F64;
+  if (!B && !f8 && !f64) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be one of peat_dtype_t");
+  if ((f8 || f64) && inj) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   float rtol, atol;
   if (!round_tol(tol, &rtol, &atol))
     return fail(h, PEAT_ERR_INVALID_ARG, "rtol and atol must be finite and >= 0 after rounding to float32");
@@ -350,6 +414,7 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (f8) return compare8_impl(h, g, c, offsets, nseg, dtype, rtol, atol, stats, hist, st);
+  if (f64) return compare64_impl(h, g, c, offsets, nseg, rtol, atol, stats, hist, st);
 
   peat::CompareParams p;
   std::memset(&p, 0, sizeof(p));
@@ -624,7 +689,7 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
                              peat_dtype_t dtype, uint64_t num, uint64_t den, peat_topk_t* out,
                              peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
-  if (is_fp8(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
+  if (own_compare(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   const int B = dtype_bytes(dtype);
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
   if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
@@ -671,6 +736,7 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
                                 peat_dtype_t dtype, const double* rtols, int nr, const double* atols, int na,
                                 uint64_t* counts_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
+  if (dtype == PEAT_F64) return fail(h, PEAT_ERR_UNSUPPORTED, "binary64 operands: peat_compare only");
   const int B = is_fp8(dtype) ? 1 : dtype_bytes(dtype);
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be one of peat_dtype_t");
   if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
@@ -732,7 +798,7 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
 peat_status_t peat_tensor_stats(peat_handle_t h, const void* x, const int64_t* offsets, int64_t nseg,
                                 peat_dtype_t dtype, peat_tstats_t* stats_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
-  if (is_fp8(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
+  if (own_compare(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   const int B = dtype_bytes(dtype);
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
   if (nseg < 0) return fail(h, PEAT_ERR_INVALID_ARG, "nseg < 0");
@@ -878,7 +944,7 @@ peat_status_t peat_inject_compare(peat_handle_t h, const void* golden, int64_t n
                                   const peat_inject_t* models, int nmodels, uint64_t seed, peat_tol_t tol,
                                   peat_stats_t* stats_out, uint64_t* hist_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
-  if (is_fp8(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
+  if (own_compare(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   if (!dtype_bytes(dtype)) return fail(h, PEAT_ERR_INVALID_ARG, "bad dtype");
   if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
   if (nmodels < 1 || nmodels > peat::INJ_MAX) return fail(h, PEAT_ERR_INVALID_ARG, "nmodels outside [1, 8]");
@@ -913,7 +979,7 @@ peat_status_t peat_pseudo_error_inject(peat_handle_t h, void* dst, const void* s
                                        peat_dtype_t dtype, const peat_inject_t* models, int nmodels,
                                        uint64_t seed, uint64_t* counts_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
-  if (is_fp8(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
+  if (own_compare(dtype)) return fail(h, PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   int B = dtype_bytes(dtype);
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "bad dtype");
   if (n < 0 || nmodels < 0 || nmodels > 64) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0 or nmodels outside [0, 64]");
@@ -1048,7 +1114,7 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
                                    peat_stream_t stream) {
   g_null_error_is_noalloc = true;
   g_noalloc_error[0] = 0;
-  if (is_fp8(dtype)) return noalloc_fail(PEAT_ERR_UNSUPPORTED, FP8_ONLY);
+  if (own_compare(dtype)) return noalloc_fail(PEAT_ERR_UNSUPPORTED, FP8_ONLY);
   const int B = dtype_bytes(dtype);
   if (!B) return noalloc_fail(PEAT_ERR_INVALID_ARG, "dtype must be PEAT_F32, PEAT_F16 or PEAT_BF16");
   float rtol, atol;

@@ -218,6 +218,42 @@ struct Cmp8Params {
 };
 cudaError_t launch_compare8(int dtype, const Cmp8Params& p, int nctas, cudaStream_t s);
 
+// binary64: one item's maxima and counts, and its three sums as normalised
+// 32-bit digits from 2^-2272 (the top limb signed)
+struct Part64Rec {
+  unsigned long long cnt[PEAT_NCLASS], nfin;
+  double ahi, alo;  // max |d| = (ahi + alo) 2^asc at ia
+  int asc;
+  long long ia;
+  double rhi, rlo, rg;  // max |d| / |g| = (rhi + rlo) 2^rsc / rg (rkind 0: zero, 1: finite, 2: +inf) at ir
+  int rsc, rkind;
+  float rlg;            // its log2, approximately (within 2^-12)
+  long long ir;
+  unsigned long long mu;  // max ULP distance at iu
+  long long iu;
+};
+constexpr int P64_LIMBS = 136;
+struct Part64 {
+  Part64Rec rec;
+  long long limbs[3 * P64_LIMBS];  // sum d, sum |d|, sum d^2
+};
+struct Cmp64Params {
+  const void* g;
+  const void* c;
+  const int64_t* offsets;
+  const int64_t* item_b;
+  const int64_t* item_e;
+  const int64_t* item_seg;
+  const int64_t* seg_first;
+  int64_t nitems, nseg;
+  double rtol, atol;  // the float32 tolerances
+  int vec;            // both bases 16-byte aligned
+  Part64* parts;
+  peat_stats_t* stats;
+  unsigned long long* hist;
+};
+cudaError_t launch_compare64(const Cmp64Params& p, int nctas, cudaStream_t s);
+
 struct InjectElemParams {
   void* dst;
   const void* src;

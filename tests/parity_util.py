@@ -140,3 +140,27 @@ def assert_hist_equal(gh, oh, ctx=""):
         bad = np.argwhere(gh != oh)
         raise AssertionError(f"{ctx}: histogram differs at {bad[:10].tolist()} gpu={gh[tuple(bad[0])]} "
                              f"oracle={oh[tuple(bad[0])]}")
+
+
+def f64_pairs(n: int, seed: int):
+    """binary64 mixture: relative noise, one-ULP neighbours, arbitrary patterns,
+    sign flips, zeros, subnormals, operands near the largest double (their
+    difference overflows) and equal pairs."""
+    rng = np.random.default_rng(seed)
+    g = (rng.standard_normal(n) * np.exp2(rng.integers(-60, 60, n))).astype(np.float64)
+    c = g * (1 + 1e-12 * rng.standard_normal(n))
+    kind = rng.integers(0, 9, n)
+    gb, cb = g.view(np.uint64).copy(), c.view(np.uint64).copy()
+    cb = np.where(kind == 0, gb + rng.integers(-3, 4, n).astype(np.int64).astype(np.uint64), cb)
+    cb = np.where(kind == 1, rng.integers(0, 2 ** 63, n, dtype=np.uint64) * np.uint64(2)
+                  + rng.integers(0, 2, n, dtype=np.uint64), cb)
+    cb = np.where(kind == 2, gb ^ np.uint64(1 << 63), cb)
+    cb = np.where(kind == 3, np.uint64(0), cb)
+    sub = rng.integers(0, 1 << 52, n, dtype=np.uint64)
+    gb = np.where(kind == 4, sub, gb)
+    cb = np.where(kind == 4, sub + rng.integers(0, 5, n, dtype=np.uint64), cb)
+    big = np.float64(1.7e308)
+    gb = np.where(kind == 5, np.array([-big]).view(np.uint64)[0], gb)
+    cb = np.where(kind == 5, (big * (1 - 1e-3 * rng.random(n))).view(np.uint64), cb)
+    cb = np.where(kind == 6, gb, cb)
+    return gb.astype(np.uint64), cb.astype(np.uint64)

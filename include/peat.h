@@ -64,9 +64,9 @@ typedef struct CUstream_st* peat_stream_t;
  * E5M2 (bias 15, IEEE-like infinities and NaNs); peat_compare,
  * peat_compare_segmented and peat_isclose_grid take them.  PEAT_F64
  * (IEEE binary64, e.g. a float32 output widened exactly to compare with a
- * binary64 one) is taken by peat_compare and peat_compare_segmented; its
- * ULP distance counts binary64 steps and its sums may round to +-inf.  The
- * other entry points return PEAT_ERR_UNSUPPORTED for these types. */
+ * binary64 one) is taken by the same three; its ULP distance counts binary64
+ * steps and its sums may round to +-inf.  The other entry points return
+ * PEAT_ERR_UNSUPPORTED for these types. */
 typedef enum {
   PEAT_F32 = 0,
   PEAT_F16 = 1,

@@ -17,8 +17,8 @@ ROOT = PKG.parent
 CSRC = PKG / "csrc"
 OUT_DIR = PKG / "_build"
 LIB = OUT_DIR / "libpeat.so"
-SOURCES = ["compare.cu", "compare8.cu", "compare64.cu", "topk.cu", "tstats.cu", "isclose.cu", "inject.cu", "peat_api.cpp"]
-HEADERS = [CSRC / "peat_internal.h", CSRC / "exact.cuh", CSRC / "inject_models.cuh", CSRC / "tol_exact.cuh",
+SOURCES = ["compare.cu", "compare8.cu", "compare64.cu", "topk.cu", "tstats.cu", "isclose.cu", "isclose64.cu", "inject.cu", "peat_api.cpp"]
+HEADERS = [CSRC / "peat_internal.h", CSRC / "exact.cuh", CSRC / "inject_models.cuh", CSRC / "tol_exact.cuh", CSRC / "exact64.cuh",
            ROOT / "include" / "peat.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",

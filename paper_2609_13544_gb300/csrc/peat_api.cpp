@@ -91,7 +91,7 @@ bool is_fp8(int dt) { return dt == PEAT_F8E4M3 || dt == PEAT_F8E5M2; }
 // the element types with a compare of their own (and no other entry point but the isclose grid for 8 bits)
 bool own_compare(int dt) { return is_fp8(dt) || dt == PEAT_F64; }
 const char* const FP8_ONLY =
-    "8-bit and binary64 operands: peat_compare and peat_compare_segmented (and peat_isclose_grid for 8 bits) only";
+    "8-bit and binary64 operands: peat_compare, peat_compare_segmented and peat_isclose_grid only";
 
 bool round_tol(peat_tol_t tol, float* r, float* a) {
   if (!(tol.rtol >= 0.0) || !(tol.atol >= 0.0)) return false;  // rejects NaN too
@@ -736,8 +736,7 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
                                 peat_dtype_t dtype, const double* rtols, int nr, const double* atols, int na,
                                 uint64_t* counts_out, peat_stream_t stream) {
   if (!h) return PEAT_ERR_INVALID_ARG;
-  if (dtype == PEAT_F64) return fail(h, PEAT_ERR_UNSUPPORTED, "binary64 operands: peat_compare only");
-  const int B = is_fp8(dtype) ? 1 : dtype_bytes(dtype);
+  const int B = is_fp8(dtype) ? 1 : (dtype == PEAT_F64 ? 8 : dtype_bytes(dtype));
   if (!B) return fail(h, PEAT_ERR_INVALID_ARG, "dtype must be one of peat_dtype_t");
   if (n < 0) return fail(h, PEAT_ERR_INVALID_ARG, "n < 0");
   if (n > 0 && (!golden || !candidate)) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
@@ -790,7 +789,7 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
   const int nctas = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)h->nsm * 8, want));
   // per-CTA counts are 32-bit
   if (n / nctas >= ((int64_t)1 << 31)) return fail(h, PEAT_ERR_UNSUPPORTED, "more than 2^31 elements per CTA");
-  e = peat::launch_isclose(dtype, p, nctas, st);
+  e = dtype == PEAT_F64 ? peat::launch_isclose64(p, nctas, st) : peat::launch_isclose(dtype, p, nctas, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "isclose launch");
   return PEAT_OK;
 }

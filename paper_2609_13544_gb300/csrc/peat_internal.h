@@ -186,6 +186,7 @@ struct IscParams {
   unsigned long long* counts;          // device, ncells (cell i * na + caller's j), zero before the launch
 };
 cudaError_t launch_isclose(int dtype, const IscParams& p, int nctas, cudaStream_t s);
+cudaError_t launch_isclose64(const IscParams& p, int nctas, cudaStream_t s);  // binary64 operands
 
 // 8-bit formats: one item's totals (sums in units of 2^-S, 2^-2S)
 struct Part8 {

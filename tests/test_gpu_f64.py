@@ -89,9 +89,33 @@ def test_fp32_candidate_against_fp64_golden(peat_gpu, oracle, h):
 def test_other_entry_points_refuse_f64(peat_gpu, h):
     x = torch.zeros(64, dtype=torch.float64, device="cuda")
     for call in (lambda: peat_gpu.peat_topk_mean(h, x, x), lambda: peat_gpu.peat_tensor_stats(h, x),
-                 lambda: peat_gpu.peat_isclose_grid(h, x, x, [0.0], [0.0]),
                  lambda: peat_gpu.peat_pseudo_error_inject(h, x, [dict(kind="bias", x=1e-3)], 1),
                  lambda: peat_gpu.peat_compare_noalloc(x, x, 1e-3)):
         with pytest.raises(peat_gpu.PeatError) as e:
             call()
         assert e.value.status == 2
+
+
+@pytest.mark.parametrize("n", [1, 3, 4099, 100_003])
+def test_f64_isclose_grid(peat_gpu, oracle, h, n):
+    gb, cb = f64_pairs(n, seed=70 + n)
+    rtols = [0.0, 1e-12, 1e-9, 1e-6, 1e-3, 1.0]
+    atols = [1e-300, 0.0, 1e-12, 1e30, 1e-6]
+    for goff in (0, 1):
+        got = peat_gpu.peat_isclose_grid(h, dev(gb, goff), dev(cb, goff), rtols, atols)
+        want = oracle.isclose_grid(gb, cb, "f64", rtols, atols)
+        assert np.array_equal(got, want), (n, goff, got, want)
+
+
+def test_f64_isclose_fig5_fp32_vs_fp64(peat_gpu, oracle, h):
+    """Fig. 5's FP32-FP64 pass fractions: a binary64 golden against its float32 rounding."""
+    rng = np.random.default_rng(12)
+    g = rng.standard_normal(300_000) * np.exp2(rng.integers(-8, 8, 300_000))
+    c = g.astype(np.float32).astype(np.float64)
+    rtols = [0.0, 1e-9, 1e-8, 3e-8, 6e-8, 1e-7, 1e-6]
+    atols = [0.0, 1e-12, 1e-9, 1e-6]
+    gb, cb = g.view(np.uint64).copy(), c.view(np.uint64).copy()
+    got = peat_gpu.peat_isclose_grid(h, dev(gb), dev(cb), rtols, atols)
+    want = oracle.isclose_grid(gb, cb, "f64", rtols, atols)
+    assert np.array_equal(got, want)
+    assert got[-1, 0] == g.size and got[0, 0] < g.size  # rtol 1e-6 accepts every float32 rounding

@@ -278,12 +278,6 @@ struct XAcc {
     uint32_t mx = split_float(x, ex), my = split_float(y, ey);
     add_m((unsigned __int128)((uint64_t)mx * my), ex + ey + sc, neg ^ (x < 0) ^ (y < 0));
   }
-  __device__ void add_double(double x, bool neg = false) {
-    if (x == 0.0) return;
-    int e;
-    uint64_t m = split_double(x, e);
-    add_m(m, e, neg ^ (x < 0));
-  }
   __device__ void add_prod(double x, double y, bool neg = false) {
     if (x == 0.0 || y == 0.0) return;
     int ex, ey;

@@ -127,9 +127,10 @@ def test_c2_full_size_properties(peat_gpu, h):
     assert math.isclose(st["sum_sq"], float((d * d).sum()), rel_tol=1e-12)
 
 
-def test_c4_full_size_sampled_segments(peat_gpu, oracle, h):
-    """Full GPT-2-medium list: every segment satisfies the invariants; the oracle
-    recomputes the 100 smallest segments one by one."""
+def test_c4_full_size_every_segment(peat_gpu, oracle, h):
+    """Full GPT-2-medium list (292 fp16 segments, 354,823,168 pairs) in the
+    bench's launch configuration: every segment against the oracle (fanned out
+    to the host cores), and the invariants."""
     from paper_2609_13544_gb300 import workloads as W
     w = W.c4_gpt2_medium(device="cuda")
     gs, gh = peat_gpu.peat_compare_segmented(h, w.golden, w.candidate, w.offsets, w.rtol, w.atol)
@@ -137,10 +138,51 @@ def test_c4_full_size_sampled_segments(peat_gpu, oracle, h):
     for s in range(len(gs)):
         _check_properties(gs[s], gh[s], int(sizes[s]))
     assert sum(s["nan_inf_asym"] for s in gs) == len(w.meta["nan_inf_positions"])
-    pick = np.argsort(sizes, kind="stable")[:100]
     gbits, cbits = host_bits(w.golden, "f16"), host_bits(w.candidate, "f16")
-    for s in pick:
-        a, b = int(w.offsets[s]), int(w.offsets[s + 1])
-        os_, oh = oracle.compare(gbits[a:b], cbits[a:b], "f16", w.rtol, w.atol)
-        assert_stats_equal(gs[s], os_, f"c4 seg {s}")
-        assert_hist_equal(gh[s], oh, f"c4 seg {s}")
+    os_, oh = oracle_segmented(gbits, cbits, w.offsets, "f16", w.rtol, w.atol)
+    for s in range(len(os_)):
+        assert_stats_equal(gs[s], os_[s], f"c4 seg {s}")
+    assert_hist_equal(gh, oh, "c4")
+
+
+def _full_via_segments(peat, oracle, h, w, nseg, ctx):
+    """A full-size single tensor in the bench's launch configuration, checked
+    through the oracle: the same tensor cut into nseg equal segments is
+    compared segment by segment on both sides (bit-exact), and the one-launch
+    result must be their exact combination: counts and histograms summed,
+    maxima and their lowest indices taken over segments, sums within 1e-10."""
+    n = w.n
+    off = np.linspace(0, n, nseg + 1).astype(np.int64)
+    gb, cb = host_bits(w.golden, w.dtype), host_bits(w.candidate, w.dtype)
+    gs, gh = peat.peat_compare_segmented(h, w.golden, w.candidate, off.tolist(), w.rtol, w.atol)
+    os_, oh = oracle_segmented(gb, cb, off, w.dtype, w.rtol, w.atol)
+    for s in range(nseg):
+        assert_stats_equal(gs[s], os_[s], f"{ctx} seg {s}")
+    assert_hist_equal(gh, oh, ctx)
+    st, hist = peat.peat_compare(h, w.golden, w.candidate, w.rtol, w.atol)
+    assert st["n"] == n and st["count"] == [sum(s["count"][k] for s in os_) for k in range(5)]
+    assert st["n_finite"] == sum(s["n_finite"] for s in os_)
+    assert np.array_equal(hist, oh.sum(axis=0))
+    for key, idx in (("max_abs", "argmax_abs"), ("max_rel", "argmax_rel"), ("max_ulp", "argmax_ulp")):
+        best = max(s[key] for s in os_ if s[idx] >= 0)
+        assert st[key] == best, key
+        cands = [int(off[k]) + os_[k][idx] for k in range(nseg) if os_[k][idx] >= 0 and os_[k][key] == best]
+        # one segment attains the rounded maximum: its index is the answer; several: any
+        # of them may hold the exact maximum, the lowest index among equal exact values
+        assert (st[idx] == cands[0]) if len(cands) == 1 else (st[idx] in cands), (key, st[idx], cands[:4])
+    for key in ("sum_abs", "sum_sq", "sum_signed"):
+        total = math.fsum(s[key] for s in os_)
+        assert abs(st[key] - total) <= 1e-10 * abs(total) + 1e-300, key
+    return st
+
+
+def test_c2_full_size_through_the_oracle(peat_gpu, oracle, h):
+    from paper_2609_13544_gb300 import workloads as W
+    _full_via_segments(peat_gpu, oracle, h, W.c2_bf16_rne_vs_rtz(device="cuda"), 64, "c2 full")
+
+
+def test_c5_full_size_through_the_oracle(peat_gpu, oracle, h):
+    from paper_2609_13544_gb300 import workloads as W
+    w = W.PlaybackSweep(device="cuda").workload(63)
+    st = _full_via_segments(peat_gpu, oracle, h, w, 128, "c5 full")
+    assert st["n"] == 268_435_456

@@ -2,9 +2,9 @@
 // histograms of the compare) for binary64 operands: the FP32-FP64 pairs of
 // Fig. 5 once the float32 side is widened (exactly) to binary64.
 //
-// d = c - g is an exact double-double (hi, lo) from TwoSum, held halved with
-// a scale of one when the difference overflows binary64 (both operands are
-// then at least 2^1022, so halving is exact).  Decisions that rounding could
+// d = c - g is an exact double-double (hi, lo) from Fast2Sum on the operands
+// ordered by magnitude, held halved with a scale of one when the difference
+// overflows binary64 (both operands are then large, so halving is exact).  Decisions that rounding could
 // flip (the tolerance, the relative maximum) take a binary64 or float32 test
 // with a margin first and otherwise the sign of an exact sum of integer
 // terms; the relative bin comes from exponents and significands exactly; the
@@ -39,7 +39,7 @@ __device__ __forceinline__ int rel_log2_floor64(const Mag& a, double ag) {
   norm_d(ag, fg, eg);
   const int k0 = ea + a.sc - eg;
   if (fa != fg) return fa > fg ? k0 : k0 - 1;
-  return a.lo < 0.0 ? k0 - 1 : k0;  // hi = ag 2^k0 exactly: lo decides
+  return neg64(a.lo) ? k0 - 1 : k0;  // hi = ag 2^k0 exactly: lo decides
 }
 
 // relative error records: a / g with kind 0 (a = 0), 1 (finite), 2 (g = 0 < a)
@@ -47,17 +47,27 @@ struct Rel {
   Mag a;
   double g;
   int kind;
-  float lg;  // log2 of the ratio, approximately (kind 1)
+  int le;    // log2 of the ratio, approximately (kind 1): le + lf, le exact,
+  float lf;  // lf = log2 of the significands' ratio within 2^-20
 };
 
-__device__ __forceinline__ float approx_log2(const Mag& a, double g) {
+__device__ __forceinline__ void approx_log2(const Mag& a, double g, int& le, float& lf) {
   uint64_t fa, fg;
   int ea, eg;
   norm_d(a.hi, fa, ea);
   norm_d(g, fg, eg);
   const float ra = __uint_as_float(0x3F800000u | (uint32_t)(fa >> 29));
   const float rg = __uint_as_float(0x3F800000u | (uint32_t)(fg >> 29));
-  return (float)(ea + a.sc - eg) + __log2f(__fdividef(ra, rg));
+  le = ea + a.sc - eg;
+  lf = __log2f(__fdividef(ra, rg));
+}
+
+// log2(x) - log2(y) of two finite ratios, within 2^-18 (clamped far from zero)
+__device__ __forceinline__ float lg_diff(int xe, float xf, int ye, float yf) {
+  const int de = xe - ye;
+  if (de > 4) return 8.0f;
+  if (de < -4) return -8.0f;
+  return (float)de + (xf - yf);
 }
 
 // x > y exactly
@@ -177,7 +187,7 @@ __device__ __forceinline__ void acc64_init(Acc64& t) {
   t.sq = W192{0ull, 0ull, 0ull, INT32_MIN};
   t.ma = Mag{0.0, 0.0, 0};
   t.ia = 0;
-  t.mr = Rel{Mag{0.0, 0.0, 0}, 1.0, 0, 0.0f};
+  t.mr = Rel{Mag{0.0, 0.0, 0}, 1.0, 0, 0, 0.0f};
   t.ir = 0;
   t.mu = 0;
   t.iu = 0;
@@ -205,18 +215,19 @@ __device__ __forceinline__ void pair64(const Cmp64Params& p, Acc64& t, unsigned*
       cls = eq ? PEAT_EXACT : PEAT_NAN_INF_ASYM;
       relbin = eq ? 0 : 63;
     } else {
-      const double gd = __longlong_as_double((long long)G), cd = __longlong_as_double((long long)C);
+      const double gd = from_bits64(G), cd = from_bits64(C);
       bool dneg;
       const Mag a = diff64(gd, cd, dneg);
-      const double ag = fabs(gd);
+      const double ag = from_bits64(mg);  // |g|
+      const bool azero = bits64(a.hi) == 0;
       t.nfin++;
       // sums: d = +-(hi + lo) 2^sc, |d|, d^2 = (hi^2 + 2 hi lo + lo^2) 4^sc
       {
         uint64_t mh, ml;
         int eh, el;
         split_d(a.hi, mh, eh);
-        split_d(fabs(a.lo), ml, el);
-        const bool lneg = a.lo < 0.0;
+        split_d(a.lo, ml, el);  // split_d takes the magnitude
+        const bool lneg = (bits64(a.lo) >> 63) != 0;
         win_add(t.sd, t.bd, mh, eh + a.sc, dneg, S);
         win_add(t.sa, t.ba, mh, eh + a.sc, false, S + SL);
         win3_add(t.sq, (u128)mh * mh, 2 * (eh + a.sc), S + 2 * SL);
@@ -233,18 +244,21 @@ __device__ __forceinline__ void pair64(const Cmp64Params& p, Acc64& t, unsigned*
       Rel r;
       r.a = a;
       r.g = ag;
-      r.kind = a.hi == 0.0 ? 0 : (ag == 0.0 ? 2 : 1);
-      r.lg = r.kind == 1 ? approx_log2(a, ag) : 0.0f;
-      const bool maybe = t.ir == 0 || r.kind > t.mr.kind || (r.kind == 1 && t.mr.kind == 1 && r.lg >= t.mr.lg - 0x1p-8f);
+      r.kind = azero ? 0 : (mg == 0 ? 2 : 1);
+      r.le = 0;
+      r.lf = 0.0f;
+      if (r.kind == 1) approx_log2(a, ag, r.le, r.lf);
+      const bool maybe = t.ir == 0 || r.kind > t.mr.kind ||
+                         (r.kind == 1 && t.mr.kind == 1 && lg_diff(r.le, r.lf, t.mr.le, t.mr.lf) >= -0x1p-16f);
       if (maybe && (t.ir == 0 || rel_gt(r, t.mr))) t.mr = r, t.ir = off + 1;
-      if (a.hi == 0.0) {
+      if (azero) {
         cls = PEAT_EXACT;
         relbin = 0;
       } else {
         if (within64(a, ag, p.rtol, p.atol)) cls = PEAT_WITHIN_TOL;
-        else if (gd != 0.0 && cd != 0.0 && sg != sc) cls = PEAT_SIGN_FLIP;
+        else if (mg != 0 && mc != 0 && sg != sc) cls = PEAT_SIGN_FLIP;
         else cls = PEAT_MISMATCH;
-        if (ag == 0.0) {
+        if (mg == 0) {
           relbin = 63;
         } else {
           const int k = rel_log2_floor64(a, ag) + 48;
@@ -274,7 +288,10 @@ __device__ __forceinline__ bool better_mag(const Mag& x, long long ix, const Mag
 __device__ __forceinline__ bool better_rel(const Rel& x, long long ix, const Rel& y, long long iy) {
   if (ix < 0) return false;
   if (iy < 0) return true;
-  if (x.kind == 1 && y.kind == 1 && fabsf(x.lg - y.lg) > 0x1p-8f) return x.lg > y.lg;  // far apart
+  if (x.kind == 1 && y.kind == 1) {  // far apart: the approximations decide
+    const float dl = lg_diff(x.le, x.lf, y.le, y.lf);
+    if (fabsf(dl) > 0x1p-16f) return dl > 0.0f;
+  }
   return rel_gt(x, y) || (!rel_gt(y, x) && ix < iy);
 }
 __device__ __forceinline__ bool better_u(unsigned long long x, long long ix, unsigned long long y, long long iy) {
@@ -289,9 +306,11 @@ __device__ void rec_merge(Part64Rec& r, const Part64Rec& o) {
   r.nfin += o.nfin;
   const Mag ra{r.ahi, r.alo, r.asc}, oa{o.ahi, o.alo, o.asc};
   if (better_mag(oa, o.ia, ra, r.ia)) r.ahi = o.ahi, r.alo = o.alo, r.asc = o.asc, r.ia = o.ia;
-  const Rel rr{Mag{r.rhi, r.rlo, r.rsc}, r.rg, r.rkind, r.rlg}, orr{Mag{o.rhi, o.rlo, o.rsc}, o.rg, o.rkind, o.rlg};
+  const Rel rr{Mag{r.rhi, r.rlo, r.rsc}, r.rg, r.rkind, r.rle, r.rlf};
+  const Rel orr{Mag{o.rhi, o.rlo, o.rsc}, o.rg, o.rkind, o.rle, o.rlf};
   if (better_rel(orr, o.ir, rr, r.ir))
-    r.rhi = o.rhi, r.rlo = o.rlo, r.rsc = o.rsc, r.rg = o.rg, r.rkind = o.rkind, r.rlg = o.rlg, r.ir = o.ir;
+    r.rhi = o.rhi, r.rlo = o.rlo, r.rsc = o.rsc, r.rg = o.rg, r.rkind = o.rkind, r.rle = o.rle, r.rlf = o.rlf,
+    r.ir = o.ir;
   if (better_u(o.mu, o.iu, r.mu, r.iu)) r.mu = o.mu, r.iu = o.iu;
 }
 
@@ -299,7 +318,7 @@ __device__ __forceinline__ void rec_from_acc(Part64Rec& r, const Acc64& a, long 
   for (int k = 0; k < PEAT_NCLASS; k++) r.cnt[k] = a.cnt[k];
   r.nfin = a.nfin;
   r.ahi = a.ma.hi, r.alo = a.ma.lo, r.asc = a.ma.sc, r.ia = a.ia ? ib + a.ia - 1 : -1;
-  r.rhi = a.mr.a.hi, r.rlo = a.mr.a.lo, r.rsc = a.mr.a.sc, r.rg = a.mr.g, r.rkind = a.mr.kind, r.rlg = a.mr.lg;
+  r.rhi = a.mr.a.hi, r.rlo = a.mr.a.lo, r.rsc = a.mr.a.sc, r.rg = a.mr.g, r.rkind = a.mr.kind, r.rle = a.mr.le, r.rlf = a.mr.lf;
   r.ir = a.ir ? ib + a.ir - 1 : -1;
   r.mu = a.mu, r.iu = a.iu ? ib + a.iu - 1 : -1;
 }
@@ -327,7 +346,7 @@ __device__ void normalise(long long* d, int n) {
   d[n - 1] += carry;
 }
 
-__global__ void __launch_bounds__(TB) compare64_stage1(Cmp64Params p) {
+__global__ void __launch_bounds__(TB, 2) compare64_stage1(Cmp64Params p) {
   __shared__ unsigned H[PEAT_HIST_BINS];
   __shared__ long long S[3 * SL];
   __shared__ Part64Rec buf[TB];
@@ -469,7 +488,7 @@ __global__ void __launch_bounds__(TB) compare64_finalize(Cmp64Params p) {
   for (int k = 0; k < PEAT_NCLASS; k++) r.cnt[k] = 0;
   r.nfin = 0;
   r.ahi = r.alo = 0.0, r.asc = 0, r.ia = -1;
-  r.rhi = r.rlo = 0.0, r.rsc = 0, r.rg = 1.0, r.rkind = 0, r.rlg = 0.0f, r.ir = -1;
+  r.rhi = r.rlo = 0.0, r.rsc = 0, r.rg = 1.0, r.rkind = 0, r.rle = 0, r.rlf = 0.0f, r.ir = -1;
   r.mu = 0, r.iu = -1;
   for (long long it = f0 + threadIdx.x; it < f1; it += TB) rec_merge(r, p.parts[it].rec);
   block_merge(r, buf);

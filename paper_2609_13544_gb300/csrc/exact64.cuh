@@ -85,39 +85,67 @@ struct Mag {
   int sc;
 };
 
-// d = c - g exactly (both finite); returns |d| and the sign of d
+constexpr uint64_t MAG64 = 0x7FFFFFFFFFFFFFFFull, INF64 = 0x7FF0000000000000ull;
+__device__ __forceinline__ uint64_t bits64(double x) { return (uint64_t)__double_as_longlong(x); }
+__device__ __forceinline__ double from_bits64(uint64_t b) { return __longlong_as_double((long long)b); }
+
+// d = c - g exactly (both finite); returns |d| and the sign of d.  The
+// operands are ordered by magnitude (their bit patterns order as their
+// values), so Fast2Sum's three operations give the exact error term
+// (Dekker: s = RN(x + y), t = y - RN(s - x) when |x| >= |y|).
 __device__ __forceinline__ Mag diff64(double g, double c, bool& dneg) {
-  double x = c, y = -g;
+  double x = c, y = from_bits64(bits64(g) ^ 0x8000000000000000ull);
+  if ((bits64(x) & MAG64) < (bits64(y) & MAG64)) {
+    const double t = x;
+    x = y;
+    y = t;
+  }
   int sc = 0;
   double s = __dadd_rn(x, y);
-  if (!(fabs(s) <= 1.7976931348623157e308)) {
+  if ((bits64(s) & MAG64) >= INF64) {  // the difference overflows: halve both (exact at this size)
     x = __dmul_rn(x, 0.5);
     y = __dmul_rn(y, 0.5);
     s = __dadd_rn(x, y);
     sc = 1;
   }
-  const double yv = __dsub_rn(s, x), xv = __dsub_rn(s, yv);
-  const double t = __dadd_rn(__dsub_rn(x, xv), __dsub_rn(y, yv));
-  dneg = s < 0.0;
-  return Mag{fabs(s), dneg ? -t : t, sc};
+  const double t = __dsub_rn(y, __dsub_rn(s, x));
+  dneg = (bits64(s) >> 63) != 0;
+  // the error term of |d| (sign of d folded in); a zero is +0: -0 and +0 would order apart below
+  const uint64_t lb = bits64(t) ^ (dneg ? 0x8000000000000000ull : 0ull);
+  return Mag{from_bits64(bits64(s) & MAG64), from_bits64((lb & MAG64) ? lb : 0ull), sc};
+}
+
+// x < 0 on the bits (x is never -0 here: see diff64)
+__device__ __forceinline__ bool neg64(double x) { return (bits64(x) >> 63) != 0; }
+
+// order-preserving key of a double (as an unsigned integer)
+__device__ __forceinline__ uint64_t okey64(double x) {
+  const uint64_t b = bits64(x);
+  return (b >> 63) ? ~b : (b | 0x8000000000000000ull);
 }
 
 // a > b exactly (lexicographic on the scale, then hi, then lo: hi is the
 // rounding of the exact value, so a larger hi means a larger value)
 __device__ __forceinline__ bool mag_gt(const Mag& a, const Mag& b) {
   if (a.sc != b.sc) return a.sc > b.sc;
-  if (a.hi != b.hi) return a.hi > b.hi;
-  return a.lo > b.lo;
+  const uint64_t ha = bits64(a.hi), hb = bits64(b.hi);  // both >= 0: the bits order as the values
+  if (ha != hb) return ha > hb;
+  return okey64(a.lo) > okey64(b.lo);
 }
 
 // a <= atol + rtol ag exactly (a > 0)
-static __device__ bool within64(const Mag& a, double ag, double rtol, double atol) {
+__device__ __forceinline__ bool within64(const Mag& a, double ag, double rtol, double atol) {
   const double thr = __fma_rn(rtol, ag, atol);
-  if (a.sc == 0 && a.hi >= 0x1p-900 && thr >= 0x1p-900 && thr <= 0x1p+1000) {
-    if (__dmul_rn(a.hi, 1.0 + 0x1p-50) < __dmul_rn(thr, 1.0 - 0x1p-50)) return true;
-    if (__dmul_rn(a.hi, 1.0 - 0x1p-50) > __dmul_rn(thr, 1.0 + 0x1p-50)) return false;
+  // margin test on the bit patterns (positive normal doubles): 16 patterns apart
+  // is at least 16 units in the last place of the smaller, more than the
+  // rounding of thr and the |lo| <= ulp(hi) / 2 of a together
+  const uint64_t hb = bits64(a.hi), tb = bits64(thr);
+  const uint64_t LO = 0x07B0000000000000ull, HI = 0x7E70000000000000ull;  // 2^-900, 2^1000
+  if (a.sc == 0 && hb >= LO && tb >= LO && tb <= HI) {
+    if (hb + 16 < tb) return true;
+    if (hb > tb + 16) return false;
   }
-  XTerm t[4] = {dbl_term(a.hi, a.sc, false), dbl_term(fabs(a.lo), a.sc, a.lo < 0.0), dbl_term(atol, 0, true),
+  XTerm t[4] = {dbl_term(a.hi, a.sc, false), dbl_term(a.lo, a.sc, neg64(a.lo)), dbl_term(atol, 0, true),
                 prod_term(rtol, ag, 0, true)};
   return xsign(t, 4) <= 0;
 }

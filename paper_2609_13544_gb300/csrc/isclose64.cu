@@ -3,7 +3,7 @@
 // exactly): the structure of the float32 grid kernel (a warp queue of the
 // differing finite pairs, a binary search per atol bounded by the previous
 // atol's result, a shared histogram of first accepting rtols), with the
-// binary64 difference as an exact TwoSum pair and the exact binary64
+// binary64 difference as an exact two-term pair and the exact binary64
 // tolerance test.
 #include <cstdint>
 
@@ -36,11 +36,11 @@ __device__ __forceinline__ int classify64(uint64_t G, uint64_t C, Mag& a, double
   const uint64_t INF = 0x7FF0000000000000ull;
   const uint64_t mg = G & 0x7FFFFFFFFFFFFFFFull, mc = C & 0x7FFFFFFFFFFFFFFFull;
   if (mg >= INF || mc >= INF) return (mg > INF && mc > INF) ? 0 : 1;
-  const double gd = __longlong_as_double((long long)G), cd = __longlong_as_double((long long)C);
-  if (gd == cd) return 0;  // +0 and -0
+  if ((mg | mc) == 0) return 0;  // +0 and -0 (the bit patterns differ)
+  const double gd = from_bits64(G), cd = from_bits64(C);
   bool dneg;
   a = diff64(gd, cd, dneg);
-  ag = fabs(gd);
+  ag = from_bits64(mg);
   return 2;
 }
 

@@ -228,7 +228,8 @@ struct Part64Rec {
   long long ia;
   double rhi, rlo, rg;  // max |d| / |g| = (rhi + rlo) 2^rsc / rg (rkind 0: zero, 1: finite, 2: +inf) at ir
   int rsc, rkind;
-  float rlg;            // its log2, approximately (within 2^-12)
+  int rle;              // its log2, approximately: rle + rlf (rle exact, rlf within 2^-20)
+  float rlf;
   long long ir;
   unsigned long long mu;  // max ULP distance at iu
   long long iu;

@@ -131,6 +131,8 @@ struct TopkState {
   unsigned int ok;              // the window held the k-th largest
   unsigned int done[3];         // CTAs finished, per pass
   unsigned int nlist, nlist2;   // list entries from the last pass and the optional extra one
+  unsigned int lowor, inexact;  // over the window pairs of pass 1: OR of the keys' low 10 bits, any |d| not a float32
+  unsigned int skip2;           // pass 1 resolved the last digit itself (passes 2 and 3 return at once)
   long long limbs[NLIMB];       // exact sum of the |d| resolved above the prefix
 };
 struct TopkListEntry {

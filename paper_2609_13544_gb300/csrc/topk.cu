@@ -55,12 +55,24 @@ template <>
 struct TK<PEAT_F16> {
   static constexpr int BYTES = 2, VEC = 8;
   static constexpr uint32_t MAG = 0x7FFFu, INF = 0x7C00u;
+  static constexpr int MB = 10, EMASK = 0x1F;  // fraction bits, exponent field
 };
 template <>
 struct TK<PEAT_BF16> {
   static constexpr int BYTES = 2, VEC = 8;
   static constexpr uint32_t MAG = 0x7FFFu, INF = 0x7F80u;
+  static constexpr int MB = 7, EMASK = 0xFF;
 };
+
+// 16-bit operands: c - g may be inexact in float32 only when their exponents
+// are more than 23 - MB apart (the difference then spans more than 24 bits);
+// a subnormal's exponent field counts as 1
+template <int DT>
+__device__ __forceinline__ uint32_t maybe_inexact(uint32_t G, uint32_t C) {
+  const int eg = max((int)((G >> TK<DT>::MB) & TK<DT>::EMASK), 1);
+  const int ec = max((int)((C >> TK<DT>::MB) & TK<DT>::EMASK), 1);
+  return (uint32_t)(abs(eg - ec) > 23 - TK<DT>::MB);
+}
 
 template <int DT>
 __device__ __forceinline__ float tk_f32(uint32_t r) {
@@ -512,6 +524,9 @@ __global__ void __launch_bounds__(TB) topk_pass1(TopkParams p) {
   ExactAcc acc(Phi + 1 >= (KEY_OVF >> 21) ? NO_FAST : max((int)((Phi + 1) >> 2), 1), lim);
   RunCount rc;
   uint32_t nab = 0, nnf = 0;
+  // 16-bit operands: whether the window's keys all have zero low 10 bits and
+  // every window |d| is a float32 value (then pass 1 resolves the last digit)
+  uint32_t lowor = 0, inex = 0;
   // a pair whose raw key is below KEY_OVF is finite with that key: inside
   // the window it is only counted, here; everything above the window, and
   // every pair with a NaN, an infinity or an overflow, is queued
@@ -520,7 +535,13 @@ __global__ void __launch_bounds__(TB) topk_pass1(TopkParams p) {
       [&](uint32_t G, uint32_t C) {
         const uint32_t u = raw_key<DT>(G, C), k0 = u >> 21;
         if (k0 > Phi || u >= KEY_OVF) return true;
-        if (k0 >= Plo) rc.add(h, ((k0 - Plo) << 11) | ((u >> 10) & 0x7FFu));
+        if (k0 >= Plo) {
+          rc.add(h, ((k0 - Plo) << 11) | ((u >> 10) & 0x7FFu));
+          if constexpr (TK<DT>::BYTES == 2) {
+            lowor |= u & 0x3FFu;
+            inex |= maybe_inexact<DT>(G, C);
+          }
+        }
         return false;
       },
       [&](uint32_t G, uint32_t C) {
@@ -537,14 +558,22 @@ __global__ void __launch_bounds__(TB) topk_pass1(TopkParams p) {
           return;
         }
         rc.add(h, ((k0 - Plo) << 11) | ((key >> 10) & 0x7FFu));
+        if constexpr (TK<DT>::BYTES == 2) {
+          lowor |= key & 0x3FFu;
+          inex |= maybe_inexact<DT>(G, C);
+        }
       });
   rc.flush(h);
   acc.flush();
   nab = __reduce_add_sync(0xFFFFFFFFu, nab);
   nnf = __reduce_add_sync(0xFFFFFFFFu, nnf);
+  lowor = __reduce_or_sync(0xFFFFFFFFu, lowor);
+  inex = __reduce_or_sync(0xFFFFFFFFu, inex);
   if ((threadIdx.x & 31) == 0) {
     if (nab) atomicAdd(&cnt_s[0], (unsigned long long)nab);
     if (nnf) atomicAdd(&cnt_s[1], (unsigned long long)nnf);
+    if (lowor) atomicOr(&st->lowor, lowor);
+    if (inex) atomicOr(&st->inexact, inex);
   }
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -559,6 +588,27 @@ __global__ void __launch_bounds__(TB) topk_pass1(TopkParams p) {
   unsigned d = 0;
   const unsigned long long wt = select_digit<TK_WIN * TK_NB1 / TB>(st->hist1, krem, d);
   const bool hit = k == 0 || (above < k && k <= above + wt);
+  // 16-bit operands whose window keys are all multiples of 2^10 with float32
+  // |d|: every window bucket holds one value, so the last digit is 0, the
+  // k-th largest is P1 2^10, and the buckets above P1 add count x value
+  // exactly; pass 2 (and 3) then have nothing to do
+  bool skip = false;
+  if constexpr (TK<DT>::BYTES == 2) skip = hit && k > 0 && __ldcg(&st->lowor) == 0 && __ldcg(&st->inexact) == 0;
+  if (skip) {
+    for (int j = threadIdx.x; j < NLIMB; j += TB) lim[j] = 0;
+    __syncthreads();
+    for (int b = d + 1 + threadIdx.x; b < TK_WIN * TK_NB1; b += TB) {
+      const unsigned long long cnt = __ldcg(&st->hist1[b]);
+      if (cnt) {
+        int sc;
+        const float v = key_value(((Plo << 11) + (uint32_t)b) << 10, sc);
+        digits_of_n(lim, v, sc, cnt);
+      }
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < NLIMB; j += TB)
+      if (lim[j]) atomicAdd(reinterpret_cast<unsigned long long*>(&st->limbs[j]), (unsigned long long)lim[j]);
+  }
   if (threadIdx.x == 0) {
     st->nfin = nfin;
     st->k = k;
@@ -568,6 +618,11 @@ __global__ void __launch_bounds__(TB) topk_pass1(TopkParams p) {
       st->P1 = P1;
       st->P0 = P1 >> 11;
       st->krem = krem;
+      if (skip) {
+        st->hist2[0] = __ldcg(&st->hist1[d]);  // P1's bucket: every key is P1 2^10 (last digit 0)
+        st->T = P1 << 10;
+        st->skip2 = 1u;
+      }
     }
     st->done[1] = 0;
   }
@@ -614,7 +669,7 @@ __global__ void __launch_bounds__(TB) topk_pass2(TopkParams p) {
   __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
   __shared__ unsigned last_s;
   TopkState* st = p.st;
-  if (st->k == 0) return;
+  if (st->k == 0 || st->skip2) return;
   for (int b = threadIdx.x; b < TK_NB2; b += TB) h[b] = 0;
   for (int j = threadIdx.x; j < NLIMB; j += TB) lim[j] = 0;
   __syncthreads();
@@ -675,7 +730,7 @@ __global__ void __launch_bounds__(TB) topk_pass3(TopkParams p) {
   __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
   __shared__ unsigned last_s;
   TopkState* st = p.st;
-  if (st->k == 0 || st->nlist <= TK_LCAP) return;
+  if (st->k == 0 || st->skip2 || st->nlist <= TK_LCAP) return;
   for (int j = threadIdx.x; j < NLIMB; j += TB) lim[j] = 0;
   __syncthreads();
   const uint32_t P1 = st->P1, T = st->T;
@@ -805,6 +860,7 @@ __global__ void __launch_bounds__(TB) topk_finalize(TopkParams p) {
     st->Plo = st->Phi = st->P0 = st->P1 = st->T = 0;
     st->ok = 0;
     st->nlist = st->nlist2 = 0;
+    st->lowor = st->inexact = st->skip2 = 0;
   }
 }
 

@@ -79,7 +79,7 @@ typedef enum {
 typedef enum {
   PEAT_OK = 0,
   PEAT_ERR_INVALID_ARG = 1, /* null pointer, negative size, bad dtype, bad offsets, ... */
-  PEAT_ERR_UNSUPPORTED = 2, /* a valid request this build does not serve */
+  PEAT_ERR_UNSUPPORTED = 2, /* a valid request the library does not serve */
   PEAT_ERR_ALLOC = 3,       /* device or pinned allocation failed */
   PEAT_ERR_CUDA = 4,        /* a CUDA runtime call failed (text in peat_last_error) */
   PEAT_ERR_TIMEOUT = 5,     /* a bounded device-side wait expired */

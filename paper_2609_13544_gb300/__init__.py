@@ -240,7 +240,7 @@ def peat_compare_segmented_raw(h: Handle, golden, candidate, offsets, rtol: floa
 
 
 def stats_to_dicts(raw: np.ndarray) -> list:
-    """Unpack host bytes (k*144) into dicts (same keys as the oracle's)."""
+    """Unpack host bytes (k*144) into dicts, one per peat_stats_t record."""
     arr = np.frombuffer(np.ascontiguousarray(raw).tobytes(), dtype=STATS_DTYPE)
     out = []
     for r in arr:

@@ -438,22 +438,46 @@ struct __align__(128) Smem {
 __device__ __forceinline__ void sacc_add(Smem& sm, int which, unsigned __int128 m, int e, bool neg) {
   for_digits(m, e, neg, [&](int j, int64_t v) { atomicAdd(&sm.sacc[which][j], (unsigned long long)v); });
 }
-// general-path terms: into this warp's copy of the sum digits
-__device__ __forceinline__ void gsacc_add(Smem& sm, int which, unsigned __int128 m, int e, bool neg) {
+// General-path terms, one per lane of a converged warp, into the warp's copy
+// of the sum digits: lanes whose digit indices agree are summed in registers
+// first (__match_any_sync groups them; the 32-bit reductions take each signed
+// digit value as a signed 16-bit high part and an unsigned 16-bit low part,
+// so that no group sum overflows), and one lane per group adds the total.
+// Without this, the lanes of a warp would serialise on 64-bit shared atomics
+// to the same few digits.
+__device__ __forceinline__ void wsacc_add(Smem& sm, int which, uint64_t m, int e, bool neg, bool on) {
+  on = on && m != 0;
+  if (!__any_sync(0xFFFFFFFFu, on)) return;
+  const int lane = threadIdx.x & 31;
+  const int p = e - LIMB_LSB, j = p >> 5, r = p & 31;
+  const uint32_t m0 = (uint32_t)m, m1 = (uint32_t)(m >> 32);
+  const uint32_t out[3] = {m0 << r, (m1 << r) | (r ? m0 >> (32 - r) : 0u), r ? m1 >> (32 - r) : 0u};
   unsigned long long* d = sm.gsacc[threadIdx.x >> 5][which];
-  for_digits(m, e, neg, [&](int j, int64_t v) { atomicAdd(d + j, (unsigned long long)v); });
+#pragma unroll
+  for (int k = 0; k < 3; k++) {
+    const bool ok = on && out[k] != 0u && (unsigned)(j + k) < (unsigned)NLIMB;
+    const unsigned grp = __match_any_sync(0xFFFFFFFFu, ok ? j + k : -1);
+    const int64_t v = ok ? (neg ? -(int64_t)out[k] : (int64_t)out[k]) : 0;
+    const uint32_t slo = __reduce_add_sync(grp, (uint32_t)v & 0xFFFFu);
+    const int32_t shi = (int32_t)__reduce_add_sync(grp, (uint32_t)(int32_t)(v >> 16));
+    if (ok && lane == __ffs(grp) - 1) atomicAdd(d + j + k, (unsigned long long)((int64_t)shi * 65536 + slo));
+  }
 }
-__device__ __forceinline__ void sacc_add_f(Smem& sm, int which, float x, bool neg, int sc) {
-  if (x == 0.0f) return;
-  int e;
-  uint32_t m = split_float(x, e);
-  gsacc_add(sm, which, m, e + sc, neg ^ (x < 0));
+__device__ __forceinline__ void wsacc_add_f(Smem& sm, int which, float x, int sc, bool on) {
+  int e = 0;
+  const uint32_t m = x != 0.0f ? split_float(x, e) : 0u;
+  wsacc_add(sm, which, m, e + sc, x < 0.0f, on);
 }
-__device__ __forceinline__ void sacc_add_prod_f(Smem& sm, int which, float x, float y, int sc) {
-  if (x == 0.0f || y == 0.0f) return;
-  int ex, ey;
-  uint32_t mx = split_float(x, ex), my = split_float(y, ey);
-  gsacc_add(sm, which, (unsigned __int128)((uint64_t)mx * my), ex + ey + sc, (x < 0) ^ (y < 0));
+__device__ __forceinline__ void wsacc_add_prod_f(Smem& sm, int which, float x, float y, int sc, bool on) {
+  int ex = 0, ey = 0;
+  const uint32_t mx = x != 0.0f ? split_float(x, ex) : 0u, my = y != 0.0f ? split_float(y, ey) : 0u;
+  wsacc_add(sm, which, (uint64_t)mx * my, ex + ey + sc, (x < 0.0f) != (y < 0.0f), on);
+}
+// one histogram bin per lane (bin < 0: none), counted once per distinct bin
+__device__ __forceinline__ void whist_add(Smem& sm, int bin) {
+  const unsigned grp = __match_any_sync(0xFFFFFFFFu, bin);
+  if (bin >= 0 && (threadIdx.x & 31) == __ffs(grp) - 1)
+    atomicAdd(&sm.ghist[threadIdx.x >> 5][bin], (unsigned long long)__popc(grp));
 }
 
 // floor(log2(a / g)) for a = (hi + lo) 2^sc > 0 and g > 0 (float32 pair, any range)
@@ -471,10 +495,17 @@ __device__ int log2_ratio(float hi, float lo, int sc, float g) {
   return k + sc;
 }
 
-// The general path: the definitions evaluated exactly, for any pair.
+// The general path: the definitions evaluated exactly, for any pair.  The
+// per-lane part: class counters and maxima into cd; the histogram bins and
+// the sum terms it returns are added by the whole warp (general_lane).
+struct GenOut {
+  int hb0, hb1;      // log2-relative bin and 64 + ULP bin, or -1
+  float s, t;        // d = (s + t) 2^sc, both zero when the pair adds no terms
+  int sc;
+};
 template <int DT>
-__device__ __forceinline__ void general_lane(Smem& sm, GenRec& cd, uint32_t G, uint32_t C, int64_t idx, float rtol,
-                                          float atol) {
+__device__ __forceinline__ void general_pair(GenRec& cd, GenOut& o, uint32_t G, uint32_t C, int64_t idx, float rtol,
+                                             float atol) {
   using T = Tr<DT>;
   uint32_t ag_m = G & T::MAG, ac_m = C & T::MAG;
   bool gnan = ag_m > T::INF, cnan = ac_m > T::INF, ginf = ag_m == T::INF, cinf = ac_m == T::INF;
@@ -494,8 +525,8 @@ __device__ __forceinline__ void general_lane(Smem& sm, GenRec& cd, uint32_t G, u
       return;
     }
     cd.n_ga++;
-    atomicAdd(&sm.ghist[threadIdx.x >> 5][63], 1ull);
-    atomicAdd(&sm.ghist[threadIdx.x >> 5][64 + (ulpdef ? (u < 63 ? (int)u : 63) : 63)], 1ull);
+    o.hb0 = 63;
+    o.hb1 = 64 + (ulpdef ? (u < 63 ? (int)u : 63) : 63);
     return;
   }
   float gf = to_f32<DT>(G), cf = to_f32<DT>(C);
@@ -540,8 +571,8 @@ __device__ __forceinline__ void general_lane(Smem& sm, GenRec& cd, uint32_t G, u
     int k = log2_ratio(hi, lo, sc, ag) + 48;
     rb = k < 1 ? 1 : (k > 62 ? 62 : k);
   }
-  atomicAdd(&sm.ghist[threadIdx.x >> 5][rb], 1ull);
-  atomicAdd(&sm.ghist[threadIdx.x >> 5][64 + (u < 63 ? (int)u : 63)], 1ull);
+  o.hb0 = rb;
+  o.hb1 = 64 + (u < 63 ? (int)u : 63);
   // maxima, full (value, index) order
   {
     int c = cd.abs_idx < 0 ? 1 : cmp_mag(hi, lo, sc, cd.abs_hi, cd.abs_lo, cd.abs_sc);
@@ -567,14 +598,31 @@ __device__ __forceinline__ void general_lane(Smem& sm, GenRec& cd, uint32_t G, u
       }
     }
   }
-  // exact sums: d = (s + t) 2^sc, |d| = (hi + lo) 2^sc, d^2 = (s^2 + 2st + t^2) 4^sc
-  sacc_add_f(sm, 0, s, false, sc);
-  sacc_add_f(sm, 0, t, false, sc);
-  sacc_add_f(sm, 1, hi, false, sc);
-  sacc_add_f(sm, 1, lo, false, sc);
-  sacc_add_prod_f(sm, 2, s, s, 2 * sc);
-  sacc_add_prod_f(sm, 2, s, t, 2 * sc + 1);
-  sacc_add_prod_f(sm, 2, t, t, 2 * sc);
+  o.s = s;
+  o.t = t;
+  o.sc = sc;
+}
+// One general pair per lane of a converged warp (valid: the lane has one):
+// the per-lane part, then the histogram bins and the exact sums, d = (s + t)
+// 2^sc, |d| = (hi + lo) 2^sc with (hi, lo) = +-(s, t), d^2 = (s^2 + 2st +
+// t^2) 4^sc, added by the whole warp.
+template <int DT>
+__device__ __forceinline__ void general_lane(Smem& sm, GenRec& cd, uint32_t G, uint32_t C, int64_t idx, float rtol,
+                                             float atol, bool valid) {
+  GenOut o{-1, -1, 0.0f, 0.0f, 0};
+  if (valid) general_pair<DT>(cd, o, G, C, idx, rtol, atol);
+  whist_add(sm, o.hb0);
+  whist_add(sm, o.hb1);
+  const bool on = o.s != 0.0f;
+  const bool neg = o.s < 0.0f;
+  const float hi = neg ? -o.s : o.s, lo = neg ? -o.t : o.t;
+  wsacc_add_f(sm, 0, o.s, o.sc, on);
+  wsacc_add_f(sm, 0, o.t, o.sc, on);
+  wsacc_add_f(sm, 1, hi, o.sc, on);
+  wsacc_add_f(sm, 1, lo, o.sc, on);
+  wsacc_add_prod_f(sm, 2, o.s, o.s, 2 * o.sc, on);
+  wsacc_add_prod_f(sm, 2, o.s, o.t, 2 * o.sc + 1, on);
+  wsacc_add_prod_f(sm, 2, o.t, o.t, 2 * o.sc, on);
 }
 
 // ---------------------------------------------------------------------------
@@ -1247,44 +1295,60 @@ __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p
   const int64_t lo = sm.lo;
   GenRec cd;
   gen_init(cd);
+  // whole warps in every round (general_lane adds with the whole warp)
+  const uint32_t lane = threadIdx.x & 31u, w0 = threadIdx.x & ~31u;
   if (n <= (uint32_t)GCAP) {
-    for (uint32_t e = threadIdx.x; e < n; e += BLOCK) {
-      const int64_t i = lo + sm.glist[e];
-      const uint32_t G = load_scalar<DT>(p.g, i);
-      general_lane<DT>(sm, cd, G, cand_at<DT, INJ>(p, i, G), i, W.rtol, W.atol);
+    for (uint32_t b = w0; b < n; b += BLOCK) {
+      const bool valid = b + lane < n;
+      int64_t i = 0;
+      uint32_t G = 0, C = 0;
+      if (valid) {
+        i = lo + sm.glist[b + lane];
+        G = load_scalar<DT>(p.g, i);
+        C = cand_at<DT, INJ>(p, i, G);
+      }
+      general_lane<DT>(sm, cd, G, C, i, W.rtol, W.atol, valid);
     }
   } else {
-    for (int64_t i = pb + threadIdx.x; i < pe; i += BLOCK) {
-      const uint32_t G = load_scalar<DT>(p.g, i), C = cand_at<DT, INJ>(p, i, G);
-      if (G == C) continue;
-      uint32_t gr = G, cr = C;
-      if constexpr (DT == PEAT_BF16) {
-        gr = G << 16;
-        cr = C << 16;
+    for (int64_t b = pb + w0; b < pe; b += BLOCK) {
+      const int64_t i = b + lane;
+      bool want = false;
+      uint32_t G = 0, C = 0;
+      if (i < pe) {
+        G = load_scalar<DT>(p.g, i);
+        C = cand_at<DT, INJ>(p, i, G);
+        want = G != C;
       }
-      // the window this pair was tested with: the head ran with the initial
-      // window, a body chunk with its warp's window of that time, the tail
-      // with its thread's warp's last window
-      int w = 0;
-      uint32_t ik = 0;
-      if (vb < ve && i >= vb) {
-        if (i >= ve) {
-          w = (int)(((i - ve) % BLOCK) >> 5);
-          ik = 0xFFFFFFFFu;
-        } else {
-          const int64_t k = (i - vb) / (CHV * Tr<DT>::VEC);
-          w = (int)(k % NW);
-          ik = (uint32_t)(k / NW);
+      if (want) {
+        uint32_t gr = G, cr = C;
+        if constexpr (DT == PEAT_BF16) {
+          gr = G << 16;
+          cr = C << 16;
         }
+        // the window this pair was tested with: the head ran with the initial
+        // window, a body chunk with its warp's window of that time, the tail
+        // with its thread's warp's last window
+        int w = 0;
+        uint32_t ik = 0;
+        if (vb < ve && i >= vb) {
+          if (i >= ve) {
+            w = (int)(((i - ve) % BLOCK) >> 5);
+            ik = 0xFFFFFFFFu;
+          } else {
+            const int64_t k = (i - vb) / (CHV * Tr<DT>::VEC);
+            w = (int)(k % NW);
+            ik = (uint32_t)(k / NW);
+          }
+        }
+        int r = (int)sm.nwin[w];
+        while (r > 0 && sm.wstart[w][r] > ik) r--;
+        Win Wi = W;
+        set_window_lb<DT>(Wi, sm.wlb[w][r]);
+        uint32_t ud;
+        float s, a, thr;
+        want = !in_window<DT>(gr, cr, to_f32<DT>(G), to_f32<DT>(C), Wi, ud, s, a, thr);
       }
-      int r = (int)sm.nwin[w];
-      while (r > 0 && sm.wstart[w][r] > ik) r--;
-      Win Wi = W;
-      set_window_lb<DT>(Wi, sm.wlb[w][r]);
-      uint32_t ud;
-      float s, a, thr;
-      if (!in_window<DT>(gr, cr, to_f32<DT>(G), to_f32<DT>(C), Wi, ud, s, a, thr))
-        general_lane<DT>(sm, cd, G, C, i, W.rtol, W.atol);
+      general_lane<DT>(sm, cd, G, C, i, W.rtol, W.atol, want);
     }
   }
   gen_counts(cd, sm);

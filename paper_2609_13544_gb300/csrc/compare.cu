@@ -382,11 +382,10 @@ struct GenRec {
 };
 
 // Maxima of the window pairs one thread evaluated exactly (offsets from the
-// CTA's first element; ties to the lower offset).  The rel record keeps the
-// ratio in normalised form an / mg with mg = |g| / 2^e(g) in [1, 2) and
-// an = |d| / 2^e(g).
+// CTA's first element; ties to the lower offset).  The rel record keeps |d|
+// and |g| of its pair (rd = 0: none).
 struct WinRec {
-  float amax, ra, rm;
+  float amax, rd, rg;
   uint32_t aidx, umax, uidx, ridx, pad;
 };
 
@@ -404,6 +403,7 @@ struct FinScratch {
 constexpr int NSTAGE = 2;  // a power of two: stage and phase are bit fields of the use count
 constexpr int RWMAX = 6;   // window moves per warp and piece
 constexpr int CHV = 64;
+constexpr int GSM = 128;   // general pairs per piece kept in shared memory
 
 struct __align__(128) Smem {
   uint4 ring_g[NW][NSTAGE][CHV];
@@ -417,8 +417,11 @@ struct __align__(128) Smem {
   long long ff, fu;                // first finite pair, first pair without NaN (search result)
   uint32_t* glist;                 // this CTA's list of general pairs (offsets), GCAP entries
   uint32_t gn;                     // entries appended in this piece (may exceed GCAP)
+  // the first GSM entries of the list stay here, with the pairs' bits
+  uint32_t gs_off[GSM], gs_g[GSM], gs_c[GSM];
   uint32_t nfe;                    // bitwise-equal pairs holding NaN or Inf
   int last;                        // this CTA finished the last piece of a one-segment call
+  unsigned pieces;                 // a one-segment call's pieces: the CTAs whose ranges are not empty
   FinScratch fin;
   int lb, ub;
   // each warp's windows in the current piece: window r applies from the warp's
@@ -696,8 +699,8 @@ __device__ __forceinline__ void thr_init(Thr& T) {
   T.trm = 1.0f;
 }
 __device__ __forceinline__ void rec_init(WinRec& r) {
-  r.amax = r.ra = 0.0f;
-  r.rm = 1.0f;
+  r.amax = r.rd = 0.0f;
+  r.rg = 1.0f;
   r.aidx = r.uidx = r.ridx = 0xFFFFFFFFu;
   r.umax = 0;
   r.pad = 0;
@@ -768,9 +771,10 @@ __device__ __forceinline__ void norm_ratio(float a, float gf, float& an, float& 
   mg = __uint_as_float((gb & 0x007FFFFFu) | 0x3F800000u);
 }
 
-// a pair outside the window: append its offset to the CTA's general list
-// (evaluated at the end of the piece; past GCAP entries the piece is rescanned)
-__device__ __forceinline__ void defer_pair(uint32_t li, Smem& sm) {
+// a pair outside the window: append it to the CTA's general list (evaluated
+// at the end of the piece; past GCAP entries the piece is rescanned).  G, C:
+// the pair's raw bits, kept with the first GSM entries.
+__device__ __forceinline__ void defer_pair(uint32_t li, uint32_t G, uint32_t C, Smem& sm) {
   const uint32_t slot = atomicAdd(&sm.gn, 1u);
   if (slot < (uint32_t)GCAP) sm.glist[slot] = li;
 }
@@ -785,7 +789,7 @@ __device__ __forceinline__ bool pair_proc(Lane& L, const Thr& T, uint32_t gr, ui
   uint32_t ud;
   float s, a, thr;
   if (!in_window<DT>(gr, cr, gf, cf, W, ud, s, a, thr)) {
-    defer_pair(li, sm);
+    defer_pair(li, DT == PEAT_BF16 ? gr >> 16 : gr, DT == PEAT_BF16 ? cr >> 16 : cr, sm);
     L.ndef++;
     return false;
   }
@@ -827,8 +831,8 @@ __device__ __forceinline__ void rescan_pair(uint32_t gr, uint32_t cr, float gf, 
   if (rel_greater<DT>(an, mg, T.tra, T.trm)) {
     T.tra = an;
     T.trm = mg;
-    r.ra = an;
-    r.rm = mg;
+    r.rd = a;
+    r.rg = fabsf(gf);
     r.ridx = li;
   }
 }
@@ -1155,12 +1159,20 @@ __device__ __forceinline__ void do_scalar(Lane& L, Thr& T, uint32_t G, uint32_t 
 // ---------------------------------------------------------------------------
 // CTA ranges: boundaries precomputed on the host
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ int cta_of(int64_t i, const CompareParams& p) {
-  int lo = 0, hi = p.nctas - 1;
+// The last CTA b with bounds[b] <= i (0 <= i), searched by a whole warp:
+// each round the lanes probe 32 evenly spaced bounds of the bracket and a
+// ballot keeps the last one at or below i, so 32^r CTAs take r rounds of
+// parallel loads instead of a chain of log2(nctas) dependent ones.
+__device__ __forceinline__ int cta_of_warp(int64_t i, const CompareParams& p) {
+  const int lane = threadIdx.x & 31;
+  int lo = 0, hi = p.nctas - 1;  // bounds[lo] = 0 <= i: the answer lies in [lo, hi]
   while (lo < hi) {
-    int mid = (lo + hi + 1) >> 1;
-    if (p.bounds[mid] <= i) lo = mid;
-    else hi = mid - 1;
+    const int step = (hi - lo + 32) / 32;
+    const int q = lo + lane * step;
+    const bool ok = lane == 0 || (q <= hi && __ldg(p.bounds + q) <= i);  // a prefix of the lanes (bounds ascend)
+    const int t = 31 - __clz(__ballot_sync(0xFFFFFFFFu, ok));
+    lo += t * step;
+    hi = min(hi, lo + step - 1);
   }
   return lo;
 }
@@ -1299,11 +1311,12 @@ __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p
   const uint32_t lane = threadIdx.x & 31u, w0 = threadIdx.x & ~31u;
   if (n <= (uint32_t)GCAP) {
     for (uint32_t b = w0; b < n; b += BLOCK) {
-      const bool valid = b + lane < n;
+      const uint32_t e = b + lane;
+      const bool valid = e < n;
       int64_t i = 0;
       uint32_t G = 0, C = 0;
       if (valid) {
-        i = lo + sm.glist[b + lane];
+        i = lo + sm.glist[e];
         G = load_scalar<DT>(p.g, i);
         C = cand_at<DT, INJ>(p, i, G);
       }
@@ -1373,18 +1386,12 @@ __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p
 
 // [pb, pe): the lowest index of a finite pair and of a pair without NaN
 // (the argmax when every error is zero), searched BLOCK elements at a time
+// (the piece's first pair, which settles both unless it holds NaN or Inf, is
+// tested when the piece starts; this search runs only when it did not)
 template <int DT, bool INJ>
 __device__ __noinline__ void first_pairs(Smem& sm, const CompareParams& p, int64_t pb, int64_t pe) {
   using Ty = Tr<DT>;
   constexpr long long NONE = 0x7FFFFFFFFFFFFFFFll;
-  if (threadIdx.x == 0) {
-    // the piece's first pair settles both unless it holds NaN or Inf
-    const uint32_t G0 = load_scalar<DT>(p.g, pb);
-    const uint32_t ag = G0 & Ty::MAG, ac = cand_at<DT, INJ>(p, pb, G0) & Ty::MAG;
-    const bool fin = ag < Ty::INF && ac < Ty::INF;
-    sm.ff = fin ? pb : NONE;
-    sm.fu = fin ? pb : NONE;
-  }
   for (int64_t base = pb;; base += BLOCK) {
     __syncthreads();
     if (base >= pe || (sm.ff != NONE && sm.fu != NONE)) break;
@@ -1462,7 +1469,7 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
     }
     (&sm.sacc[0][0])[j] += v;
   }
-  first_pairs<DT, INJ>(sm, p, pb, pe);
+  if (sm.ff == 0x7FFFFFFFFFFFFFFFll || sm.fu == 0x7FFFFFFFFFFFFFFFll) first_pairs<DT, INJ>(sm, p, pb, pe);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t lo = sm.lo;
   // window pairs = unequal pairs - general pairs; EXACT = the piece length -
@@ -1492,13 +1499,10 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
       w.abs_hi = r.amax;
       w.abs_idx = lo + r.aidx;
     }
-    if (r.ra > 0.0f) {
-      const int64_t i = lo + r.ridx;
-      const uint32_t Gi = load_scalar<DT>(p.g, i);
-      const float gf = to_f32<DT>(Gi), cf = to_f32<DT>(cand_at<DT, INJ>(p, i, Gi));
-      w.rel_hi = fabsf(__fsub_rn(cf, gf));
-      w.rel_g = fabsf(gf);
-      w.rel_idx = i;
+    if (r.rd > 0.0f) {
+      w.rel_hi = r.rd;
+      w.rel_g = r.rg;
+      w.rel_idx = lo + r.ridx;
     }
     if (r.umax > 0u) {
       w.ulp = DT == PEAT_BF16 ? r.umax >> 16 : r.umax;
@@ -1532,14 +1536,14 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
     if (v) atomicAdd(reinterpret_cast<unsigned long long*>(&acc->limbs[0][0]) + j, v);
   }
   // publish, then count this piece: the segment's pieces are the CTAs whose
-  // ranges meet it
-  __threadfence();
+  // ranges meet it (a multi-segment call finalizes in a second launch, after
+  // this one)
+  if (p.nseg == 1) __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) {
     sm.last = 0;
     if (p.nseg == 1) {  // one segment: its last CTA finalizes it (else a second launch does, in parallel)
-      const unsigned int pieces = (unsigned int)(cta_of(p.n_total - 1, p) - cta_of(0, p) + 1);
-      sm.last = atomicAdd(&acc->done, 1u) == pieces - 1u;
+      sm.last = atomicAdd(&acc->done, 1u) == sm.pieces - 1u;
     }
   }
   // reset the CTA totals for the next piece
@@ -1597,6 +1601,10 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
   W.inc = tid < HALF ? 1u : 65536u;
   Lane L;
   lane_init(L);
+  if (p.nseg == 1 && p.n_total > 0 && warp == 0) {  // (counted here, off the tail of the last piece)
+    const int b1 = cta_of_warp(p.n_total - 1, p), b0 = cta_of_warp(0, p);
+    if (lane == 0) sm.pieces = (unsigned)(b1 - b0 + 1);
+  }
   __syncthreads();
   if (blockIdx.x == 0 && p.has_empty) write_empty_segments(p);
   uint32_t seq = 0;      // this warp's bulk-copy stage uses so far (stage = seq % NSTAGE)
@@ -1635,6 +1643,12 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
     // exponent and the largest same-sign ULP distance of the first vectors
     if (tid == 0) sm.lb = sm.ub = 0;
     __syncthreads();
+    // the piece's first pair (its loads overlap the sample's)
+    uint32_t G0 = 0, C0 = 0;
+    if (tid == 0) {
+      G0 = load_scalar<DT>(p.g, pb);
+      C0 = cand_at<DT, INJ>(p, pb, G0);
+    }
     if (tid < nvec) {
       const uint4 gv = load_vec(p.g, (vb + (int64_t)tid * VEC) * Ty::BYTES);
       const uint4 cv = INJ ? inj_one<DT>(p, gv, vb + (int64_t)tid * VEC)
@@ -1652,6 +1666,12 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
       }
       atomicMax(&sm.lb, (int)emax);
       atomicMax(&sm.ub, (int)(32 - __clz(umax)));
+    }
+    if (tid == 0) {
+      constexpr long long NONE = 0x7FFFFFFFFFFFFFFFll;
+      const bool fin = (G0 & Ty::MAG) < Ty::INF && (C0 & Ty::MAG) < Ty::INF;
+      sm.ff = fin ? pb : NONE;
+      sm.fu = fin ? pb : NONE;
     }
     __syncthreads();
     // the piece's initial window, the first entry of every warp's window log
@@ -1808,7 +1828,7 @@ __device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s,
   Partial x;
   part_none(x);
   {
-    const int b0 = cta_of(s0, p), b1 = cta_of(s1 - 1, p);
+    const int b0 = cta_of_warp(s0, p), b1 = cta_of_warp(s1 - 1, p);
     for (int b = b0 + tid; b <= b1; b += BLOCK) part_merge(x, load_partial(p.partials + s + b));
   }
   part_warp_reduce(x);

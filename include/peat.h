@@ -371,13 +371,16 @@ const char* peat_last_error(peat_handle_t h);
  *     device and stall every stream;
  * and it does not need a handle (creating one allocates its workspace).
  *
- * Arguments, outputs and errors are those of peat_compare (one tensor, no
- * segments).  Instead of a handle's workspace it uses one fixed block of
- * device memory per device, reserved when the library's device code is
- * loaded (about 21 MB: per-CTA lists of general-path pairs for up to 320
- * CTAs, their partial results, the CTA bounds and one accumulator).  Nothing
- * is allocated by a call, on the device or on the host.
- *   - n above 320 * (2^31 - 65) elements is rejected with PEAT_ERR_UNSUPPORTED.
+ * Arguments and outputs are those of peat_compare (one tensor, no segments)
+ * for PEAT_F32, PEAT_F16 and PEAT_BF16 operands; PEAT_F64, PEAT_F8E4M3 and
+ * PEAT_F8E5M2 return PEAT_ERR_UNSUPPORTED.  Instead of a handle's workspace
+ * it uses one fixed block of device memory per device, reserved when the
+ * library's device code is loaded (about 21 MB: per-CTA lists of
+ * general-path pairs for up to 320 CTAs, their partial results, the CTA
+ * bounds, a status word and one accumulator).  Nothing is allocated by a
+ * call, on the device or on the host.
+ *   - Each CTA's range must stay below 2^31 - 64 elements (at most 320
+ *     CTAs, two per SM): a larger n is rejected with PEAT_ERR_UNSUPPORTED.
  *   - The block's accumulator must be zero when a call starts.  It is zero
  *     when the code loads and every call that runs to completion leaves it
  *     zero; a call that fails to launch clears it with cudaMemsetAsync.
@@ -387,14 +390,23 @@ const char* peat_last_error(peat_handle_t h);
  *   - The first call on each device does a one-time setup (it looks up the
  *     block's address with cudaGetSymbolAddress and sets kernel attributes);
  *     make it before any stream capture.
- *   - It launches two kernels on `stream` (the CTA bounds, then the compare).
- *   - A bounded device-side wait that expires leaves the outputs invalid;
- *     without a handle this entry point has no place to report it later.
- * Errors: as peat_compare, plus PEAT_ERR_UNSUPPORTED (n or device ordinal
- * beyond the limits); the text is in peat_last_error(NULL). */
+ *   - It launches two kernels on `stream`: the CTA bounds (which also
+ *     clears the block's status word), then the compare.
+ *   - A bounded device-side wait that expires leaves the outputs invalid and
+ *     marks them: argmax_abs, argmax_rel and argmax_ulp are then -2 (a value
+ *     no valid call produces).  peat_compare marks them the same way and also
+ *     reports PEAT_ERR_TIMEOUT on the handle's next call.
+ * Errors: as peat_compare, plus PEAT_ERR_UNSUPPORTED (n, dtype or device
+ * ordinal beyond the limits); the text is in peat_last_error(NULL). */
 peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, int64_t n, peat_dtype_t dtype,
                                    peat_tol_t tol, peat_stats_t* stats_out, uint64_t* hist_out,
                                    peat_stream_t stream);
+
+/* Testing aid for peat_compare_noalloc (the counterpart of
+ * PEAT_FLAG_TEST_EXPIRE_WAITS): on != 0 makes every bounded device-side wait
+ * of later calls give up at its first poll, so that the expired-wait marking
+ * can be exercised without a real stall; on = 0 restores the normal limit. */
+void peat_test_noalloc_expire_waits(int on);
 
 #ifdef __cplusplus
 }

@@ -77,7 +77,8 @@ class InjectModel(ctypes.Structure):
 
 EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
            "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc", "peat_topk_mean",
-           "peat_tensor_stats", "peat_spearman", "peat_mean_std", "peat_isclose_grid", "peat_inject_compare")
+           "peat_tensor_stats", "peat_spearman", "peat_mean_std", "peat_isclose_grid", "peat_inject_compare",
+           "peat_test_noalloc_expire_waits")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -111,6 +112,8 @@ def load(path: Optional[Path] = None) -> ctypes.CDLL:
     L.peat_last_error.restype = ctypes.c_char_p
     L.peat_compare_noalloc.argtypes = [vp, vp, i64, i32, Tol, vp, vp, vp]
     L.peat_compare_noalloc.restype = i32
+    L.peat_test_noalloc_expire_waits.argtypes = [i32]
+    L.peat_test_noalloc_expire_waits.restype = None
     L.peat_topk_mean.argtypes = [vp, vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, vp, vp]
     L.peat_topk_mean.restype = i32
     L.peat_isclose_grid.argtypes = [vp, vp, vp, i64, i32, vp, i32, vp, i32, vp, vp]
@@ -261,6 +264,11 @@ def peat_compare(h: Handle, golden, candidate, rtol: float, atol: float = 0.0, s
     _sync(stream)
     s = stats_to_dicts(stats.cpu().numpy())[0]
     return s, hist.cpu().numpy().view(np.uint64).reshape(2, 64)
+
+
+def peat_test_noalloc_expire_waits(on: bool) -> None:
+    """Testing aid: every bounded device-side wait of later peat_compare_noalloc calls gives up at once."""
+    load().peat_test_noalloc_expire_waits(1 if on else 0)
 
 
 def peat_compare_noalloc(golden, candidate, rtol: float, atol: float = 0.0, stream=None):

@@ -1878,6 +1878,8 @@ __device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s,
     r.sum_sq = f.sums[2];
     r.rtol_eff = p.rtol;
     r.atol_eff = p.atol;
+    if (p.status && (*reinterpret_cast<volatile unsigned int*>(p.status) & 1u))
+      r.argmax_abs = r.argmax_rel = r.argmax_ulp = -2;  // a bounded wait expired: the outputs are invalid
     p.stats[s] = r;
   }
   if (p.hist && tid < HBINS) p.hist[s * HBINS + tid] = hv + ((tid == 0 || tid == 64) ? f.cnt[0] : 0ull);
@@ -1926,24 +1928,27 @@ __host__ __device__ int64_t bound_t(int64_t b, int nctas, int64_t n, int64_t p0)
   return lo < n ? lo : n;
 }
 
-// offsets {0, n} and the CTA bounds of a one-tensor call, written on the device
+// offsets {0, n} and the CTA bounds of a one-tensor call, written on the
+// device; a non-null status word is cleared for the compare that follows
 template <int DT>
-__global__ void compare_bounds(int64_t* offsets, int64_t* bounds, int nctas, int64_t n, int64_t p0) {
+__global__ void compare_bounds(int64_t* offsets, int64_t* bounds, int nctas, int64_t n, int64_t p0,
+                               unsigned int* status) {
   for (int b = threadIdx.x; b <= nctas; b += blockDim.x) bounds[b] = bound_t<DT>(b, nctas, n, p0);
   if (threadIdx.x == 0) {
     offsets[0] = 0;
     offsets[1] = n;
+    if (status) *status = 0u;
   }
 }
 
 }  // namespace
 
 cudaError_t launch_bounds_on_device(int dtype, int64_t* offsets, int64_t* bounds, int nctas, int64_t n, int64_t p0,
-                                    cudaStream_t s) {
+                                    unsigned int* status, cudaStream_t s) {
   switch (dtype) {
-    case PEAT_F32: compare_bounds<PEAT_F32><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0); break;
-    case PEAT_F16: compare_bounds<PEAT_F16><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0); break;
-    case PEAT_BF16: compare_bounds<PEAT_BF16><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0); break;
+    case PEAT_F32: compare_bounds<PEAT_F32><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0, status); break;
+    case PEAT_F16: compare_bounds<PEAT_F16><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0, status); break;
+    case PEAT_BF16: compare_bounds<PEAT_BF16><<<1, BLOCK, 0, s>>>(offsets, bounds, nctas, n, p0, status); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

@@ -167,7 +167,7 @@ static cudaError_t single_bounds(peat_handle_t h, int dtype, int nctas, int64_t 
       h->single_nctas == nctas && h->single_stream == st)
     return cudaSuccess;
   h->single_valid = false;
-  cudaError_t e = peat::launch_bounds_on_device(dtype, h->d_single, h->d_single + 2, nctas, n, p0, st);
+  cudaError_t e = peat::launch_bounds_on_device(dtype, h->d_single, h->d_single + 2, nctas, n, p0, nullptr, st);
   if (e != cudaSuccess) return e;
   h->single_valid = true;
   h->single_dtype = dtype;
@@ -540,13 +540,15 @@ constexpr int NOALLOC_MAX_CTAS = 320;     // grid cap of the allocation-free com
 constexpr int NOALLOC_MAX_DEVICES = 64;
 struct NoallocScratch {
   peat::SegAcc acc;                                  // zero between calls
-  unsigned int status;                               // set by an expired device-side wait
+  unsigned int status;                               // set by an expired device-side wait, cleared per call
   unsigned int pad;
   int64_t offsets[2];                                // {0, n}, written by the bounds kernel
   int64_t bounds[NOALLOC_MAX_CTAS + 1];
   peat::Partial partials[1 + NOALLOC_MAX_CTAS];
   uint32_t glist[(size_t)NOALLOC_MAX_CTAS * peat::GCAP];
 };
+// testing aid: every bounded wait of the allocation-free compare gives up at once
+std::atomic<unsigned int> g_noalloc_wait_limit{1u << 24};
 
 struct NoallocDevice {
   std::atomic<int> ready{0};
@@ -1122,9 +1124,6 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
   if (n < 0) return noalloc_fail(PEAT_ERR_INVALID_ARG, "n < 0");
   if (n > 0 && (!golden || !candidate)) return noalloc_fail(PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
   if (!stats_out) return noalloc_fail(PEAT_ERR_INVALID_ARG, "stats_out is NULL");
-  // the per-CTA offsets of stage 1 are 32-bit: n / nctas must stay below 2^31 - 64
-  const int64_t max_n = (int64_t)NOALLOC_MAX_CTAS * (((int64_t)1 << 31) - 65);
-  if (n > max_n) return noalloc_fail(PEAT_ERR_UNSUPPORTED, "n exceeds the allocation-free limit (320 * (2^31 - 65))");
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return noalloc_cuda_fail(e, "cudaGetDevice");
@@ -1162,6 +1161,9 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
     p.p0 = -1;
   const int max_ctas = std::min(NOALLOC_MAX_CTAS, D.nsm * peat::compare_ctas_per_sm());
   p.nctas = (int)std::max<int64_t>(1, std::min<int64_t>(max_ctas, (n + 4095) / 4096));
+  // the per-CTA element offsets of stage 1 are 32-bit
+  if (n / p.nctas >= ((int64_t)1 << 31) - 64)
+    return noalloc_fail(PEAT_ERR_UNSUPPORTED, "n is too large for one call (2^31 - 64 elements or more per CTA)");
   p.offsets = S->offsets;
   p.bounds = S->bounds;
   p.partials = S->partials;
@@ -1169,12 +1171,14 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
   p.glist = S->glist;
   p.has_empty = n == 0;
   p.status = &S->status;
-  p.wait_limit = 1u << 24;
+  p.wait_limit = g_noalloc_wait_limit.load(std::memory_order_relaxed);
   p.rtol = rtol;
   p.atol = atol;
   p.stats = stats_out;
   p.hist = hist_out;
-  e = peat::launch_bounds_on_device(dtype, S->offsets, S->bounds, p.nctas, n, p.p0, st);
+  // the bounds kernel also clears the status word: a wait that expired in an
+  // earlier call must not mark this call's outputs
+  e = peat::launch_bounds_on_device(dtype, S->offsets, S->bounds, p.nctas, n, p.p0, &S->status, st);
   if (e != cudaSuccess) return noalloc_cuda_fail(e, "bounds launch");
   e = peat::launch_compare(dtype, p, st);
   if (e != cudaSuccess) {
@@ -1183,6 +1187,8 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
   }
   return PEAT_OK;
 }
+
+void peat_test_noalloc_expire_waits(int on) { g_noalloc_wait_limit.store(on ? 0u : (1u << 24)); }
 
 const char* peat_last_error(peat_handle_t h) {
   if (!h) return g_null_error_is_noalloc ? g_noalloc_error : g_create_error.c_str();

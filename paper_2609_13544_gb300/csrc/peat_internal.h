@@ -106,7 +106,7 @@ size_t compare_segacc_bytes();
 // offsets {0, n} and the nctas + 1 CTA bounds of a one-tensor call, computed
 // by a one-CTA kernel (for the caller that has no host staging buffer)
 cudaError_t launch_bounds_on_device(int dtype, int64_t* offsets, int64_t* bounds, int nctas, int64_t n, int64_t p0,
-                                    cudaStream_t s);
+                                    unsigned int* status, cudaStream_t s);
 
 // ---- mean of the top errors (topk.cu) ----
 // key(|d|) is an order-preserving 31-bit key of |c - g|.  A sample picks a

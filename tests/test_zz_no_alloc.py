@@ -84,10 +84,10 @@ def test_rejections_touch_nothing(peat_gpu):
     x = torch.zeros(16, dtype=torch.bfloat16, device="cuda")
     s, _ = outputs()
     tol = peat_gpu.Tol(1e-3, 0.0)
-    # n beyond the allocation-free limit: rejected before any device work
+    # n beyond the per-SM limit: rejected before any device work
     rc = L.peat_compare_noalloc(x.data_ptr(), x.data_ptr(), 1 << 40, 2, tol, s.data_ptr(), None, None)
     assert rc == 2
-    assert "allocation-free limit" in peat_gpu.peat_last_error(None)
+    assert "too large" in peat_gpu.peat_last_error(None)
     rc = L.peat_compare_noalloc(x.data_ptr(), x.data_ptr(), 16, 7, tol, s.data_ptr(), None, None)
     assert rc == 1
     rc = L.peat_compare_noalloc(x.data_ptr(), x.data_ptr(), -1, 2, tol, s.data_ptr(), None, None)
@@ -96,3 +96,19 @@ def test_rejections_touch_nothing(peat_gpu):
                                 None)
     assert rc == 1
     torch.cuda.synchronize()
+
+
+def test_expired_wait_marks_the_outputs_and_the_next_call_is_clean(peat_gpu, h):
+    """With every bounded wait giving up at once (testing aid), the outputs
+    carry the documented mark (argmax fields -2); the status word is cleared
+    per call, so the next normal call equals peat_compare again."""
+    import torch
+    gb, cb = noise_pairs("bf16", 1_000_003, seed=23)
+    g, c = to_device(gb, "bf16"), to_device(cb, "bf16")
+    peat_gpu.peat_test_noalloc_expire_waits(True)
+    try:
+        st, _ = peat_gpu.peat_compare_noalloc(g, c, 1e-3, 0.0)
+    finally:
+        peat_gpu.peat_test_noalloc_expire_waits(False)
+    assert st["argmax_abs"] == st["argmax_rel"] == st["argmax_ulp"] == -2
+    run_both(peat_gpu, h, g, c, 1e-3, 0.0)

@@ -83,7 +83,14 @@ typedef enum {
   PEAT_ERR_ALLOC = 3,       /* device or pinned allocation failed */
   PEAT_ERR_CUDA = 4,        /* a CUDA runtime call failed (text in peat_last_error) */
   PEAT_ERR_TIMEOUT = 5,     /* a bounded device-side wait expired */
-  PEAT_ERR_INTERNAL = 6     /* an internal consistency check failed */
+  PEAT_ERR_INTERNAL = 6     /* an internal consistency check failed: an exact
+                               accumulator of an earlier call needed a digit
+                               outside its range (the kernels never write it out
+                               of bounds but raise a library-wide mapped status
+                               word; the next handle call of any handle, or the
+                               next peat_compare_noalloc, returns this once and
+                               clears it; the outputs since the previous check
+                               are invalid) */
 } peat_status_t;
 
 /* Classes, in the order of peat_stats_t.count. */
@@ -120,7 +127,7 @@ typedef struct {
  * Outputs of calls on such a handle are not valid. */
 #define PEAT_FLAG_TEST_EXPIRE_WAITS 0x80000000u
 
-/* Signature of one tensor (or one segment).  144 bytes, no padding holes. */
+/* Signature of one tensor (or one segment).  160 bytes, no padding holes. */
 typedef struct {
   uint64_t n;                   /* pairs compared */
   uint64_t count[PEAT_NCLASS];  /* class counts; they sum to n */
@@ -136,6 +143,13 @@ typedef struct {
   double sum_signed;            /* RN64(sum d) */
   double rtol_eff;              /* the float32 tolerances actually used */
   double atol_eff;
+  /* The paper's Mean and Variance of Errors scores (Section IV-B-3) over the
+   * n_finite pairs, each the exact value rounded once (RN-even binary64,
+   * computed on the device from the exact sums; 0 if n_finite = 0):
+   *   mean_abs = sum |d| / n_finite,
+   *   var_abs  = (n_finite sum d^2 - (sum |d|)^2) / n_finite^2 (population). */
+  double mean_abs;
+  double var_abs;
 } peat_stats_t;
 
 /* Histograms of one tensor: 128 uint64 counters, [0..63] log2-relative-error
@@ -258,11 +272,7 @@ typedef struct {
   double threshold;   /* RN64 of the k-th largest |c - g| (0 if k = 0) */
   double sum;         /* RN64 of the exact sum of the k largest |c - g| */
   double mean;        /* RN64 of that exact sum divided by k (0 if k = 0) */
-  uint32_t exact;     /* 1: every field exact as defined.  0: more than 65536 pairs whose
-                         |c - g| is not a float32 value (float32 or float16 operands of
-                         different magnitudes) share the float32 rounding of the k-th
-                         largest; the excess were taken at that rounding, so sum, mean
-                         and threshold may be off by their rounding errors */
+  uint32_t exact;     /* always 1: every field is exact as defined (kept for the layout) */
   uint32_t reserved;
 } peat_topk_t;
 
@@ -275,7 +285,9 @@ typedef struct {
  * Streams both tensors three times (a radix select over an order-preserving
  * key of |c - g|, 10 + 11 + 10 bits, that sums exactly what it has resolved
  * as it goes), a fourth time only when more than 65536 pairs whose |c - g| is
- * not a float32 value lie within 1024 float32 steps of the k-th largest;
+ * not a float32 value lie within 1024 float32 steps of the k-th largest, and
+ * a fifth and sixth time only when more than 65536 of them share the float32
+ * rounding of the k-th largest (a radix select over their rounding errors);
  * asynchronously on `stream`.  The handle's workspace is shared with its
  * other calls (do not overlap them).
  * Errors: INVALID_ARG (null pointer with n > 0, n < 0, bad dtype, num = 0,
@@ -355,10 +367,26 @@ peat_status_t peat_tensor_stats(peat_handle_t h, const void* x, const int64_t* o
 peat_status_t peat_spearman(const double* x, const double* y, int64_t n, double* rho_out);
 peat_status_t peat_mean_std(const double* x, int64_t n, int ddof, double* mean_out, double* std_out);
 
+/* The cross-step trend of an error score over replayed epochs (Alg. 1 runs
+ * the Err step once per recorded epoch; Section IV-C-1 reads each layer's
+ * scores across epochs): the least-squares line log y = intercept +
+ * slope log x through the points (x[i], y[i]) with x[i] > 0 and y[i] > 0
+ * finite (the others, e.g. a step whose score is 0, are left out), so that
+ * y ~ exp(intercept) x^slope; an error growing like sqrt(step) gives slope
+ * 1/2.  Two passes over the log values with compensated sums (host code).
+ *   slope_out, intercept_out  NaN when fewer than two points remain or all
+ *                             their x are equal;
+ *   r2_out                    the fit's coefficient of determination, NaN
+ *                             when all remaining log y are equal;
+ *   used_out                  the number of points used (may be NULL).
+ * Errors: INVALID_ARG (null pointer, n < 0); text in peat_last_error(NULL). */
+peat_status_t peat_trend(const double* x, const double* y, int64_t n, double* slope_out, double* intercept_out,
+                         double* r2_out, int64_t* used_out);
+
 /* Text of the last error reported on h (never NULL; "" if none).  With
  * h == NULL, the last error on this thread of the calls that take no handle
  * (peat_signature_create, peat_compare_noalloc, peat_spearman,
- * peat_mean_std), whichever failed last. */
+ * peat_mean_std, peat_trend), whichever failed last. */
 const char* peat_last_error(peat_handle_t h);
 
 /* peat_compare without a handle and without any allocation.  The paper has no
@@ -402,11 +430,29 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
                                    peat_tol_t tol, peat_stats_t* stats_out, uint64_t* hist_out,
                                    peat_stream_t stream);
 
+/* Profiling aid: with event != NULL (a cudaEvent_t created on h's device),
+ * every later peat_compare, peat_compare_segmented and peat_inject_compare
+ * call on h records it on the call's stream right after enqueuing stage 1,
+ * i.e. before the per-segment finalize launch of a multi-segment call (a
+ * one-segment call finalizes inside stage 1).  Events recorded around the
+ * call then time stage 1 alone and the finalize alone.  NULL stops it.  The
+ * event must outlive its use.  Errors: INVALID_ARG (h NULL). */
+peat_status_t peat_set_stage1_event(peat_handle_t h, void* event);
+
 /* Testing aid for peat_compare_noalloc (the counterpart of
  * PEAT_FLAG_TEST_EXPIRE_WAITS): on != 0 makes every bounded device-side wait
  * of later calls give up at its first poll, so that the expired-wait marking
  * can be exercised without a real stall; on = 0 restores the normal limit. */
 void peat_test_noalloc_expire_waits(int on);
+
+/* Testing aid for the range check of the exact accumulators (runs on the
+ * host, no GPU involved): the kernels' split of +-m 2^e (m = m_hi 2^64 +
+ * m_lo, neg != 0 for the minus sign) into the signed 32-bit digits of their
+ * fixed-point sums.  digits_out (24 entries) receives the digit of weight
+ * 2^(32 j - 416) at index j.  Returns 1 if a nonzero digit fell outside those
+ * 24 (it is not written; the kernels report this case as PEAT_ERR_INTERNAL),
+ * else 0. */
+int32_t peat_test_for_digits(uint64_t m_lo, uint64_t m_hi, int32_t e, int32_t neg, int64_t* digits_out);
 
 #ifdef __cplusplus
 }

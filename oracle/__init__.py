@@ -7,7 +7,10 @@ from it.
 
 Everything is computed by ``peat_oracle.c`` (see its header comment for the
 definitions, which follow Section IV-B-3 "FI Assessment Scores" and the Err
-step of Alg. 1 / Alg. 2).  This module only marshals numpy arrays.
+step of Alg. 1 / Alg. 2).  This module marshals numpy arrays, and forms the
+last exact step of a few scores with Python integers and ``Fraction``: the
+mean and variance of |d| from the C code's exact sums, and the context
+statistics' mean and variance.
 """
 from __future__ import annotations
 
@@ -96,6 +99,8 @@ def lib() -> ctypes.CDLL:
         L.orc_compare.restype = i32
         L.orc_compare_segmented.argtypes = [vp, vp, vp, i64, i32, dbl, dbl, ctypes.POINTER(Stats), vp]
         L.orc_compare_segmented.restype = i32
+        L.orc_compare_segmented_sums.argtypes = [vp, vp, vp, i64, i32, dbl, dbl, ctypes.POINTER(Stats), vp, vp]
+        L.orc_compare_segmented_sums.restype = i32
         L.orc_topk_mean.argtypes = [vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, ctypes.POINTER(TopK)]
         L.orc_topk_mean.restype = i32
         L.orc_tensor_stats.argtypes = [vp, i64, i32, ctypes.POINTER(TStats)]
@@ -148,13 +153,28 @@ def compare(g, c, dtype: str, rtol: float, atol: float = 0.0):
     gb, cb = _bits(g, dtype), _bits(c, dtype)
     if gb.size != cb.size:
         raise ValueError("golden and candidate differ in length")
-    st = Stats()
-    hist = np.zeros((2, 64), np.uint64)
-    rc = lib().orc_compare(gb.ctypes.data, cb.ctypes.data, gb.size, DTYPES[dtype], rtol, atol,
-                           ctypes.byref(st), hist.ctypes.data)
-    if rc:
-        raise ValueError(f"oracle rejected the arguments (code {rc})")
-    return _stats_dict(st), hist
+    stats, hist = compare_segmented(gb, cb, [0, gb.size], dtype, rtol, atol)
+    return stats[0], hist[0]
+
+
+def mean_var(S1, S2, n_finite: int) -> tuple:
+    """The Mean and Variance of Errors scores (Section IV-B-3) over the n_f
+    finite pairs, from the exact sums S1 = sum |d| and S2 = sum d^2
+    (Fractions): mean = S1 / n_f and var = (n_f S2 - S1^2) / n_f^2
+    (population variance), each the exact rational rounded once
+    (float(Fraction) rounds to nearest even; past the largest double: inf)."""
+    if n_finite == 0:
+        return 0.0, 0.0
+    nf = int(n_finite)
+    return _rn(S1 / nf), _rn((nf * S2 - S1 * S1) / (nf * nf))
+
+
+def _rn(q) -> float:
+    """RN-even binary64 of a non-negative rational, +inf past the largest double."""
+    try:
+        return float(q)
+    except OverflowError:
+        return float("inf")
 
 
 def topk_mean(g, c, dtype: str, num: int = 1, den: int = 10) -> dict:
@@ -279,6 +299,35 @@ def mean_std(x, ddof: int = 0):
     return float(m), float(sd)
 
 
+def trend(x, y) -> dict:
+    """The cross-step trend of a score over replayed epochs (Alg. 1's Err step
+    per recorded epoch, read across epochs as in Section IV-C-1): the
+    least-squares line log y = intercept + slope log x through the points with
+    x, y finite and positive.  math.log per point, then the normal equations
+    in exact rationals on those logs, each result rounded once."""
+    import math
+    from fractions import Fraction
+    pts = [(math.log(float(a)), math.log(float(b))) for a, b in zip(x, y)
+           if math.isfinite(a) and math.isfinite(b) and a > 0 and b > 0]
+    out = {"slope": float("nan"), "intercept": float("nan"), "r2": float("nan"), "used": len(pts)}
+    m = len(pts)
+    if m < 2:
+        return out
+    lx = [Fraction(a) for a, _ in pts]
+    ly = [Fraction(b) for _, b in pts]
+    mx, my = sum(lx) / m, sum(ly) / m
+    sxx = sum((a - mx) ** 2 for a in lx)
+    if sxx == 0:
+        return out
+    sxy = sum((a - mx) * (b - my) for a, b in zip(lx, ly))
+    syy = sum((b - my) ** 2 for b in ly)
+    slope = sxy / sxx
+    out["slope"], out["intercept"] = float(slope), float(my - slope * mx)
+    if syy != 0:
+        out["r2"] = float(1 - (syy - slope * sxy) / syy)  # the residual sum of squares is syy - slope sxy
+    return out
+
+
 def compare_segmented(g, c, offsets: Sequence[int], dtype: str, rtol: float, atol: float = 0.0):
     """Per-segment signatures: (list of stats dicts, hist uint64[nseg, 2, 64])."""
     gb, cb = _bits(g, dtype), _bits(c, dtype)
@@ -288,11 +337,22 @@ def compare_segmented(g, c, offsets: Sequence[int], dtype: str, rtol: float, ato
         raise ValueError("bad offsets or lengths")
     st = (Stats * max(nseg, 1))()
     hist = np.zeros((max(nseg, 1), 2, 64), np.uint64)
-    rc = lib().orc_compare_segmented(gb.ctypes.data, cb.ctypes.data, off.ctypes.data, nseg,
-                                     DTYPES[dtype], rtol, atol, st, hist.ctypes.data)
+    words = np.zeros((max(nseg, 1), 2, ACC_WORDS), np.uint64)
+    rc = lib().orc_compare_segmented_sums(gb.ctypes.data, cb.ctypes.data, off.ctypes.data, nseg,
+                                          DTYPES[dtype], rtol, atol, st, hist.ctypes.data, words.ctypes.data)
     if rc:
         raise ValueError(f"oracle rejected the arguments (code {rc})")
-    return [_stats_dict(st[s]) for s in range(nseg)], hist[:nseg]
+    from fractions import Fraction
+    unit = 1 << (-ACC_LSB)
+    out = []
+    for s in range(nseg):
+        d = _stats_dict(st[s])
+        # the exact sums themselves (they let a caller combine segments exactly)
+        d["S1_exact"] = Fraction(_acc_int(words[s, 0]), unit)
+        d["S2_exact"] = Fraction(_acc_int(words[s, 1]), unit)
+        d["mean_abs"], d["var_abs"] = mean_var(d["S1_exact"], d["S2_exact"], d["n_finite"])
+        out.append(d)
+    return out, hist[:nseg]
 
 
 def ulp_key(bits: int, dtype: str) -> int:

@@ -418,8 +418,10 @@ static int tol_ok(double rtol, double atol, double* rtol_eff, double* atol_eff) 
   return 1;
 }
 
+/* words, if not NULL, receives the exact sums of |c-g| and of (c-g)^2 over
+ * the finite pairs: 2 * ORC_ACC_WORDS words (see orc_compare_segmented_sums) */
 static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, double rtol,
-                          double atol, orc_stats* st, uint64_t* hist) {
+                          double atol, orc_stats* st, uint64_t* hist, uint64_t* words) {
   memset(st, 0, sizeof(*st));
   memset(hist, 0, sizeof(uint64_t) * 128);
   st->n = (uint64_t)n;
@@ -540,6 +542,10 @@ static void compare_range(const void* gb, const void* cb, int64_t n, int dtype, 
   st->sum_abs = acc_to_double(&s_abs);
   st->sum_sq = acc_to_double(&s_sq);
   st->sum_signed = acc_to_double(&s_signed);
+  if (words) {
+    memcpy(words, s_abs.w, sizeof(s_abs.w));
+    memcpy(words + ACC_W, s_sq.w, sizeof(s_sq.w));
+  }
 }
 
 static int dtype_ok(int dtype) { return dtype == ORC_F32 || dtype == ORC_F16 || dtype == ORC_BF16; }
@@ -556,12 +562,18 @@ int orc_compare(const void* g, const void* c, int64_t n, int dtype, double rtol,
   double r, a;
   if (!dtype_ok_cmp(dtype) || n < 0 || !st || !hist || (n > 0 && (!g || !c))) return ORC_BAD_ARG;
   if (!tol_ok(rtol, atol, &r, &a)) return ORC_BAD_ARG;
-  compare_range(g, c, n, dtype, r, a, st, hist);
+  compare_range(g, c, n, dtype, r, a, st, hist, NULL);
   return ORC_OK;
 }
 
 int orc_compare_segmented(const void* g, const void* c, const int64_t* offsets, int64_t nseg,
                           int dtype, double rtol, double atol, orc_stats* st, uint64_t* hist) {
+  return orc_compare_segmented_sums(g, c, offsets, nseg, dtype, rtol, atol, st, hist, NULL);
+}
+
+int orc_compare_segmented_sums(const void* g, const void* c, const int64_t* offsets, int64_t nseg,
+                               int dtype, double rtol, double atol, orc_stats* st, uint64_t* hist,
+                               uint64_t* words) {
   double r, a;
   if (!dtype_ok_cmp(dtype) || nseg < 0 || !offsets || (nseg > 0 && (!st || !hist))) return ORC_BAD_ARG;
   if (!tol_ok(rtol, atol, &r, &a)) return ORC_BAD_ARG;
@@ -573,7 +585,7 @@ int orc_compare_segmented(const void* g, const void* c, const int64_t* offsets, 
   for (int64_t s = 0; s < nseg; s++) {
     int64_t b = offsets[s], e = offsets[s + 1];
     compare_range((const char*)g + sz * b, (const char*)c + sz * b, e - b, dtype, r, a, st + s,
-                  hist + 128 * s);
+                  hist + 128 * s, words ? words + (size_t)s * 2 * ACC_W : NULL);
   }
   return ORC_OK;
 }

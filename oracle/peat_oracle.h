@@ -33,9 +33,10 @@ enum { ORC_EXACT = 0, ORC_WITHIN_TOL = 1, ORC_MISMATCH = 2, ORC_NAN_INF_ASYM = 3
 /* return codes */
 enum { ORC_OK = 0, ORC_BAD_ARG = 1 };
 
-/* Per-tensor (or per-segment) signature.  Field order and types are chosen
- * to be bit-compatible with the library's result record so that tests can
- * compare the two byte by byte. */
+/* Per-tensor (or per-segment) signature.  Field order and types are those of
+ * the first 144 bytes of the library's result record; the record's last two
+ * fields (the mean and variance of |d|) are formed from the exact sums that
+ * orc_compare_segmented_sums returns. */
 typedef struct {
   uint64_t n;                 /* pairs compared */
   uint64_t count[ORC_NCLASS]; /* class counts */
@@ -61,6 +62,15 @@ int orc_compare(const void* g, const void* c, int64_t n, int dtype, double rtol,
  * Argmax indices are local to the segment. */
 int orc_compare_segmented(const void* g, const void* c, const int64_t* offsets, int64_t nseg,
                           int dtype, double rtol, double atol, orc_stats* st, uint64_t* hist);
+
+/* orc_compare_segmented, plus (words != NULL) the exact sums of |c-g| and of
+ * (c-g)^2 over each segment's finite pairs, in the fixed-point format below:
+ * segment s gets words[2 s ORC_ACC_WORDS ...] (sum |d|) followed by
+ * ORC_ACC_WORDS words of sum d^2.  The Mean and Variance of Errors scores
+ * (Section IV-B-3) are formed from them exactly (oracle/__init__.py). */
+int orc_compare_segmented_sums(const void* g, const void* c, const int64_t* offsets, int64_t nseg,
+                               int dtype, double rtol, double atol, orc_stats* st, uint64_t* hist,
+                               uint64_t* words);
 
 /* Mean of the top errors (Section IV-B-3, "Mean of Top 10% Errors"): over
  * the pairs with both operands finite, the k = ceil(n_finite * num / den)

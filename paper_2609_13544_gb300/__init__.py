@@ -21,7 +21,7 @@ from .buildlib import LIB, build  # noqa: F401
 DTYPE_CODES = {"f32": 0, "f16": 1, "bf16": 2}
 CLASSES = ("exact", "within_tol", "mismatch", "nan_inf_asym", "sign_flip")
 HIST_BINS = 128
-STATS_BYTES = 144
+STATS_BYTES = 160
 INJECT_KINDS = {
     "rz": 0, "rv": 1, "bitflip": 2, "nan_inf": 3, "signflip": 4, "rel_gauss": 5,
     "add_gauss": 6, "bias": 7, "cast_f16_rne": 8, "cast_f16_rtz": 9, "cast_bf16_rne": 10,
@@ -50,7 +50,7 @@ STATS_DTYPE = np.dtype([
     ("n", "<u8"), ("count", "<u8", (5,)), ("n_finite", "<u8"),
     ("max_abs", "<f8"), ("argmax_abs", "<i8"), ("max_rel", "<f8"), ("argmax_rel", "<i8"),
     ("max_ulp", "<u8"), ("argmax_ulp", "<i8"), ("sum_abs", "<f8"), ("sum_sq", "<f8"),
-    ("sum_signed", "<f8"), ("rtol_eff", "<f8"), ("atol_eff", "<f8"),
+    ("sum_signed", "<f8"), ("rtol_eff", "<f8"), ("atol_eff", "<f8"), ("mean_abs", "<f8"), ("var_abs", "<f8"),
 ])
 assert STATS_DTYPE.itemsize == STATS_BYTES
 
@@ -78,7 +78,7 @@ class InjectModel(ctypes.Structure):
 EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
            "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc", "peat_topk_mean",
            "peat_tensor_stats", "peat_spearman", "peat_mean_std", "peat_isclose_grid", "peat_inject_compare",
-           "peat_test_noalloc_expire_waits")
+           "peat_test_noalloc_expire_waits", "peat_test_for_digits", "peat_trend", "peat_set_stage1_event")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -114,6 +114,13 @@ def load(path: Optional[Path] = None) -> ctypes.CDLL:
     L.peat_compare_noalloc.restype = i32
     L.peat_test_noalloc_expire_waits.argtypes = [i32]
     L.peat_test_noalloc_expire_waits.restype = None
+    L.peat_test_for_digits.argtypes = [ctypes.c_uint64, ctypes.c_uint64, i32, i32, ctypes.c_void_p]
+    L.peat_test_for_digits.restype = i32
+    L.peat_trend.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p,
+                             ctypes.c_void_p, ctypes.c_void_p]
+    L.peat_trend.restype = i32
+    L.peat_set_stage1_event.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    L.peat_set_stage1_event.restype = i32
     L.peat_topk_mean.argtypes = [vp, vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, vp, vp]
     L.peat_topk_mean.restype = i32
     L.peat_isclose_grid.argtypes = [vp, vp, vp, i64, i32, vp, i32, vp, i32, vp, vp]
@@ -205,7 +212,7 @@ def _dev_tensor_check(*ts):
 
 def peat_compare_raw(h: Handle, golden, candidate, rtol: float, atol: float, stats_out, hist_out=None,
                      stream=None) -> None:
-    """peat_compare on preallocated device outputs (stats_out: uint8[144], hist_out: int64[128])."""
+    """peat_compare on preallocated device outputs (stats_out: uint8[160], hist_out: int64[128])."""
     _dev_tensor_check(golden, candidate)
     if golden.numel() != candidate.numel() or golden.dtype != candidate.dtype:
         raise ValueError("golden and candidate differ in size or dtype")
@@ -243,7 +250,7 @@ def peat_compare_segmented_raw(h: Handle, golden, candidate, offsets, rtol: floa
 
 
 def stats_to_dicts(raw: np.ndarray) -> list:
-    """Unpack host bytes (k*144) into dicts, one per peat_stats_t record."""
+    """Unpack host bytes (k*160) into dicts, one per peat_stats_t record."""
     arr = np.frombuffer(np.ascontiguousarray(raw).tobytes(), dtype=STATS_DTYPE)
     out = []
     for r in arr:
@@ -269,6 +276,14 @@ def peat_compare(h: Handle, golden, candidate, rtol: float, atol: float = 0.0, s
 def peat_test_noalloc_expire_waits(on: bool) -> None:
     """Testing aid: every bounded device-side wait of later peat_compare_noalloc calls gives up at once."""
     load().peat_test_noalloc_expire_waits(1 if on else 0)
+
+
+def peat_test_for_digits(m: int, e: int, neg: bool):
+    """Testing aid (host only): the kernels' digit split of +-m 2^e -> (24 signed
+    digits of weight 2^(32 j - 416), True if a digit fell outside them)."""
+    out = np.zeros(24, np.int64)
+    rc = load().peat_test_for_digits(m & (2 ** 64 - 1), m >> 64, int(e), 1 if neg else 0, out.ctypes.data)
+    return out, rc == 1
 
 
 def peat_compare_noalloc(golden, candidate, rtol: float, atol: float = 0.0, stream=None):
@@ -392,6 +407,28 @@ def peat_mean_std(x, ddof: int = 0):
     return m.value, sd.value
 
 
+def peat_set_stage1_event(h: Handle, event) -> None:
+    """Profiling aid: record `event` (a torch.cuda.Event that has been recorded
+    once, so that it exists; None: stop) after each later compare's stage-1 launch."""
+    ptr = None if event is None else ctypes.c_void_p(event.cuda_event)
+    _check(load().peat_set_stage1_event(h.ptr, ptr), h)
+
+
+def peat_trend(x, y) -> dict:
+    """Least-squares power-law trend of y against x (log y = intercept + slope log x)
+    over the points with both values finite and positive: dict of slope,
+    intercept, r2 and used (the number of points kept)."""
+    a, b = _host_doubles(x), _host_doubles(y)
+    if a.size != b.size:
+        raise ValueError("x and y differ in length")
+    sl, ic, r2 = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+    used = ctypes.c_int64()
+    rc = load().peat_trend(a.ctypes.data, b.ctypes.data, a.size, ctypes.byref(sl), ctypes.byref(ic),
+                           ctypes.byref(r2), ctypes.byref(used))
+    _check(rc, None)
+    return {"slope": sl.value, "intercept": ic.value, "r2": r2.value, "used": used.value}
+
+
 def inject_model(kind: str, k: int = 0, bit_lo: int = 0, bit_hi: int = 0, x: float = 0.0) -> dict:
     return {"kind": kind, "k": k, "bit_lo": bit_lo, "bit_hi": bit_hi, "x": x}
 
@@ -434,7 +471,7 @@ def _model_array(models: Sequence[dict]):
 
 def peat_inject_compare_raw(h: Handle, golden, models: Sequence[dict], seed: int, rtol: float, atol: float,
                             stats_out, hist_out=None, stream=None) -> None:
-    """peat_inject_compare on preallocated device outputs (stats_out: uint8[144], hist_out: int64[128])."""
+    """peat_inject_compare on preallocated device outputs (stats_out: uint8[160], hist_out: int64[128])."""
     _dev_tensor_check(golden)
     rc = load().peat_inject_compare(h.ptr, golden.data_ptr(), golden.numel(), dtype_code(golden),
                                     _model_array(models), len(models), ctypes.c_uint64(seed), Tol(rtol, atol),
@@ -458,11 +495,12 @@ def peat_inject_compare(h: Handle, golden, models: Sequence[dict], seed: int, rt
 
 
 def derived_scores(st: dict) -> dict:
-    """Host-side scores of Section IV-B-3 from one signature: mean, variance of |e|, bias, L2, RMS."""
+    """The scores of Section IV-B-3 from one signature.  Max, Mean and Variance
+    of |e| are the record's own fields (the mean and the variance computed on
+    the device, exact and rounded once); bias, L2 and RMS are conveniences
+    derived here from the rounded sums."""
     import math
     nf = st["n_finite"]
-    mean = st["sum_abs"] / nf if nf else 0.0
-    out = {"max": st["max_abs"], "mean": mean, "bias": st["sum_signed"] / nf if nf else 0.0,
-           "l2": math.sqrt(st["sum_sq"]), "rms": math.sqrt(st["sum_sq"] / nf) if nf else 0.0,
-           "var": (st["sum_sq"] / nf - mean * mean) if nf else 0.0}
-    return out
+    return {"max": st["max_abs"], "mean": st["mean_abs"], "var": st["var_abs"],
+            "bias": st["sum_signed"] / nf if nf else 0.0, "l2": math.sqrt(st["sum_sq"]),
+            "rms": math.sqrt(st["sum_sq"] / nf) if nf else 0.0}

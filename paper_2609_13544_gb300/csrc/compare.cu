@@ -43,6 +43,8 @@
 
 #include "exact.cuh"
 #include "inject_models.cuh"
+#include "meanvar.cuh"
+#include <nvtx3/nvToolsExt.h>
 #include "peat_internal.h"
 
 namespace peat {
@@ -393,6 +395,11 @@ struct WinRec {
 // tile of CHV 16-byte vectors of each tensor (two vectors per lane).
 constexpr int NW = BLOCK / 32;
 
+// scratch of the mean and variance of |d|: S1 = sum |d| and S2 = sum d^2,
+// both NLIMB digits weighing 2^(32 j + LIMB_LSB) (two more after carrying)
+using MV = MeanVarScratch<NLIMB + 2, NLIMB + 2, -LIMB_LSB / 32>;
+static_assert(LIMB_LSB % 32 == 0, "the S2 shift is a whole number of digits");
+
 // scratch of a segment's finalization
 struct FinScratch {
   unsigned long long cnt[8];
@@ -406,7 +413,10 @@ constexpr int CHV = 64;
 constexpr int GSM = 128;   // general pairs per piece kept in shared memory
 
 struct __align__(128) Smem {
-  uint4 ring_g[NW][NSTAGE][CHV];
+  union {  // the mean/variance scratch of a finalizing CTA reuses the (by then idle) staging ring
+    uint4 ring_g[NW][NSTAGE][CHV];
+    MV mv;
+  };
   uint4 ring_c[NW][NSTAGE][CHV];
   unsigned long long bar[NW][NSTAGE];
   unsigned long long hist[HBINS];
@@ -479,7 +489,7 @@ __device__ __forceinline__ void wsacc_add_prod_f(Smem& sm, int which, float x, f
 // one histogram bin per lane (bin < 0: none), counted once per distinct bin
 __device__ __forceinline__ void whist_add(Smem& sm, int bin) {
   const unsigned grp = __match_any_sync(0xFFFFFFFFu, bin);
-  if (bin >= 0 && (threadIdx.x & 31) == __ffs(grp) - 1)
+  if (bin >= 0 && (threadIdx.x & 31) == __ffs(grp) - 1 && PEAT_CHECK(bin < HBINS))
     atomicAdd(&sm.ghist[threadIdx.x >> 5][bin], (unsigned long long)__popc(grp));
 }
 
@@ -1317,6 +1327,7 @@ __device__ __noinline__ void run_general(Win W, Smem& sm, const CompareParams& p
       uint32_t G = 0, C = 0;
       if (valid) {
         i = lo + sm.glist[e];
+        if (!PEAT_CHECK(i >= 0 && i < p.n_total)) i = lo;  // a listed offset outside the tensor
         G = load_scalar<DT>(p.g, i);
         C = cand_at<DT, INJ>(p, i, G);
       }
@@ -1425,13 +1436,13 @@ __device__ void fold_round(Lane& L, Smem& sm, int lexp) {
     sum = __reduce_add_sync(0xFFFFFFFFu, sum);
     if (lane == 0 && sum) {
       const int bin = r < NUR ? 64 + r + 1 : 48 + Rows<DT>::KLO + (r - NUR);
-      sm.hist[bin] += sum;
+      if (PEAT_CHECK(bin >= 0 && bin < HBINS)) sm.hist[bin] += sum;
     }
   }
   __syncthreads();
 }
 
-__device__ void finalize_segment(const CompareParams& p, int64_t s, FinScratch& f);
+__device__ void finalize_segment(const CompareParams& p, int64_t s, FinScratch& f, MV& mv);
 __device__ void write_empty_segments(const CompareParams& p);
 
 // End of one segment piece [pb, pe): the integer totals go to the segment's
@@ -1525,7 +1536,9 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
       constexpr long long NONE = 0x7FFFFFFFFFFFFFFFll;
       x.first_fin = sm.ff == NONE ? -1 : sm.ff;
       x.first_ulp = sm.fu == NONE ? -1 : sm.fu;
-      *out = x;
+      if (PEAT_CHECK(seg >= 0 && seg < p.nseg && seg + (int64_t)blockIdx.x < p.nseg + p.nctas && pb <= pe &&
+                     pe <= p.n_total))
+        *out = x;
     }
   }
   for (int b = threadIdx.x; b < HBINS; b += BLOCK)
@@ -1556,7 +1569,7 @@ __device__ __forceinline__ void finish_piece(Lane& L, const Win& W, Smem& sm, co
   __syncthreads();
   if (sm.last) {
     __threadfence();
-    finalize_segment(p, seg, sm.fin);
+    finalize_segment(p, seg, sm.fin, sm.mv);
   }
 }
 
@@ -1719,7 +1732,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
           fail_seq = seq;
           if (lane == 0) atomicOr(p.status, 1u);
         }
-        if (!failed) {
+        if (!failed && PEAT_CHECK(k * CHV < nvec && vb + k * CHV * VEC - lo < ((int64_t)1 << 32))) {
           const int64_t v0 = k * CHV;
           const int nvalid = (int)min((int64_t)CHV, nvec - v0);
           if constexpr (INJ) {
@@ -1804,7 +1817,7 @@ __device__ __forceinline__ Partial load_partial(const Partial* src) {
 // maxima in CTA order, round the exact sums once, write the outputs and clear
 // the accumulator for the next call.  Uses the CTA's totals in shared memory
 // as scratch (they are zero on entry and on exit).
-__device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s, FinScratch& f) {
+__device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s, FinScratch& f, MV& mv) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t s0 = p.offsets[s], s1 = p.offsets[s + 1];
   SegAcc* acc = p.acc + s;
@@ -1840,7 +1853,10 @@ __device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s,
     else part_none(x);
     part_warp_reduce(x);
   }
-  __syncthreads();
+  if (tid == 64) carry_to_digits(limbs + 1 * NLIMB, NLIMB, mv.A);  // S1 = sum |d|
+  if (tid == 96) carry_to_digits(limbs + 2 * NLIMB, NLIMB, mv.B);  // S2 = sum d^2
+  // the mean and variance of |d| over the finite pairs (synchronises the block)
+  mean_var_block(mv, (uint64_t)(s1 - s0) - f.cnt[3], LIMB_LSB);
   if (tid == 0) {
     const unsigned long long* cnt = f.cnt;
     peat_stats_t r;
@@ -1878,6 +1894,8 @@ __device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s,
     r.sum_sq = f.sums[2];
     r.rtol_eff = p.rtol;
     r.atol_eff = p.atol;
+    r.mean_abs = mv.mean;
+    r.var_abs = mv.var;
     if (p.status && (*reinterpret_cast<volatile unsigned int*>(p.status) & 1u))
       r.argmax_abs = r.argmax_rel = r.argmax_ulp = -2;  // a bounded wait expired: the outputs are invalid
     p.stats[s] = r;
@@ -1889,7 +1907,8 @@ __device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s,
 // Segments of a multi-segment call, one CTA each, after stage 1.
 __global__ void __launch_bounds__(BLOCK) compare_finalize(CompareParams p) {
   __shared__ FinScratch f;
-  if (p.offsets[blockIdx.x] < p.offsets[blockIdx.x + 1]) finalize_segment(p, blockIdx.x, f);
+  __shared__ MV mv;
+  if (p.offsets[blockIdx.x] < p.offsets[blockIdx.x + 1]) finalize_segment(p, blockIdx.x, f, mv);
 }
 
 // The outputs of every empty segment (no pairs): zero counts and sums, argmax -1.
@@ -1909,12 +1928,19 @@ __device__ __noinline__ void write_empty_segments(const CompareParams& p) {
 
 template <int DT>
 cudaError_t launch_t(const CompareParams& p, cudaStream_t st) {
+  // NVTX ranges (host-side enqueue of each stage) for profilers; no cost without one attached
+  nvtxRangePushA(p.inj_n > 0 ? "peat inject+compare stage 1" : "peat compare stage 1");
   if (p.inj_n > 0) compare_stage1<DT, true><<<p.nctas, BLOCK, sizeof(Smem), st>>>(p);
   else compare_stage1<DT, false><<<p.nctas, BLOCK, sizeof(Smem), st>>>(p);
   cudaError_t e = cudaGetLastError();
+  nvtxRangePop();
+  if (e == cudaSuccess && p.stage1_event) e = cudaEventRecord(static_cast<cudaEvent_t>(p.stage1_event), st);
   if (e != cudaSuccess || p.nseg <= 1) return e;
+  nvtxRangePushA("peat compare stage 2 (per-segment finalize)");
   compare_finalize<<<(unsigned)p.nseg, BLOCK, 0, st>>>(p);
-  return cudaGetLastError();
+  e = cudaGetLastError();
+  nvtxRangePop();
+  return e;
 }
 
 template <int DT>
@@ -1996,5 +2022,16 @@ cudaError_t compare_prepare() {
 int compare_ctas_per_sm() { return CTAS_PER_SM; }
 size_t compare_partial_bytes() { return sizeof(Partial); }
 size_t compare_segacc_bytes() { return sizeof(SegAcc); }
+
+cudaError_t register_digit_status_compare(unsigned int* word) { return set_digit_status_here(word); }
+
+// The index arithmetic of for_digits run on the host (a test of the digit
+// split and of its range check; no GPU involved).
+int test_for_digits(uint64_t m_lo, uint64_t m_hi, int e, int neg, int64_t* out) {
+  for (int j = 0; j < NLIMB; j++) out[j] = 0;
+  t_host_digit_dropped = false;
+  for_digits(((unsigned __int128)m_hi << 64) | m_lo, e, neg != 0, [&](int j, int64_t v) { out[j] += v; });
+  return t_host_digit_dropped ? 1 : 0;
+}
 
 }  // namespace peat

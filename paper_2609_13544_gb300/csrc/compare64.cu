@@ -13,6 +13,7 @@
 #include <cstdint>
 
 #include "exact64.cuh"
+#include "meanvar.cuh"
 #include "peat_internal.h"
 
 namespace peat {
@@ -498,6 +499,13 @@ __global__ void __launch_bounds__(TB) compare64_finalize(Cmp64Params p) {
     S[k] = v;
   }
   __syncthreads();
+  // the mean and variance of |d| from S1 = sum |d| and S2 = sum d^2, both SL
+  // digits weighing 2^(32 j + SLSB) (two more after carrying)
+  __shared__ MeanVarScratch<SL + 2, SL + 2, -SLSB / 32> mv;
+  static_assert(SLSB % 32 == 0, "the S2 shift is a whole number of digits");
+  if (threadIdx.x == 0) carry_to_digits(S + SL, SL, mv.A);
+  if (threadIdx.x == 32) carry_to_digits(S + 2 * SL, SL, mv.B);
+  mean_var_block(mv, r.nfin, SLSB);
   if (threadIdx.x != 0) return;
   peat_stats_t o;
   o.n = (uint64_t)(p.offsets[seg + 1] - p.offsets[seg]);
@@ -517,6 +525,8 @@ __global__ void __launch_bounds__(TB) compare64_finalize(Cmp64Params p) {
   o.sum_sq = limbs_rn64(S + 2 * SL);
   o.rtol_eff = p.rtol;
   o.atol_eff = p.atol;
+  o.mean_abs = mv.mean;
+  o.var_abs = mv.var;
   p.stats[seg] = o;
 }
 

@@ -14,6 +14,7 @@
 #include <cstdint>
 #include <type_traits>
 
+#include "meanvar.cuh"
 #include "peat_internal.h"
 
 namespace peat {
@@ -408,6 +409,10 @@ __device__ double u128_to_double(u128 x) {
 template <int DT>
 __global__ void __launch_bounds__(TB) compare8_finalize(Cmp8Params p) {
   __shared__ Tot warp_tot[NW];
+  // S1 = s1 2^-S and S2 = s2 2^-2S: four digits each, no shift between them
+  __shared__ MeanVarScratch<4, 4, 0> mv;
+  __shared__ unsigned long long nfin;
+  constexpr int S = F8<DT>::S;
   const long long seg = blockIdx.x;
   Tot t;
   tot_init(t);
@@ -417,8 +422,16 @@ __global__ void __launch_bounds__(TB) compare8_finalize(Cmp8Params p) {
     tot_merge(t, o);
   }
   block_total(t, warp_tot);
+  if (threadIdx.x == 0) {
+    for (int j = 0; j < 4; j++) {
+      mv.A[j] = (uint32_t)(t.s1 >> (32 * j));
+      mv.B[j] = (uint32_t)(t.s2 >> (32 * j));
+    }
+    nfin = t.nfin;
+  }
+  __syncthreads();
+  mean_var_block(mv, nfin, -S);
   if (threadIdx.x != 0) return;
-  constexpr int S = F8<DT>::S;
   peat_stats_t r;
   r.n = (uint64_t)(p.offsets[seg + 1] - p.offsets[seg]);
   for (int k = 0; k < PEAT_NCLASS; k++) r.count[k] = t.cnt[k];
@@ -437,6 +450,8 @@ __global__ void __launch_bounds__(TB) compare8_finalize(Cmp8Params p) {
   r.sum_signed = t.sd < 0 ? -sdm : sdm;
   r.rtol_eff = (double)p.rtol;
   r.atol_eff = (double)p.atol;
+  r.mean_abs = mv.mean;
+  r.var_abs = mv.var;
   p.stats[seg] = r;
 }
 

@@ -3,6 +3,8 @@
 // (digit j weighs 2^(32 j + LIMB_LSB)), and the one rounding of such an
 // accumulator to binary64.
 #pragma once
+#include <cuda_runtime.h>
+
 #include <cstdint>
 
 #include "peat_internal.h"
@@ -32,11 +34,44 @@ __device__ __forceinline__ uint64_t split_double(double x, int& e) {
   return m | (1ull << 52);
 }
 
+// Where a digit outside an accumulator's range is reported: a mapped host
+// word shared by the whole library (bit STATUS_DIGIT_RANGE; the handle calls
+// return PEAT_ERR_INTERNAL once they see it).  Every source file that
+// includes this header has its own copy of the pointer, set on each device
+// by register_digit_status before its kernels run (null: not reported).
+static __device__ unsigned int* g_digit_status = nullptr;
+static inline cudaError_t set_digit_status_here(unsigned int* word) {
+  return cudaMemcpyToSymbol(g_digit_status, &word, sizeof(word));
+}
+#ifdef PEAT_CHECKED
+__device__ __forceinline__ bool check_ok(bool c) {
+  if (!c && g_digit_status) atomicOr(g_digit_status, STATUS_CHECK);
+  return c;
+}
+#define PEAT_CHECK(cond) (::peat::check_ok(cond))
+#else
+#define PEAT_CHECK(cond) true
+#endif
+
+// the host side of for_digits (only the index check of the test hook runs there)
+static thread_local bool t_host_digit_dropped = false;
+
+#pragma nv_exec_check_disable
+__host__ __device__ __forceinline__ void digit_dropped() {
+#ifdef __CUDA_ARCH__
+  if (g_digit_status) atomicOr(g_digit_status, STATUS_DIGIT_RANGE);
+#else
+  t_host_digit_dropped = true;
+#endif
+}
+
 // Signed 32-bit digits of +-m * 2^e (m < 2^128), delivered to f(digit, value).
-// Every value that occurs is a multiple of 2^LIMB_LSB and below 2^352; a digit
-// outside [0, NLIMB) is dropped rather than written out of bounds.
+// Every value that occurs is a multiple of 2^LIMB_LSB and below 2^352, so
+// every digit index lies in [0, NLIMB); a digit outside it (an internal
+// error) is not written out of bounds but reported through the status word.
+#pragma nv_exec_check_disable
 template <class F>
-__device__ __forceinline__ void for_digits(unsigned __int128 m, int e, bool neg, F&& f) {
+__host__ __device__ __forceinline__ void for_digits(unsigned __int128 m, int e, bool neg, F&& f) {
   if (m == 0) return;
   int p = e - LIMB_LSB;
   int j = p >> 5, r = p & 31;
@@ -47,8 +82,11 @@ __device__ __forceinline__ void for_digits(unsigned __int128 m, int e, bool neg,
   for (int k = 1; k < 4; k++) out[k] = (md[k] << r) | (r ? (md[k - 1] >> (32 - r)) : 0u);
   out[4] = r ? (md[3] >> (32 - r)) : 0u;
 #pragma unroll
-  for (int k = 0; k < 5; k++)
-    if (out[k] && (unsigned)(j + k) < (unsigned)NLIMB) f(j + k, neg ? -(int64_t)out[k] : (int64_t)out[k]);
+  for (int k = 0; k < 5; k++) {
+    if (!out[k]) continue;
+    if ((unsigned)(j + k) < (unsigned)NLIMB) f(j + k, neg ? -(int64_t)out[k] : (int64_t)out[k]);
+    else digit_dropped();
+  }
 }
 
 // RN-even binary64 of the exact value of NLIMB carry-save digits (digit j

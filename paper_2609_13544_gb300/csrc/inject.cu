@@ -12,6 +12,7 @@
 #include <cstdint>
 
 #include "inject_models.cuh"
+#include <nvtx3/nvToolsExt.h>
 #include "peat_internal.h"
 
 namespace peat {
@@ -94,6 +95,10 @@ cudaError_t elem_t(const InjectElemParams& p, cudaStream_t s) {
   if (p.n <= 0) return cudaSuccess;
   int64_t blocks = ((p.n + 3) / 4 + 255) / 256;
   if (blocks > 152 * 16) blocks = 152 * 16;
+  nvtxRangePushA("peat pseudo-error inject");
+  struct Pop {
+    ~Pop() { nvtxRangePop(); }
+  } pop;
   switch (p.kind) {
     case PEAT_INJ_NAN_INF: inject_elem<DT, PEAT_INJ_NAN_INF><<<(unsigned)blocks, 256, 0, s>>>(p); break;
     case PEAT_INJ_SIGNFLIP: inject_elem<DT, PEAT_INJ_SIGNFLIP><<<(unsigned)blocks, 256, 0, s>>>(p); break;
@@ -111,7 +116,9 @@ cudaError_t elem_t(const InjectElemParams& p, cudaStream_t s) {
 template <int DT>
 cudaError_t scatter_t(const InjectScatterParams& p, cudaStream_t s) {
   if (p.k <= 0) return cudaSuccess;
+  nvtxRangePushA("peat pseudo-error inject (fixed-count scatter)");
   inject_scatter<DT><<<(unsigned)((p.k + 255) / 256), 256, 0, s>>>(p);
+  nvtxRangePop();
   return cudaGetLastError();
 }
 

@@ -280,4 +280,6 @@ cudaError_t launch_isclose(int dtype, const IscParams& p, int nctas, cudaStream_
   return cudaErrorInvalidValue;
 }
 
+cudaError_t register_digit_status_isclose(unsigned int* word) { return set_digit_status_here(word); }
+
 }  // namespace peat

@@ -28,6 +28,7 @@ struct peat_handle_s {
   unsigned int* status_host = nullptr;  // mapped pinned error word written by the kernels
   unsigned int* status_dev = nullptr;
   unsigned int wait_limit = 1u << 24;   // polls before a pipeline wait gives up
+  void* stage1_event = nullptr;         // profiling aid: recorded after each compare's stage-1 launch
   int64_t* d_offsets = nullptr;  // offsets (nseg + 1) then CTA bounds (nctas + 1)
   int64_t* h_offsets = nullptr;  // pinned staging of the same
   int64_t* d_single = nullptr;   // one-tensor calls: {0, n} then CTA bounds, written on the device
@@ -84,6 +85,53 @@ peat_status_t cuda_fail(peat_handle_t h, cudaError_t e, const char* what) {
   cudaGetLastError();  // clear a sticky non-fatal error state
   return fail(h, PEAT_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }
+
+// The library-wide word of the exact accumulators' range check (bit
+// peat::STATUS_DIGIT_RANGE): one mapped, portable host word, allocated with
+// the first handle (or the first allocation-free call) and registered with
+// every kernel source once per device.
+std::mutex g_digit_mu;
+unsigned int* g_digit_host = nullptr;
+uint64_t g_digit_devices = 0;  // ordinals below 64 whose kernels report to it
+
+cudaError_t register_digit_status(int dev) {
+  std::lock_guard<std::mutex> lk(g_digit_mu);
+  if (dev >= 0 && dev < 64 && (g_digit_devices >> dev) & 1) return cudaSuccess;
+  cudaError_t e = cudaSuccess;
+  if (!g_digit_host) {
+    e = cudaHostAlloc((void**)&g_digit_host, sizeof(unsigned int), cudaHostAllocMapped | cudaHostAllocPortable);
+    if (e != cudaSuccess) {
+      g_digit_host = nullptr;
+      return e;
+    }
+    *(volatile unsigned int*)g_digit_host = 0;
+  }
+  unsigned int* dptr = nullptr;
+  e = cudaHostGetDevicePointer((void**)&dptr, g_digit_host, 0);
+  if (e == cudaSuccess) e = peat::register_digit_status_compare(dptr);
+  if (e == cudaSuccess) e = peat::register_digit_status_topk(dptr);
+  if (e == cudaSuccess) e = peat::register_digit_status_tstats(dptr);
+  if (e == cudaSuccess) e = peat::register_digit_status_isclose(dptr);
+  if (e == cudaSuccess && dev >= 0 && dev < 64) g_digit_devices |= 1ull << dev;
+  return e;
+}
+
+// true (and the word cleared) if a kernel reported a lost digit, or a failed
+// assertion of the checked build, since the last look; DIGIT_FAULT says which
+const char* g_digit_what = "";
+bool digit_fault_pending() {
+  if (!g_digit_host) return false;
+  const unsigned int w = __atomic_exchange_n(g_digit_host, 0u, __ATOMIC_RELAXED);
+  if (!w) return false;
+  g_digit_what = (w & peat::STATUS_DIGIT_RANGE)
+                     ? "an exact accumulator needed a digit outside its range in an earlier call (an internal "
+                       "error): the outputs of the calls since the previous check are invalid"
+                     : "an index or range assertion of the checked build failed in an earlier call: the outputs "
+                       "of the calls since the previous check are invalid";
+  return true;
+}
+#define DIGIT_FAULT g_digit_what
+
 
 // the element types of the main kernels (the 8-bit formats have their own compare)
 int dtype_bytes(int dt) { return dt == PEAT_F32 ? 4 : (dt == PEAT_F16 || dt == PEAT_BF16 ? 2 : 0); }
@@ -404,6 +452,7 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   const int64_t n = offsets[nseg];
   if (n > 0 && (!g || (!c && !inj))) return fail(h, PEAT_ERR_INVALID_ARG, "golden/candidate is NULL");
   if (nseg > 0 && !stats) return fail(h, PEAT_ERR_INVALID_ARG, "stats_out is NULL");
+  if (digit_fault_pending()) return fail(h, PEAT_ERR_INTERNAL, DIGIT_FAULT);
   if (h->status_host && *(volatile unsigned int*)h->status_host) {
     *(volatile unsigned int*)h->status_host = 0;
     return fail(h, PEAT_ERR_TIMEOUT,
@@ -474,6 +523,7 @@ peat_status_t compare_impl(peat_handle_t h, const void* g, const void* c, const 
   p.has_empty = 0;
   for (int64_t s = 0; s < nseg && !p.has_empty; s++) p.has_empty = offsets[s + 1] == offsets[s];
   p.status = h->status_dev;
+  p.stage1_event = h->stage1_event;
   p.wait_limit = h->wait_limit;
   p.rtol = rtol;
   p.atol = atol;
@@ -607,6 +657,12 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
     return PEAT_ERR_CUDA;
   }
   cudaDeviceGetAttribute(&h->nsm, cudaDevAttrMultiProcessorCount, h->device);
+  if (register_digit_status(h->device) != cudaSuccess) {
+    cudaGetLastError();
+    g_create_error = "could not set up the library's status word";
+    delete h;
+    return PEAT_ERR_CUDA;
+  }
   if (peat::compare_prepare() != cudaSuccess) {
     cudaGetLastError();
     g_create_error = "could not configure the compare kernels";
@@ -623,6 +679,7 @@ peat_status_t peat_signature_create(peat_handle_t* out, const peat_config_t* cfg
             cudaMalloc(&h->glist, sizeof(uint32_t) * (size_t)peat::GCAP * 2 * (size_t)h->max_ctas) == cudaSuccess &&
             cudaHostAlloc((void**)&h->status_host, sizeof(unsigned int), cudaHostAllocMapped) == cudaSuccess &&
             cudaHostGetDevicePointer((void**)&h->status_dev, h->status_host, 0) == cudaSuccess &&
+            (*(volatile unsigned int*)h->status_host = 0u, true) &&  // pinned memory starts undefined
             cudaMemset(h->acc, 0, acc_bytes) == cudaSuccess &&
             cudaMalloc(&h->d_offsets, sizeof(int64_t) * staging) == cudaSuccess &&
             cudaMallocHost(&h->h_offsets, sizeof(int64_t) * staging) == cudaSuccess &&
@@ -700,6 +757,7 @@ peat_status_t peat_topk_mean(peat_handle_t h, const void* golden, const void* ca
   if (!out) return fail(h, PEAT_ERR_INVALID_ARG, "out is NULL");
   DeviceGuard dg(h->device);
   if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
+  if (digit_fault_pending()) return fail(h, PEAT_ERR_INTERNAL, DIGIT_FAULT);
   peat::TopkParams p;
   std::memset(&p, 0, sizeof(p));
   p.g = golden;
@@ -766,6 +824,7 @@ peat_status_t peat_isclose_grid(peat_handle_t h, const void* golden, const void*
   for (int j = 0; j < na; j++) p.atol[j] = at[p.aperm[j]];
   DeviceGuard dg(h->device);
   if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
+  if (digit_fault_pending()) return fail(h, PEAT_ERR_INTERNAL, DIGIT_FAULT);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   p.g = golden;
   p.c = candidate;
@@ -817,6 +876,7 @@ peat_status_t peat_tensor_stats(peat_handle_t h, const void* x, const int64_t* o
   if (nseg == 0) return PEAT_OK;
   DeviceGuard dg(h->device);
   if (!dg.ok) return fail(h, PEAT_ERR_CUDA, "cudaSetDevice failed");
+  if (digit_fault_pending()) return fail(h, PEAT_ERR_INTERNAL, DIGIT_FAULT);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   peat::TsParams p;
   std::memset(&p, 0, sizeof(p));
@@ -938,6 +998,48 @@ peat_status_t peat_mean_std(const double* x, int64_t n, int ddof, double* mean_o
   }
   const double ss = csum([x, mean](int64_t i) { return (x[i] - mean) * (x[i] - mean); });
   *std_out = std::sqrt(ss / (double)(n - ddof));
+  return PEAT_OK;
+}
+
+peat_status_t peat_trend(const double* x, const double* y, int64_t n, double* slope_out, double* intercept_out,
+                         double* r2_out, int64_t* used_out) {
+  if (!slope_out || !intercept_out || !r2_out || n < 0 || (n > 0 && (!x || !y)))
+    return host_fail("null pointer or n < 0");
+  std::vector<double> lx, ly;
+  for (int64_t i = 0; i < n; i++)
+    if (std::isfinite(x[i]) && std::isfinite(y[i]) && x[i] > 0.0 && y[i] > 0.0) {
+      lx.push_back(std::log(x[i]));
+      ly.push_back(std::log(y[i]));
+    }
+  const int64_t m = (int64_t)lx.size();
+  if (used_out) *used_out = m;
+  *slope_out = *intercept_out = *r2_out = std::nan("");
+  if (m < 2) return PEAT_OK;
+  auto csum = [m](auto f) {  // compensated (Neumaier) sum of f(0..m-1)
+    double s = 0.0, c = 0.0;
+    for (int64_t i = 0; i < m; i++) {
+      const double v = f(i), t = s + v;
+      c += std::fabs(s) >= std::fabs(v) ? (s - t) + v : (v - t) + s;
+      s = t;
+    }
+    return s + c;
+  };
+  const double mx = csum([&](int64_t i) { return lx[i]; }) / (double)m;
+  const double my = csum([&](int64_t i) { return ly[i]; }) / (double)m;
+  const double sxx = csum([&](int64_t i) { return (lx[i] - mx) * (lx[i] - mx); });
+  const double sxy = csum([&](int64_t i) { return (lx[i] - mx) * (ly[i] - my); });
+  const double syy = csum([&](int64_t i) { return (ly[i] - my) * (ly[i] - my); });
+  if (!(sxx > 0.0)) return PEAT_OK;
+  const double b = sxy / sxx, a0 = my - b * mx;
+  *slope_out = b;
+  *intercept_out = a0;
+  if (syy > 0.0) {
+    const double sse = csum([&](int64_t i) {
+      const double r = ly[i] - (a0 + b * lx[i]);
+      return r * r;
+    });
+    *r2_out = 1.0 - sse / syy;
+  }
   return PEAT_OK;
 }
 
@@ -1138,6 +1240,8 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
       if (e != cudaSuccess || !ptr) return noalloc_cuda_fail(e, "cudaGetSymbolAddress(scratch)");
       e = peat::compare_prepare();
       if (e != cudaSuccess) return noalloc_cuda_fail(e, "could not configure the compare kernels");
+      e = register_digit_status(dev);
+      if (e != cudaSuccess) return noalloc_cuda_fail(e, "could not set up the library's status word");
       int nsm = 0;
       e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
       if (e != cudaSuccess || nsm <= 0) return noalloc_cuda_fail(e, "cudaDeviceGetAttribute(SM count)");
@@ -1146,6 +1250,7 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
       D.ready.store(1, std::memory_order_release);
     }
   }
+  if (digit_fault_pending()) return noalloc_fail(PEAT_ERR_INTERNAL, DIGIT_FAULT);
   NoallocScratch* S = D.scratch;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   peat::CompareParams p;
@@ -1188,7 +1293,18 @@ peat_status_t peat_compare_noalloc(const void* golden, const void* candidate, in
   return PEAT_OK;
 }
 
+peat_status_t peat_set_stage1_event(peat_handle_t h, void* event) {
+  if (!h) return PEAT_ERR_INVALID_ARG;
+  h->stage1_event = event;
+  return PEAT_OK;
+}
+
 void peat_test_noalloc_expire_waits(int on) { g_noalloc_wait_limit.store(on ? 0u : (1u << 24)); }
+
+int32_t peat_test_for_digits(uint64_t m_lo, uint64_t m_hi, int32_t e, int32_t neg, int64_t* digits_out) {
+  if (!digits_out) return -1;
+  return peat::test_for_digits(m_lo, m_hi, e, neg, digits_out);
+}
 
 const char* peat_last_error(peat_handle_t h) {
   if (!h) return g_null_error_is_noalloc ? g_noalloc_error : g_create_error.c_str();

@@ -92,6 +92,7 @@ struct CompareParams {
   float rtol, atol;        // float32 tolerances
   peat_stats_t* stats;
   uint64_t* hist;          // may be null
+  void* stage1_event;      // host side only: a cudaEvent_t recorded after the stage-1 launch (or null)
 };
 
 // Host-side launchers (compare.cu / inject.cu).
@@ -117,6 +118,7 @@ cudaError_t launch_bounds_on_device(int dtype, int64_t* offsets, int64_t* bounds
 constexpr int TK_NB0 = 1024, TK_NB1 = 2048, TK_NB2 = 1024, TK_WIN = 3;
 constexpr int64_t TK_SAMPLE = 1 << 18;  // pairs in the sample
 constexpr unsigned TK_LCAP = 65536;     // listed pairs whose |d| is not a float32 value
+constexpr int TK_NBL = 65536;           // bins of each 16-bit digit of the order key of a rounding error
 
 // Device state of one peat_topk_mean call, zero between calls.
 struct TopkState {
@@ -134,6 +136,12 @@ struct TopkState {
   unsigned int lowor, inexact;  // over the window pairs of pass 1: OR of the keys' low 10 bits, any |d| not a float32
   unsigned int skip2;           // pass 1 resolved the last digit itself (passes 2 and 3 return at once)
   long long limbs[NLIMB];       // exact sum of the |d| resolved above the prefix
+  // only when T's bucket has more than TK_LCAP pairs whose |d| is not a
+  // float32 value: a radix select over the order key of their rounding
+  // errors, high and low 16 bits (counts zero between calls)
+  unsigned long long histl[2][TK_NBL];
+  unsigned long long kreml[2];  // the rank left inside the selected high digit, then inside the low one
+  unsigned int dl[2];           // the selected high and low digits
 };
 struct TopkListEntry {
   float lo;      // |d| = (value of key + lo), the value of key taken as in the key's definition
@@ -283,5 +291,23 @@ cudaError_t launch_inject_elem(int dtype, const InjectElemParams& p, cudaStream_
 cudaError_t launch_inject_scatter(int dtype, const InjectScatterParams& p, cudaStream_t s);
 cudaError_t launch_gather(int dtype, const void* src, const int64_t* from, int64_t* out, int64_t k,
                           cudaStream_t s);
+
+// The range check of the exact accumulators (for_digits): each kernel source
+// sets bit STATUS_DIGIT_RANGE of a library-wide word when a digit would fall
+// outside its accumulator (an internal error: the bounds on the terms exclude
+// it); each
+// kernel source reports to `word` (a device pointer of a mapped host word),
+// set per device.
+constexpr unsigned int STATUS_DIGIT_RANGE = 2u;
+// The checked build (compiled with -DPEAT_CHECKED): index and range
+// assertions in the compare kernels.  A failed one sets STATUS_CHECK in the
+// same word and its guarded access is skipped; nothing traps.  Without the
+// macro every check is the constant true and compiles away.
+constexpr unsigned int STATUS_CHECK = 4u;
+cudaError_t register_digit_status_compare(unsigned int* word);
+cudaError_t register_digit_status_topk(unsigned int* word);
+cudaError_t register_digit_status_tstats(unsigned int* word);
+cudaError_t register_digit_status_isclose(unsigned int* word);
+int test_for_digits(uint64_t m_lo, uint64_t m_hi, int e, int neg, int64_t* out);
 
 }  // namespace peat

@@ -20,7 +20,10 @@
 //           of the pairs with key >> 10 = P1 whose |d| is not a float32 value
 //           (their rounding errors lo, |d| = value(key) + lo);
 //   pass 3  only if that list overflowed: the pairs with key >> 10 = P1 and
-//           key > T summed exactly, and T's inexact pairs listed again.
+//           key > T summed exactly, and T's inexact pairs listed again;
+//   pass 4, 5  only if even T's inexact pairs overflow the list: a radix
+//           select over the order key of T's rounding errors (16 + 16 bits),
+//           summing exactly the errors above the resolved prefix.
 // The last CTA to finish a pass selects its digit.  A one-CTA finalize adds
 // the P1 range above T from the histogram (every key there is one float32
 // value), m value(T) for the m pairs of T's bucket that belong to the top k,
@@ -722,6 +725,14 @@ __global__ void __launch_bounds__(TB) topk_pass2(TopkParams p) {
   }
 }
 
+__device__ __forceinline__ uint32_t order_key(float x) {
+  const uint32_t b = __float_as_uint(x);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float from_order_key(uint32_t u) {
+  return __uint_as_float((u & 0x80000000u) ? (u & 0x7FFFFFFFu) : ~u);
+}
+
 // Only when the list of the last pass overflowed: the pairs with key >> 10 =
 // P1 above T summed exactly, and T's pairs whose |d| is not a float32 listed.
 template <int DT>
@@ -763,12 +774,86 @@ __global__ void __launch_bounds__(TB) topk_pass3(TopkParams p) {
   if (pass_end(nullptr, 0, nullptr, lim, st, 2, &last_s) && threadIdx.x == 0) st->done[2] = 0;
 }
 
-__device__ __forceinline__ uint32_t order_key(float x) {
-  const uint32_t b = __float_as_uint(x);
-  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+// Only when pass 3 found more than TK_LCAP pairs of T's bucket whose |d| is
+// not a float32 value, so that their rounding errors lo (|d| = (vT + lo)
+// 2^scT) cannot all be listed: the m largest lo of the bucket (m = krem, its
+// pairs inside the top k), by a radix select on order_key(lo) in two 16-bit
+// digits.  Pairs whose |d| is a float32 value take part with lo = 0.
+// Pass 4 counts the bucket by the high digit; the last CTA selects it.
+template <int DT>
+__global__ void __launch_bounds__(TB) topk_pass4(TopkParams p) {
+  __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
+  __shared__ unsigned last_s;
+  TopkState* st = p.st;
+  if (st->k == 0 || st->skip2 || st->nlist2 <= TK_LCAP) return;
+  const uint32_t T = st->T;
+  tk_filtered<DT>(
+      p, ring + (threadIdx.x >> 5) * ring_cap<DT>(),
+      [&](uint32_t G, uint32_t C) {
+        const uint32_t u = raw_key<DT>(G, C);
+        return u >= KEY_OVF || u == T;
+      },
+      [&](uint32_t G, uint32_t C) {
+        if (!tk_finite<DT>(G, C)) return;
+        const float gf = tk_f32<DT>(G), cf = tk_f32<DT>(C);
+        if (tk_key(gf, cf) != T) return;
+        float hi, lo;
+        int sc;
+        tk_exact(gf, cf, hi, lo, sc);
+        atomicAdd(&st->histl[0][order_key(lo) >> 16], 1ull);
+      });
+  if (!pass_end(nullptr, 0, nullptr, nullptr, st, 2, &last_s)) return;
+  unsigned long long krem = __ldcg(&st->krem);
+  unsigned d;
+  select_digit<TK_NBL / TB>(st->histl[0], krem, d);
+  if (threadIdx.x == 0) {
+    st->dl[0] = d;
+    st->kreml[0] = krem;
+    st->done[2] = 0;
+  }
 }
-__device__ __forceinline__ float from_order_key(uint32_t u) {
-  return __uint_as_float((u & 0x80000000u) ? (u & 0x7FFFFFFFu) : ~u);
+
+// Pass 5: the bucket's lo above the high digit summed exactly, those at it
+// counted by the low digit; the last CTA selects the low digit.  Every bin of
+// the low digit stands for one float32 value of lo.
+template <int DT>
+__global__ void __launch_bounds__(TB) topk_pass5(TopkParams p) {
+  __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
+  __shared__ long long lim[NLIMB];
+  __shared__ unsigned last_s;
+  TopkState* st = p.st;
+  if (st->k == 0 || st->skip2 || st->nlist2 <= TK_LCAP) return;
+  for (int j = threadIdx.x; j < NLIMB; j += TB) lim[j] = 0;
+  __syncthreads();
+  const uint32_t T = st->T, dh = st->dl[0];
+  int scT;
+  key_value(T, scT);
+  tk_filtered<DT>(
+      p, ring + (threadIdx.x >> 5) * ring_cap<DT>(),
+      [&](uint32_t G, uint32_t C) {
+        const uint32_t u = raw_key<DT>(G, C);
+        return u >= KEY_OVF || u == T;
+      },
+      [&](uint32_t G, uint32_t C) {
+        if (!tk_finite<DT>(G, C)) return;
+        const float gf = tk_f32<DT>(G), cf = tk_f32<DT>(C);
+        if (tk_key(gf, cf) != T) return;
+        float hi, lo;
+        int sc;
+        tk_exact(gf, cf, hi, lo, sc);
+        const uint32_t u = order_key(lo);
+        if ((u >> 16) > dh) digits_of(lim, lo, scT);
+        else if ((u >> 16) == dh) atomicAdd(&st->histl[1][u & 0xFFFFu], 1ull);
+      });
+  if (!pass_end(nullptr, 0, nullptr, lim, st, 2, &last_s)) return;
+  unsigned long long krem = __ldcg(&st->kreml[0]);
+  unsigned d;
+  select_digit<TK_NBL / TB>(st->histl[1], krem, d);
+  if (threadIdx.x == 0) {
+    st->dl[1] = d;
+    st->kreml[1] = krem;
+    st->done[2] = 0;
+  }
 }
 
 // The P1 range, T's bucket, the rounding, the output; the state cleared for
@@ -782,7 +867,7 @@ __global__ void __launch_bounds__(TB) topk_finalize(TopkParams p) {
   r.n_finite = st->nfin;
   r.k = k;
   r.threshold = r.sum = r.mean = 0.0;
-  r.exact = 1;
+  r.exact = 1;  // every field is exact as defined, always
   r.reserved = 0;
   if (k > 0) {
     for (int j = tid; j < NLIMB; j += TB) lim[j] = st->limbs[j];
@@ -790,8 +875,8 @@ __global__ void __launch_bounds__(TB) topk_finalize(TopkParams p) {
     const uint32_t T = st->T, P1 = st->P1, d2 = T & 0x3FFu;
     const unsigned long long m = st->krem, nbT = st->hist2[d2];
     const bool ovf = st->nlist > TK_LCAP;
-    const unsigned L = ovf ? min(st->nlist2, TK_LCAP) : st->nlist;
-    if (ovf && st->nlist2 > TK_LCAP) r.exact = 0;
+    const bool radix = ovf && st->nlist2 > TK_LCAP;  // T's bucket resolved by passes 4 and 5
+    const unsigned L = radix ? 0u : ovf ? st->nlist2 : st->nlist;
     int scT;
     const float vT = key_value(T, scT);
     if (!ovf) {
@@ -814,7 +899,17 @@ __global__ void __launch_bounds__(TB) topk_finalize(TopkParams p) {
     for (unsigned i = tid; i < L; i += TB) lt += p.list[i].key == T ? 1u : 0u;
     const unsigned long long LT = block_sum(lt);
     float vstar = 0.0f;
-    if (LT > 0) {
+    if (radix) {
+      // the bucket's lo above the selected low digit: one float32 value per
+      // bin; the m-th largest lo is the selected bin's value
+      const uint32_t dh = st->dl[0], dlow = st->dl[1];
+      for (unsigned b = dlow + 1 + tid; b < (unsigned)TK_NBL; b += TB) {
+        const unsigned long long c = st->histl[1][b];
+        if (c) digits_of_n(lim, from_order_key((dh << 16) | b), scT, c);
+      }
+      vstar = from_order_key((dh << 16) | dlow);
+      if (tid == 0) digits_of_n(lim, vstar, scT, st->kreml[1]);
+    } else if (LT > 0) {
       const unsigned long long Z = nbT - LT;
       // u*: the largest order key with count(order key >= u*) >= m
       uint32_t u = 0;
@@ -855,8 +950,13 @@ __global__ void __launch_bounds__(TB) topk_finalize(TopkParams p) {
   for (int j = tid; j < TK_WIN * TK_NB1; j += TB) st->hist1[j] = 0;
   for (int j = tid; j < TK_NB2; j += TB) st->hist2[j] = 0;
   for (int j = tid; j < NLIMB; j += TB) st->limbs[j] = 0;
+  if (st->nlist > TK_LCAP && st->nlist2 > TK_LCAP)  // the radix passes ran: clear their counts
+    for (int j = tid; j < 2 * TK_NBL; j += TB) (&st->histl[0][0])[j] = 0;
+  __syncthreads();
   if (tid == 0) {
     st->nonfin = st->above = st->nfin = st->k = st->krem = 0;
+    st->kreml[0] = st->kreml[1] = 0;
+    st->dl[0] = st->dl[1] = 0;
     st->Plo = st->Phi = st->P0 = st->P1 = st->T = 0;
     st->ok = 0;
     st->nlist = st->nlist2 = 0;
@@ -874,7 +974,8 @@ int occ(K kernel) {
 template <int DT>
 int ctas_per_sm_t() {
   const int a = std::min(occ(topk_pass1<DT, false>), occ(topk_pass1<DT, true>));
-  const int b = std::min(std::min(occ(topk_pass0<DT>), occ(topk_pass2<DT>)), occ(topk_pass3<DT>));
+  const int b = std::min(std::min(occ(topk_pass0<DT>), occ(topk_pass2<DT>)),
+                         std::min(occ(topk_pass3<DT>), std::min(occ(topk_pass4<DT>), occ(topk_pass5<DT>))));
   return std::max(1, std::min(a, b));
 }
 
@@ -890,6 +991,8 @@ cudaError_t launch_t(const TopkParams& p, int nctas, cudaStream_t s) {
   topk_pass1<DT, true><<<nctas, TB, 0, s>>>(p);
   topk_pass2<DT><<<nctas, TB, 0, s>>>(p);
   topk_pass3<DT><<<nctas, TB, 0, s>>>(p);
+  topk_pass4<DT><<<nctas, TB, 0, s>>>(p);
+  topk_pass5<DT><<<nctas, TB, 0, s>>>(p);
   topk_finalize<<<1, TB, 0, s>>>(p);
   return cudaGetLastError();
 }
@@ -914,5 +1017,7 @@ cudaError_t launch_topk(int dtype, const TopkParams& p, int nctas, cudaStream_t 
   }
   return cudaErrorInvalidValue;
 }
+
+cudaError_t register_digit_status_topk(unsigned int* word) { return set_digit_status_here(word); }
 
 }  // namespace peat

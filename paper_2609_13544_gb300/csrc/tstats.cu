@@ -596,4 +596,6 @@ cudaError_t launch_tstats(int dtype, const TsParams& p, cudaStream_t s) {
   return cudaErrorInvalidValue;
 }
 
+cudaError_t register_digit_status_tstats(unsigned int* word) { return set_digit_status_here(word); }
+
 }  // namespace peat

@@ -70,16 +70,18 @@ def main():
          "counts": [2, 1, 1, 0, 0], "n_finite": 4, "max_abs": 1.0, "argmax_abs": 2, "max_rel": 0.5,
          "argmax_rel": 0, "max_ulp": 4194304, "argmax_ulp": 0, "sum_signed": -0.5, "sum_abs": 1.5,
          "sum_sq": 1.25, "relhist": {"0": 2, "46": 1, "47": 1}, "ulphist": {"0": 2, "63": 2},
-         "why": "d = (0.5, 0, -1, 0); 1 <= RN32(0.4)*3; 1->1.5 and 3->2 are both 2^22 key steps (tie -> index 0)"},
+         "mean_abs": 0.375, "var_abs": 0.171875,
+         "why": "d = (0.5, 0, -1, 0); 1 <= RN32(0.4)*3; 1->1.5 and 3->2 are both 2^22 key steps (tie -> index 0); "
+                "mean |d| = 1.5/4, var = 1.25/4 - (3/8)^2 = 11/64"},
         {"dtype": "f32", "g": [0.0, 0.0, 0.0], "c": [1.0, -1.0, 1.0], "rtol": 0.0, "atol": 0.0,
          "counts": [0, 0, 3, 0, 0], "n_finite": 3, "max_abs": 1.0, "argmax_abs": 0, "max_rel": float("inf"),
          "argmax_rel": 0, "max_ulp": 1065353216, "argmax_ulp": 0, "sum_signed": 1.0, "sum_abs": 3.0,
-         "sum_sq": 3.0, "relhist": {"63": 3}, "ulphist": {"63": 3},
-         "why": "ties resolve to the lowest index; g = 0 gives rel = +inf"},
+         "sum_sq": 3.0, "relhist": {"63": 3}, "ulphist": {"63": 3}, "mean_abs": 1.0, "var_abs": 0.0,
+         "why": "ties resolve to the lowest index; g = 0 gives rel = +inf; |d| all 1: mean 1, variance 0"},
         {"dtype": "f16", "g": [1.0, 1.0], "c": [1.0, 1.0], "rtol": 0.0, "atol": 0.0,
          "counts": [2, 0, 0, 0, 0], "n_finite": 2, "max_abs": 0.0, "argmax_abs": 0, "max_rel": 0.0,
          "argmax_rel": 0, "max_ulp": 0, "argmax_ulp": 0, "sum_signed": 0.0, "sum_abs": 0.0, "sum_sq": 0.0,
-         "relhist": {"0": 2}, "ulphist": {"0": 2},
+         "relhist": {"0": 2}, "ulphist": {"0": 2}, "mean_abs": 0.0, "var_abs": 0.0,
          "why": "identical tensors: every maximum is 0 at the first finite pair"},
     ]
     out = Path(__file__).with_name("hand_cases.json")

@@ -13,7 +13,7 @@ TORCH_DT = {"f32": "float32", "f16": "float16", "bf16": "bfloat16", "f8e4m3": "f
             "f8e5m2": "float8_e5m2"}
 WIDTH = {"f32": 32, "f16": 16, "bf16": 16, "f8e4m3": 8, "f8e5m2": 8}
 INT_KEYS = ("n", "count", "n_finite", "argmax_abs", "argmax_rel", "max_ulp", "argmax_ulp")
-EXACT_FLOAT_KEYS = ("max_abs", "max_rel", "rtol_eff", "atol_eff")
+EXACT_FLOAT_KEYS = ("max_abs", "max_rel", "rtol_eff", "atol_eff", "mean_abs", "var_abs")
 SUM_KEYS = ("sum_abs", "sum_sq", "sum_signed")
 SUM_RTOL = 1e-10  # the stated bound for the binary64 sums (the design is exact)
 

@@ -10,7 +10,7 @@ ROOT = Path(__file__).resolve().parents[1]
 
 def declared_functions():
     text = (ROOT / "include" / "peat.h").read_text()
-    return sorted(set(re.findall(r"^(?:peat_status_t|const char\*|void)\s+(peat_\w+)\s*\(", text, re.M)))
+    return sorted(set(re.findall(r"^(?:peat_status_t|const char\*|void|int32_t)\s+(peat_\w+)\s*\(", text, re.M)))
 
 
 def test_header_declares_the_boundary():
@@ -18,7 +18,8 @@ def test_header_declares_the_boundary():
         "peat_compare", "peat_compare_noalloc", "peat_compare_segmented", "peat_inject_compare", "peat_last_error",
         "peat_isclose_grid", "peat_mean_std", "peat_pseudo_error_inject", "peat_signature_create",
         "peat_signature_destroy",
-        "peat_spearman", "peat_tensor_stats", "peat_test_noalloc_expire_waits", "peat_topk_mean"])
+        "peat_set_stage1_event", "peat_spearman", "peat_tensor_stats", "peat_test_for_digits",
+        "peat_test_noalloc_expire_waits", "peat_topk_mean", "peat_trend"])
 
 
 def test_library_builds_and_exports_every_declared_symbol():
@@ -33,7 +34,7 @@ def test_binding_names_match_the_abi():
     import paper_2609_13544_gb300 as peat
     for name in declared_functions():
         assert hasattr(peat, name), name
-    assert peat.STATS_DTYPE.itemsize == 144
+    assert peat.STATS_DTYPE.itemsize == 160
     assert peat.TOPK_DTYPE.itemsize == 48
     assert peat.TSTATS_DTYPE.itemsize == 80
 
@@ -47,5 +48,41 @@ def test_last_error_without_handle_is_empty_string():
 def test_stats_layout_matches_oracle():
     import oracle
     import paper_2609_13544_gb300 as peat
-    assert ctypes.sizeof(oracle.Stats) == peat.STATS_DTYPE.itemsize
-    assert [f for f, _ in oracle.Stats._fields_] == list(peat.STATS_DTYPE.names)
+    # the library's record is the oracle's C record followed by the Mean and
+    # Variance of Errors scores, which the oracle forms from its exact sums
+    # in Python (oracle.mean_var)
+    assert ctypes.sizeof(oracle.Stats) + 16 == peat.STATS_DTYPE.itemsize
+    assert [f for f, _ in oracle.Stats._fields_] + ["mean_abs", "var_abs"] == list(peat.STATS_DTYPE.names)
+
+
+def test_digit_split_and_its_range_check():
+    """The exact accumulators' digit split (run on the host through the testing
+    aid): every in-range term comes back exactly as its digits (checked with
+    Python integers), and a term that needs a digit outside the 24 is reported,
+    never written.  The range is [2^-416, 2^352): digit j weighs 2^(32 j - 416)."""
+    import random
+    import paper_2609_13544_gb300 as peat
+    rng = random.Random(5)
+    for _ in range(2000):
+        bits = rng.choice([1, 24, 53, 64, 100, 128])
+        m = rng.getrandbits(bits) | 1
+        e = rng.randint(-416, 352 - bits)
+        neg = rng.random() < 0.5
+        d, dropped = peat.peat_test_for_digits(m, e, neg)
+        assert not dropped, (m, e)
+        total = sum(int(v) << (32 * j) for j, v in enumerate(d))  # value * 2^416
+        assert total == (-1 if neg else 1) * (m << (e + 416)), (m, e, neg)
+        assert all(abs(int(v)) < 2 ** 32 for v in d)
+    # the edges: the lowest digit's lowest bit, the highest digit's highest bit
+    d, dropped = peat.peat_test_for_digits(1, -416, False)
+    assert not dropped and int(d[0]) == 1 and not d[1:].any()
+    d, dropped = peat.peat_test_for_digits(1, 351, True)
+    assert not dropped and int(d[23]) == -(2 ** 31) and not d[:23].any()
+    # out of range below and above: reported, and nothing of it written
+    for m, e in [(1, -417), (1, 352), (3, 351), (2 ** 127 + 1, 300), (5, -1000)]:
+        d, dropped = peat.peat_test_for_digits(m, e, False)
+        assert dropped, (m, e)
+    d, dropped = peat.peat_test_for_digits(3, 351, False)  # 2^351 kept, 2^352 reported
+    assert dropped and int(d[23]) == 2 ** 31
+    d, dropped = peat.peat_test_for_digits(0, 10 ** 4, False)  # zero: nothing at all
+    assert not dropped and not d.any()

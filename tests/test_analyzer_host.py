@@ -92,3 +92,51 @@ def test_library_mean_std_matches_oracle(peat_host, oracle, ddof):
             assert math.isclose(sd, osd, rel_tol=1e-12, abs_tol=1e-300)
     with pytest.raises(peat_host.PeatError):
         peat_host.peat_mean_std([1.0], 2)
+
+
+# ---------------------------------------------------------------- cross-step trend
+def test_oracle_trend_against_polyfit_and_closed_forms(oracle):
+    """The trend against numpy.polyfit on the logs, and exact power laws."""
+    rng = np.random.default_rng(21)
+    x = np.arange(1, 64, dtype=np.float64)
+    y = 3e-5 * x ** 0.5 * np.exp(0.05 * rng.standard_normal(x.size))
+    t = oracle.trend(x, y)
+    b, a = np.polyfit(np.log(x), np.log(y), 1)
+    assert math.isclose(t["slope"], b, rel_tol=1e-12) and math.isclose(t["intercept"], a, rel_tol=1e-12)
+    r = np.log(y) - (a + b * np.log(x))
+    assert math.isclose(t["r2"], 1 - (r @ r) / np.sum((np.log(y) - np.log(y).mean()) ** 2), rel_tol=1e-10)
+    for p in (0.5, 1.0, -2.0):
+        t = oracle.trend(x, 7.0 * x ** p)
+        assert abs(t["slope"] - p) < 1e-13 and abs(t["intercept"] - math.log(7.0)) < 1e-12
+        assert abs(t["r2"] - 1.0) < 1e-12
+    # points outside the log domain are left out; too few points give NaN
+    t = oracle.trend([0.0, 1.0, 2.0, 4.0, 5.0], [1.0, 2.0, 4.0, 0.0, math.inf])
+    assert t["used"] == 2 and abs(t["slope"] - 1.0) < 1e-15
+    assert math.isnan(oracle.trend([1.0], [1.0])["slope"])
+    assert math.isnan(oracle.trend([2.0, 2.0], [1.0, 3.0])["slope"])
+    assert math.isnan(oracle.trend([1.0, 2.0], [3.0, 3.0])["r2"])
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_library_trend_matches_oracle(peat_host, oracle, seed):
+    rng = np.random.default_rng(seed)
+    n = [2, 64, 5000][seed]
+    x = np.arange(n, dtype=np.float64)  # x = 0 is left out on both sides
+    y = np.abs(rng.standard_normal(n)) * (x + 1) ** 0.7
+    y[rng.integers(0, n, max(1, n // 10))] = 0.0
+    got, want = peat_host.peat_trend(x, y), oracle.trend(x, y)
+    assert got["used"] == want["used"]
+    for k in ("slope", "intercept", "r2"):
+        if math.isnan(want[k]):
+            assert math.isnan(got[k]), k
+        else:
+            assert math.isclose(got[k], want[k], rel_tol=1e-11, abs_tol=1e-13), (k, got[k], want[k])
+
+
+def test_library_trend_edges(peat_host):
+    t = peat_host.peat_trend([1.0, 2.0, 4.0], [3.0, 6.0, 12.0])
+    assert abs(t["slope"] - 1.0) < 1e-15 and t["used"] == 3 and abs(t["r2"] - 1.0) < 1e-15
+    t = peat_host.peat_trend([1.0], [1.0])
+    assert t["used"] == 1 and math.isnan(t["slope"]) and math.isnan(t["r2"])
+    t = peat_host.peat_trend([], [])
+    assert t["used"] == 0 and math.isnan(t["intercept"])

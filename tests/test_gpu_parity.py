@@ -135,7 +135,7 @@ def test_determinism(peat_gpu, h):
     import torch
     gb, cb = noise_pairs("bf16", 3_000_001, seed=3)
     g, c = to_device(gb, "bf16"), to_device(cb, "bf16")
-    stats = [torch.empty(144, dtype=torch.uint8, device="cuda") for _ in range(3)]
+    stats = [torch.empty(160, dtype=torch.uint8, device="cuda") for _ in range(3)]
     hists = [torch.empty(128, dtype=torch.int64, device="cuda") for _ in range(3)]
     for s, hh in zip(stats, hists):
         peat_gpu.peat_compare_raw(h, g, c, 1e-3, 0.0, s, hh)
@@ -147,7 +147,7 @@ def test_determinism(peat_gpu, h):
 def test_invalid_arguments(peat_gpu, h):
     import torch
     g = torch.zeros(10, device="cuda")
-    s = torch.empty(144, dtype=torch.uint8, device="cuda")
+    s = torch.empty(160, dtype=torch.uint8, device="cuda")
     with pytest.raises(peat_gpu.PeatError) as e:
         peat_gpu.peat_compare_raw(h, g, g, -1.0, 0.0, s)
     assert e.value.status == 1
@@ -171,7 +171,7 @@ def test_forced_wait_expiry_reports_timeout_and_context_survives(peat_gpu, oracl
     import torch
     gb, cb = noise_pairs("bf16", 1_000_003, seed=17)
     g, c = to_device(gb, "bf16"), to_device(cb, "bf16")
-    s = torch.empty(144, dtype=torch.uint8, device="cuda")
+    s = torch.empty(160, dtype=torch.uint8, device="cuda")
     bad = peat_gpu.Handle(0, flags=peat_gpu.PEAT_FLAG_TEST_EXPIRE_WAITS)
     peat_gpu.peat_compare_raw(bad, g, c, 1e-3, 0.0, s)
     torch.cuda.synchronize()

@@ -5,6 +5,7 @@ configuration the bench times, compare the outputs the oracle can compute one
 by one (whole small segments) and check properties that hold at any size.
 """
 import math
+from fractions import Fraction
 
 import numpy as np
 import pytest
@@ -27,6 +28,16 @@ def h(peat_gpu):
 
 def host_bits(t, dtype):
     return t.contiguous().view(ITYPE[dtype]).cpu().numpy().view(NPT[dtype])
+
+
+def value_at(bits, i, dtype):
+    """The value of element i (a Python float, exact for every format here)."""
+    b = int(bits[i])
+    if dtype == "f32":
+        return float(np.array([b], np.uint32).view(np.float32)[0])
+    if dtype == "f16":
+        return float(np.array([b], np.uint16).view(np.float16)[0])
+    return float(np.array([b << 16], np.uint32).view(np.float32)[0])  # bf16
 
 
 def compare_workload(peat, oracle, h, w, ctx):
@@ -102,6 +113,31 @@ def test_c5_playback_reduced(peat_gpu, oracle, h, step):
         assert st["exact"] == w.n
 
 
+def test_c5_sweep_step_by_step_and_trend(peat_gpu, oracle, h):
+    """Config 5 as a sweep (Alg. 1's Err step once per recorded epoch): eight
+    steps spanning 0..63 of a 1,048,576-element bf16 sweep, each compared on
+    the device and by the oracle (every output bit for bit); the library's
+    cross-step trend of the device's mean |d| series equals the oracle's
+    trend of its own series."""
+    from paper_2609_13544_gb300 import workloads as W
+    sweep = W.PlaybackSweep(n=1 << 20, device="cuda")
+    steps = [0, 9, 18, 27, 36, 45, 54, 63]
+    dev_mean, orc_mean = [], []
+    for s in steps:
+        w = sweep.workload(s)
+        st = compare_workload(peat_gpu, oracle, h, w, f"c5 sweep step {s}")
+        if s == 0:
+            assert st["exact"] == w.n
+        dev_mean.append(st["mean_abs"])
+        gb, cb = host_bits(w.golden, "bf16"), host_bits(w.candidate, "bf16")
+        orc_mean.append(oracle.compare(gb, cb, "bf16", w.rtol, w.atol)[0]["mean_abs"])
+    assert dev_mean == orc_mean
+    got, want = peat_gpu.peat_trend(steps, dev_mean), oracle.trend(steps, orc_mean)
+    assert got["used"] == want["used"] >= 2
+    for k in ("slope", "intercept", "r2"):
+        assert math.isclose(got[k], want[k], rel_tol=1e-11), k
+
+
 def _check_properties(st, hist, n):
     assert sum(st["count"]) == n == st["n"]
     assert int(hist[0].sum()) == n and int(hist[1].sum()) == n
@@ -163,16 +199,38 @@ def _full_via_segments(peat, oracle, h, w, nseg, ctx):
     assert st["n"] == n and st["count"] == [sum(s["count"][k] for s in os_) for k in range(5)]
     assert st["n_finite"] == sum(s["n_finite"] for s in os_)
     assert np.array_equal(hist, oh.sum(axis=0))
+    def seg_of(i):
+        return int(np.searchsorted(off, i, side="right")) - 1
+
+    def exact(key, i):
+        """The exact value (a Fraction) of pair i's quantity behind `key`."""
+        if key == "max_ulp":  # an integer: the segment's own maximum is exact
+            return os_[seg_of(i)]["max_ulp"]
+        gv, cv = value_at(gb, i, w.dtype), value_at(cb, i, w.dtype)
+        a = abs(Fraction(cv) - Fraction(gv))
+        if key == "max_abs":
+            return a
+        return a / abs(Fraction(gv)) if gv != 0 else math.inf
+
     for key, idx in (("max_abs", "argmax_abs"), ("max_rel", "argmax_rel"), ("max_ulp", "argmax_ulp")):
         best = max(s[key] for s in os_ if s[idx] >= 0)
         assert st[key] == best, key
+        # the segments whose maximum rounds to the same value; among them the
+        # exact maximum (each segment's own argmax holds its exact maximum),
+        # and of equal exact values the lowest index, is the only answer
         cands = [int(off[k]) + os_[k][idx] for k in range(nseg) if os_[k][idx] >= 0 and os_[k][key] == best]
-        # one segment attains the rounded maximum: its index is the answer; several: any
-        # of them may hold the exact maximum, the lowest index among equal exact values
-        assert (st[idx] == cands[0]) if len(cands) == 1 else (st[idx] in cands), (key, st[idx], cands[:4])
+        top = max(exact(key, i) for i in cands)
+        want = min(i for i in cands if exact(key, i) == top)
+        assert st[idx] == want, (key, st[idx], want, cands[:4])
     for key in ("sum_abs", "sum_sq", "sum_signed"):
         total = math.fsum(s[key] for s in os_)
         assert abs(st[key] - total) <= 1e-10 * abs(total) + 1e-300, key
+    # the Mean and Variance of Errors scores of the whole tensor, bit for bit,
+    # from the segments' exact sums combined exactly
+    S1 = sum(s["S1_exact"] for s in os_)
+    S2 = sum(s["S2_exact"] for s in os_)
+    nf = sum(s["n_finite"] for s in os_)
+    assert (st["mean_abs"], st["var_abs"]) == oracle.mean_var(S1, S2, nf)
     return st
 
 

@@ -97,6 +97,18 @@ def ref_pair(gb: int, cb: int, dtype: str, rtol: float, atol: float, rank=None):
     return out
 
 
+def check_mean_var(st, absd):
+    """The Mean and Variance of Errors scores (Section IV-B-3) against the
+    statistics module run on the exact |d| values (Fractions in, Fractions
+    out: statistics.fmean would round, mean and pvariance do not)."""
+    import statistics
+    if not absd:
+        assert st["mean_abs"] == 0.0 and st["var_abs"] == 0.0
+        return
+    assert st["mean_abs"] == rn64(statistics.mean(absd))
+    assert st["var_abs"] == rn64(statistics.pvariance(absd))
+
+
 # ---------------------------------------------------------------- hand cases
 @pytest.mark.parametrize("case", GOLD["cases"], ids=lambda c: f"{c['dtype']}:{c['g']}:{c['c']}:{c['why'][:20]}")
 def test_hand_case(oracle, case):
@@ -119,7 +131,7 @@ def test_hand_aggregate(oracle, agg):
     st, h = oracle.compare(np.array(agg["g"], npt), np.array(agg["c"], npt), agg["dtype"], agg["rtol"], agg["atol"])
     assert st["count"] == agg["counts"]
     for k in ("n_finite", "max_abs", "argmax_abs", "max_rel", "argmax_rel", "max_ulp", "argmax_ulp",
-              "sum_signed", "sum_abs", "sum_sq"):
+              "sum_signed", "sum_abs", "sum_sq", "mean_abs", "var_abs"):
         assert st[k] == agg[k], k
     assert {str(i): int(v) for i, v in enumerate(h[0]) if v} == agg["relhist"]
     assert {str(i): int(v) for i, v in enumerate(h[1]) if v} == agg["ulphist"]
@@ -275,10 +287,12 @@ def test_f64_aggregate_against_exact_rationals(oracle):
     S0 = S1 = S2 = Fraction(0)
     best_a = best_r = None
     ia = ir = -1
+    absd = []
     for i in range(g.size):
         ref = ref_pair(int(g[i]), int(c[i]), "f64", 1e-6, 0.0)
         if not ref["finite"]:
             continue
+        absd.append(ref["a"])
         S0 += ref["d"]
         S1 += ref["a"]
         S2 += ref["d"] ** 2
@@ -288,6 +302,7 @@ def test_f64_aggregate_against_exact_rationals(oracle):
         if best_r is None or r > best_r:
             best_r, ir = r, i
     assert (st["sum_signed"], st["sum_abs"], st["sum_sq"]) == (rn64(S0), rn64(S1), rn64(S2))
+    check_mean_var(st, absd)
     assert st["argmax_abs"] == ia and st["max_abs"] == rn64(best_a)
     assert st["argmax_rel"] == ir
     assert st["max_rel"] == (math.inf if best_r == math.inf else rn64(best_r))
@@ -399,10 +414,12 @@ def test_aggregate_against_exact_rationals(oracle, dtype):
     S0 = S1 = S2 = Fraction(0)
     best_a = best_r = None
     ia = ir = -1
+    absd = []
     for i in range(g.size):
         ref = ref_pair(int(g[i]), int(c[i]), dtype, 1e-2, 0.0)
         if not ref["finite"]:
             continue
+        absd.append(ref["a"])
         S0 += ref["d"]
         S1 += ref["a"]
         S2 += ref["d"] ** 2
@@ -414,9 +431,70 @@ def test_aggregate_against_exact_rationals(oracle, dtype):
     assert st["sum_signed"] == float(S0)
     assert st["sum_abs"] == float(S1)
     assert st["sum_sq"] == float(S2)
+    check_mean_var(st, absd)
     assert st["argmax_abs"] == ia and st["max_abs"] == float(best_a)
     assert st["argmax_rel"] == ir
     assert st["max_rel"] == (math.inf if best_r == math.inf else float(best_r))
+
+
+def test_mean_var_cancellation_and_binary64_range(oracle):
+    """The variance is formed exactly, then rounded once: a variance nine
+    orders below mean^2 (where S2/n - mean^2 in doubles is off in the third
+    digit), |d| past the largest double (mean +inf, variance 0 or +inf) and a
+    variance on the subnormal grid, each against Fractions of the raw values."""
+    import statistics
+    c = (1 + np.arange(3) * 2.0 ** -23).astype(np.float32)
+    st, _ = oracle.compare(np.zeros(3, np.float32), c, "f32", 0.0)
+    vals = [Fraction(float(x)) for x in c]
+    assert st["mean_abs"] == float(statistics.mean(vals))
+    assert st["var_abs"] == float(statistics.pvariance(vals)) > 0
+    assert st["sum_sq"] / 3 - (st["sum_abs"] / 3) ** 2 != st["var_abs"]  # the naive formula is off
+    big = np.finfo(np.float64).max
+    st, _ = oracle.compare(np.array([-big, -big]), np.array([big, big]), "f64", 0.0)
+    assert st["mean_abs"] == math.inf and st["var_abs"] == 0.0
+    st, _ = oracle.compare(np.array([-big, 0.0]), np.array([big, 0.0]), "f64", 0.0)
+    assert st["mean_abs"] == big and st["var_abs"] == math.inf
+    d = [3 * 2.0 ** -520, 0.0, 2.0 ** -520]
+    st, _ = oracle.compare(np.zeros(3), np.array(d), "f64", 0.0)
+    var = statistics.pvariance([Fraction(x) for x in d])
+    assert 0 < st["var_abs"] < 2.0 ** -1022 and st["var_abs"] == float(var)
+    # non-finite pairs are left out of both scores
+    st, _ = oracle.compare(np.array([0.0, 0.0, 1.0], np.float32), np.array([2.0, np.nan, np.inf], np.float32),
+                           "f32", 0.0)
+    assert st["n_finite"] == 1 and st["mean_abs"] == 2.0 and st["var_abs"] == 0.0
+
+
+def test_playback_sweep_against_its_closed_form(oracle):
+    """Config 5's recipe at a small size.  Step 0 compares every snapshot with
+    itself: all EXACT.  At step s the candidate is the bf16 rounding of
+    g (1 + 1e-4 sqrt(s) z), z ~ N(0, 1), for a bf16 golden g, so it differs
+    from g exactly when the noise carries g out of g's own rounding interval:
+    above by more than half the step up, below by more than half the step
+    down (a quarter of the step at a power of two).  The expected number of
+    non-EXACT pairs is the sum of those two Gaussian tails over the pairs
+    (scipy.special.erfc); the oracle's count lies within 5 standard
+    deviations of it.  (So the measured error does not grow like sqrt(s): the
+    noise stays below half a bf16 step for small s, and the count follows the
+    tail beyond it.)"""
+    from scipy.special import erfc
+    from paper_2609_13544_gb300 import workloads as W
+    sweep = W.PlaybackSweep(n=262_144, device="cpu")
+    st, _ = oracle.compare(sweep.workload(0).golden, sweep.workload(0).candidate, "bf16", 2.0 ** -7)
+    assert st["exact"] == st["n"] == 262_144 and st["mean_abs"] == 0.0
+    for s in (16, 32, 48, 63):
+        w = sweep.workload(s)
+        st, _ = oracle.compare(w.golden, w.candidate, "bf16", w.rtol)
+        gb = w.golden.view(torch.int16).numpy().view(np.uint16).astype(np.uint32)
+        ef, mant = (gb >> 7) & 0xFF, gb & 0x7F
+        g = np.abs((gb << 16).view(np.float32).astype(np.float64))
+        ok = (ef > 0) & (ef < 255)  # normal goldens (zero stays zero; none is subnormal here)
+        step_up = np.exp2(ef.astype(np.float64) - 127 - 7)
+        step_dn = np.where(mant == 0, step_up / 2, step_up)
+        sig = 1e-4 * np.sqrt(s)
+        p = 0.5 * (erfc(step_up / 2 / g / sig / np.sqrt(2)) + erfc(step_dn / 2 / g / sig / np.sqrt(2)))
+        p = np.where(ok, p, 0.0)
+        mu, sd = p.sum(), np.sqrt((p * (1 - p)).sum())
+        assert abs((st["n"] - st["exact"]) - mu) <= 5 * sd + 1, (s, st["n"] - st["exact"], mu, sd)
 
 
 # ---------------------------------------------------------------- library routines

@@ -120,6 +120,90 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+class NvmlSampler:
+    """SM clock, its maximum, power and the clock event reasons of one GPU,
+    read in-process through NVML (read-only queries) every `period` seconds
+    on a background thread.  The GPU is found by the PCI bus id the CUDA
+    driver reports for the process's device (CUDA and NVML ordinals differ
+    under CUDA_VISIBLE_DEVICES).  available is False when NVML or the CUDA
+    driver library cannot be loaded; the caller then falls back to
+    nvidia-smi."""
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+               0x80: "hw_power_brake_slowdown", 0x2: "applications_clocks_setting"}
+
+    def __init__(self, cuda_ordinal: int, period: float = 0.01):
+        import ctypes
+        import threading
+        self.period = period
+        self.rows = []
+        self.available = False
+        self._stop = threading.Event()
+        self._thread = None
+        try:
+            self.nv = ctypes.CDLL("libnvidia-ml.so.1")
+            cu = ctypes.CDLL("libcuda.so.1")
+            if cu.cuInit(0) != 0:
+                return
+            dev = ctypes.c_int()
+            if cu.cuDeviceGet(ctypes.byref(dev), cuda_ordinal) != 0:
+                return
+            bus = ctypes.create_string_buffer(64)
+            if cu.cuDeviceGetPCIBusId(bus, 64, dev) != 0:
+                return
+            if self.nv.nvmlInit_v2() != 0:
+                return
+            self.h = ctypes.c_void_p()
+            if self.nv.nvmlDeviceGetHandleByPciBusId_v2(bus, ctypes.byref(self.h)) != 0:
+                return
+            mx = ctypes.c_uint()
+            self.max_mhz = mx.value if self.nv.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(mx)) == 0 else None
+            self.reasons_fn = getattr(self.nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                getattr(self.nv, "nvmlDeviceGetCurrentClocksThrottleReasons")
+            self.available = True
+        except (OSError, AttributeError):
+            self.available = False
+
+    def sample(self):
+        import ctypes
+        mhz, mw, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        ok = self.nv.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(mhz)) == 0  # NVML_CLOCK_SM
+        self.nv.nvmlDeviceGetPowerUsage(self.h, ctypes.byref(mw))
+        self.reasons_fn(self.h, ctypes.byref(rs))
+        if ok:
+            self.rows.append((time.perf_counter(), mhz.value, mw.value / 1000.0, rs.value))
+
+    def _run(self):
+        while not self._stop.is_set():
+            self.sample()
+            self._stop.wait(self.period)
+
+    def __enter__(self):
+        import threading
+        self.rows = []
+        if self.available:
+            self._stop.clear()
+            self._thread = threading.Thread(target=self._run, daemon=True)
+            self._thread.start()
+        return self
+
+    def __exit__(self, *a):
+        if self._thread is not None:
+            self._stop.set()
+            self._thread.join()
+            self.sample()
+
+    def summary(self, t0=None, t1=None) -> dict:
+        rows = [r for r in self.rows if (t0 is None or r[0] >= t0) and (t1 is None or r[0] <= t1)] or self.rows
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0, "source": "nvml"}
+        busy = [r for r in rows if not (r[3] & 0x1)] or rows  # samples not flagged idle
+        reasons = sorted({name for r in busy for bit, name in self.REASONS.items() if r[3] & bit})
+        return {"sm_mhz": statistics.median(r[1] for r in busy), "sm_max_mhz": self.max_mhz,
+                "sm_mhz_min": min(r[1] for r in busy), "power_w_max": max(r[2] for r in rows),
+                "reasons": reasons, "samples": len(rows), "samples_not_idle": len(busy),
+                "period_ms": self.period * 1e3, "source": "nvml in-process (read-only queries)"}
+
+
 def make_workload(name: str, device: str):
     from paper_2609_13544_gb300 import workloads as W
     if name == "c1":
@@ -232,6 +316,206 @@ def run_reference(args) -> None:
     print(json.dumps(line), flush=True)
 
 
+# --------------------------------------------------------------------------- oracle sample + parity
+INT_KEYS = ("n", "count", "n_finite", "argmax_abs", "argmax_rel", "max_ulp", "argmax_ulp")
+EXACT_KEYS = ("max_abs", "max_rel", "rtol_eff", "atol_eff", "mean_abs", "var_abs")
+SUM_KEYS = ("sum_abs", "sum_sq", "sum_signed")
+
+
+def _oracle_job(args):
+    import oracle
+    g, c, offs, dtype, rtol, atol = args
+    t0 = time.perf_counter()
+    st, hist = oracle.compare_segmented(g, c, offs, dtype, rtol, atol)
+    for d in st:  # the exact sums are Fractions; only the rounded outputs travel back
+        d.pop("S1_exact", None)
+        d.pop("S2_exact", None)
+    return time.perf_counter() - t0, st, hist
+
+
+def oracle_sample(w, pool, cores: int, pairs: int):
+    """The oracle on the first `pairs` pairs of a workload, cut at the
+    workload's own segment boundaries and at `cores` equal chunks (one
+    process each): (pairs/s, seconds, pairs, cut offsets, stats, hist)."""
+    import numpy as np
+    P = int(min(pairs, w.n))
+    chunks = np.linspace(0, P, cores + 1).astype(np.int64)
+    cuts = set(int(x) for x in chunks)
+    if w.offsets is not None:
+        cuts |= {int(o) for o in w.offsets if 0 <= int(o) <= P}
+    off = np.array(sorted(cuts), np.int64)
+    gb, cb = host_bits(w.golden[:P], w.dtype), host_bits(w.candidate[:P], w.dtype)
+    jobs = []
+    for a, b in zip(chunks[:-1], chunks[1:]):
+        if b > a:
+            sub = off[(off >= a) & (off <= b)]
+            jobs.append((gb[a:b], cb[a:b], sub - a, w.dtype, w.rtol, w.atol))
+    t0 = time.perf_counter()
+    res = list(pool.map(_oracle_job, jobs))
+    dt = time.perf_counter() - t0
+    stats = [d for r in res for d in r[1]]
+    hist = np.concatenate([r[2] for r in res])
+    return P / dt, dt, P, off, stats, hist
+
+
+def parity_on_sample(peat, h, w, off, ostats, ohist) -> dict:
+    """The CUDA path on the oracle's sample, cut the same way (one segmented
+    call): every integer output and maximum bit for bit, the binary64 sums
+    within 1e-10 relative."""
+    import numpy as np
+    P = int(off[-1])
+    gs, gh = peat.peat_compare_segmented(h, w.golden[:P], w.candidate[:P], off.tolist(), w.rtol, w.atol)
+    bad = None
+    for k, (a, b) in enumerate(zip(gs, ostats)):
+        for key in INT_KEYS + EXACT_KEYS:
+            if a[key] != b[key]:
+                bad = bad or f"segment {k}: {key} gpu={a[key]!r} oracle={b[key]!r}"
+        for key in SUM_KEYS:
+            if not (a[key] == b[key] or abs(a[key] - b[key]) <= 1e-10 * abs(b[key])):
+                bad = bad or f"segment {k}: {key} gpu={a[key]!r} oracle={b[key]!r}"
+    if not np.array_equal(np.asarray(gh), np.asarray(ohist)):
+        bad = bad or "histograms differ"
+    return {"status": "ok" if bad is None else "MISMATCH", "pairs": P, "segments": len(gs),
+            "checked": "counts, maxima, argmax, mean/var bit for bit; sums within 1e-10; both histograms",
+            **({"first_mismatch": bad} if bad else {})}
+
+
+# --------------------------------------------------------------------------- per-config timings
+def events_ms(torch, stream, fn, calls: int) -> float:
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(calls):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / calls
+
+
+def config_block(peat, h, name: str, w, stream, peak: float, cold: bool) -> dict:
+    """Hot timing (back-to-back calls, about 50 ms of them), cold timing with
+    L2 flushed between calls (a 512 MiB write) where asked, and for a
+    segmented call stage 1 alone against stage 1 + the finalize."""
+    import torch
+    nseg = 1 if w.offsets is None else len(w.offsets) - 1
+    dev = w.golden.device
+    stats = torch.empty(nseg * peat.STATS_BYTES, dtype=torch.uint8, device=dev)
+    hist = torch.empty(nseg * peat.HIST_BINS, dtype=torch.int64, device=dev)
+
+    def call():
+        if w.offsets is None:
+            peat.peat_compare_raw(h, w.golden, w.candidate, w.rtol, w.atol, stats, hist, stream)
+        else:
+            peat.peat_compare_segmented_raw(h, w.golden, w.candidate, w.offsets, w.rtol, w.atol, stats, hist, stream)
+
+    for _ in range(3):
+        call()
+    est = events_ms(torch, stream, call, 3)
+    calls = int(min(5000, max(10, 50.0 / max(est, 1e-3))))
+    ms = events_ms(torch, stream, call, calls)
+    nbytes = 2 * w.n * (4 if w.dtype == "f32" else 2)
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    out = {"workload": WORKLOAD_NAMES[name], "element": w.dtype, "pairs": w.n, "segments": nseg,
+           "algorithmic_bytes_per_call": nbytes,
+           "hot": {"calls": calls, "us_per_call": ms * 1e3, "pairs_per_s": w.n / (ms * 1e-3), "gbs": gbs,
+                   "frac": gbs / peak, "l2": "back to back" + (" (inputs fit in L2: re-read from L2)"
+                                                             if nbytes < 120e6 else " (inputs larger than L2)")}}
+    if cold:
+        flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+        times = []
+        for i in range(30):
+            flush.fill_(i & 255)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            call()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+        del flush
+        cm = statistics.median(times)
+        out["cold"] = {"calls": len(times), "us_per_call_median": cm * 1e3, "pairs_per_s": w.n / (cm * 1e-3),
+                       "gbs": nbytes / (cm * 1e-3) / 1e9, "frac": nbytes / (cm * 1e-3) / 1e9 / peak,
+                       "l2": "flushed before every call (512 MiB write, outside the timed call)"}
+    if nseg > 1:
+        mid = torch.cuda.Event(enable_timing=True)
+        mid.record(stream)
+        torch.cuda.synchronize()
+        peat.peat_set_stage1_event(h, mid)
+        s1, s2 = [], []
+        try:
+            for _ in range(20):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                call()
+                e1.record(stream)
+                torch.cuda.synchronize()
+                s1.append(e0.elapsed_time(mid))
+                s2.append(mid.elapsed_time(e1))
+        finally:
+            peat.peat_set_stage1_event(h, None)
+        a, b = statistics.median(s1), statistics.median(s2)
+        out["stage1_alone"] = {"us_stage1": a * 1e3, "us_finalize": b * 1e3, "us_total": (a + b) * 1e3,
+                               "stage1_gbs": nbytes / (a * 1e-3) / 1e9, "stage1_frac": nbytes / (a * 1e-3) / 1e9 / peak,
+                               "how": "events around each call and one the library records after the stage-1 "
+                                      "launch (peat_set_stage1_event); medians of 20 calls"}
+    del stats, hist
+    return out
+
+
+def c5_sweep(peat, h, stream, peak: float) -> dict:
+    """Config 5 as specified: 64 successive step snapshots of the
+    268,435,456-element bf16 tensor, generated beforehand (about 69 GB in
+    HBM), compared back to back in one timed region; the per-step series and
+    the cross-step trends (peat_trend) of mean |d| and max |d|."""
+    import numpy as np
+    import torch
+    from paper_2609_13544_gb300 import workloads as W
+    sweep = W.PlaybackSweep(device="cuda")
+    n, S = sweep.n, 64
+    G = torch.empty((S, n), dtype=torch.bfloat16, device="cuda")
+    C = torch.empty((S, n), dtype=torch.bfloat16, device="cuda")
+    for s in range(S):
+        sweep.step(s, out_g=G[s], out_c=C[s])
+    del sweep
+    rtol = 2.0 ** -7
+    stats = torch.empty(S * peat.STATS_BYTES, dtype=torch.uint8, device="cuda")
+    hist = torch.empty(S * peat.HIST_BINS, dtype=torch.int64, device="cuda")
+
+    def one(s):
+        peat.peat_compare_raw(h, G[s], C[s], rtol, 0.0, stats[s * peat.STATS_BYTES:(s + 1) * peat.STATS_BYTES],
+                              hist[s * peat.HIST_BINS:(s + 1) * peat.HIST_BINS], stream)
+
+    for s in range(3):
+        one(s)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for s in range(S):
+        one(s)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    st = peat.stats_to_dicts(stats.cpu().numpy())
+    del G, C, stats, hist
+    torch.cuda.empty_cache()
+    steps = list(range(S))
+    mean_abs = [d["mean_abs"] for d in st]
+    max_abs = [d["max_abs"] for d in st]
+    nbytes = 2 * n * 2
+    return {"workload": "playback sweep: steps 0..63 of a 268,435,456-element bf16 tensor, golden_s = x0 + s drift, "
+                        "candidate_s = golden_s (1 + 1e-4 sqrt(s) z) rounded to bf16, rtol 2^-7",
+            "steps": S, "pairs_per_step": n, "ms_total": ms, "us_per_step": ms * 1e3 / S,
+            "pairs_per_s": S * n / (ms * 1e-3), "gbs": S * nbytes / (ms * 1e-3) / 1e9,
+            "frac": S * nbytes / (ms * 1e-3) / 1e9 / peak,
+            "step0_all_exact": st[0]["exact"] == n,
+            "series": {"max_abs": max_abs, "mean_abs": mean_abs, "var_abs": [d["var_abs"] for d in st],
+                       "non_exact": [d["n"] - d["exact"] for d in st], "mismatch": [d["mismatch"] for d in st],
+                       "max_ulp": [d["max_ulp"] for d in st]},
+            "trend_mean_abs": peat.peat_trend(steps, mean_abs), "trend_max_abs": peat.peat_trend(steps, max_abs),
+            "note": "trend = least-squares slope of log score against log step over the steps with a nonzero "
+                    "score (peat_trend); the injected noise grows like sqrt(s) but a bf16 candidate differs "
+                    "only where it exceeds half a bf16 step, so mean |d| follows that Gaussian tail"}
+
+
 # --------------------------------------------------------------------------- the CUDA path
 def run_gpu(args) -> None:
     import numpy as np
@@ -265,6 +549,8 @@ def run_gpu(args) -> None:
     torch.cuda.synchronize()
     st = peat.stats_to_dicts(stats.cpu().numpy())
     assert sum(sum(s["count"]) for s in st) == w.n, "counts do not add up to n"
+    peaks = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", 6800.0))
 
     def barrier():
         if world > 1:
@@ -272,11 +558,42 @@ def run_gpu(args) -> None:
             dist.barrier()
         torch.cuda.synchronize()
 
+    # N = 1: the oracle leg first (the cpu_baseline of every config, and on
+    # the same sample the parity of the CUDA path, before anything is timed),
+    # then each config's own timings
+    cpu, parity, configs = None, None, None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        cores = os.cpu_count() or 1
+        configs = {}
+        with make_pool(cores) as pool:
+            for name in sorted(WORKLOAD_NAMES):
+                wn = w if name == args.workload else make_workload(name, "cuda")
+                r0 = oracle_sample(wn, pool, cores, min(wn.n, 50_000 * cores))[0]
+                seconds = 15.0 if name == args.workload else 3.0  # oracle work per config (wall)
+                rate, dt, done, off, ost, oh = oracle_sample(wn, pool, cores, int(max(1_000_000, r0 * seconds)))
+                c_cpu = {"value": rate, "unit": "pairs/s", "cores": cores, "kind": "oracle",
+                         "sample": f"first {done} pairs of {name} cut into {len(off) - 1} segments "
+                                   f"(its own boundaries and {cores} equal chunks), {cores} processes, {dt:.1f} s wall"}
+                c_par = parity_on_sample(peat, h, wn, off, ost, oh)
+                del ost, oh
+                blk = config_block(peat, h, name, wn, stream, peak, cold=name in ("c1", "c3"))
+                blk["cpu_baseline"] = c_cpu
+                blk["parity_before_timing"] = c_par
+                blk["gpu_over_oracle"] = blk["hot"]["pairs_per_s"] / rate
+                configs[name] = blk
+                if name == args.workload:
+                    cpu, parity = c_cpu, c_par
+                del wn
+                torch.cuda.empty_cache()
+
     for _ in range(args.warmup):
         step()
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local) as clk:
+    nvml = NvmlSampler(local)
+    with (nvml if nvml.available else ClockSampler(local)) as clk:
         time.sleep(0.25)
         barrier()
         wall0 = time.perf_counter()
@@ -285,16 +602,41 @@ def run_gpu(args) -> None:
             step()
         e1.record(stream)
         barrier()
-        wall = time.perf_counter() - wall0
+        wall1 = time.perf_counter()
+        wall = wall1 - wall0
+        # a clock-covered region of at least a second: the same call repeated
+        per = max(e0.elapsed_time(e1) / args.steps, 1e-3)
+        sus_calls = int(max(args.steps, 1.2e3 / per))
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier()
+        sw0 = time.perf_counter()
+        s0.record(stream)
+        for _ in range(sus_calls):
+            step()
+        s1.record(stream)
+        barrier()
+        sw1 = time.perf_counter()
         time.sleep(0.25)
     ms = max_over_ranks(e0.elapsed_time(e1), dev)
-    clocks = clk.summary()
+    if nvml.available:
+        clocks = nvml.summary(wall0, wall1)
+        clocks_sus = nvml.summary(sw0, sw1)
+    else:
+        clocks = clocks_sus = clk.summary()
     ms_per_step = ms / args.steps
     value = whole_job_rate(w.n, world, args.steps, ms)
     bytes_per_step = 2 * w.n * (4 if w.dtype == "f32" else 2)
     gbs = bytes_per_step / (ms_per_step * 1e-3) / 1e9
-    peaks = measured_peaks()
-    peak = float(peaks.get("hbm_gbs", 6800.0))
+    sus_ms = max_over_ranks(s0.elapsed_time(s1), dev) / sus_calls
+    sustained = {"calls": sus_calls, "seconds": sus_ms * sus_calls * 1e-3, "us_per_call": sus_ms * 1e3,
+                 "pairs_per_s": w.n / (sus_ms * 1e-3), "gbs": bytes_per_step / (sus_ms * 1e-3) / 1e9,
+                 "frac": bytes_per_step / (sus_ms * 1e-3) / 1e9 / peak, "clocks": clocks_sus,
+                 "us_x_sm_mhz": (sus_ms * 1e3 * clocks_sus["sm_mhz"]) if clocks_sus.get("sm_mhz") else None}
+    if clocks.get("sm_mhz"):
+        clocks["ms_per_step_x_sm_mhz"] = ms_per_step * clocks["sm_mhz"]
+    sweep = None
+    if rank == 0 and world == 1 and not args.no_sweep:
+        sweep = c5_sweep(peat, h, stream, peak)
 
     # the mean of the top 10 % of the errors (Section IV-B-3) on the same
     # tensor: its own timing, reported beside the compare's line
@@ -525,19 +867,6 @@ def run_gpu(args) -> None:
                        "step's compare (two buffer sets); stats and histograms read back every step"}
         del bufs
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        import oracle
-        oracle.build()
-        cores = os.cpu_count() or 1
-        wc = w
-        with make_pool(cores) as pool:
-            r0, _, _ = oracle_rate(wc, pool, cores, min(wc.n, 100_000 * cores))
-            target = int(min(wc.n, max(1_000_000, r0 * 20.0)))  # about 20 s of CPU work in total
-            rate, dt, done = oracle_rate(wc, pool, cores, target)
-        cpu = {"value": rate, "unit": "pairs/s", "cores": cores, "kind": "oracle",
-               "sample": f"first {done} pairs of the same workload, {cores} processes, {dt:.1f} s wall"}
-
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "pairs/s", "n_gpus": world, "steps": args.steps,
@@ -557,6 +886,7 @@ def run_gpu(args) -> None:
                          "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy)" if not peaks.get("fallback")
                          else "fallback 6.8 TB/s"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": (1 if nseg == 1 else 2) * args.steps, "clocks": clocks,
+            "parity_before_timing": parity, "sustained": sustained, "configs": configs, "c5_sweep": sweep,
             "next_rows": {"f1_top10_mean": topk, "f2_fused_inject_compare": fused, "f3_context_stats": tstats,
                           "f4_isclose_grid": isc, "f4_fp8_compare": fp8, "f4_f64_compare": f64},
             "wall_s_timed": wall,
@@ -576,6 +906,7 @@ def main():
     ap.add_argument("--workload", default="c2", choices=sorted(WORKLOAD_NAMES))
     ap.add_argument("--impl", default="peat", choices=["peat", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the 64-step config-5 sweep")
     ap.add_argument("--no-topk", action="store_true",
                     help="skip the timings of the next rows (top-10 %% mean, fused inject + compare, "
                          "context statistics, isclose grid)")

@@ -454,6 +454,13 @@ void peat_test_noalloc_expire_waits(int on);
  * else 0. */
 int32_t peat_test_for_digits(uint64_t m_lo, uint64_t m_hi, int32_t e, int32_t neg, int64_t* digits_out);
 
+/* Testing aid for the one rounding of the Mean and Variance of Errors scores
+ * (runs on the host, no GPU involved): RN-even binary64 of (W + f) 2^e / d
+ * with W = w_hi 2^64 + w_lo (w_hi's top bit set), 0 < f < 1 when sticky != 0
+ * and f = 0 otherwise, 1 <= d < 2^64 -- the routine the kernels round both
+ * scores with.  NaN for arguments outside that domain. */
+double peat_test_quot_rn(uint64_t w_hi, uint64_t w_lo, int32_t sticky, int32_t e, uint64_t d);
+
 #ifdef __cplusplus
 }
 #endif

@@ -78,7 +78,8 @@ class InjectModel(ctypes.Structure):
 EXPORTS = ("peat_signature_create", "peat_signature_destroy", "peat_compare", "peat_compare_segmented",
            "peat_pseudo_error_inject", "peat_last_error", "peat_compare_noalloc", "peat_topk_mean",
            "peat_tensor_stats", "peat_spearman", "peat_mean_std", "peat_isclose_grid", "peat_inject_compare",
-           "peat_test_noalloc_expire_waits", "peat_test_for_digits", "peat_trend", "peat_set_stage1_event")
+           "peat_test_noalloc_expire_waits", "peat_test_for_digits", "peat_trend", "peat_set_stage1_event",
+           "peat_test_quot_rn")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -121,6 +122,8 @@ def load(path: Optional[Path] = None) -> ctypes.CDLL:
     L.peat_trend.restype = i32
     L.peat_set_stage1_event.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
     L.peat_set_stage1_event.restype = i32
+    L.peat_test_quot_rn.argtypes = [ctypes.c_uint64, ctypes.c_uint64, i32, i32, ctypes.c_uint64]
+    L.peat_test_quot_rn.restype = ctypes.c_double
     L.peat_topk_mean.argtypes = [vp, vp, vp, i64, i32, ctypes.c_uint64, ctypes.c_uint64, vp, vp]
     L.peat_topk_mean.restype = i32
     L.peat_isclose_grid.argtypes = [vp, vp, vp, i64, i32, vp, i32, vp, i32, vp, vp]
@@ -412,6 +415,11 @@ def peat_set_stage1_event(h: Handle, event) -> None:
     once, so that it exists; None: stop) after each later compare's stage-1 launch."""
     ptr = None if event is None else ctypes.c_void_p(event.cuda_event)
     _check(load().peat_set_stage1_event(h.ptr, ptr), h)
+
+
+def peat_test_quot_rn(W: int, sticky: bool, e: int, d: int) -> float:
+    """Testing aid (host only): the kernels' RN-even binary64 of (W + f) 2^e / d."""
+    return load().peat_test_quot_rn(W >> 64, W & (2 ** 64 - 1), 1 if sticky else 0, int(e), int(d))
 
 
 def peat_trend(x, y) -> dict:

@@ -2034,4 +2034,10 @@ int test_for_digits(uint64_t m_lo, uint64_t m_hi, int e, int neg, int64_t* out) 
   return t_host_digit_dropped ? 1 : 0;
 }
 
+// The binary64 rounding of the exact quotients behind the mean and the
+// variance, run on the host (a test of quot_rn; no GPU involved).
+double test_quot_rn(uint64_t w_hi, uint64_t w_lo, int sticky, int e, uint64_t d) {
+  return quot_rn(((unsigned __int128)w_hi << 64) | w_lo, sticky != 0, e, d);
+}
+
 }  // namespace peat

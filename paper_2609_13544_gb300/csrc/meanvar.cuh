@@ -8,6 +8,7 @@
 // counts and the weight of the last digit differ between them.
 #pragma once
 #include <cstdint>
+#include <cstring>
 
 namespace peat {
 
@@ -42,7 +43,7 @@ __device__ double digits_rn(const uint32_t (&w)[NWD], int E, bool sticky) {
 // digits below them and the remainders only set the sticky bit.  As floor
 // (floor(W / k) / k) = floor(W / k^2) and W >= 2^224, the quotient keeps at
 // least 96 significant bits, so it rounds as the exact quotient does.
-__device__ inline double digits_div_rn(const uint32_t* N, int nd, uint64_t k, int times, int scale) {
+static __device__ __noinline__ double digits_div_rn(const uint32_t* N, int nd, uint64_t k, int times, int scale) {
   int top = nd - 1;
   while (top >= 0 && N[top] == 0) top--;
   if (top < 0) return 0.0;
@@ -68,6 +69,114 @@ __device__ inline double digits_div_rn(const uint32_t* N, int nd, uint64_t k, in
   return digits_rn(w, E, sticky);
 }
 
+// host and device spellings of the few bit operations used below
+__host__ __device__ inline int clz64(uint64_t x) {
+#ifdef __CUDA_ARCH__
+  return __clzll((long long)x);
+#else
+  return x ? __builtin_clzll(x) : 64;
+#endif
+}
+__host__ __device__ inline double bits_to_double(uint64_t b) {
+#ifdef __CUDA_ARCH__
+  return __longlong_as_double((long long)b);
+#else
+  double d;
+  memcpy(&d, &b, sizeof(d));
+  return d;
+#endif
+}
+
+// floor(W / Dn) and W mod Dn for W < 2^128 and Dn in [2^63, 2^64): the
+// quotient is built from digits of about 20 bits, each estimated in float32
+// from the remainder's leading 24 bits and Dn's leading 24 bits, scaled down
+// by 1 - 2^-20 so that it never exceeds the true digit (the estimate is
+// within 3 2^-24 of rem / Dn), and each removed from the remainder exactly;
+// a digit that comes out as 0 while rem >= Dn is taken as 1.  Every step
+// shrinks the remainder by about 2^20 (a digit is at least 2^-19 short of
+// the true quotient only in relative terms), so five or six steps reach
+// rem < Dn; the loops are bounded all the same.
+__host__ __device__ inline void divmod_128_64(unsigned __int128 W, uint64_t Dn, unsigned __int128& Q, uint64_t& R) {
+  const float rd = 1.0f / (float)(uint32_t)(Dn >> 40);  // Dn >> 40 in [2^23, 2^24): exact in float32
+  unsigned __int128 rem = W, q = 0;
+  for (int it = 0; it < 16 && rem >= Dn; it++) {
+    const uint64_t rh64 = (uint64_t)(rem >> 64);
+    const int lz = rh64 ? clz64(rh64) : 64 + clz64((uint64_t)rem);
+    const int s = 104 - lz;  // rem's leading 24 bits are rem >> s
+    const uint32_t top = (uint32_t)(rem >> s);
+    // rem / Dn ~ top 2^s / (dtop 2^40) with dtop = Dn >> 40: est 2^(s - 40)
+    // with est = top rd in (1/2, 2), taken as the 25-bit integer est 2^24
+    const uint64_t e24 = (uint64_t)((float)top * rd * (1.0f - 9.5367431640625e-7f) * 16777216.0f);  // (1 - 2^-20) 2^24
+    // rem >= Dn >= 2^63 has at least 64 bits, so k = s - 40 >= 0
+    const int k = s - 40 - 24;
+    unsigned __int128 t = k >= 0 ? (unsigned __int128)e24 << k : (unsigned __int128)(e24 >> -k);
+    if (t == 0) t = 1;  // rem >= Dn: at least one more
+    rem -= t * Dn;      // t Dn <= rem: never below zero
+    q += t;
+  }
+  for (int it = 0; it < 4 && rem >= Dn; it++) {  // not reached: the loop above ends with rem < Dn
+    rem -= Dn;
+    q += 1;
+  }
+  Q = q;
+  R = (uint64_t)rem;
+}
+
+// RN-even binary64 of X = (W + f) 2^E / D for W >= 2^127 (its top bit
+// set), 0 <= f < 1 (f > 0 exactly when sticky) and 1 <= D < 2^64, in integer
+// and float32 arithmetic only: with Dn = D 2^z normalised to [2^63, 2^64),
+// Q = floor(W / Dn) (2^63 <= Q < 2^65) and X = (Q + e) 2^(E + z), 0 <= e < 1,
+// e > 0 exactly when the remainder or f is nonzero.  Q keeps at least 63
+// bits, more than the 53 + 1 the rounding reads, so the remainder only
+// enters as the sticky bit.  The binary64 bits are assembled directly
+// (normal, subnormal, or +inf past the largest double).
+__host__ __device__ inline double quot_rn(unsigned __int128 W, bool sticky, int E, uint64_t D) {
+  const int z = clz64(D);
+  const uint64_t Dn = D << z;
+  unsigned __int128 Q;
+  uint64_t rem;
+  divmod_128_64(W, Dn, Q, rem);
+  sticky = sticky || rem != 0;
+  const int t = (uint64_t)(Q >> 64) ? 64 : 63;  // Q's leading one
+  const int P = E + z, lead = t + P;
+  if (lead >= 1024) return bits_to_double(0x7FF0000000000000ull);
+  const bool normal = lead >= -1022;
+  const int pos = normal ? t - 52 : -1074 - P;  // Q's bit of the result's last place (>= 1)
+  uint64_t m = 0;
+  bool half = false, below = sticky || Q != 0;
+  if (pos < 128) {
+    m = (uint64_t)(Q >> pos);
+    half = ((Q >> (pos - 1)) & 1) != 0;
+    below = sticky || (pos >= 2 && (Q << (129 - pos)) != 0);
+  }
+  if (half && (below || (m & 1ull))) m++;
+  // normal: the implicit bit of m carries into the exponent field (and a
+  // rounding to 2^53 moves it up one); subnormal: m itself (2^52 is 2^-1022)
+  const uint64_t bits = normal ? ((uint64_t)(lead + 1022) << 52) + m : m;
+  if (bits >= 0x7FF0000000000000ull) return bits_to_double(0x7FF0000000000000ull);
+  return bits_to_double(bits);
+}
+
+// RN-even binary64 of N 2^scale / D for the nd-digit magnitude N and
+// 1 <= D < 2^64: N's leading 128 bits as W (top bit set), the rest as the
+// sticky bit, then quot_rn.
+// Out of line: the mean and the variance share one copy of the code (it runs
+// once per call, so a second copy would be a second cold fetch).
+static __host__ __device__ __noinline__ double digits_quot_rn(const uint32_t* N, int nd, uint64_t D, int scale) {
+  int top = nd - 1;
+  while (top >= 0 && N[top] == 0) top--;
+  if (top < 0) return 0.0;
+  const int lz = clz64(N[top]) - 32;
+  auto dig = [&](int i) -> uint32_t { return i >= 0 ? N[i] : 0u; };
+  const unsigned __int128 win = ((unsigned __int128)dig(top) << 96) | ((unsigned __int128)dig(top - 1) << 64) |
+                                ((unsigned __int128)dig(top - 2) << 32) | dig(top - 3);
+  const uint32_t next = dig(top - 4);
+  const unsigned __int128 W = lz ? (win << lz) | (next >> (32 - lz)) : win;
+  bool sticky = lz ? (uint32_t)(next << lz) != 0 : next != 0;
+  for (int i = top - 5; i >= 0 && !sticky; i--) sticky = N[i] != 0;  // usually stops at once
+  return quot_rn(W, sticky, scale + 32 * (top - 3) - lz, D);
+}
+
 // Shared scratch of mean_var_block: S1 = A 2^e1 (NA digits) and
 // S2 = B 2^(2 e1 + 32 SHB) (NB digits), both non-negative magnitudes.
 template <int NA, int NB, int SHB>
@@ -75,6 +184,7 @@ struct MeanVarScratch {
   static constexpr int ND = (2 * NA > NB + SHB + 2 ? 2 * NA : NB + SHB + 2) + 1;
   uint32_t A[NA], B[NB];
   unsigned __int128 col[2 * NA];  // column sums of A * A
+  long long t[ND];                // N as signed carry-save digits
   uint32_t N[ND];
   double mean, var;
 };
@@ -101,37 +211,59 @@ template <int NA, int NB, int SHB>
 __device__ void mean_var_block(MeanVarScratch<NA, NB, SHB>& s, uint64_t nf, int e1) {
   constexpr int ND = MeanVarScratch<NA, NB, SHB>::ND;
   __syncthreads();
-  for (int c = threadIdx.x; c < 2 * NA - 1; c += blockDim.x) {
+  // the nonzero digit ranges: the loops below skip the zeros around them
+  int la = NA, ta = -1, lb = NB, tb = -1;
+  for (int i = 0; i < NA; i++)
+    if (s.A[i]) {
+      la = min(la, i);
+      ta = i;
+    }
+  for (int i = 0; i < NB; i++)
+    if (s.B[i]) {
+      lb = min(lb, i);
+      tb = i;
+    }
+  for (int c = 2 * la + (int)threadIdx.x; c <= 2 * ta; c += blockDim.x) {
     unsigned __int128 acc = 0;
-    const int i0 = c < NA ? 0 : c - NA + 1, i1 = c < NA ? c : NA - 1;
+    const int i0 = max(la, c - ta), i1 = min(ta, c - la);
     for (int i = i0; i <= i1; i++) acc += (unsigned __int128)((uint64_t)s.A[i] * s.A[c - i]);
-    s.col[c] = acc;
+    s.col[c] = acc;  // below 2^(64 + 8): three digits
   }
-  if (threadIdx.x == 0) s.col[2 * NA - 1] = 0;
+  // N = n_f B 2^(32 SHB) - A^2 as signed carry-save digits, every digit on
+  // its own thread: the three 32-bit parts of the products B[k] n_f that
+  // land on digit j, minus those of the column sums (each part below 2^32,
+  // so |t[j]| < 2^34).  Digits below j0 are zero, and so are those from j1
+  // on (past the last carry).
+  const int j0 = ta < 0 ? 0 : (tb >= 0 ? min(2 * la, SHB + lb) : 2 * la);
+  const int j1 = ta < 0 ? 0 : min(ND, max(2 * ta + 4, tb >= 0 ? SHB + tb + 4 : 0));
+  __syncthreads();
+  for (int j = j0 + (int)threadIdx.x; j < j1; j += blockDim.x) {
+    long long v = 0;
+#pragma unroll
+    for (int q = 0; q < 3; q++) {
+      const int k = j - SHB - q;  // B[k] n_f contributes its part q to digit j
+      if (k >= lb && k <= tb) v += (long long)(uint32_t)(((unsigned __int128)s.B[k] * nf) >> (32 * q));
+      const int c = j - q;  // so does the column sum c
+      if (c >= 2 * la && c <= 2 * ta) v -= (long long)(uint32_t)(s.col[c] >> (32 * q));
+    }
+    s.t[j] = v;
+  }
   __syncthreads();
   if (threadIdx.x == 0) {
-    if (nf == 0) {
+    if (nf == 0 || ta < 0) {
       s.mean = s.var = 0.0;
     } else {
-      // N = n_f B 2^(32 SHB) - A^2, digit by digit: the minuend's digit x
-      // from the running product, the subtrahend's digit y from the column
-      // sums with their carries, and the borrow
-      unsigned __int128 prod = 0, carry = 0;
-      uint32_t borrow = 0;
-      for (int j = 0; j < ND; j++) {
-        if (j >= SHB && j < SHB + NB) prod += (unsigned __int128)s.B[j - SHB] * nf;
-        const uint32_t x = (uint32_t)prod;
-        prod >>= 32;
-        unsigned __int128 cs = carry;
-        if (j < 2 * NA) cs += s.col[j];
-        const uint32_t y = (uint32_t)cs;
-        carry = cs >> 32;
-        const uint64_t sub = (uint64_t)y + borrow;
-        s.N[j] = x - (uint32_t)sub;
-        borrow = (uint64_t)x < sub ? 1u : 0u;
+      // carry propagation (64-bit arithmetic shifts; the final carry is 0 as N >= 0)
+      for (int j = 0; j < j0; j++) s.N[j] = 0;
+      long long carry = 0;
+      for (int j = j0; j < j1; j++) {
+        const long long v = s.t[j] + carry;
+        s.N[j] = (uint32_t)v;
+        carry = v >> 32;
       }
-      s.mean = digits_div_rn(s.A, NA, nf, 1, e1);
-      s.var = digits_div_rn(s.N, ND, nf, 2, 2 * e1);
+      for (int j = j1; j < ND; j++) s.N[j] = 0;
+      s.mean = digits_quot_rn(s.A, ta + 1, nf, e1);
+      s.var = nf < (1ull << 32) ? digits_quot_rn(s.N, j1, nf * nf, 2 * e1) : digits_div_rn(s.N, j1, nf, 2, 2 * e1);
     }
   }
   __syncthreads();

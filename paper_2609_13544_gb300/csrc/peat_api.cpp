@@ -1301,6 +1301,11 @@ peat_status_t peat_set_stage1_event(peat_handle_t h, void* event) {
 
 void peat_test_noalloc_expire_waits(int on) { g_noalloc_wait_limit.store(on ? 0u : (1u << 24)); }
 
+double peat_test_quot_rn(uint64_t w_hi, uint64_t w_lo, int32_t sticky, int32_t e, uint64_t d) {
+  if (d == 0 || !(w_hi >> 63)) return std::nan("");
+  return peat::test_quot_rn(w_hi, w_lo, sticky, e, d);
+}
+
 int32_t peat_test_for_digits(uint64_t m_lo, uint64_t m_hi, int32_t e, int32_t neg, int64_t* digits_out) {
   if (!digits_out) return -1;
   return peat::test_for_digits(m_lo, m_hi, e, neg, digits_out);

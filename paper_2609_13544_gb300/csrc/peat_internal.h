@@ -309,5 +309,6 @@ cudaError_t register_digit_status_topk(unsigned int* word);
 cudaError_t register_digit_status_tstats(unsigned int* word);
 cudaError_t register_digit_status_isclose(unsigned int* word);
 int test_for_digits(uint64_t m_lo, uint64_t m_hi, int e, int neg, int64_t* out);
+double test_quot_rn(uint64_t w_hi, uint64_t w_lo, int sticky, int e, uint64_t d);
 
 }  // namespace peat

@@ -1,5 +1,6 @@
 """The C-ABI library builds, loads and exports every symbol include/peat.h declares (CPU only)."""
 import ctypes
+import math
 import re
 from pathlib import Path
 
@@ -10,7 +11,7 @@ ROOT = Path(__file__).resolve().parents[1]
 
 def declared_functions():
     text = (ROOT / "include" / "peat.h").read_text()
-    return sorted(set(re.findall(r"^(?:peat_status_t|const char\*|void|int32_t)\s+(peat_\w+)\s*\(", text, re.M)))
+    return sorted(set(re.findall(r"^(?:peat_status_t|const char\*|void|int32_t|double)\s+(peat_\w+)\s*\(", text, re.M)))
 
 
 def test_header_declares_the_boundary():
@@ -19,7 +20,7 @@ def test_header_declares_the_boundary():
         "peat_isclose_grid", "peat_mean_std", "peat_pseudo_error_inject", "peat_signature_create",
         "peat_signature_destroy",
         "peat_set_stage1_event", "peat_spearman", "peat_tensor_stats", "peat_test_for_digits",
-        "peat_test_noalloc_expire_waits", "peat_topk_mean", "peat_trend"])
+        "peat_test_noalloc_expire_waits", "peat_test_quot_rn", "peat_topk_mean", "peat_trend"])
 
 
 def test_library_builds_and_exports_every_declared_symbol():
@@ -86,3 +87,53 @@ def test_digit_split_and_its_range_check():
     assert dropped and int(d[23]) == 2 ** 31
     d, dropped = peat.peat_test_for_digits(0, 10 ** 4, False)  # zero: nothing at all
     assert not dropped and not d.any()
+
+
+def _rn(q):
+    from fractions import Fraction  # noqa: F401
+    try:
+        return float(q)
+    except OverflowError:
+        return math.inf
+
+
+def test_quotient_rounding_of_the_mean_and_variance():
+    """The one rounding of the Mean and Variance of Errors scores (run on the
+    host through the testing aid): RN-even binary64 of (W + f) 2^e / d against
+    Python's correctly rounded Fraction -> float, over random operands and the
+    edges: exact quotients, ties to even, the subnormal grid, the overflow
+    threshold, d = 1 and d = 2^64 - 1.  f = 1/2 stands for any 0 < f < 1 (the
+    quotient keeps 63 bits or more, so no rounding boundary lies inside)."""
+    import random
+    from fractions import Fraction
+    import paper_2609_13544_gb300 as peat
+    rng = random.Random(11)
+
+    def want(W, sticky, e, d):
+        return _rn(Fraction(2 * W + (1 if sticky else 0), 2 * d) * Fraction(2) ** e)
+
+    cases = []
+    for _ in range(4000):
+        W = (1 << 127) | rng.getrandbits(127)
+        d = rng.choice([1, 2, 3, 7, 10, rng.getrandbits(16) | 1, rng.getrandbits(32) | 1, rng.getrandbits(63) | 1,
+                        (1 << 64) - 1, rng.getrandbits(64) | 1])
+        e = rng.choice([rng.randint(-1300, 1000), rng.randint(-1250, -1150), rng.randint(-200, 200)])
+        cases.append((W, rng.random() < 0.5, e, d))
+    # exact quotients on the grid and ties between grid points
+    for _ in range(500):
+        d = rng.getrandbits(rng.choice([8, 30, 60])) | 1
+        q = ((1 << 52) | rng.getrandbits(52)) * 2 + rng.choice([0, 1])  # a grid value or a midpoint (54 bits)
+        W = q * d
+        sh = 128 - W.bit_length()
+        cases.append((W << sh, False, rng.randint(-1200, 900) - sh, d))
+        cases.append((W << sh, True, rng.randint(-1200, 900) - sh, d))
+    # the overflow threshold (2^54 - 1) 2^970 and the largest double
+    for d in (1, 3, (1 << 64) - 1):
+        for q in ((1 << 54) - 1, (1 << 54) - 2, (1 << 53) - 1):
+            W = q * d
+            sh = 128 - W.bit_length()
+            cases.append((W << sh, False, 970 - sh, d))
+            cases.append((W << sh, True, 970 - sh, d))
+    for W, sticky, e, d in cases:
+        got, exp = peat.peat_test_quot_rn(W, sticky, e, d), want(W, sticky, e, d)
+        assert got == exp, (hex(W), sticky, e, d, got, exp)

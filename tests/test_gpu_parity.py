@@ -203,3 +203,34 @@ def test_tolerance_ties_float32(peat_gpu, oracle, h, rtol, atol):
     perm = rng.permutation(gb.size)
     gs = check_pair(peat_gpu, oracle, h, gb[perm], cb[perm], "f32", rtol, atol, ctx=f"ties rtol={rtol} atol={atol}")
     assert gs["within_tol"] > 0 and gs["mismatch"] > 0
+
+
+@pytest.mark.parametrize("case", ["cancel_f32", "overflow_f64", "mixed_f64", "subnormal_var_f64", "bf16_many"])
+def test_mean_var_edges_match_the_oracle(peat_gpu, oracle, h, case):
+    """The Mean and Variance of Errors scores at their edges, bit for bit: a
+    variance far below mean^2, |d| past the largest double (mean +inf), a
+    variance past it, a variance on the subnormal grid, and a long bf16 run
+    (many digits of the exact sums in use)."""
+    import torch
+    big = np.finfo(np.float64).max
+    if case == "cancel_f32":
+        g, c, dt = np.zeros(3, np.float32), (1 + np.arange(3) * 2.0 ** -23).astype(np.float32), "f32"
+    elif case == "overflow_f64":
+        g, c, dt = np.array([-big, -big]), np.array([big, big]), "f64"
+    elif case == "mixed_f64":
+        g, c, dt = np.array([-big, 0.0, 1.0]), np.array([big, 0.0, 1.0 + 2.0 ** -52]), "f64"
+    elif case == "subnormal_var_f64":
+        g, c, dt = np.zeros(3), np.array([3 * 2.0 ** -520, 0.0, 2.0 ** -520]), "f64"
+    else:
+        gb, cb = noise_pairs("bf16", 3_000_017, seed=91)
+        g, c, dt = gb, cb, "bf16"
+    if dt == "bf16":
+        gt, ct = to_device(g, "bf16"), to_device(c, "bf16")
+        gbits, cbits = g, c
+    else:
+        gt, ct = torch.from_numpy(g).cuda(), torch.from_numpy(c).cuda()
+        gbits, cbits = g.view(np.uint32 if dt == "f32" else np.uint64), c.view(np.uint32 if dt == "f32" else np.uint64)
+    st, hist = peat_gpu.peat_compare(h, gt, ct, 1e-3, 0.0)
+    ost, oh = oracle.compare(gbits, cbits, dt, 1e-3, 0.0)
+    assert_stats_equal(st, ost, case)
+    assert (st["mean_abs"], st["var_abs"]) == (ost["mean_abs"], ost["var_abs"])

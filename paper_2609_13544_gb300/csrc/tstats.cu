@@ -177,6 +177,16 @@ __device__ __forceinline__ void ts_flush(TsLane<DT>& L, int lb, long long* lim) 
   L.since = 0;
 }
 
+// an element outside the warp's window: its digits straight into the CTA's
+// accumulator (out of line: rare, and the unrolled loop stays small enough
+// for the instruction cache)
+template <int DT>
+__device__ __noinline__ void ts_slow(uint32_t m, int ee, bool neg, long long* lim) {
+  const int ex = ee - TS<DT>::BM;  // |x| = m 2^ex
+  for_digits(m, ex, neg, [&](int j, int64_t v) { lim_add(lim, j, v); });
+  for_digits((uint64_t)m * m, 2 * ex, false, [&](int j, int64_t v) { lim_add(lim + NLIMB, j, v); });
+}
+
 template <int DT>
 __device__ __forceinline__ void ts_elem(TsLane<DT>& L, uint32_t r, int lb, long long* lim) {
   using T = TS<DT>;
@@ -206,9 +216,7 @@ __device__ __forceinline__ void ts_elem(TsLane<DT>& L, uint32_t r, int lb, long 
       L.r2 += (uint64_t)t * t;  // below 2^56
     }
   } else if (m != 0) {
-    const int ex = ee - T::BM;  // |x| = m 2^ex
-    for_digits(m, ex, neg, [&](int j, int64_t v) { lim_add(lim, j, v); });
-    for_digits((uint64_t)m * m, 2 * ex, false, [&](int j, int64_t v) { lim_add(lim + NLIMB, j, v); });
+    ts_slow<DT>(m, ee, neg, lim);
     L.slow++;
   }
 }

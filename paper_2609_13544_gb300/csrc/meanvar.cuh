@@ -203,14 +203,23 @@ __device__ inline void carry_to_digits(const long long* src, int n, uint32_t* ou
   out[n + 1] = (uint32_t)((unsigned long long)carry >> 32);
 }
 
-// Called by every thread of the block once s.A and s.B hold S1 and S2 (and
-// the writes are visible to the block); leaves s.mean and s.var for every
-// thread.  n_f S2 - S1^2 is never negative (Cauchy-Schwarz over the n_f
-// values |d|), so the subtraction below ends without a borrow.
+// A barrier of nt threads (a multiple of 32): the block's own barrier for
+// id 0, else the named barrier id (only the group's threads take part).
+__device__ __forceinline__ void group_sync(int id, int nt) {
+  if (id == 0) __syncthreads();
+  else asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nt) : "memory");
+}
+
+// Called by every thread of a group of nt threads (t = 0 .. nt - 1, barrier
+// id bar) once s.A and s.B hold S1 and S2 (written by threads of the group);
+// leaves s.mean and s.var for every thread of the group.  n_f S2 - S1^2 is
+// never negative (Cauchy-Schwarz over the n_f values |d|), so the carry
+// propagation below ends without a borrow.  The mean (thread 32) and the
+// carries and the variance (thread 0) run side by side on two warps.
 template <int NA, int NB, int SHB>
-__device__ void mean_var_block(MeanVarScratch<NA, NB, SHB>& s, uint64_t nf, int e1) {
+__device__ void mean_var_group(MeanVarScratch<NA, NB, SHB>& s, uint64_t nf, int e1, int t, int nt, int bar) {
   constexpr int ND = MeanVarScratch<NA, NB, SHB>::ND;
-  __syncthreads();
+  group_sync(bar, nt);
   // the nonzero digit ranges: the loops below skip the zeros around them
   int la = NA, ta = -1, lb = NB, tb = -1;
   for (int i = 0; i < NA; i++)
@@ -223,7 +232,7 @@ __device__ void mean_var_block(MeanVarScratch<NA, NB, SHB>& s, uint64_t nf, int 
       lb = min(lb, i);
       tb = i;
     }
-  for (int c = 2 * la + (int)threadIdx.x; c <= 2 * ta; c += blockDim.x) {
+  for (int c = 2 * la + t; c <= 2 * ta; c += nt) {
     unsigned __int128 acc = 0;
     const int i0 = max(la, c - ta), i1 = min(ta, c - la);
     for (int i = i0; i <= i1; i++) acc += (unsigned __int128)((uint64_t)s.A[i] * s.A[c - i]);
@@ -236,8 +245,8 @@ __device__ void mean_var_block(MeanVarScratch<NA, NB, SHB>& s, uint64_t nf, int 
   // on (past the last carry).
   const int j0 = ta < 0 ? 0 : (tb >= 0 ? min(2 * la, SHB + lb) : 2 * la);
   const int j1 = ta < 0 ? 0 : min(ND, max(2 * ta + 4, tb >= 0 ? SHB + tb + 4 : 0));
-  __syncthreads();
-  for (int j = j0 + (int)threadIdx.x; j < j1; j += blockDim.x) {
+  group_sync(bar, nt);
+  for (int j = j0 + t; j < j1; j += nt) {
     long long v = 0;
 #pragma unroll
     for (int q = 0; q < 3; q++) {
@@ -248,10 +257,12 @@ __device__ void mean_var_block(MeanVarScratch<NA, NB, SHB>& s, uint64_t nf, int 
     }
     s.t[j] = v;
   }
-  __syncthreads();
-  if (threadIdx.x == 0) {
+  group_sync(bar, nt);
+  const int tmean = nt > 32 ? 32 : 0;
+  if (t == tmean) s.mean = (nf == 0 || ta < 0) ? 0.0 : digits_quot_rn(s.A, ta + 1, nf, e1);
+  if (t == 0) {
     if (nf == 0 || ta < 0) {
-      s.mean = s.var = 0.0;
+      s.var = 0.0;
     } else {
       // carry propagation (64-bit arithmetic shifts; the final carry is 0 as N >= 0)
       for (int j = 0; j < j0; j++) s.N[j] = 0;
@@ -262,11 +273,16 @@ __device__ void mean_var_block(MeanVarScratch<NA, NB, SHB>& s, uint64_t nf, int 
         carry = v >> 32;
       }
       for (int j = j1; j < ND; j++) s.N[j] = 0;
-      s.mean = digits_quot_rn(s.A, ta + 1, nf, e1);
       s.var = nf < (1ull << 32) ? digits_quot_rn(s.N, j1, nf * nf, 2 * e1) : digits_div_rn(s.N, j1, nf, 2, 2 * e1);
     }
   }
-  __syncthreads();
+  group_sync(bar, nt);
+}
+
+// the same with the whole block as the group (every thread calls it)
+template <int NA, int NB, int SHB>
+__device__ void mean_var_block(MeanVarScratch<NA, NB, SHB>& s, uint64_t nf, int e1) {
+  mean_var_group(s, nf, e1, (int)threadIdx.x, (int)blockDim.x, 0);
 }
 
 }  // namespace peat

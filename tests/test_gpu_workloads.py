@@ -138,6 +138,25 @@ def test_c5_sweep_step_by_step_and_trend(peat_gpu, oracle, h):
         assert math.isclose(got[k], want[k], rel_tol=1e-11), k
 
 
+def test_c5_sweep_resumes_from_its_records(peat_gpu, h, tmp_path):
+    """The sweep driver on the CUDA path: four steps recorded, a rerun reads
+    them back (no compare launched) with the same signatures, and a step
+    whose record is removed is compared again and comes out the same."""
+    from paper_2609_13544_gb300 import workloads as W
+    from paper_2609_13544_gb300.sweep import playback_sweep
+    sweep = W.PlaybackSweep(n=1 << 20, device="cuda")
+    steps = [0, 21, 42, 63]
+    r1 = playback_sweep(h, sweep.step, steps, 2.0 ** -7, record_dir=tmp_path, tag="c5-1M")
+    assert r1["computed"] == 4 and r1["records"][0]["stats"]["exact"] == 1 << 20
+    r2 = playback_sweep(h, lambda s: (_ for _ in ()).throw(AssertionError("recomputed")), steps, 2.0 ** -7,
+                        record_dir=tmp_path, tag="c5-1M")
+    assert r2["resumed"] == 4 and r2["series"] == r1["series"]
+    (tmp_path / "step_000042.json").unlink()
+    r3 = playback_sweep(h, sweep.step, steps, 2.0 ** -7, record_dir=tmp_path, tag="c5-1M")
+    assert r3["computed"] == 1 and r3["series"] == r1["series"]
+    assert r3["records"][2]["hist"] == r1["records"][2]["hist"]
+
+
 def _check_properties(st, hist, n):
     assert sum(st["count"]) == n == st["n"]
     assert int(hist[0].sum()) == n and int(hist[1].sum()) == n

@@ -887,7 +887,7 @@ peat_status_t peat_tensor_stats(peat_handle_t h, const void* x, const int64_t* o
   p.p0 = (n > 0 && ax % B == 0) ? (int64_t)(((16 - ax % 16) % 16) / B) : -1;
   // one wave of resident CTAs, about one CTA per 8K elements, within the staging area
   const int64_t want = (n + 8191) / 8192;
-  const int64_t cap = std::min<int64_t>((int64_t)peat::tstats_ctas_per_sm() * h->nsm, 2 * (int64_t)h->max_ctas);
+  const int64_t cap = std::min<int64_t>((int64_t)peat::tstats_ctas_per_sm(dtype) * h->nsm, 2 * (int64_t)h->max_ctas);
   p.nctas = (int)std::max<int64_t>(1, std::min<int64_t>(cap, want));
   cudaError_t e;
   if (nseg == 1) {  // one tensor: no host staging (see compare_impl)

@@ -179,7 +179,7 @@ struct TsParams {
   TsAcc* acc;               // nseg accumulators
   peat_tstats_t* out;       // device, nseg records
 };
-int tstats_ctas_per_sm();
+int tstats_ctas_per_sm(int dtype);  // resident CTAs of the element type's stage 1
 cudaError_t launch_tstats(int dtype, const TsParams& p, cudaStream_t s);
 
 // ---- isclose pass counts over a tolerance grid (isclose.cu) ----

@@ -372,6 +372,237 @@ __global__ void __launch_bounds__(TB) tstats_stage1(TsParams p) {
   }
 }
 
+// ---- stage 1 for 16-bit elements: a histogram of bit patterns ----
+// A 16-bit element has few values.  Per piece, the CTA places one window of
+// WS exponents (from the largest finite exponent among the first vector of
+// every thread, plus one binade of headroom) and counts every finite nonzero
+// element inside it in a shared histogram indexed by (sign, exponent - Lb,
+// significand field): one shared atomic per element, no per-element sums,
+// keys or branches beyond the window test.  Zeros have two bins of their
+// own; NaN, infinities, subnormals and elements outside the window take the
+// exact path above (digits, counted extremes).  At the end of the piece each
+// bin adds count * value and count * value^2 exactly (integers in units of
+// the window's floor), and the extreme nonzero bins give the finite minimum
+// and maximum.
+template <int DT>
+struct H16;
+template <>
+struct H16<PEAT_F16> {
+  static constexpr int WSB = 3, WS = 1 << WSB;  // 8 exponents: 16,384 bins
+};
+template <>
+struct H16<PEAT_BF16> {
+  static constexpr int WSB = 5, WS = 1 << WSB;  // 32 exponents: 8,192 bins
+};
+template <int DT>
+constexpr int h16_bins() {
+  return 2 * H16<DT>::WS << TS<DT>::MB;
+}
+
+// an element the histogram does not take: counted (NaN, infinity) or added
+// to the digits with its order key (finite), on the CTA's shared totals
+template <int DT>
+__device__ __noinline__ void h16_slow(uint32_t r, long long* lim, unsigned long long* cnt, unsigned int* kmin_s,
+                                      unsigned int* kmax_s) {
+  using T = TS<DT>;
+  const uint32_t e = (r >> T::MB) & T::EMASK, mant = r & ((1u << T::MB) - 1u);
+  if (e == T::EINF) {
+    atomicAdd(&cnt[mant ? 1 : 2], 1ull);
+    return;
+  }
+  const uint32_t k = order_key(raw_to_f32<DT>(r));
+  atomicMin(kmin_s, k);
+  atomicMax(kmax_s, k);
+  const uint32_t m = mant | (e ? (1u << T::MB) : 0u);
+  if (m) ts_slow<DT>(m, e ? (int)e : 1, (r >> (T::BITS - 1)) & 1u, lim);
+}
+
+template <int DT>
+__global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
+  using T = TS<DT>;
+  constexpr int VEC = T::VEC, B = T::BYTES, MB = T::MB, WS = H16<DT>::WS, WSB = H16<DT>::WSB;
+  constexpr int NB = h16_bins<DT>();
+  constexpr uint32_t WSM = (uint32_t)WS << MB, MAGM = (1u << (T::BITS - 1)) - 1u;
+  extern __shared__ uint32_t hist[];  // NB bins, then the bins of +0 and -0
+  __shared__ long long lim[2 * NLIMB];
+  __shared__ unsigned long long cnt[3];
+  __shared__ unsigned int kmin_s, kmax_s, emax_s;
+  __shared__ unsigned long long red[3][TB / 32][4];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t lo = p.bounds[blockIdx.x], hi = p.bounds[blockIdx.x + 1];
+  if (lo >= hi) return;
+  int64_t s0 = 0, s1 = p.nseg;
+  while (s1 - s0 > 1) {
+    const int64_t mid = (s0 + s1) / 2;
+    if (p.offsets[mid] <= lo) s0 = mid;
+    else s1 = mid;
+  }
+  int64_t seg = s0;
+  while (p.offsets[seg + 1] <= lo) seg++;
+  const uint32_t hb = (uint32_t)__cvta_generic_to_shared(hist);
+  for (int j = tid; j < NB + 2; j += TB) hist[j] = 0;
+  for (int64_t a = lo; a < hi;) {
+    const int64_t b = min(hi, p.offsets[seg + 1]);
+    for (int j = tid; j < 2 * NLIMB; j += TB) lim[j] = 0;
+    if (tid < 3) cnt[tid] = 0;
+    if (tid == 0) {
+      kmin_s = 0xFFFFFFFFu;
+      kmax_s = 0;
+      emax_s = 0;
+    }
+    // the vector grid inside the piece
+    int64_t a0 = b, nv = 0;
+    if (p.p0 >= 0 && p.p0 < p.n_total) {
+      a0 = a <= p.p0 ? p.p0 : p.p0 + ((a - p.p0 + VEC - 1) / VEC) * VEC;
+      if (a0 < b) nv = (b - a0) / VEC;
+      else a0 = b;
+    }
+    __syncthreads();
+    // the window: one binade above the largest finite exponent among the
+    // first vector of every thread (or the tail's first elements)
+    {
+      uint32_t em = 0;
+      if (tid < nv) {
+        const uint4 v = ts_vec(p.x, (a0 + (int64_t)tid * VEC) * B);  // this thread's first vector of the piece
+#pragma unroll
+        for (int j = 0; j < VEC; j++) {
+          const uint32_t e = (ts_lane<DT>(v, j) >> MB) & T::EMASK;
+          if (e != T::EINF) em = max(em, e);
+        }
+      } else if (nv == 0 && a + tid < b) {
+        const uint32_t e = (ts_load<DT>(p.x, a + tid) >> MB) & T::EMASK;
+        if (e != T::EINF) em = e;
+      }
+      em = __reduce_max_sync(0xFFFFFFFFu, em);
+      if (lane == 0 && em) atomicMax(&emax_s, em);
+    }
+    __syncthreads();
+    const int lb = max(1, min((int)emax_s + 2 - WS, (int)T::EINF - WS));  // window exponents [lb, lb + WS)
+    const uint32_t lbm = (uint32_t)lb << MB;
+    auto elem = [&](uint32_t r) {
+      const uint32_t mag = r & MAGM, t = mag - lbm;
+      if (t < WSM) {
+        asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(hb + 4u * (t | ((r >> (T::BITS - 1)) << (WSB + MB)))),
+                     "r"(1u)
+                     : "memory");
+      } else if (mag == 0) {
+        asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(hb + 4u * (NB + (r >> (T::BITS - 1)))), "r"(1u)
+                     : "memory");
+      } else {
+        h16_slow<DT>(r, lim, cnt, &kmin_s, &kmax_s);
+      }
+    };
+    constexpr int U = 4;
+    for (int64_t k0 = 0; k0 < nv; k0 += (int64_t)U * TB) {
+      uint4 v[U];
+#pragma unroll
+      for (int uu = 0; uu < U; uu++) {
+        const int64_t k = k0 + uu * TB + tid;
+        v[uu] = k < nv ? ts_vec(p.x, (a0 + k * VEC) * B) : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int uu = 0; uu < U; uu++) {
+        if (k0 + uu * TB + tid < nv) {
+#pragma unroll
+          for (int j = 0; j < VEC; j++) elem(ts_lane<DT>(v[uu], j));
+        }
+      }
+    }
+    {  // the elements outside the vector grid: [a, a0) and [a0 + nv VEC, b)
+      const int64_t h = a0 - a, t0 = a0 + nv * VEC, ns = h + (b - t0);
+      for (int64_t i = tid; i < ns; i += TB) elem(ts_load<DT>(p.x, i < h ? a + i : t0 + (i - h)));
+    }
+    __syncthreads();
+    // the bins: exact sums in units of 2^(lb - BM) (S1 by sign, S2), the
+    // extreme keys, and the bins cleared for the next piece
+    unsigned __int128 s1p = 0, s1n = 0, s2 = 0;
+    uint32_t kmn = 0xFFFFFFFFu, kmx = 0;
+    for (int bin = tid; bin < NB + 2; bin += TB) {
+      const uint32_t c = hist[bin];
+      if (!c) continue;
+      hist[bin] = 0;
+      uint32_t r;
+      if (bin >= NB) {
+        r = (uint32_t)(bin - NB) << (T::BITS - 1);  // +0 or -0
+      } else {
+        const uint32_t sg = (uint32_t)bin >> (WSB + MB), slot = ((uint32_t)bin >> MB) & (WS - 1u);
+        const uint32_t mant = (uint32_t)bin & ((1u << MB) - 1u);
+        r = (sg << (T::BITS - 1)) | ((uint32_t)(lb + (int)slot) << MB) | mant;
+        const uint64_t tt = (uint64_t)(mant | (1u << MB)) << slot;  // below 2^(MB + WS)
+        const unsigned __int128 ct = (unsigned __int128)tt * c;
+        if (sg) s1n += ct;
+        else s1p += ct;
+        s2 += ct * tt;  // below 2^(2 (MB + WS) + 32)
+      }
+      const uint32_t k = order_key(raw_to_f32<DT>(r));
+      kmn = min(kmn, k);
+      kmx = max(kmx, k);
+    }
+    // block totals: 32-bit words of each 128-bit sum summed over the warp,
+    // then over the warps by warp 0, added as digits
+    {
+      const unsigned __int128 d = s1p - s1n;  // |S1| < 2^120: two's complement in 128 bits
+#pragma unroll
+      for (int q = 0; q < 4; q++) {
+        uint64_t w1 = (uint32_t)(d >> (32 * q)), w2 = (uint32_t)(s2 >> (32 * q));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          w1 += __shfl_xor_sync(0xFFFFFFFFu, w1, o);
+          w2 += __shfl_xor_sync(0xFFFFFFFFu, w2, o);
+        }
+        if (lane == 0) {
+          red[0][warp][q] = w1;
+          red[1][warp][q] = w2;
+        }
+      }
+      kmn = __reduce_min_sync(0xFFFFFFFFu, kmn);
+      kmx = __reduce_max_sync(0xFFFFFFFFu, kmx);
+      if (lane == 0) {
+        if (kmn != 0xFFFFFFFFu) atomicMin(&kmin_s, kmn);
+        if (kmx) atomicMax(&kmax_s, kmx);
+      }
+    }
+    __syncthreads();
+    if (tid == 0) {
+      // word q of S1 (two's complement) and of S2, each summed over the block;
+      // S1's words rebuild its 128-bit value, whose sign is its top bit
+      unsigned __int128 S1 = 0, S2w[4];
+      for (int q = 0; q < 4; q++) {
+        unsigned __int128 t1 = 0, t2 = 0;
+        for (int w = 0; w < TB / 32; w++) {
+          t1 += red[0][w][q];
+          t2 += red[1][w][q];
+        }
+        S1 += t1 << (32 * q);
+        S2w[q] = t2;
+      }
+      const int u = lb - T::BM;  // weight of a unit
+      const bool neg = (S1 >> 127) != 0;
+      const unsigned __int128 mag1 = neg ? (unsigned __int128)0 - S1 : S1;
+      for_digits(mag1, u, neg, [&](int j, int64_t v) { lim_add(lim, j, v); });
+      for (int q = 0; q < 4; q++)
+        if (S2w[q]) for_digits(S2w[q], 2 * u + 32 * q, false, [&](int j, int64_t v) { lim_add(lim + NLIMB, j, v); });
+    }
+    __syncthreads();
+    TsAcc& acc = p.acc[seg];
+    for (int j = tid; j < 2 * NLIMB; j += TB)
+      if (lim[j]) atomicAdd(reinterpret_cast<unsigned long long*>(&acc.limbs[0][0] + j), (unsigned long long)lim[j]);
+    if (tid == 0) {
+      const unsigned long long nfin = (unsigned long long)(b - a) - cnt[1] - cnt[2];
+      if (nfin) atomicAdd(&acc.nfin, nfin);
+      if (cnt[1]) atomicAdd(&acc.nnan, cnt[1]);
+      if (cnt[2]) atomicAdd(&acc.ninf, cnt[2]);
+      if (nfin) {
+        atomicMax(&acc.kmin_inv, ~kmin_s);
+        atomicMax(&acc.kmax, kmax_s);
+      }
+    }
+    __syncthreads();
+    a = b;
+    while (seg < p.nseg && p.offsets[seg + 1] <= a) seg++;
+  }
+}
+
 // ---- stage 2: exact mean and variance ----
 // Every loop below has compile-time bounds and is unrolled, so the digit
 // arrays stay in registers.
@@ -572,25 +803,57 @@ __global__ void __launch_bounds__(FIN_THREADS) tstats_finalize(TsParams p) {
 }
 
 template <int DT>
+constexpr size_t hist_smem() {
+  return sizeof(uint32_t) * (size_t)(h16_bins<DT>() + 2);
+}
+
+// the dynamic shared memory of the histogram kernels, allowed once per
+// process (above the default 48 KB for fp16)
+cudaError_t hist_prepare() {
+  static const cudaError_t e = [] {
+    cudaError_t r = cudaFuncSetAttribute(tstats_hist<PEAT_F16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)hist_smem<PEAT_F16>());
+    if (r == cudaSuccess)
+      r = cudaFuncSetAttribute(tstats_hist<PEAT_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)hist_smem<PEAT_BF16>());
+    return r;
+  }();
+  return e;
+}
+
+template <int DT>
 cudaError_t launch_t(const TsParams& p, cudaStream_t s) {
-  tstats_stage1<DT><<<p.nctas, TB, 0, s>>>(p);
+  if constexpr (DT == PEAT_F32) {
+    tstats_stage1<DT><<<p.nctas, TB, 0, s>>>(p);
+  } else {
+    const cudaError_t e = hist_prepare();
+    if (e != cudaSuccess) return e;
+    tstats_hist<DT><<<p.nctas, TB, hist_smem<DT>(), s>>>(p);
+  }
   tstats_finalize<<<(unsigned)p.nseg, FIN_THREADS, 0, s>>>(p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-int tstats_ctas_per_sm() {
-  static const int v = [] {
+int tstats_ctas_per_sm(int dtype) {
+  struct Occ {
+    int v[3];
+  };
+  static const Occ o = [] {
+    Occ r{{1, 1, 1}};
+    hist_prepare();
     int a = 0, b = 0, c = 0;
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, tstats_stage1<PEAT_F32>, TB, 0);
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, tstats_stage1<PEAT_F16>, TB, 0);
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&c, tstats_stage1<PEAT_BF16>, TB, 0);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, tstats_hist<PEAT_F16>, TB, hist_smem<PEAT_F16>());
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&c, tstats_hist<PEAT_BF16>, TB, hist_smem<PEAT_BF16>());
     cudaGetLastError();
-    const int m = a < b ? a : b;
-    return (m < c ? m : c) > 0 ? (m < c ? m : c) : 1;
+    if (a > 0) r.v[0] = a;
+    if (b > 0) r.v[1] = b;
+    if (c > 0) r.v[2] = c;
+    return r;
   }();
-  return v;
+  return dtype == PEAT_F32 ? o.v[0] : dtype == PEAT_F16 ? o.v[1] : o.v[2];
 }
 
 int64_t tstats_vec_elems(int dtype) { return dtype == PEAT_F32 ? 4 : 8; }

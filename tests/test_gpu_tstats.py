@@ -85,6 +85,37 @@ def test_special_tensors(peat_gpu, oracle, h):
         check(peat_gpu, oracle, h, bits, "f32", ctx=name)
 
 
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+def test_special_16bit_tensors(peat_gpu, oracle, h, dtype):
+    """The 16-bit histogram path at its edges: NaN and infinities, signed
+    zeros (-0 below +0 for min and max), a constant, the largest finite and
+    the smallest subnormal values, every exponent once, all bit patterns,
+    and zeros next to tiny values (the window is placed by the largest
+    exponent: everything far below takes the exact digit path)."""
+    rng = np.random.default_rng(41)
+    inf, nan, mx, sub = ((0x7C00, 0x7E00, 0x7BFF, 0x0001) if dtype == "f16" else (0x7F80, 0x7FC0, 0x7F7F, 0x0001))
+    exps = 31 if dtype == "f16" else 255
+    mb = 10 if dtype == "f16" else 7
+    specials = {
+        "all NaN": np.full(5000, nan, np.uint16),
+        "all zero both signs": np.array([0, 0x8000] * 3000, np.uint16),
+        "only negative zero": np.full(700, 0x8000, np.uint16),
+        "constant": np.full(100_000, 0x3C00 if dtype == "f16" else 0x3F80, np.uint16),
+        "extremes": np.array([mx, 0x8000 | mx, sub, 0x8000 | sub, inf, 0x8000 | inf, nan, 0] * 1000, np.uint16),
+        "every exponent": np.array([(e << mb) | 3 for e in range(1, exps)] * 40
+                                   + [0x8000 | (e << mb) | 5 for e in range(1, exps)] * 40, np.uint16),
+        "every pattern": np.arange(65536, dtype=np.uint32).astype(np.uint16),
+        "zeros and tiny": np.concatenate([np.full(3000, 0x8000, np.uint16),
+                                          rng.integers(1, 1 << mb, 3000).astype(np.uint16),
+                                          np.full(10, mx, np.uint16)]),
+    }
+    for name, bits in specials.items():
+        check(peat_gpu, oracle, h, bits, dtype, ctx=name)
+        perm = rng.permutation(bits.size)
+        check(peat_gpu, oracle, h, bits[perm], dtype, ctx=name + " shuffled")
+        check(peat_gpu, oracle, h, bits, dtype, offsets=[0, bits.size // 3, bits.size // 3, bits.size], ctx=name + " segs")
+
+
 @pytest.mark.parametrize("dtype", DTYPES)
 def test_scale_changes_inside_a_warp_range(peat_gpu, oracle, h, dtype):
     """Blocks of very different magnitude in one tensor: warps move their

@@ -1588,6 +1588,7 @@ __global__ void __launch_bounds__(BLOCK, CTAS_PER_SM) compare_stage1(ComparePara
   constexpr int64_t ROUND_CHUNKS = (int64_t)NW * (65535 / (2 * VEC));
   extern __shared__ __align__(128) unsigned char smem_raw[];
   Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+  pdl_trigger();  // a multi-segment call's finalize kernel may start launching (it waits for this grid)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   for (int b = tid; b < HBINS; b += BLOCK) sm.hist[b] = 0;
   for (int j = tid; j < NSUM * NLIMB; j += BLOCK) (&sm.sacc[0][0])[j] = 0;
@@ -1908,6 +1909,7 @@ __device__ __noinline__ void finalize_segment(const CompareParams& p, int64_t s,
 __global__ void __launch_bounds__(BLOCK) compare_finalize(CompareParams p) {
   __shared__ FinScratch f;
   __shared__ MV mv;
+  pdl_wait();  // stage 1 complete
   if (p.offsets[blockIdx.x] < p.offsets[blockIdx.x + 1]) finalize_segment(p, blockIdx.x, f, mv);
 }
 
@@ -1937,8 +1939,14 @@ cudaError_t launch_t(const CompareParams& p, cudaStream_t st) {
   if (e == cudaSuccess && p.stage1_event) e = cudaEventRecord(static_cast<cudaEvent_t>(p.stage1_event), st);
   if (e != cudaSuccess || p.nseg <= 1) return e;
   nvtxRangePushA("peat compare stage 2 (per-segment finalize)");
-  compare_finalize<<<(unsigned)p.nseg, BLOCK, 0, st>>>(p);
-  e = cudaGetLastError();
+  // a programmatic dependent of stage 1 (its launch overlaps the end of stage
+  // 1), unless an event was recorded between the two
+  if (p.stage1_event) {
+    compare_finalize<<<(unsigned)p.nseg, BLOCK, 0, st>>>(p);
+    e = cudaGetLastError();
+  } else {
+    e = launch_dependent(compare_finalize, (unsigned)p.nseg, BLOCK, 0, st, p);
+  }
   nvtxRangePop();
   return e;
 }

@@ -351,6 +351,7 @@ __global__ void __launch_bounds__(TB, 2) compare64_stage1(Cmp64Params p) {
   __shared__ unsigned H[PEAT_HIST_BINS];
   __shared__ long long S[3 * SL];
   __shared__ Part64Rec buf[TB];
+  pdl_trigger();  // the finalize kernel may start launching (it waits for this grid)
   const int lane = threadIdx.x & 31;
   for (long long item = blockIdx.x; item < p.nitems; item += gridDim.x) {
     const long long b = p.item_b[item], e = p.item_e[item], seg = p.item_seg[item];
@@ -483,6 +484,7 @@ __device__ double rel_value64(const Mag& a, double g) {
 __global__ void __launch_bounds__(TB) compare64_finalize(Cmp64Params p) {
   __shared__ Part64Rec buf[TB];
   __shared__ long long S[3 * SL];
+  pdl_wait();  // stage 1 complete
   const long long seg = blockIdx.x;
   const long long f0 = p.seg_first[seg], f1 = p.seg_first[seg + 1];
   Part64Rec r;
@@ -533,9 +535,14 @@ __global__ void __launch_bounds__(TB) compare64_finalize(Cmp64Params p) {
 }  // namespace
 
 cudaError_t launch_compare64(const Cmp64Params& p, int nctas, cudaStream_t s) {
-  if (p.nitems > 0) compare64_stage1<<<nctas, TB, 0, s>>>(p);
-  compare64_finalize<<<(unsigned)p.nseg, TB, 0, s>>>(p);
-  return cudaGetLastError();
+  if (p.nitems == 0) {
+    compare64_finalize<<<(unsigned)p.nseg, TB, 0, s>>>(p);
+    return cudaGetLastError();
+  }
+  compare64_stage1<<<nctas, TB, 0, s>>>(p);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return launch_dependent(compare64_finalize, (unsigned)p.nseg, TB, 0, s, p);  // overlaps stage 1's end
 }
 
 }  // namespace peat

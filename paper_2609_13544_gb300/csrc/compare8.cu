@@ -315,6 +315,7 @@ __global__ void __launch_bounds__(TB) compare8_stage1(Cmp8Params p) {
   __shared__ unsigned H[PEAT_HIST_BINS];
   __shared__ Tot warp_tot[NW];
   __shared__ unsigned long long AM[128];
+  pdl_trigger();  // the finalize kernel may start launching (it waits for this grid)
   const int lane = threadIdx.x & 31;
   for (int k = threadIdx.x; k < 128; k += TB) AM[k] = p.amax[k];
   for (long long item = blockIdx.x; item < p.nitems; item += gridDim.x) {
@@ -412,6 +413,7 @@ __global__ void __launch_bounds__(TB) compare8_finalize(Cmp8Params p) {
   // S1 = s1 2^-S and S2 = s2 2^-2S: four digits each, no shift between them
   __shared__ MeanVarScratch<4, 4, 0> mv;
   __shared__ unsigned long long nfin;
+  pdl_wait();  // stage 1 complete
   constexpr int S = F8<DT>::S;
   const long long seg = blockIdx.x;
   Tot t;
@@ -457,9 +459,14 @@ __global__ void __launch_bounds__(TB) compare8_finalize(Cmp8Params p) {
 
 template <int DT>
 cudaError_t launch_t(const Cmp8Params& p, int nctas, cudaStream_t s) {
-  if (p.nitems > 0) compare8_stage1<DT><<<nctas, TB, 0, s>>>(p);
-  compare8_finalize<DT><<<(unsigned)p.nseg, TB, 0, s>>>(p);
-  return cudaGetLastError();
+  if (p.nitems == 0) {
+    compare8_finalize<DT><<<(unsigned)p.nseg, TB, 0, s>>>(p);
+    return cudaGetLastError();
+  }
+  compare8_stage1<DT><<<nctas, TB, 0, s>>>(p);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return launch_dependent(compare8_finalize<DT>, (unsigned)p.nseg, TB, 0, s, p);  // overlaps stage 1's end
 }
 
 }  // namespace

@@ -8,6 +8,36 @@
 
 namespace peat {
 
+#ifdef __CUDACC__
+// Programmatic dependent launch (PTX griddepcontrol, sm_90 and later). A
+// kernel started by launch_dependent may begin while the kernel before it on
+// the stream is still running, so it calls pdl_wait() before its first access
+// to anything that kernel (or any earlier one) writes; pdl_wait() returns once
+// the previous kernel has completed and its memory operations are visible,
+// and at once in a kernel launched the ordinary way. pdl_trigger() lets the
+// next dependent kernel start launching; without it that happens when this
+// kernel completes. A dependent's blocks only occupy resources that the
+// previous grid's finished blocks gave back, since the launch waits for every
+// block of the previous grid to trigger or exit.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+template <typename... KA, typename... A>
+inline cudaError_t launch_dependent(void (*kernel)(KA...), unsigned grid, unsigned block, size_t smem,
+                                    cudaStream_t s, A... args) {
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+#endif
+
 // Exact sums are carried as NLIMB signed 64-bit digits; digit j weighs
 // 2^(32 j + LIMB_LSB).  Every term that occurs (products of two float32
 // values, or of a binary64 difference and a float32 value) is a multiple of

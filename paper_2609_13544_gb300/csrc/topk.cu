@@ -456,6 +456,7 @@ __global__ void __launch_bounds__(TB) topk_sample(TopkParams p) {
   constexpr int VEC = TK<DT>::VEC, B = TK<DT>::BYTES;
   __shared__ uint32_t h[TK_NB0];
   __shared__ unsigned last_s;
+  pdl_trigger();
   TopkState* st = p.st;
   for (int b = threadIdx.x; b < TK_NB0; b += TB) h[b] = 0;
   __syncthreads();
@@ -516,6 +517,8 @@ __global__ void __launch_bounds__(TB) topk_pass1(TopkParams p) {
   __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
   __shared__ unsigned long long cnt_s[2];
   __shared__ unsigned last_s;
+  pdl_wait();
+  pdl_trigger();
   TopkState* st = p.st;
   if (FB && st->ok) return;
   for (int b = threadIdx.x; b < TK_WIN * TK_NB1; b += TB) h[b] = 0;
@@ -638,6 +641,8 @@ template <int DT>
 __global__ void __launch_bounds__(TB) topk_pass0(TopkParams p) {
   __shared__ uint32_t h[TK_NB0];
   __shared__ unsigned last_s;
+  pdl_wait();
+  pdl_trigger();
   TopkState* st = p.st;
   if (st->ok) return;
   for (int b = threadIdx.x; b < TK_NB0; b += TB) h[b] = 0;
@@ -671,6 +676,8 @@ __global__ void __launch_bounds__(TB) topk_pass2(TopkParams p) {
   __shared__ long long lim[NLIMB];
   __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
   __shared__ unsigned last_s;
+  pdl_wait();
+  pdl_trigger();
   TopkState* st = p.st;
   if (st->k == 0 || st->skip2) return;
   for (int b = threadIdx.x; b < TK_NB2; b += TB) h[b] = 0;
@@ -740,6 +747,8 @@ __global__ void __launch_bounds__(TB) topk_pass3(TopkParams p) {
   __shared__ long long lim[NLIMB];
   __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
   __shared__ unsigned last_s;
+  pdl_wait();
+  pdl_trigger();
   TopkState* st = p.st;
   if (st->k == 0 || st->skip2 || st->nlist <= TK_LCAP) return;
   for (int j = threadIdx.x; j < NLIMB; j += TB) lim[j] = 0;
@@ -784,6 +793,8 @@ template <int DT>
 __global__ void __launch_bounds__(TB) topk_pass4(TopkParams p) {
   __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
   __shared__ unsigned last_s;
+  pdl_wait();
+  pdl_trigger();
   TopkState* st = p.st;
   if (st->k == 0 || st->skip2 || st->nlist2 <= TK_LCAP) return;
   const uint32_t T = st->T;
@@ -821,6 +832,8 @@ __global__ void __launch_bounds__(TB) topk_pass5(TopkParams p) {
   __shared__ typename QT<DT>::T ring[(TB / 32) * ring_cap<DT>()];
   __shared__ long long lim[NLIMB];
   __shared__ unsigned last_s;
+  pdl_wait();
+  pdl_trigger();
   TopkState* st = p.st;
   if (st->k == 0 || st->skip2 || st->nlist2 <= TK_LCAP) return;
   for (int j = threadIdx.x; j < NLIMB; j += TB) lim[j] = 0;
@@ -859,6 +872,7 @@ __global__ void __launch_bounds__(TB) topk_pass5(TopkParams p) {
 // The P1 range, T's bucket, the rounding, the output; the state cleared for
 // the next call.  One CTA.
 __global__ void __launch_bounds__(TB) topk_finalize(TopkParams p) {
+  pdl_wait();
   TopkState* st = p.st;
   __shared__ long long lim[NLIMB];
   const int tid = threadIdx.x;
@@ -985,16 +999,22 @@ cudaError_t launch_t(const TopkParams& p, int nctas, cudaStream_t s) {
   const int64_t units = p.nvec > 0 ? std::min<int64_t>((p.nvec + 31) / 32, TK_SAMPLE / (32 * TK<DT>::VEC))
                                    : (std::min<int64_t>(p.n, TK_SAMPLE) + 31) / 32;
   const int sctas = (int)std::max<int64_t>(1, std::min<int64_t>(nctas, (units + TB / 32 - 1) / (TB / 32)));
+  // the sample waits for everything before it on the stream; each later pass
+  // is a programmatic dependent of the one before (its launch overlaps the
+  // previous pass, its first access waits for it), which hides the launch
+  // latency of the passes that find nothing to do
   topk_sample<DT><<<sctas, TB, 0, s>>>(p);
-  topk_pass1<DT, false><<<nctas, TB, 0, s>>>(p);
-  topk_pass0<DT><<<nctas, TB, 0, s>>>(p);
-  topk_pass1<DT, true><<<nctas, TB, 0, s>>>(p);
-  topk_pass2<DT><<<nctas, TB, 0, s>>>(p);
-  topk_pass3<DT><<<nctas, TB, 0, s>>>(p);
-  topk_pass4<DT><<<nctas, TB, 0, s>>>(p);
-  topk_pass5<DT><<<nctas, TB, 0, s>>>(p);
-  topk_finalize<<<1, TB, 0, s>>>(p);
-  return cudaGetLastError();
+  cudaError_t e = cudaGetLastError();
+  const unsigned g = (unsigned)nctas;
+  if (e == cudaSuccess) e = launch_dependent(topk_pass1<DT, false>, g, TB, 0, s, p);
+  if (e == cudaSuccess) e = launch_dependent(topk_pass0<DT>, g, TB, 0, s, p);
+  if (e == cudaSuccess) e = launch_dependent(topk_pass1<DT, true>, g, TB, 0, s, p);
+  if (e == cudaSuccess) e = launch_dependent(topk_pass2<DT>, g, TB, 0, s, p);
+  if (e == cudaSuccess) e = launch_dependent(topk_pass3<DT>, g, TB, 0, s, p);
+  if (e == cudaSuccess) e = launch_dependent(topk_pass4<DT>, g, TB, 0, s, p);
+  if (e == cudaSuccess) e = launch_dependent(topk_pass5<DT>, g, TB, 0, s, p);
+  if (e == cudaSuccess) e = launch_dependent(topk_finalize, 1u, TB, 0, s, p);
+  return e;
 }
 
 }  // namespace

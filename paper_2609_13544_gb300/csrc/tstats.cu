@@ -50,13 +50,13 @@ struct TS<PEAT_F32> {
 };
 template <>
 struct TS<PEAT_F16> {
-  static constexpr int BYTES = 2, VEC = 8, BITS = 16, MB = 10, BM = 25, WSPAN = 16;
-  static constexpr uint32_t EMASK = 0x1Fu, EINF = 0x1Fu, FLUSH = 1u << 20;
+  static constexpr int BYTES = 2, VEC = 8, BITS = 16, MB = 10, BM = 25;
+  static constexpr uint32_t EMASK = 0x1Fu, EINF = 0x1Fu;
 };
 template <>
 struct TS<PEAT_BF16> {
-  static constexpr int BYTES = 2, VEC = 8, BITS = 16, MB = 7, BM = 134, WSPAN = 20;
-  static constexpr uint32_t EMASK = 0xFFu, EINF = 0xFFu, FLUSH = 1u << 20;
+  static constexpr int BYTES = 2, VEC = 8, BITS = 16, MB = 7, BM = 134;
+  static constexpr uint32_t EMASK = 0xFFu, EINF = 0xFFu;
 };
 
 template <int DT>
@@ -315,6 +315,7 @@ __global__ void __launch_bounds__(TB) tstats_stage1(TsParams p) {
   __shared__ long long lim[2 * NLIMB];
   __shared__ unsigned long long cnt[3];
   __shared__ unsigned int kmin_s, kmax_s;
+  pdl_trigger();  // the finalize kernel may start launching (it waits for this grid)
   const int64_t lo = p.bounds[blockIdx.x], hi = p.bounds[blockIdx.x + 1];
   if (lo >= hi) return;
   // the segment holding lo: the last s with offsets[s] <= lo (empty segments skipped)
@@ -423,6 +424,7 @@ __global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
   constexpr int VEC = T::VEC, B = T::BYTES, MB = T::MB, WS = H16<DT>::WS, WSB = H16<DT>::WSB;
   constexpr int NB = h16_bins<DT>();
   constexpr uint32_t WSM = (uint32_t)WS << MB, MAGM = (1u << (T::BITS - 1)) - 1u;
+  pdl_trigger();  // the finalize kernel may start launching (it waits for this grid)
   extern __shared__ uint32_t hist[];  // NB bins, then the bins of +0 and -0
   __shared__ long long lim[2 * NLIMB];
   __shared__ unsigned long long cnt[3];
@@ -762,6 +764,7 @@ __device__ __noinline__ double seg_mean(const TsAcc& acc, uint64_t nf) {
 // accumulator cleared for the next call.
 constexpr int FIN_THREADS = 128;
 __global__ void __launch_bounds__(FIN_THREADS) tstats_finalize(TsParams p) {
+  pdl_wait();  // stage 1 complete
   const int64_t s = blockIdx.x;
   const int tid = threadIdx.x, warp = tid >> 5;
   TsAcc& acc = p.acc[s];
@@ -830,8 +833,10 @@ cudaError_t launch_t(const TsParams& p, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     tstats_hist<DT><<<p.nctas, TB, hist_smem<DT>(), s>>>(p);
   }
-  tstats_finalize<<<(unsigned)p.nseg, FIN_THREADS, 0, s>>>(p);
-  return cudaGetLastError();
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  // a programmatic dependent of stage 1: its launch overlaps stage 1's end
+  return launch_dependent(tstats_finalize, (unsigned)p.nseg, FIN_THREADS, 0, s, p);
 }
 
 }  // namespace

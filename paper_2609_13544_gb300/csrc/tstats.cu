@@ -396,26 +396,52 @@ constexpr int h16_bins() {
   return 2 * H16<DT>::WS << TS<DT>::MB;
 }
 
-// an element the histogram does not take: counted (NaN, infinity) or added
-// to the digits with its order key (finite), on the CTA's shared totals
+// One thread's share of the nonzero elements the histogram does not take,
+// in the thread's own shared-memory slot (no atomics, so a tensor whose bulk
+// lies outside the window does not serialise on a few addresses): NaN and
+// infinity counts, the extreme order keys of the finite ones, and the exact
+// sums over the LW binades below the window, t = m 2^(e - lw) < 2^(MB + LW)
+// in units of 2^(lw - BM) (sum of t as int64, of t^2 in 128 bits: a piece
+// holds fewer than 2^32 elements, so a thread fewer than 2^24).  Binades
+// above the window or further below go to the CTA's digits.
+constexpr int LW = 28;
+struct SlowSlot {
+  long long s1;
+  unsigned long long s2lo, s2hi;
+  uint32_t kmn, kmx, nnan, ninf;
+};
+
 template <int DT>
-__device__ __noinline__ void h16_slow(uint32_t r, long long* lim, unsigned long long* cnt, unsigned int* kmin_s,
-                                      unsigned int* kmax_s) {
+__device__ __noinline__ void h16_slow(uint32_t r, int lw, SlowSlot& q, long long* lim) {
   using T = TS<DT>;
   const uint32_t e = (r >> T::MB) & T::EMASK, mant = r & ((1u << T::MB) - 1u);
   if (e == T::EINF) {
-    atomicAdd(&cnt[mant ? 1 : 2], 1ull);
+    if (mant) q.nnan++;
+    else q.ninf++;
     return;
   }
   const uint32_t k = order_key(raw_to_f32<DT>(r));
-  atomicMin(kmin_s, k);
-  atomicMax(kmax_s, k);
+  q.kmn = min(q.kmn, k);
+  q.kmx = max(q.kmx, k);
   const uint32_t m = mant | (e ? (1u << T::MB) : 0u);
-  if (m) ts_slow<DT>(m, e ? (int)e : 1, (r >> (T::BITS - 1)) & 1u, lim);
+  if (!m) return;
+  const int ee = e ? (int)e : 1;
+  const bool neg = (r >> (T::BITS - 1)) & 1u;
+  if (ee >= lw && ee - lw < LW) {
+    const uint64_t t = (uint64_t)m << (ee - lw);
+    q.s1 += neg ? -(long long)t : (long long)t;
+    const unsigned __int128 s2 = (((unsigned __int128)q.s2hi << 64) | q.s2lo) + (unsigned __int128)t * t;
+    q.s2lo = (uint64_t)s2;
+    q.s2hi = (uint64_t)(s2 >> 64);
+  } else {
+    ts_slow<DT>(m, ee, neg, lim);
+  }
 }
 
 template <int DT>
-__global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
+// four CTAs per SM (at most 64 registers: the piece end's wider sums must not
+// cost the element loop its occupancy)
+__global__ void __launch_bounds__(TB, 4) tstats_hist(TsParams p) {
   using T = TS<DT>;
   constexpr int VEC = T::VEC, B = T::BYTES, MB = T::MB, WS = H16<DT>::WS, WSB = H16<DT>::WSB;
   constexpr int NB = h16_bins<DT>();
@@ -425,7 +451,9 @@ __global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
   __shared__ long long lim[2 * NLIMB];
   __shared__ unsigned long long cnt[3];
   __shared__ unsigned int kmin_s, kmax_s, emax_s;
-  __shared__ unsigned long long red[3][TB / 32][4];
+  __shared__ unsigned long long red[4][TB / 32][4];
+  __shared__ SlowSlot slow[TB];
+  __shared__ int took_s;  // some warp of the piece took elements outside the window
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t lo = p.bounds[blockIdx.x], hi = p.bounds[blockIdx.x + 1];
   if (lo >= hi) return;
@@ -447,7 +475,9 @@ __global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
       kmin_s = 0xFFFFFFFFu;
       kmax_s = 0;
       emax_s = 0;
+      took_s = 0;
     }
+    slow[tid] = SlowSlot{0, 0, 0, 0xFFFFFFFFu, 0u, 0u, 0u};
     // the vector grid inside the piece
     int64_t a0 = b, nv = 0;
     if (p.p0 >= 0 && p.p0 < p.n_total) {
@@ -476,6 +506,7 @@ __global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
     }
     __syncthreads();
     const int lb = max(1, min((int)emax_s + 2 - WS, (int)T::EINF - WS));  // window exponents [lb, lb + WS)
+    const int lw = max(1, lb - LW);                                        // the slots' binades [lw, lw + LW)
     const uint32_t lbm = (uint32_t)lb << MB;
     auto elem = [&](uint32_t r) {
       const uint32_t mag = r & MAGM, t = mag - lbm;
@@ -487,7 +518,7 @@ __global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
         asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(hb + 4u * (NB + (r >> (T::BITS - 1)))), "r"(1u)
                      : "memory");
       } else {
-        h16_slow<DT>(r, lim, cnt, &kmin_s, &kmax_s);
+        h16_slow<DT>(r, lw, slow[tid], lim);
       }
     };
     constexpr int U = 4;
@@ -536,9 +567,11 @@ __global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
       kmn = min(kmn, k);
       kmx = max(kmx, k);
     }
-    // block totals: 32-bit words of each 128-bit sum summed over the warp,
-    // then over the warps by warp 0, added as digits
+    // block totals: 32-bit words of each 128-bit sum (the window's, and the
+    // slots' below it) summed over the warp, then over the warps by thread 0,
+    // added as digits; the slots' counts and extreme keys with them
     {
+      const SlowSlot q0 = slow[tid];
       const unsigned __int128 d = s1p - s1n;  // |S1| < 2^120: two's complement in 128 bits
 #pragma unroll
       for (int q = 0; q < 4; q++) {
@@ -552,6 +585,36 @@ __global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
           red[0][warp][q] = w1;
           red[1][warp][q] = w2;
         }
+      }
+      // the slots: only a warp that took elements outside the window has work here
+      const bool took = q0.kmn != 0xFFFFFFFFu || (q0.nnan | q0.ninf) != 0u;
+      if (__any_sync(0xFFFFFFFFu, took)) {
+        const unsigned __int128 dl = (unsigned __int128)(__int128)q0.s1;
+        const unsigned __int128 s2l = ((unsigned __int128)q0.s2hi << 64) | q0.s2lo;
+#pragma unroll
+        for (int q = 0; q < 4; q++) {
+          uint64_t w1 = (uint32_t)(dl >> (32 * q)), w2 = (uint32_t)(s2l >> (32 * q));
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+            w1 += __shfl_xor_sync(0xFFFFFFFFu, w1, o);
+            w2 += __shfl_xor_sync(0xFFFFFFFFu, w2, o);
+          }
+          if (lane == 0) {
+            red[2][warp][q] = w1;
+            red[3][warp][q] = w2;
+          }
+        }
+        kmn = min(kmn, q0.kmn);
+        kmx = max(kmx, q0.kmx);
+        const uint32_t nn = __reduce_add_sync(0xFFFFFFFFu, q0.nnan), ni = __reduce_add_sync(0xFFFFFFFFu, q0.ninf);
+        if (lane == 0) {
+          if (nn) atomicAdd(&cnt[1], (unsigned long long)nn);
+          if (ni) atomicAdd(&cnt[2], (unsigned long long)ni);
+          took_s = 1;
+        }
+      } else if (lane < 4) {
+        red[2][warp][lane] = 0;
+        red[3][warp][lane] = 0;
       }
       kmn = __reduce_min_sync(0xFFFFFFFFu, kmn);
       kmx = __reduce_max_sync(0xFFFFFFFFu, kmx);
@@ -580,6 +643,21 @@ __global__ void __launch_bounds__(TB) tstats_hist(TsParams p) {
       for_digits(mag1, u, neg, [&](int j, int64_t v) { lim_add(lim, j, v); });
       for (int q = 0; q < 4; q++)
         if (S2w[q]) for_digits(S2w[q], 2 * u + 32 * q, false, [&](int j, int64_t v) { lim_add(lim + NLIMB, j, v); });
+      // the slots' sums, in units of 2^(lw - BM)
+      unsigned __int128 L1 = 0;
+      for (int q = 0; q < 4 && took_s; q++) {
+        unsigned __int128 t1 = 0, t2 = 0;
+        for (int w = 0; w < TB / 32; w++) {
+          t1 += red[2][w][q];
+          t2 += red[3][w][q];
+        }
+        L1 += t1 << (32 * q);
+        const int ul = lw - T::BM;
+        if (t2) for_digits(t2, 2 * ul + 32 * q, false, [&](int j, int64_t v) { lim_add(lim + NLIMB, j, v); });
+      }
+      const bool negl = (L1 >> 127) != 0;
+      const unsigned __int128 magl = negl ? (unsigned __int128)0 - L1 : L1;
+      if (magl) for_digits(magl, lw - T::BM, negl, [&](int j, int64_t v) { lim_add(lim, j, v); });
     }
     __syncthreads();
     TsAcc& acc = p.acc[seg];

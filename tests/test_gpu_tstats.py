@@ -145,6 +145,34 @@ def test_workload_c3_segments(peat_gpu, oracle, h):
     check(peat_gpu, oracle, h, bits, "f32", offsets=w.offsets, ctx="c3 goldens")
 
 
+def test_workload_c4_checkpoint_sample(peat_gpu, oracle, h):
+    """The fp16 GPT-2-medium checkpoint (Laplace values over about 20 binades):
+    its first 8 M elements with the workload's own segment boundaries."""
+    from paper_2609_13544_gb300 import workloads as W
+    w = W.c4_gpt2_medium(device="cuda")
+    P = 8_000_000
+    offsets = [int(o) for o in w.offsets if int(o) < P] + [P]
+    bits = w.golden[:P].cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+    del w
+    check(peat_gpu, oracle, h, bits, "f16", offsets=offsets, ctx="c4 goldens")
+
+
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+def test_wide_range_16bit(peat_gpu, oracle, h, dtype):
+    """Magnitudes log-uniform over every binade of the format (fp16 30, bf16
+    250) with random signs, zeros and subnormals: most elements fall outside
+    any window and take the exact path."""
+    rng = np.random.default_rng(41)
+    n = 1_000_003
+    e = rng.integers(0, 31 if dtype == "f16" else 255, n, dtype=np.uint32)
+    m = rng.integers(0, 1 << (10 if dtype == "f16" else 7), n, dtype=np.uint32)
+    sgn = rng.integers(0, 2, n, dtype=np.uint32)
+    bits = ((sgn << 15) | (e << (10 if dtype == "f16" else 7)) | m).astype(np.uint16)
+    check(peat_gpu, oracle, h, bits, dtype, ctx="wide")
+    offsets = [0, 17, 300_000, 300_000, 999_999, n]
+    check(peat_gpu, oracle, h, bits, dtype, offsets=offsets, ctx="wide segmented")
+
+
 def test_workload_c2_full_against_torch(peat_gpu, h):
     """The [8,2048,4096] bf16 activation: every bf16 value and square is exact in
     binary64, so torch's float64 sums agree to their own rounding."""

@@ -661,7 +661,7 @@ def run_gpu(args) -> None:
         for _ in range(3):
             peat.peat_topk_mean_raw(h, g, c, 1, 10, tk_out, stream)
         barrier()
-        tk_calls = max(20, min(200, args.steps // 2))
+        tk_calls = max(100, min(400, 5 * args.steps))
         t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         t0.record(stream)
         for _ in range(tk_calls):
@@ -688,7 +688,7 @@ def run_gpu(args) -> None:
         for _ in range(3):
             peat.peat_tensor_stats_raw(h, g, off, ts_out, stream)
         barrier()
-        ts_calls = max(20, min(200, args.steps // 2))
+        ts_calls = max(100, min(400, 5 * args.steps))
         t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         t0.record(stream)
         for _ in range(ts_calls):

@@ -380,11 +380,11 @@ __global__ void __launch_bounds__(TB) tstats_stage1(TsParams p) {
 // element inside it in a shared histogram indexed by (sign, exponent - Lb,
 // significand field): one shared atomic per element, no per-element sums,
 // keys or branches beyond the window test.  Zeros have two bins of their
-// own; NaN, infinities, subnormals and elements outside the window take the
-// exact path above (digits, counted extremes).  At the end of the piece each
-// bin adds count * value and count * value^2 exactly (integers in units of
-// the window's floor), and the extreme nonzero bins give the finite minimum
-// and maximum.
+// own; NaN, infinities, subnormals and elements outside the window go to the
+// thread's slot (h16_slow below) or, further out, to the digits.  At the end
+// of the piece each bin adds count * value and count * value^2 exactly
+// (integers in units of the window's floor), and the extreme nonzero bins
+// give the finite minimum and maximum.
 template <int DT>
 struct H16;
 template <>
